@@ -1,0 +1,223 @@
+"""CPU oracle for the Kernel Quantization hot path (arXiv 2003.05148).
+
+TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the CPU
+baseline leg of ``bench.py`` are the only callers. The CUDA library never imports,
+links or runs anything here, and nothing here imports the CUDA library.
+
+The compute-heavy steps live in ``kq_oracle.c`` (plain C, built with
+``-ffp-contract=off`` so that only the ``fmaf`` calls written in the source fuse);
+this module loads it with ctypes and adds the storage accounting of Eq. 4-7,
+which is exact integer / rational arithmetic done here in Python.
+
+Parity pins for every function are in ``tests/test_oracle.py``.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+import subprocess
+from fractions import Fraction
+from typing import Optional
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "kq_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "libkq_oracle.so")
+_CFLAGS = ["-O2", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared", "-pthread"]
+
+D = 9
+LEVELS = 64
+
+
+def build(force: bool = False) -> str:
+    """Compile kq_oracle.c into oracle/_build/libkq_oracle.so (gcc)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        subprocess.run(["gcc", *_CFLAGS, _SRC, "-o", tmp, "-lm"], check=True)
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+_lib = None
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        lib = ctypes.CDLL(build())
+        P = ctypes.c_void_p
+        i64, i32, f64 = ctypes.c_int64, ctypes.c_int32, ctypes.c_double
+        lib.kqo_assign.argtypes = [P, i64, P, i32, P, P, P, P, i32]
+        lib.kqo_assign.restype = None
+        lib.kqo_update.argtypes = [P, i64, P, i32, P, P, P]
+        lib.kqo_update.restype = None
+        lib.kqo_objective.argtypes = [P, i64]
+        lib.kqo_objective.restype = f64
+        lib.kqo_fit.argtypes = [P, i64, i32, P, i32, P, P, P, P, i32]
+        lib.kqo_fit.restype = i32
+        lib.kqo_level_scale.argtypes = [P, i32, P]
+        lib.kqo_level_scale.restype = i32
+        lib.kqo_level_fit.argtypes = [P, i32, P, i32, P, P]
+        lib.kqo_level_fit.restype = i32
+        lib.kqo_reconstruct.argtypes = [P, i64, P, P, P, P]
+        lib.kqo_reconstruct.restype = None
+        lib.kqo_encode.argtypes = [P, i64, P, P]
+        lib.kqo_encode.restype = None
+        lib.kqo_gather_rows.argtypes = [P, P, i32, P]
+        lib.kqo_gather_rows.restype = None
+        _lib = lib
+    return _lib
+
+
+def _ptr(a: Optional[np.ndarray]):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _f32(a) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=np.float32)
+
+
+def _i32(a) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=np.int32)
+
+
+def default_threads() -> int:
+    try:
+        return max(1, len(os.sched_getaffinity(0)))
+    except AttributeError:  # pragma: no cover
+        return max(1, os.cpu_count() or 1)
+
+
+def assign(W, C, threads: int = 1, gap: bool = False):
+    """Eq. 1 assignment (Sec. 3.1). Returns (idx int32, dist fp32[, d1, d2 fp64]).
+
+    idx_i = argmin_k d(W_i, C_k) with the fp32 direct-form distance and the
+    lowest index on ties. With ``gap`` also the fp64 best and second-best
+    distances of every row, for judging how close each decision was.
+    """
+    W, C = _f32(W).reshape(-1, D), _f32(C).reshape(-1, D)
+    n, K = W.shape[0], C.shape[0]
+    idx = np.empty(n, np.int32)
+    dist = np.empty(n, np.float32)
+    d1 = np.empty(n, np.float64) if gap else None
+    d2 = np.empty(n, np.float64) if gap else None
+    _load().kqo_assign(_ptr(W), n, _ptr(C), K, _ptr(idx), _ptr(dist), _ptr(d1), _ptr(d2), threads)
+    return (idx, dist, d1, d2) if gap else (idx, dist)
+
+
+def update(W, idx, C_prev):
+    """Eq. 1 centroid step (Sec. 3.1): (C_next fp32 (K, 9), counts int32 (K,))."""
+    W, C_prev, idx = _f32(W).reshape(-1, D), _f32(C_prev).reshape(-1, D), _i32(idx)
+    K = C_prev.shape[0]
+    C_next = np.empty_like(C_prev)
+    counts = np.empty(K, np.int32)
+    _load().kqo_update(_ptr(W), W.shape[0], _ptr(idx), K, _ptr(C_prev), _ptr(C_next), _ptr(counts))
+    return C_next, counts
+
+
+def objective(dist) -> float:
+    """Eq. 1 objective: fp64 sum of per-kernel distances in ascending order."""
+    dist = _f32(dist)
+    return float(_load().kqo_objective(_ptr(dist), dist.shape[0]))
+
+
+def fit(W, C_init, iters: int, threads: int = 1):
+    """k-means of Eq. 1 for a fixed number of iterations.
+
+    Returns (C_T, idx_T, counts_T, objective[0..T]).
+    """
+    W, C0 = _f32(W).reshape(-1, D), _f32(C_init).reshape(-1, D)
+    n, K = W.shape[0], C0.shape[0]
+    C = np.empty_like(C0)
+    idx = np.empty(n, np.int32)
+    counts = np.empty(K, np.int32)
+    obj = np.empty(iters + 1, np.float64)
+    _load().kqo_fit(_ptr(W), n, K, _ptr(C0), iters, _ptr(C), _ptr(idx), _ptr(counts), _ptr(obj), threads)
+    return C, idx, counts, obj
+
+
+def level_scale(C, counts) -> int:
+    """Exponent S of the fixed-point scale 2^S used for the exact level sums."""
+    C, counts = _f32(C).reshape(-1, D), _i32(counts)
+    return int(_load().kqo_level_scale(_ptr(C), C.shape[0], _ptr(counts)))
+
+
+def level_fit(C, counts, max_iters: int = 100):
+    """Sec. 3.2 6-bit codebook quantisation: (levels fp32 (64,), codes uint8 (K, 9), updates)."""
+    C, counts = _f32(C).reshape(-1, D), _i32(counts)
+    K = C.shape[0]
+    levels = np.empty(LEVELS, np.float32)
+    codes = np.empty((K, D), np.uint8)
+    it = _load().kqo_level_fit(_ptr(C), K, _ptr(counts), max_iters, _ptr(levels), _ptr(codes))
+    return levels, codes, int(it)
+
+
+def encode(values, levels):
+    """Sec. 3.2 encode: nearest of the 64 levels by fp32 |v - level|, lower index on ties."""
+    v, levels = _f32(values).reshape(-1), _f32(levels)
+    codes = np.empty(v.shape[0], np.uint8)
+    _load().kqo_encode(_ptr(v), v.shape[0], _ptr(levels), _ptr(codes))
+    return codes
+
+
+def reconstruct(idx, C, codes=None, levels=None):
+    """Sec. 3.2 testing phase: W' (n, 9) from kernel indices and the (decoded) codebook."""
+    idx, C = _i32(idx), _f32(C).reshape(-1, D)
+    out = np.empty((idx.shape[0], D), np.float32)
+    if codes is not None:
+        codes = np.ascontiguousarray(codes, dtype=np.uint8).reshape(-1, D)
+        levels = _f32(levels)
+    _load().kqo_reconstruct(_ptr(idx), idx.shape[0], _ptr(C), _ptr(codes), _ptr(levels), _ptr(out))
+    return out
+
+
+def gather_rows(W, sel):
+    """Codeword initialisation: C_0[j] = W[sel[j]]."""
+    W = _f32(W).reshape(-1, D)
+    sel = np.ascontiguousarray(sel, dtype=np.int64)
+    C0 = np.empty((sel.shape[0], D), np.float32)
+    _load().kqo_gather_rows(_ptr(W), _ptr(sel), sel.shape[0], _ptr(C0))
+    return C0
+
+
+# ---------------------------------------------------------------------------
+# Storage accounting, Sec. 3.2-3.3 and Sec. 4.1 (Eq. 4-7). Exact arithmetic.
+# ---------------------------------------------------------------------------
+
+def ceil_log2(k: int) -> int:
+    """ceil(log2 k) for an integer k >= 1, by integer bit length (k = 1 -> 0)."""
+    if k < 1:
+        raise ValueError("codebook size must be >= 1")
+    return (k - 1).bit_length()
+
+
+@dataclasses.dataclass(frozen=True)
+class Report:
+    index_bits: int
+    codebook_bits: int
+    total_bits: int
+    beta: Fraction  # Eq. 7, bits per parameter
+    ratio_kq: Fraction  # Eq. 6, C_KQ
+
+
+def report(n: int, k: int, omega: int = 3, b_c: int = 32, b_fp: int = 32) -> Report:
+    """Eq. 4 (B), Eq. 6 (C_KQ) and Eq. 7 (beta) for one layer.
+
+    B = k * omega^2 * b_c + n * ceil(log2 k); beta = B / (n omega^2);
+    C_KQ = n omega^2 b_FP / B. b_c = 32 for kernel-level only (K), 6 after
+    codebook quantisation (K+C); the 64-entry level table is not counted.
+    """
+    idx_bits = n * ceil_log2(k)
+    cb_bits = k * omega * omega * b_c
+    total = idx_bits + cb_bits
+    return Report(idx_bits, cb_bits, total, Fraction(total, n * omega * omega),
+                  Fraction(n * omega * omega * b_fp, total))
+
+
+def ratio_conventional(n: int, omega: int, u: int, b_1: int, b_fp: int = 32) -> Fraction:
+    """Eq. 5: C_con = n omega^2 b_FP / (u b_1 + n omega^2 ceil(log2 u))."""
+    return Fraction(n * omega * omega * b_fp, u * b_1 + n * omega * omega * ceil_log2(u))

@@ -1,0 +1,350 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+No GPU. Each test checks the oracle against something other than itself: values
+the paper prints (tests/golden), exact rational arithmetic on small inputs,
+closed forms, invariants and textbook special cases.
+"""
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "paper_tables.txt")
+
+
+def _golden_rows():
+    rows = []
+    with open(GOLDEN) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            rows.append(line.split())
+    return rows
+
+
+# ---------------------------------------------------------------------------
+# Eq. 4-7 storage accounting against Tables 4-5 and the Sec. 4.2.1 ablation.
+# ---------------------------------------------------------------------------
+
+def _cell(s):
+    return float(s.rstrip("!")), s.endswith("!")
+
+
+@pytest.mark.parametrize("row", [r for r in _golden_rows() if r[0].startswith("table")], ids=lambda r: r[0] + r[1])
+def test_report_tables_4_5(row):
+    src, layer, n, k = row[0], row[1], int(row[2]), int(row[3])
+    pK, pKC, bK, bKC = (_cell(c) for c in row[4:8])
+    rK = oracle.report(n, k, 3, 32)
+    rKC = oracle.report(n, k, 3, 6)
+    checks = [(float(rK.beta), bK, 0.01), (float(rKC.beta), bKC, 0.01),
+              (float(rK.beta) * 100 / 32, pK, 0.03), (float(rKC.beta) * 100 / 32, pKC, 0.03)]
+    for exact, (printed, bad), tol in checks:
+        if bad:
+            # The printed cell is one the paper got wrong for this (n, k).
+            assert abs(exact - printed) > tol, (src, layer, exact, printed)
+        else:
+            assert abs(exact - printed) <= tol, (src, layer, exact, printed)
+
+
+@pytest.mark.parametrize("row", [r for r in _golden_rows() if r[0].startswith("ablation")], ids=lambda r: r[1])
+def test_report_ablation_k128(row):
+    n, k = int(row[2]), int(row[3])
+    ratioK, ratioKC, betaKC = float(row[4]), float(row[5]), float(row[6])
+    rK, rKC = oracle.report(n, k, 3, 32), oracle.report(n, k, 3, 6)
+    # printed to two decimals, sometimes truncated rather than rounded
+    assert abs(float(rK.ratio_kq) - ratioK) <= 0.01
+    assert abs(float(rKC.ratio_kq) - ratioKC) <= 0.01
+    assert abs(float(rKC.beta) - betaKC) <= 0.001
+    # Eq. 7 is the reciprocal of Eq. 6 times 32
+    assert rKC.beta * rKC.ratio_kq == 32
+
+
+def test_report_closed_forms():
+    # Sec. 4.2.2: 256 entries need 8-bit indices, 512 need 9, 614 need 10.
+    assert oracle.ceil_log2(256) == 8
+    assert oracle.ceil_log2(512) == 9
+    assert oracle.ceil_log2(614) == 10
+    assert oracle.ceil_log2(1) == 0
+    assert oracle.ceil_log2(2) == 1
+    assert oracle.ceil_log2(3) == 2
+    with pytest.raises(ValueError):
+        oracle.ceil_log2(0)
+    # Sec. 3.3: conventional quantisation is limited to 32x (u = 2, one bit per weight) ...
+    n = 10 ** 12
+    con = oracle.ratio_conventional(n, 3, 2, 32)
+    assert con < 32 and float(con) == pytest.approx(32, rel=1e-9)
+    # ... and KQ with 3x3 kernels to 288x (k = 2, one bit per kernel).
+    kq = oracle.report(n, 2, 3, 32).ratio_kq
+    assert kq < 288 and float(kq) == pytest.approx(288, rel=1e-9)
+    # bit counts: B = k w^2 b_c + n ceil(log2 k)
+    r = oracle.report(4096, 128, 3, 6)
+    assert (r.index_bits, r.codebook_bits, r.total_bits) == (4096 * 7, 128 * 9 * 6, 4096 * 7 + 128 * 54)
+
+
+# ---------------------------------------------------------------------------
+# Eq. 1 assignment against exhaustive exact argmin.
+# ---------------------------------------------------------------------------
+
+def _exact_d(x, c):
+    return sum((Fraction(float(a)) - Fraction(float(b))) ** 2 for a, b in zip(x, c))
+
+
+def _int_case(n, K, seed, lo=-6, hi=7):
+    rng = np.random.default_rng(seed)
+    W = rng.integers(lo, hi, size=(n, 9)).astype(np.float32)
+    C = rng.integers(lo, hi, size=(K, 9)).astype(np.float32)
+    return W, C
+
+
+@pytest.mark.parametrize("n,K,seed", [(64, 16, 0), (37, 5, 1), (50, 1, 2), (20, 13, 3)])
+def test_assign_brute_force_integers(n, K, seed):
+    # Small integers: every fp32 difference, square and partial sum is exact,
+    # so the fp32 direct form equals the exact distance and the argmin (lowest
+    # index on ties) must equal exhaustive exact search, ties included.
+    W, C = _int_case(n, K, seed)
+    C[K // 2] = C[0]  # duplicate codeword: the lower index must win
+    W[0] = C[K - 1]
+    idx, dist = oracle.assign(W, C)
+    for i in range(n):
+        ds = [_exact_d(W[i], C[k]) for k in range(K)]
+        m = min(ds)
+        assert idx[i] == ds.index(m)
+        assert Fraction(float(dist[i])) == m
+    first = next(k for k in range(K) if np.array_equal(C[k], C[K - 1]))
+    assert idx[0] == first and dist[0] == 0
+
+
+def test_assign_constructed_ties():
+    # x equidistant from c_3 and c_1 (mirror images): index 1 must win.
+    C = np.zeros((5, 9), np.float32)
+    C[:, 0] = [9, 1, 7, -5, 3]
+    C[3, 0] = -1
+    W = np.zeros((1, 9), np.float32)  # d = 1 to both c_1 (x0=1) and c_3 (x0=-1)
+    idx, dist = oracle.assign(W, C)
+    assert idx[0] == 1 and dist[0] == 1.0
+    # all codewords identical -> index 0
+    idx, _ = oracle.assign(W, np.ones((7, 9), np.float32))
+    assert idx[0] == 0
+
+
+def test_assign_float_against_exact():
+    # Random floats: the fp32 decision equals the exact argmin wherever the exact
+    # relative gap is far above fp32 rounding; the fp64 best/second-best the
+    # oracle reports agree with exact arithmetic.
+    W = synth.random_kernels(40, 9, 11, 0.05)
+    C = synth.random_kernels(12, 9, 12, 0.05)
+    idx, dist, d1, d2 = oracle.assign(W, C, gap=True)
+    for i in range(W.shape[0]):
+        ds = sorted((_exact_d(W[i], C[k]), k) for k in range(12))
+        (e1, k1), (e2, _) = ds[0], ds[1]
+        assert float(d1[i]) == pytest.approx(float(e1), rel=1e-12)
+        assert float(d2[i]) == pytest.approx(float(e2), rel=1e-12)
+        assert float(dist[i]) == pytest.approx(float(e1), rel=1e-6)
+        if (e2 - e1) / e1 > 1e-5:
+            assert idx[i] == k1
+
+
+def test_assign_threads_do_not_change_result():
+    W = synth.random_kernels(1001, 9, 5)
+    C = synth.random_kernels(33, 9, 6)
+    a = oracle.assign(W, C, threads=1)
+    b = oracle.assign(W, C, threads=7)
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1].view(np.int32), b[1].view(np.int32))
+
+
+def test_assign_nonfinite_rules():
+    # a NaN kernel never beats the initial (+inf, 0): index 0
+    W = np.full((1, 9), np.nan, np.float32)
+    idx, dist = oracle.assign(W, synth.random_kernels(4, 9, 1))
+    assert idx[0] == 0 and np.isinf(dist[0])
+
+
+# ---------------------------------------------------------------------------
+# Eq. 1 update: each codeword is the mean of its members.
+# ---------------------------------------------------------------------------
+
+def _f32_ulps(a, b):
+    ai = np.array([a], np.float32).view(np.int32)[0]
+    bi = np.array([b], np.float32).view(np.int32)[0]
+    return abs(int(ai) - int(bi))
+
+
+def test_update_mean_of_members_exact():
+    n, K = 300, 9
+    W = synth.random_kernels(n, 9, 21, 0.1)
+    idx = synth.below(synth.stream_key(22, 2), n, K - 1).astype(np.int32)  # codeword K-1 stays empty
+    C_prev = synth.random_kernels(K, 9, 23)
+    C_next, counts = oracle.update(W, idx, C_prev)
+    for k in range(K):
+        members = np.nonzero(idx == k)[0]
+        assert counts[k] == len(members)
+        if len(members) == 0:
+            assert np.array_equal(C_next[k].view(np.int32), C_prev[k].view(np.int32))
+            continue
+        for j in range(9):
+            exact = sum(Fraction(float(W[i, j])) for i in members) / len(members)
+            assert _f32_ulps(C_next[k, j], np.float32(float(exact))) <= 1
+
+
+def test_update_dyadic_bit_exact():
+    # values on a 2^-10 grid: fp64 sums are exact and the mean rounds once.
+    rng = np.random.default_rng(3)
+    W = (rng.integers(-512, 512, size=(257, 9)) / 1024.0).astype(np.float32)
+    idx = rng.integers(0, 6, size=257).astype(np.int32)
+    C_next, counts = oracle.update(W, idx, np.zeros((6, 9), np.float32))
+    for k in range(6):
+        m = idx == k
+        for j in range(9):
+            exact = Fraction(int(round(W[m, j].astype(np.float64).sum() * 1024)), 1024 * int(m.sum()))
+            assert C_next[k, j] == np.float32(float(exact))
+
+
+def test_k1_global_mean():
+    W = synth.random_kernels(500, 9, 31, 0.2)
+    C, idx, counts, obj = oracle.fit(W, W[:1], iters=3)
+    assert np.all(idx == 0) and counts[0] == 500
+    for j in range(9):
+        exact = sum(Fraction(float(v)) for v in W[:, j]) / 500
+        assert _f32_ulps(C[0, j], np.float32(float(exact))) <= 1
+
+
+def test_k_equals_n_identity():
+    W = synth.random_kernels(64, 9, 41)
+    C, idx, counts, obj = oracle.fit(W, W, iters=2)
+    assert np.array_equal(idx, np.arange(64))
+    assert np.all(counts == 1)
+    assert np.all(obj == 0.0)
+    assert np.array_equal(C.view(np.int32), W.view(np.int32))
+
+
+def test_fit_objective_non_increasing_and_consistent():
+    lay = synth.workload(1).layers[0]
+    W, sel = synth.layer_inputs(lay)
+    C0 = oracle.gather_rows(W, sel)
+    assert np.array_equal(C0, W[sel])
+    C, idx, counts, obj = oracle.fit(W, C0, iters=10, threads=4)
+    assert np.all(obj[1:] <= obj[:-1] * (1 + 1e-6))
+    assert obj[-1] < obj[0]
+    assert counts.sum() == W.shape[0]
+    assert np.array_equal(counts, np.bincount(idx, minlength=C.shape[0]))
+    # the fit is the composition of its steps
+    Ct = C0
+    for _ in range(10):
+        i_t, d_t = oracle.assign(W, Ct)
+        Ct, _ = oracle.update(W, i_t, Ct)
+    i_T, d_T = oracle.assign(W, Ct)
+    assert np.array_equal(Ct, C) and np.array_equal(i_T, idx)
+    assert oracle.objective(d_T) == obj[-1]
+
+
+# ---------------------------------------------------------------------------
+# Sec. 3.2: weighted 64-level codebook quantisation.
+# ---------------------------------------------------------------------------
+
+def test_level_fit_equally_spaced_is_fixed_point():
+    # scalars 0..63 (plus repeats): linspace init hits them exactly, nothing moves.
+    C = np.concatenate([np.arange(64), np.arange(8)]).astype(np.float32).reshape(8, 9)
+    counts = np.ones(8, np.int32)
+    levels, codes, it = oracle.level_fit(C, counts)
+    assert np.array_equal(levels, np.arange(64, dtype=np.float32))
+    assert np.array_equal(codes.reshape(-1), C.reshape(-1).astype(np.uint8))
+    assert it == 1
+
+
+def _exact_weighted_means(C, counts, codes):
+    out = {}
+    v = C.reshape(-1)
+    z = np.repeat(counts, 9)
+    for l in np.unique(codes):
+        m = (codes.reshape(-1) == l) & (z > 0)
+        if m.any():
+            out[int(l)] = sum(Fraction(float(a)) * int(w) for a, w in zip(v[m], z[m])) / int(z[m].sum())
+    return out
+
+
+def test_level_fit_converged_levels_are_weighted_means():
+    rng = np.random.default_rng(7)
+    C = (rng.integers(-4096, 4096, size=(200, 9)) / 65536.0).astype(np.float32)
+    counts = rng.integers(0, 50, size=200).astype(np.int32)
+    levels, codes, it = oracle.level_fit(C, counts, max_iters=100)
+    assert it < 100  # converged
+    assert np.all(np.diff(levels) >= 0)
+    means = _exact_weighted_means(C, counts, codes)
+    for l, mval in means.items():
+        assert _f32_ulps(levels[l], np.float32(float(mval))) <= 1
+    # every scalar sits at its nearest level (exact arithmetic; lower index on ties)
+    for v, c in zip(C.reshape(-1), codes.reshape(-1)):
+        d = [abs(Fraction(float(v)) - Fraction(float(L))) for L in levels]
+        assert c == d.index(min(d))
+
+
+def test_level_fit_weights_equal_repetition():
+    # Weighted k-means with integer weights equals plain k-means on the multiset
+    # in which each codeword appears z_k times (the reconstructed K-only weights).
+    C = synth.random_kernels(60, 9, 51, 0.05)
+    counts = synth.random_counts(60, 52, 6)
+    counts[3] = 0
+    levels, codes, it = oracle.level_fit(C, counts)
+    rep = np.repeat(C, counts, axis=0)
+    lv2, cd2, it2 = oracle.level_fit(rep, np.ones(rep.shape[0], np.int32))
+    assert np.array_equal(levels.view(np.int32), lv2.view(np.int32))
+    assert it == it2
+    assert np.array_equal(np.repeat(codes, counts, axis=0), cd2)
+    # ignoring the weights gives a different answer on this input
+    lv3, _, _ = oracle.level_fit(C[counts > 0], np.ones(int((counts > 0).sum()), np.int32))
+    assert not np.array_equal(levels, lv3)
+
+
+def test_level_fit_codes_round_trip():
+    C = synth.random_kernels(300, 9, 61, 0.05)
+    counts = synth.random_counts(300, 62, 100)
+    levels, codes, _ = oracle.level_fit(C, counts)
+    assert codes.max() < 64
+    assert np.unique(levels).size == 64
+    # encoding a level value gives back its own code
+    assert np.array_equal(oracle.encode(levels, levels), np.arange(64))
+    # encoding is what the fit stored for the codebook scalars
+    assert np.array_equal(oracle.encode(C.reshape(-1), levels), codes.reshape(-1))
+    # decoding then re-encoding is the identity on codes
+    assert np.array_equal(oracle.encode(levels[codes].reshape(-1), levels), codes.reshape(-1))
+
+
+def test_level_scale_bounds():
+    C = synth.random_kernels(100, 9, 71, 0.05)
+    counts = synth.random_counts(100, 72, 1000)
+    S = oracle.level_scale(C, counts)
+    A = int(counts.sum()) * 9
+    M = float(np.abs(C[counts > 0]).max())
+    assert A * M * 2.0 ** S < 2 ** 62 <= A * M * 2.0 ** (S + 1)
+
+
+# ---------------------------------------------------------------------------
+# Sec. 3.2 testing phase: reconstruction.
+# ---------------------------------------------------------------------------
+
+def test_reconstruct_round_trip():
+    C = synth.random_kernels(50, 9, 81)
+    idx = synth.below(synth.stream_key(82, 2), 400, 50).astype(np.int32)
+    Wr = oracle.reconstruct(idx, C)
+    # every reconstructed kernel is a codeword, so assignment recovers idx
+    i2, d2 = oracle.assign(Wr, C)
+    assert np.array_equal(i2, idx) and np.all(d2 == 0)
+    assert np.array_equal(oracle.reconstruct(np.arange(50, dtype=np.int32), C), C)
+
+
+def test_reconstruct_with_codes_uses_levels():
+    C = synth.random_kernels(40, 9, 91, 0.05)
+    counts = synth.random_counts(40, 92, 9)
+    levels, codes, _ = oracle.level_fit(C, counts)
+    idx = synth.below(synth.stream_key(93, 2), 123, 40).astype(np.int32)
+    Wr = oracle.reconstruct(idx, C, codes, levels)
+    # each reconstructed weight is the level nearest to the codebook scalar
+    for i in range(123):
+        for j in range(9):
+            v = C[idx[i], j]
+            assert abs(Wr[i, j] - v) == np.min(np.abs(levels - v))
