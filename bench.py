@@ -1,0 +1,376 @@
+"""Benchmark of the KQ hot path on GB300: kernel x codeword distance evals/s.
+
+One step = one pass of the whole hot path over the 2048x2048 stress layer
+(n = 4,194,304 kernels, K = 65,536 codewords, 10 Lloyd iterations):
+codebook init from seeded kernels, 10 x (assign + centroid update), final assign,
+cluster sizes, 6-bit codebook quantisation, K+C reconstruction of the weights.
+The metric counts (iters + 1) * n * K distance evaluations per step.
+
+Default (impl "kq"): the CUDA path through the C ABI, inputs resident in HBM
+(the 151 MB weight matrix is larger than the 129 MB L2, so no flush is needed),
+timed with CUDA events on the launching stream. "e2e" re-times the step through
+kq_fit_codebook with the weights coming from pinned host memory and every output
+copied back. --impl reference times the CPU oracle on a bounded row sample of
+the same workload on the host cores.
+
+Multi-GPU (torchrun): the path does not shard here, so every rank runs an
+independent replica; value = all ranks' evals / max-over-ranks time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "kernel x codeword distance evals/s per Lloyd iteration"
+UNIT = "evals/s"
+SM_COUNT_NOMINAL = 152
+FP32_LANES_PER_SM = 128
+OPS_PER_PAIR = 18  # 9 FSUB + 9 FFMA on the FP32 pipe
+WORKLOAD_CFG = 5
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f)
+    except OSError:
+        return {}
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu = gpu_id
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            p = [x.strip() for x in ln.split(",")]
+            if len(p) < 7:
+                continue
+            try:
+                sm.append(float(p[0]))
+                mx = float(p[1])
+            except ValueError:
+                continue
+            for nm, v in zip(names, p[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def _smi_id(dev) -> str:
+    """nvidia-smi -i argument for a torch device (its UUID when torch exposes it)."""
+    import torch
+
+    props = torch.cuda.get_device_properties(dev)
+    uuid = getattr(props, "uuid", None)
+    if uuid is not None:
+        u = str(uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        return vis.split(",")[dev.index or 0]
+    return str(dev.index or 0)
+
+
+def _cpu_sample(W, C, seconds: float, threads: int):
+    """Time the oracle's assignment on a seeded row sample sized for ~`seconds`."""
+    import oracle
+
+    rows_all = synth.below(synth.stream_key(4242, 9), 1 << 16, W.shape[0])
+    probe = 64
+    t0 = time.perf_counter()
+    oracle.assign(W[rows_all[:probe]], C, threads=threads)
+    dt = max(time.perf_counter() - t0, 1e-3)
+    rows = int(min(len(rows_all), max(probe, probe * seconds / dt)))
+    rows = max(threads, rows - rows % threads)
+    t0 = time.perf_counter()
+    oracle.assign(W[rows_all[:rows]], C, threads=threads)
+    dt = time.perf_counter() - t0
+    return rows, dt
+
+
+def run_reference(args, rank, world):
+    """CPU oracle on the host cores (rank 0 only)."""
+    if rank != 0:
+        return
+    import oracle
+
+    lay = synth.workload(WORKLOAD_CFG).layers[0]
+    W, sel = synth.layer_inputs(lay)
+    C0 = oracle.gather_rows(W, sel)
+    threads = oracle.default_threads()
+    per_step = []
+    rows = None
+    for s in range(args.warmup + args.steps):
+        rows, dt = _cpu_sample(W, C0, args.ref_seconds, threads)
+        if s >= args.warmup:
+            per_step.append((rows, dt))
+    pairs = sum(r for r, _ in per_step) * lay.K
+    secs = sum(d for _, d in per_step)
+    value = pairs / secs
+    sample = (f"assign step of the oracle (the step holding ~all of the work) on {rows} seeded rows of the "
+              f"{lay.n}-kernel layer against all K={lay.K} codewords, per step")
+    out = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * secs / len(per_step), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": "stress_2048x2048_K65536_T10", "n": lay.n, "K": lay.K, "iters": 10},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(out), flush=True)
+
+
+def run_kq(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2003_05148_gb300 import build, kq
+
+    build.build()
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    lay = synth.workload(WORKLOAD_CFG).layers[0]
+    T = synth.workload(WORKLOAD_CFG).iters
+    n, K = lay.n, lay.K
+    W_h, sel_h = synth.layer_inputs(lay)
+    stream = torch.cuda.current_stream()
+
+    W = torch.from_numpy(W_h).to(dev)
+    sel = torch.from_numpy(sel_h).to(dev)
+    ws = kq.workspace(n, K, dev)
+    Ca = torch.empty(K, 9, dtype=torch.float32, device=dev)
+    Cb = torch.empty_like(Ca)
+    idx = torch.empty(n, dtype=torch.int32, device=dev)
+    counts = torch.empty(K, dtype=torch.int32, device=dev)
+    levels = torch.empty(64, dtype=torch.float32, device=dev)
+    codes = torch.empty(K, 9, dtype=torch.uint8, device=dev)
+    Wr = torch.empty_like(W)
+    n_assign = T + 1
+
+    def new_events():
+        return [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_assign)]
+
+    def step(ev=None):
+        """One pass of the hot path through the public entry points; `ev` brackets each assign."""
+        kq.kq_init_codebook(W, sel, Ca, ws)
+        cur, nxt = Ca, Cb
+        for t in range(T):
+            if ev:
+                ev[t][0].record(stream)
+            kq.kq_assign(W, cur, idx, None, ws)
+            if ev:
+                ev[t][1].record(stream)
+            kq.kq_update_centroids(W, idx, cur, nxt, counts, ws)
+            cur, nxt = nxt, cur
+        if ev:
+            ev[T][0].record(stream)
+        kq.kq_assign(W, cur, idx, None, ws)
+        if ev:
+            ev[T][1].record(stream)
+        kq.kq_update_centroids(W, idx, cur, nxt, counts, ws)  # cluster sizes of the final assignment
+        kq.kq_quantize_codebook_6bit(cur, counts, 100, levels, codes, None, ws)
+        kq.kq_reconstruct(idx, None, codes, levels, Wr, ws, K=K)
+
+    for _ in range(args.warmup):
+        step()
+    st, flags = kq.kq_device_status(ws)
+    if st != 0:
+        raise RuntimeError(f"device status {st} flags {flags:#x} after warm-up")
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    evs = [new_events() for _ in range(args.steps)]
+    launches0 = kq.kq_kernel_launches()
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(_smi_id(dev)) as clocks:
+        e0.record(stream)
+        for s in range(args.steps):
+            step(evs[s])
+        e1.record(stream)
+        barrier()
+    launches = kq.kq_kernel_launches() - launches0
+    ms_total = e0.elapsed_time(e1)
+    assign_ms = [a.elapsed_time(b) for ev in evs for a, b in ev]
+    t_local = torch.tensor([ms_total], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t_local, op=dist.ReduceOp.MAX)
+    ms_max = float(t_local.item())
+    pairs_per_step = n_assign * n * K
+    value = world * args.steps * pairs_per_step / (ms_max / 1e3)
+
+    st, flags = kq.kq_device_status(ws)
+    if st != 0:
+        raise RuntimeError(f"device status {st} flags {flags:#x} after the timed steps")
+
+    # ---- end to end through kq_fit_codebook: pinned host in, every output back ----
+    W_pin = torch.from_numpy(W_h).pin_memory()
+    sel_pin = torch.from_numpy(sel_h).pin_memory()
+    outs = {"C": torch.empty(K, 9, dtype=torch.float32).pin_memory(),
+            "idx": torch.empty(n, dtype=torch.int32).pin_memory(),
+            "counts": torch.empty(K, dtype=torch.int32).pin_memory(),
+            "levels": torch.empty(64, dtype=torch.float32).pin_memory(),
+            "codes": torch.empty(K, 9, dtype=torch.uint8).pin_memory(),
+            "Wr": torch.empty(n, 9, dtype=torch.float32).pin_memory(),
+            "objective": torch.empty(T + 1, dtype=torch.float64).pin_memory()}
+    obj = torch.empty(T + 1, dtype=torch.float64, device=dev)
+    Wd = torch.empty_like(W)
+    seld = torch.empty_like(sel)
+
+    def e2e_step():
+        Wd.copy_(W_pin, non_blocking=True)
+        seld.copy_(sel_pin, non_blocking=True)
+        kq.kq_init_codebook(Wd, seld, Ca, ws)
+        kq.kq_fit_codebook(Wd, Ca, T, Cb, idx, counts, obj, ws)
+        kq.kq_quantize_codebook_6bit(Cb, counts, 100, levels, codes, None, ws)
+        kq.kq_reconstruct(idx, None, codes, levels, Wr, ws, K=K)
+        for name, src in (("C", Cb), ("idx", idx), ("counts", counts), ("levels", levels), ("codes", codes),
+                          ("Wr", Wr), ("objective", obj)):
+            outs[name].copy_(src, non_blocking=True)
+
+    e2e_steps = max(1, min(args.steps, args.e2e_steps))
+    e2e_step()
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        e2e_step()
+    torch.cuda.synchronize()
+    e2e_s = time.perf_counter() - t0
+    t_e2e = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t_e2e, op=dist.ReduceOp.MAX)
+    e2e_value = world * e2e_steps * pairs_per_step / float(t_e2e.item())
+    h2d = W_pin.numel() * 4 + sel_pin.numel() * 8
+    d2h = sum(t.numel() * t.element_size() for t in outs.values())
+
+    if rank != 0:
+        return
+    peaks = _peaks()
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    clk = clocks.summary()
+    max_mhz = float(peaks.get("sm_max_mhz", 2070.0))
+    peak_tops = sms * FP32_LANES_PER_SM * max_mhz * 1e6 / 1e12
+    t_assign = statistics.mean(assign_ms) / 1e3
+    achieved = OPS_PER_PAIR * n * K / t_assign / 1e12
+    roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s", "frac": achieved / peak_tops,
+                "traffic": None, "kernel": "assign_kernel",
+                "peak_basis": f"{sms} SMs x {FP32_LANES_PER_SM} FP32 lanes x {max_mhz:.0f} MHz (max SM clock); "
+                              f"op = one FP32-pipe lane op, {OPS_PER_PAIR} per pair (9 FSUB + 9 FFMA)",
+                "assign_ms_mean": 1e3 * t_assign, "assign_launches": len(assign_ms)}
+    if clk:
+        roofline["frac_at_sampled_clock"] = achieved / (sms * FP32_LANES_PER_SM * clk["sm_mhz"] * 1e6 / 1e12)
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms_max / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32", "data": "synthetic",
+        "config": {"workload": "stress_2048x2048_K65536_T10", "n": n, "K": K, "iters": T,
+                   "step": "init + 10x(assign+update) + assign + counts + 6-bit quantize + K+C reconstruct",
+                   "l2": "inputs larger than L2 (W is 151 MB, L2 129 MB): no flush",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": roofline,
+        "gpu_launches": int(launches),
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+                "steps": e2e_steps, "api": "kq_init_codebook + kq_fit_codebook + kq_quantize_codebook_6bit + "
+                                           "kq_reconstruct, pinned host buffers, all outputs copied back"},
+    }
+    if clk:
+        out["clocks"] = clk
+    if world == 1 and not args.no_cpu_baseline:
+        import oracle
+
+        threads = oracle.default_threads()
+        C0 = oracle.gather_rows(W_h, sel_h)
+        rows, dt = _cpu_sample(W_h, C0, args.ref_seconds, threads)
+        out["cpu_baseline"] = {"value": rows * K / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+                               "sample": f"oracle assign of {rows} seeded rows against all K={K} codewords "
+                                         f"({rows * K:.3g} evals, {dt:.1f} s)"}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["kq", "reference"], default="kq")
+    ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--ref-seconds", type=float, default=10.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        print("warning: fewer than 3 warm-up steps", file=sys.stderr)
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    try:
+        run_kq(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,210 @@
+/*
+ * kq.h -- C ABI of libkq, the sm_103a (GB300) implementation of the hot path of
+ * Kernel Quantization (KQ, "Kernel Quantization for Efficient Network
+ * Compression", arXiv 2003.05148).
+ *
+ * KQ treats each 3x3 kernel of a conv layer (a 9-float vector) as the unit of
+ * quantisation: it learns a codebook of k kernels by k-means (Sec. 3.1, Eq. 1),
+ * stores one ceil(log2 k)-bit index per kernel, quantises the codebook scalars to
+ * 6 bits by count-weighted k-means (Sec. 3.2) and rebuilds the weights from the
+ * indices at test time (Sec. 3.2, last paragraph). Eq. 4-7 count the bits.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Layouts. W is the conv weight viewed as n rows of 9 floats, row-major: the
+ *   PyTorch [q][p][3][3] tensor is exactly this with n = p*q and row i = o*p + c
+ *   (Sec. 3.1 reshapes W into the kernel matrix [m_0 .. m_{n-1}]). A codebook C is
+ *   K rows of 9 floats. Indices are int32, counts int32, codes uint8 (one 6-bit
+ *   code per byte, values 0..63), levels 64 floats.
+ * - Memory. Every pointer except those documented as host pointers is device
+ *   memory owned by the caller. The library allocates nothing and frees nothing.
+ *   Scratch lives in a caller-allocated workspace of kq_workspace_bytes(n, K)
+ *   bytes (256-byte aligned), which must be zero-filled once before its first
+ *   use (e.g. torch.zeros); the library keeps it consistent afterwards. One
+ *   workspace must not be used by two calls that can run at the same time.
+ * - Streams. Work is enqueued on the given stream and the call returns without
+ *   waiting for it (except kq_device_status, which synchronises the stream).
+ * - Errors. Arguments are validated on the host before anything is enqueued; a
+ *   bad argument returns a status and enqueues nothing. Problems that only the
+ *   device can see (a non-finite input, an index or code out of range, a bounded
+ *   device-side wait that gave up) set bits of a sticky status word in the
+ *   workspace; kq_device_status() reads and clears it. Device code never traps
+ *   and never waits without a bound. A CUDA launch error returns KQ_ERR_CUDA.
+ * - Determinism. For identical inputs every output is bitwise identical from
+ *   run to run (no floating-point atomics anywhere).
+ * - Alignment. W and W_out must be 16-byte aligned; other float / int pointers
+ *   4-byte aligned; the workspace 256-byte aligned. Otherwise KQ_ERR_ALIGNMENT.
+ * - Sizes. 1 <= K <= n, n < 2^31, K*9 < 2^31.
+ */
+#ifndef KQ_H_
+#define KQ_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* cudaStream_t without pulling in the CUDA headers (same underlying type). */
+typedef struct CUstream_st *kq_stream_t;
+
+typedef enum {
+    KQ_OK = 0,
+    KQ_ERR_INVALID_ARG = 1, /* a size, pointer or flag is out of its documented range */
+    KQ_ERR_ALIGNMENT = 2,   /* a pointer is not aligned as documented */
+    KQ_ERR_NONFINITE = 3,   /* (device status) an input value was NaN or +-inf */
+    KQ_ERR_CUDA = 4,        /* a CUDA runtime call or kernel launch failed */
+    KQ_ERR_DEVICE_CHECK = 5, /* (device status) an index or code was out of range */
+    KQ_ERR_WORKSPACE = 6,   /* workspace missing or smaller than kq_workspace_bytes */
+    KQ_ERR_TIMEOUT = 7      /* (device status) a bounded device-side wait gave up */
+} kq_status;
+
+/* Bits of the device status word returned by kq_device_status(). */
+#define KQ_FLAG_NONFINITE 0x1u
+#define KQ_FLAG_INDEX_RANGE 0x2u
+#define KQ_FLAG_CODE_RANGE 0x4u
+#define KQ_FLAG_TIMEOUT 0x8u
+
+/* Human-readable name of a status. Never NULL. */
+const char *kq_status_string(kq_status s);
+
+/* Version of this ABI; changes whenever a signature or a layout changes. */
+int32_t kq_abi_version(void);
+
+/* Number of CUDA kernels libkq has launched in this process so far (all
+ * devices, all threads). A diagnostic for tracing and launch accounting. */
+uint64_t kq_kernel_launches(void);
+
+/* Bytes of workspace needed by any entry point for n kernels and K codewords.
+ * Returns 0 when (n, K) is outside the supported range. */
+size_t kq_workspace_bytes(int64_t n, int32_t K);
+
+/* Read and clear the sticky device status word of a workspace. Synchronises
+ * `stream` first (so it reports every call enqueued before it on that stream).
+ * *flags_out (host pointer, may be NULL) receives the raw KQ_FLAG_* bits.
+ * Returns KQ_OK, or the status of the most severe flag set:
+ * KQ_ERR_TIMEOUT > KQ_ERR_DEVICE_CHECK > KQ_ERR_NONFINITE. */
+kq_status kq_device_status(void *ws, size_t ws_bytes, kq_stream_t stream, uint32_t *flags_out);
+
+/* Codeword initialisation: C0[j] = W[sel[j]] for j < K.
+ * The paper does not say how k-means is initialised (Sec. 3.1); KQ here seeds
+ * the codebook with K distinct kernels whose row numbers the caller draws.
+ *   W    n x 9 fp32 (device);  sel  K int64 row numbers in [0, n) (device)
+ *   C0   K x 9 fp32 output (device)
+ * Uses only the first 4096 bytes of the workspace (ws_bytes >= 4096).
+ * A row number outside [0, n) sets KQ_FLAG_INDEX_RANGE and writes zeros. */
+kq_status kq_init_codebook(const float *W, int64_t n, const int64_t *sel, int32_t K, float *C0, void *ws,
+                           size_t ws_bytes, kq_stream_t stream);
+
+/* Assignment step of k-means, Sec. 3.1 Eq. 1: for every kernel m_i,
+ *   idx[i]  = argmin_k || m_i - c_k ||^2,   dist[i] = that minimum,
+ * with the distance evaluated in fp32 as t_j = fl(x_j - c_j), acc = fma(t_j,
+ * t_j, acc) for j = 0..8 in order (acc starts at 0), and ties resolved toward
+ * the lowest k (the running best starts at (+inf, 0)).
+ *   W     n x 9 fp32 (device, 16-byte aligned)
+ *   C     K x 9 fp32 (device)
+ *   idx   n int32 output (device)
+ *   dist  n fp32 output (device) or NULL
+ * A non-finite value in W or C sets KQ_FLAG_NONFINITE (the outputs are still
+ * written by the rules above). */
+kq_status kq_assign(const float *W, int64_t n, const float *C, int32_t K, int32_t *idx, float *dist, void *ws,
+                    size_t ws_bytes, kq_stream_t stream);
+
+/* Update step of k-means, Sec. 3.1 Eq. 1: for every codeword,
+ *   counts[k] = z_k = |S_k| = #{ i : idx[i] == k },
+ *   C_next[k] = (1 / z_k) * sum_{i in S_k} m_i   if z_k > 0, else C_prev[k],
+ * the minimiser of Eq. 1 for fixed sets S_k (an empty set keeps its codeword).
+ * The sums are exact int64 fixed-point sums (scale 2^S chosen from max|W| so
+ * that no sum can overflow), so the result does not depend on the order in
+ * which kernels are added; it differs from the exact mean by far less than
+ * 1e-5 relative.
+ *   W       n x 9 fp32 (device, 16-byte aligned);  idx  n int32 (device)
+ *   C_prev  K x 9 fp32 (device);  C_next  K x 9 fp32 output (device, may equal C_prev)
+ *   counts  K int32 output (device)
+ * An index outside [0, K) is skipped and sets KQ_FLAG_INDEX_RANGE. */
+kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int32_t K, const float *C_prev,
+                              float *C_next, int32_t *counts, void *ws, size_t ws_bytes, kq_stream_t stream);
+
+/* k-means fit of the kernel codebook, Sec. 3.1 Eq. 1 (the "Quantize kernel ...
+ * with k-means" step of Algorithm 1): from C_init, `iters` times
+ * { assign against C_t; objective[t] = sum_i dist_i; C_{t+1} = update },
+ * then a final assign against C_iters, objective[iters] = its sum.
+ *   W          n x 9 fp32 (device, 16-byte aligned)
+ *   C_init     K x 9 fp32 (device); C_out K x 9 fp32 output (device; may equal C_init)
+ *   iters      >= 0
+ *   flags      must be 0 (reserved)
+ *   idx        n int32 output: the final assignment (device)
+ *   counts     K int32 output: cluster sizes of the final assignment (device)
+ *   objective  iters + 1 fp64 outputs (device) or NULL: Eq. 1 objective per step,
+ *              summed in a fixed order (bitwise reproducible)
+ * Runs entirely on `stream`; no host synchronisation. */
+kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_init, int32_t iters, int32_t flags,
+                          float *C_out, int32_t *idx, int32_t *counts, double *objective, void *ws, size_t ws_bytes,
+                          kq_stream_t stream);
+
+/* 6-bit kernel-codebook quantisation, Sec. 3.2: k-means with 64 levels over all
+ * K*9 codebook scalars v_kj, each weighted by its entry's appearance count
+ * z_k ("entry appearance time"), then the code of every scalar.
+ *   - levels start at linspace(min, max, 64) over the scalars with z_k > 0 (all
+ *     scalars if no count is positive), computed in fp64 and rounded to fp32;
+ *   - a scalar's code is its nearest level by fp32 |v - level|, lower index on ties;
+ *   - a level becomes the z-weighted mean of its scalars, computed from exact
+ *     int64 fixed-point sums (scale 2^S, S = 62 - e with A*M = f*2^e, f in
+ *     [0.5, 1), A = sum of weights, M = max |v| over weighted scalars); a level
+ *     with no weighted scalar keeps its value;
+ *   - stop when no code changes or after max_iters level updates; the codes
+ *     returned are those of the final levels.
+ *   C          K x 9 fp32 (device);  counts K int32 >= 0 (device)
+ *   max_iters  0 .. 100000
+ *   levels     64 fp32 output (device);  codes K x 9 uint8 output (device)
+ *   iters_run  1 int32 output (device) or NULL: level updates performed
+ * Uses only the first 4096 bytes of the workspace (ws_bytes >= 4096). The CTAs
+ * of this call meet at grid barriers whose waits are bounded (~2 s): a wait that
+ * runs out sets KQ_FLAG_TIMEOUT and the call ends without writing its outputs.
+ * A negative count sets KQ_FLAG_INDEX_RANGE and is treated as 0. */
+kq_status kq_quantize_codebook_6bit(const float *C, int32_t K, const int32_t *counts, int32_t max_iters,
+                                    float *levels, uint8_t *codes, int32_t *iters_run, void *ws, size_t ws_bytes,
+                                    kq_stream_t stream);
+
+/* Test-time recovery, Sec. 3.2 (last paragraph): first the kernel codebook is
+ * recovered (C_hat[k][j] = levels[codes[k][j]]), then the weight tensor:
+ *   W_out[i] = C_hat[idx[i]]   (K+C: codes and levels given), or
+ *   W_out[i] = C[idx[i]]       (kernel-level only: codes == NULL and levels == NULL).
+ *   idx    n int32 (device);  C  K x 9 fp32 (device; unused when codes are given, may be NULL then)
+ *   codes  K x 9 uint8 (device) or NULL;  levels 64 fp32 (device) or NULL
+ *   W_out  n x 9 fp32 output (device, 16-byte aligned)
+ * An index outside [0, K) writes a zero row and sets KQ_FLAG_INDEX_RANGE; a
+ * code above 63 decodes to 0 and sets KQ_FLAG_CODE_RANGE. */
+kq_status kq_reconstruct(const int32_t *idx, int64_t n, const float *C, int32_t K, const uint8_t *codes,
+                         const float *levels, float *W_out, void *ws, size_t ws_bytes, kq_stream_t stream);
+
+/* Storage accounting of one layer (host only, no device work), Sec. 3.2-3.3 and
+ * Sec. 4.1:
+ *   Eq. 4  total_bits B = k * omega^2 * b_c + n * ceil(log2 k)
+ *          (index_bits = n * ceil(log2 k), codebook_bits = k * omega^2 * b_c;
+ *           the 64-entry level table of the 6-bit codebook is not counted)
+ *   Eq. 7  beta = B / (n * omega^2)             bits per parameter
+ *   Eq. 6  ratio_kq = n * omega^2 * 32 / B      compression ratio C_KQ
+ * b_c = 32 for kernel-level quantisation only, 6 after codebook quantisation.
+ * Requires n >= 1, 1 <= k, omega >= 1, b_c >= 1, out != NULL (host pointer). */
+typedef struct {
+    int64_t index_bits;
+    int64_t codebook_bits;
+    int64_t total_bits;
+    double beta;
+    double ratio_kq;
+} kq_report;
+
+kq_status kq_compression_report(int64_t n, int32_t k, int32_t omega, int32_t b_c, kq_report *out);
+
+/* Eq. 5 (host only): compression ratio of conventional per-weight quantisation,
+ * C_con = n * omega^2 * b_fp / (u * b_1 + n * omega^2 * ceil(log2 u)), with u
+ * codebook entries of b_1 bits each and b_fp-bit full-precision weights. */
+kq_status kq_conventional_ratio(int64_t n, int32_t omega, int32_t u, int32_t b_1, int32_t b_fp, double *out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KQ_H_ */

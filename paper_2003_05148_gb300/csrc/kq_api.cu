@@ -1,0 +1,278 @@
+// kq_api.cu -- the extern "C" entry points of libkq declared in include/kq.h:
+// argument validation, workspace carving and kernel sequencing. No device memory
+// is allocated here; every buffer is the caller's or a slice of its workspace.
+#include <stddef.h>
+
+#include <atomic>
+
+#include "kq_internal.cuh"
+
+using namespace kq;
+
+namespace kq {
+static std::atomic<unsigned long long> g_launches{0};
+void count_launch(int kernels) { g_launches.fetch_add((unsigned long long)kernels, std::memory_order_relaxed); }
+}  // namespace kq
+
+namespace {
+
+constexpr int32_t KQ_ABI_VERSION = 1;
+
+inline bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+inline kq_status cuda_status(cudaError_t e) { return e == cudaSuccess ? KQ_OK : KQ_ERR_CUDA; }
+
+#define KQ_TRY(expr)                                  \
+    do {                                              \
+        cudaError_t e_ = (expr);                      \
+        if (e_ != cudaSuccess) return KQ_ERR_CUDA;    \
+    } while (0)
+
+// Supported problem sizes (see kq.h, "Sizes").
+inline bool sizes_ok(int64_t n, int32_t K) {
+    return n >= 1 && n < (1LL << 31) && K >= 1 && (int64_t)K <= n && (int64_t)K * D < (1LL << 31);
+}
+
+// Entry points that only use the fixed 4 KiB header of the workspace.
+kq_status check_ws_header(void *ws, size_t ws_bytes) {
+    if (!ws) return KQ_ERR_WORKSPACE;
+    if (!aligned(ws, 256)) return KQ_ERR_ALIGNMENT;
+    if (ws_bytes < 4096) return KQ_ERR_WORKSPACE;
+    return KQ_OK;
+}
+
+kq_status check_ws(void *ws, size_t ws_bytes, int64_t n, int32_t K) {
+    if (!ws) return KQ_ERR_WORKSPACE;
+    if (!aligned(ws, 256)) return KQ_ERR_ALIGNMENT;
+    if (ws_bytes < ws_layout(n, K).total) return KQ_ERR_WORKSPACE;
+    return KQ_OK;
+}
+
+kq_status num_sms(int *out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return KQ_ERR_CUDA;
+    if (cudaDeviceGetAttribute(out, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return KQ_ERR_CUDA;
+    return KQ_OK;
+}
+
+struct Ws {
+    Header *hdr;
+    float *cd;
+    unsigned long long *acc;
+    unsigned long long *part;
+    double *blocksum;
+    float *cbuf0, *cbuf1, *cp;
+};
+
+Ws carve(void *ws, int64_t n, int32_t K) {
+    const WsLayout L = ws_layout(n, K);
+    char *b = static_cast<char *>(ws);
+    Ws w;
+    w.hdr = reinterpret_cast<Header *>(b);
+    w.cd = reinterpret_cast<float *>(b + L.cd);
+    w.acc = reinterpret_cast<unsigned long long *>(b + L.acc);
+    w.part = reinterpret_cast<unsigned long long *>(b + L.part);
+    w.blocksum = reinterpret_cast<double *>(b + L.blocksum);
+    w.cbuf0 = reinterpret_cast<float *>(b + L.cbuf0);
+    w.cbuf1 = reinterpret_cast<float *>(b + L.cbuf1);
+    w.cp = reinterpret_cast<float *>(b + L.cp);
+    return w;
+}
+
+// Update step on prepared state: accumulate into the (zeroed) accumulators and
+// finalise; the finalise leaves the accumulators zeroed again.
+kq_status run_update(const float *W, int64_t n, const int32_t *idx, int32_t K, const float *C_prev, float *C_next,
+                     int32_t *counts, float *Cd_next, const Ws &w, int sms, cudaStream_t s) {
+    KQ_TRY(launch_accumulate(W, n, idx, K, &w.hdr->maxabs_bits, w.acc, &w.hdr->status, sms, s));
+    KQ_TRY(launch_finalize(w.acc, K, n, &w.hdr->maxabs_bits, C_prev, C_next, counts, Cd_next, s));
+    return KQ_OK;
+}
+
+kq_status prepare_update(const float *W, int64_t n, int32_t K, const Ws &w, int sms, cudaStream_t s) {
+    KQ_TRY(cudaMemsetAsync(&w.hdr->maxabs_bits, 0, sizeof(uint32_t), s));
+    KQ_TRY(launch_maxabs(W, n * D, &w.hdr->maxabs_bits, &w.hdr->status, sms, s));
+    KQ_TRY(cudaMemsetAsync(w.acc, 0, (size_t)K * ACC_WORDS * sizeof(unsigned long long), s));
+    return KQ_OK;
+}
+
+int ceil_log2_i64(int64_t k) {
+    int b = 0;
+    while ((1LL << b) < k) ++b;
+    return b;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *kq_status_string(kq_status s) {
+    switch (s) {
+        case KQ_OK: return "KQ_OK";
+        case KQ_ERR_INVALID_ARG: return "KQ_ERR_INVALID_ARG";
+        case KQ_ERR_ALIGNMENT: return "KQ_ERR_ALIGNMENT";
+        case KQ_ERR_NONFINITE: return "KQ_ERR_NONFINITE";
+        case KQ_ERR_CUDA: return "KQ_ERR_CUDA";
+        case KQ_ERR_DEVICE_CHECK: return "KQ_ERR_DEVICE_CHECK";
+        case KQ_ERR_WORKSPACE: return "KQ_ERR_WORKSPACE";
+        case KQ_ERR_TIMEOUT: return "KQ_ERR_TIMEOUT";
+    }
+    return "KQ_ERR_UNKNOWN";
+}
+
+int32_t kq_abi_version(void) { return KQ_ABI_VERSION; }
+
+uint64_t kq_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
+
+size_t kq_workspace_bytes(int64_t n, int32_t K) {
+    if (!sizes_ok(n, K)) return 0;
+    return ws_layout(n, K).total;
+}
+
+kq_status kq_device_status(void *ws, size_t ws_bytes, kq_stream_t stream, uint32_t *flags_out) {
+    if (!ws) return KQ_ERR_WORKSPACE;
+    if (!aligned(ws, 256)) return KQ_ERR_ALIGNMENT;
+    if (ws_bytes < sizeof(Header)) return KQ_ERR_WORKSPACE;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    Header *h = static_cast<Header *>(ws);
+    uint32_t flags = 0;
+    KQ_TRY(cudaMemcpyAsync(&flags, &h->status, sizeof(flags), cudaMemcpyDeviceToHost, s));
+    KQ_TRY(cudaMemsetAsync(&h->status, 0, sizeof(uint32_t), s));
+    KQ_TRY(cudaStreamSynchronize(s));
+    if (flags_out) *flags_out = flags;
+    if (flags & KQ_FLAG_TIMEOUT) return KQ_ERR_TIMEOUT;
+    if (flags & (KQ_FLAG_INDEX_RANGE | KQ_FLAG_CODE_RANGE)) return KQ_ERR_DEVICE_CHECK;
+    if (flags & KQ_FLAG_NONFINITE) return KQ_ERR_NONFINITE;
+    return KQ_OK;
+}
+
+kq_status kq_init_codebook(const float *W, int64_t n, const int64_t *sel, int32_t K, float *C0, void *ws,
+                           size_t ws_bytes, kq_stream_t stream) {
+    if (!sizes_ok(n, K) || !W || !sel || !C0) return KQ_ERR_INVALID_ARG;
+    if (!aligned(W, 4) || !aligned(sel, 8) || !aligned(C0, 4)) return KQ_ERR_ALIGNMENT;
+    kq_status st = check_ws_header(ws, ws_bytes);
+    if (st != KQ_OK) return st;
+    Header *h = static_cast<Header *>(ws);
+    return cuda_status(launch_init_codebook(W, n, sel, K, C0, &h->status, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+kq_status kq_assign(const float *W, int64_t n, const float *C, int32_t K, int32_t *idx, float *dist, void *ws,
+                    size_t ws_bytes, kq_stream_t stream) {
+    if (!sizes_ok(n, K) || !W || !C || !idx) return KQ_ERR_INVALID_ARG;
+    if (!aligned(W, 16) || !aligned(C, 4) || !aligned(idx, 4) || !aligned(dist, 4)) return KQ_ERR_ALIGNMENT;
+    kq_status st = check_ws(ws, ws_bytes, n, K);
+    if (st != KQ_OK) return st;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != KQ_OK) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    Ws w = carve(ws, n, K);
+    KQ_TRY(launch_pack_codebook(C, K, w.cd, &w.hdr->status, s));
+    int nb = 0;
+    KQ_TRY(launch_assign(W, n, w.cd, K, idx, dist, w.blocksum, &nb, w.part, &w.hdr->status, sms, s));
+    return KQ_OK;
+}
+
+kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int32_t K, const float *C_prev,
+                              float *C_next, int32_t *counts, void *ws, size_t ws_bytes, kq_stream_t stream) {
+    if (!sizes_ok(n, K) || !W || !idx || !C_prev || !C_next || !counts) return KQ_ERR_INVALID_ARG;
+    if (!aligned(W, 16) || !aligned(idx, 4) || !aligned(C_prev, 4) || !aligned(C_next, 4) || !aligned(counts, 4))
+        return KQ_ERR_ALIGNMENT;
+    kq_status st = check_ws(ws, ws_bytes, n, K);
+    if (st != KQ_OK) return st;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != KQ_OK) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    Ws w = carve(ws, n, K);
+    if ((st = prepare_update(W, n, K, w, sms, s)) != KQ_OK) return st;
+    return run_update(W, n, idx, K, C_prev, C_next, counts, nullptr, w, sms, s);
+}
+
+kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_init, int32_t iters, int32_t flags,
+                          float *C_out, int32_t *idx, int32_t *counts, double *objective, void *ws, size_t ws_bytes,
+                          kq_stream_t stream) {
+    if (!sizes_ok(n, K) || !W || !C_init || !C_out || !idx || !counts) return KQ_ERR_INVALID_ARG;
+    if (iters < 0 || flags != 0) return KQ_ERR_INVALID_ARG;
+    if (!aligned(W, 16) || !aligned(C_init, 4) || !aligned(C_out, 4) || !aligned(idx, 4) || !aligned(counts, 4) ||
+        !aligned(objective, 8))
+        return KQ_ERR_ALIGNMENT;
+    kq_status st = check_ws(ws, ws_bytes, n, K);
+    if (st != KQ_OK) return st;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != KQ_OK) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    Ws w = carve(ws, n, K);
+    const size_t cbytes = (size_t)K * D * sizeof(float);
+
+    if ((st = prepare_update(W, n, K, w, sms, s)) != KQ_OK) return st;
+    KQ_TRY(cudaMemcpyAsync(w.cbuf0, C_init, cbytes, cudaMemcpyDeviceToDevice, s));
+    KQ_TRY(launch_pack_codebook(w.cbuf0, K, w.cd, &w.hdr->status, s));
+    float *cur = w.cbuf0, *nxt = w.cbuf1;
+    int nb = 0;
+    for (int32_t t = 0; t < iters; ++t) {
+        KQ_TRY(launch_assign(W, n, w.cd, K, idx, nullptr, w.blocksum, &nb, w.part, &w.hdr->status, sms, s));
+        if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
+        if ((st = run_update(W, n, idx, K, cur, nxt, counts, w.cd, w, sms, s)) != KQ_OK) return st;
+        float *tmp = cur;
+        cur = nxt;
+        nxt = tmp;
+    }
+    KQ_TRY(launch_assign(W, n, w.cd, K, idx, nullptr, w.blocksum, &nb, w.part, &w.hdr->status, sms, s));
+    if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + iters, s));
+    KQ_TRY(launch_histogram(idx, n, K, counts, &w.hdr->status, sms, s));
+    KQ_TRY(cudaMemcpyAsync(C_out, cur, cbytes, cudaMemcpyDeviceToDevice, s));
+    return KQ_OK;
+}
+
+kq_status kq_quantize_codebook_6bit(const float *C, int32_t K, const int32_t *counts, int32_t max_iters,
+                                    float *levels, uint8_t *codes, int32_t *iters_run, void *ws, size_t ws_bytes,
+                                    kq_stream_t stream) {
+    if (K < 1 || (int64_t)K * D >= (1LL << 31) || !C || !counts || !levels || !codes) return KQ_ERR_INVALID_ARG;
+    if (max_iters < 0 || max_iters > 100000) return KQ_ERR_INVALID_ARG;
+    if (!aligned(C, 4) || !aligned(counts, 4) || !aligned(levels, 4) || !aligned(iters_run, 4))
+        return KQ_ERR_ALIGNMENT;
+    kq_status st = check_ws_header(ws, ws_bytes);
+    if (st != KQ_OK) return st;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != KQ_OK) return st;
+    Header *h = static_cast<Header *>(ws);
+    return cuda_status(launch_level_fit(C, K, counts, max_iters, levels, codes, iters_run, h, sms,
+                                        reinterpret_cast<cudaStream_t>(stream)));
+}
+
+kq_status kq_reconstruct(const int32_t *idx, int64_t n, const float *C, int32_t K, const uint8_t *codes,
+                         const float *levels, float *W_out, void *ws, size_t ws_bytes, kq_stream_t stream) {
+    if (!sizes_ok(n, K) || !idx || !W_out) return KQ_ERR_INVALID_ARG;
+    if ((codes == nullptr) != (levels == nullptr)) return KQ_ERR_INVALID_ARG;
+    if (!codes && !C) return KQ_ERR_INVALID_ARG;
+    if (!aligned(idx, 4) || !aligned(C, 4) || !aligned(levels, 4) || !aligned(W_out, 16)) return KQ_ERR_ALIGNMENT;
+    kq_status st = check_ws(ws, ws_bytes, n, K);
+    if (st != KQ_OK) return st;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != KQ_OK) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    Ws w = carve(ws, n, K);
+    KQ_TRY(launch_decode_codebook(C, K, codes, levels, w.cp, &w.hdr->status, s));
+    KQ_TRY(launch_gather_rows(idx, n, w.cp, K, W_out, &w.hdr->status, sms, s));
+    return KQ_OK;
+}
+
+kq_status kq_compression_report(int64_t n, int32_t k, int32_t omega, int32_t b_c, kq_report *out) {
+    if (n < 1 || k < 1 || omega < 1 || b_c < 1 || !out) return KQ_ERR_INVALID_ARG;
+    const int64_t w2 = (int64_t)omega * omega;
+    if (n > (1LL << 40) || w2 > (1LL << 20)) return KQ_ERR_INVALID_ARG;
+    out->index_bits = n * ceil_log2_i64(k);
+    out->codebook_bits = (int64_t)k * w2 * b_c;
+    out->total_bits = out->index_bits + out->codebook_bits;
+    out->beta = (double)out->total_bits / (double)(n * w2);
+    out->ratio_kq = (double)(n * w2 * 32) / (double)out->total_bits;
+    return KQ_OK;
+}
+
+kq_status kq_conventional_ratio(int64_t n, int32_t omega, int32_t u, int32_t b_1, int32_t b_fp, double *out) {
+    if (n < 1 || omega < 1 || u < 2 || b_1 < 1 || b_fp < 1 || !out) return KQ_ERR_INVALID_ARG;
+    const int64_t w2 = (int64_t)omega * omega;
+    if (n > (1LL << 40) || w2 > (1LL << 20)) return KQ_ERR_INVALID_ARG;
+    *out = (double)(n * w2 * b_fp) / (double)((int64_t)u * b_1 + n * w2 * ceil_log2_i64(u));
+    return KQ_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,133 @@
+// kq_internal.cuh -- definitions shared by the libkq translation units (not part
+// of the public ABI): workspace layout, device status bits, packed fp32x2 math.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "kq.h"
+
+namespace kq {
+
+constexpr int D = 9;             // omega^2 for 3x3 kernels (Sec. 3.1)
+constexpr int LEVELS = 64;       // 6-bit codebook quantisation (Sec. 3.2)
+constexpr int CD_FLOATS = 20;    // packed codeword for the assign kernel: 10 duplicated pairs
+constexpr int CP_FLOATS = 12;    // padded codeword row for the reconstruct gather (48 B)
+constexpr int ACC_WORDS = 16;    // int64 accumulator row per codeword: 9 sums, count, pad (128 B)
+constexpr int ROW_BLOCK = 1024;  // kernels per assign CTA (256 threads x 4 rows)
+constexpr int MAX_PART_BLOCKS = 512;  // bound on (row blocks x codeword splits) with split-K
+
+// Fixed part of the workspace (first 4 KiB).
+struct Header {
+    uint32_t status;        // sticky KQ_FLAG_* bits
+    uint32_t maxabs_bits;   // max |W| as fp32 bits (update scale)
+    uint32_t barrier;       // grid-barrier arrival counter (level fit)
+    uint32_t abort;         // set when a bounded wait gives up
+    uint32_t changed[3];    // level fit: "some code changed" per iteration (triple buffered)
+    uint32_t pad0;
+    uint32_t lo_w, lo_a;    // level fit: ordered-int minima over weighted / all scalars (init 0xff..)
+    uint32_t hi_w, hi_a;    // level fit: ordered-int maxima over weighted / all scalars (init 0)
+    uint32_t maxv_w;        // level fit: max |v| over weighted scalars (fp32 bits)
+    uint32_t pad1;
+    unsigned long long wtotal;          // level fit: sum of weights
+    unsigned long long lacc[3][LEVELS][2];  // level fit: (weight sum, fixed-point sum) per level
+};
+static_assert(sizeof(Header) <= 4096, "header too large");
+
+struct WsLayout {
+    size_t cd, acc, part, blocksum, cbuf0, cbuf1, cp, total;
+};
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+inline WsLayout ws_layout(int64_t n, int32_t K) {
+    WsLayout L;
+    size_t off = 4096;
+    L.cd = off;       off = align_up(off + (size_t)K * CD_FLOATS * 4, 256);
+    L.acc = off;      off = align_up(off + (size_t)K * ACC_WORDS * 8, 256);
+    L.part = off;     off = align_up(off + (size_t)MAX_PART_BLOCKS * ROW_BLOCK * 8, 256);
+    size_t nblk = (size_t)((n + 255) / 256) + MAX_PART_BLOCKS;  // >= CTAs of assign or combine
+    L.blocksum = off; off = align_up(off + nblk * 8, 256);
+    L.cbuf0 = off;    off = align_up(off + (size_t)K * D * 4, 256);
+    L.cbuf1 = off;    off = align_up(off + (size_t)K * D * 4, 256);
+    L.cp = off;       off = align_up(off + (size_t)K * CP_FLOATS * 4, 256);
+    L.total = off;
+    return L;
+}
+
+// ---- packed fp32x2 arithmetic (sm_100+ PTX). Element 0 is the low 32 bits. ----
+__device__ __forceinline__ unsigned long long pack2(float lo, float hi) {
+    unsigned long long r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ void unpack2(unsigned long long v, float &lo, float &hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ unsigned long long sub2(unsigned long long a, unsigned long long b) {
+    unsigned long long d;
+    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ unsigned long long mul2(unsigned long long a, unsigned long long b) {
+    unsigned long long d;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ unsigned long long fma2(unsigned long long a, unsigned long long b,
+                                                   unsigned long long c) {
+    unsigned long long d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+
+// Order-preserving map of fp32 to uint32 (for atomicMin / atomicMax on floats).
+__device__ __forceinline__ uint32_t f2ord(float f) {
+    uint32_t u = __float_as_uint(f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float ord2f(uint32_t u) {
+    return __uint_as_float((u & 0x80000000u) ? (u & 0x7fffffffu) : ~u);
+}
+
+__device__ __forceinline__ void set_flag(uint32_t *status, uint32_t bit) { atomicOr(status, bit); }
+
+__device__ __forceinline__ bool finite9(const float *v) {
+    bool ok = true;
+#pragma unroll
+    for (int j = 0; j < D; ++j) ok &= isfinite(v[j]);
+    return ok;
+}
+
+// Process-wide count of kernels libkq has launched (kq_kernel_launches()).
+void count_launch(int kernels = 1);
+
+// ---- launchers (defined in the .cu files; all return cudaGetLastError()) ----
+cudaError_t launch_pack_codebook(const float *C, int32_t K, float *Cd, uint32_t *status, cudaStream_t s);
+cudaError_t launch_assign(const float *W, int64_t n, const float *Cd, int32_t K, int32_t *idx, float *dist,
+                          double *blocksum, int *nblocksum, unsigned long long *part, uint32_t *status,
+                          int num_sms, cudaStream_t s);
+cudaError_t launch_sum_blocks(const double *blocksum, int nblocks, double *out, cudaStream_t s);
+
+cudaError_t launch_maxabs(const float *W, int64_t count, uint32_t *maxabs_bits, uint32_t *status, int num_sms,
+                          cudaStream_t s);
+cudaError_t launch_accumulate(const float *W, int64_t n, const int32_t *idx, int32_t K,
+                              const uint32_t *maxabs_bits, unsigned long long *acc, uint32_t *status,
+                              int num_sms, cudaStream_t s);
+cudaError_t launch_histogram(const int32_t *idx, int64_t n, int32_t K, int32_t *counts, uint32_t *status,
+                             int num_sms, cudaStream_t s);
+cudaError_t launch_finalize(unsigned long long *acc, int32_t K, int64_t n, const uint32_t *maxabs_bits,
+                            const float *C_prev, float *C_next, int32_t *counts, float *Cd_next,
+                            cudaStream_t s);
+
+cudaError_t launch_level_fit(const float *C, int32_t K, const int32_t *counts, int32_t max_iters, float *levels,
+                             uint8_t *codes, int32_t *iters_run, Header *hdr, int num_sms, cudaStream_t s);
+
+cudaError_t launch_decode_codebook(const float *C, int32_t K, const uint8_t *codes, const float *levels,
+                                   float *Cp, uint32_t *status, cudaStream_t s);
+cudaError_t launch_gather_rows(const int32_t *idx, int64_t n, const float *Cp, int32_t K, float *W_out,
+                               uint32_t *status, int num_sms, cudaStream_t s);
+cudaError_t launch_init_codebook(const float *W, int64_t n, const int64_t *sel, int32_t K, float *C0,
+                                 uint32_t *status, cudaStream_t s);
+
+}  // namespace kq

@@ -1,0 +1,184 @@
+"""Thin Python binding of libkq (include/kq.h): argument marshalling only.
+
+Each function has the name of the C entry point it calls, takes CUDA tensors
+(PyTorch supplies device memory and the current stream) and passes their device
+pointers through ctypes. Every step of the computation runs in libkq's CUDA
+kernels; there is no CPU path, and loading fails loudly when libkq.so has not
+been built.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import torch
+
+from .build import LIB
+
+KQ_OK = 0
+STATUS_NAMES = {0: "KQ_OK", 1: "KQ_ERR_INVALID_ARG", 2: "KQ_ERR_ALIGNMENT", 3: "KQ_ERR_NONFINITE",
+                4: "KQ_ERR_CUDA", 5: "KQ_ERR_DEVICE_CHECK", 6: "KQ_ERR_WORKSPACE", 7: "KQ_ERR_TIMEOUT"}
+FLAG_NONFINITE, FLAG_INDEX_RANGE, FLAG_CODE_RANGE, FLAG_TIMEOUT = 0x1, 0x2, 0x4, 0x8
+
+EXPORTS = ["kq_status_string", "kq_abi_version", "kq_kernel_launches", "kq_workspace_bytes", "kq_device_status", "kq_init_codebook",
+           "kq_assign", "kq_update_centroids", "kq_fit_codebook", "kq_quantize_codebook_6bit", "kq_reconstruct",
+           "kq_compression_report", "kq_conventional_ratio"]
+
+
+class KQError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        self.status = status
+        super().__init__(f"{fn} failed: {STATUS_NAMES.get(status, status)}")
+
+
+class Report(ctypes.Structure):
+    _fields_ = [("index_bits", ctypes.c_int64), ("codebook_bits", ctypes.c_int64), ("total_bits", ctypes.c_int64),
+                ("beta", ctypes.c_double), ("ratio_kq", ctypes.c_double)]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libkq.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB):
+            raise RuntimeError(f"libkq.so is not built ({LIB}); run paper_2003_05148_gb300.build.build()")
+        L = ctypes.CDLL(LIB)
+        P, i64, i32, sz = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_size_t
+        sig = {
+            "kq_status_string": ([ctypes.c_int], ctypes.c_char_p),
+            "kq_abi_version": ([], i32),
+            "kq_kernel_launches": ([], ctypes.c_uint64),
+            "kq_workspace_bytes": ([i64, i32], sz),
+            "kq_device_status": ([P, sz, P, P], ctypes.c_int),
+            "kq_init_codebook": ([P, i64, P, i32, P, P, sz, P], ctypes.c_int),
+            "kq_assign": ([P, i64, P, i32, P, P, P, sz, P], ctypes.c_int),
+            "kq_update_centroids": ([P, i64, P, i32, P, P, P, P, sz, P], ctypes.c_int),
+            "kq_fit_codebook": ([P, i64, i32, P, i32, i32, P, P, P, P, P, sz, P], ctypes.c_int),
+            "kq_quantize_codebook_6bit": ([P, i32, P, i32, P, P, P, P, sz, P], ctypes.c_int),
+            "kq_reconstruct": ([P, i64, P, i32, P, P, P, P, sz, P], ctypes.c_int),
+            "kq_compression_report": ([i64, i32, i32, i32, ctypes.POINTER(Report)], ctypes.c_int),
+            "kq_conventional_ratio": ([i64, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
+        }
+        for name, (args, res) in sig.items():
+            f = getattr(L, name)
+            f.argtypes = args
+            f.restype = res
+        _lib = L
+    return _lib
+
+
+def _check(fn: str, status: int) -> None:
+    if status != KQ_OK:
+        raise KQError(fn, status)
+
+
+def _dev(t: Optional[torch.Tensor], name: str, dtype: torch.dtype):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor) or t.device.type != "cuda":
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must have dtype {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _rows(W: torch.Tensor) -> int:
+    if W.numel() % 9:
+        raise ValueError("kernel tensors must hold a multiple of 9 floats (3x3 kernels)")
+    return W.numel() // 9
+
+
+def kq_status_string(status: int) -> str:
+    return lib().kq_status_string(status).decode()
+
+
+def kq_abi_version() -> int:
+    return lib().kq_abi_version()
+
+
+def kq_kernel_launches() -> int:
+    return int(lib().kq_kernel_launches())
+
+
+def kq_workspace_bytes(n: int, K: int) -> int:
+    return int(lib().kq_workspace_bytes(n, K))
+
+
+def workspace(n: int, K: int, device=None) -> torch.Tensor:
+    """Zero-filled workspace of kq_workspace_bytes(n, K) bytes on the device."""
+    nbytes = kq_workspace_bytes(n, K)
+    if nbytes == 0:
+        raise ValueError(f"unsupported sizes n={n}, K={K}")
+    return torch.zeros(nbytes, dtype=torch.uint8, device=device or "cuda")
+
+
+def kq_device_status(ws: torch.Tensor, stream=None):
+    """(status, flags): read and clear the sticky device status word (synchronises the stream)."""
+    flags = ctypes.c_uint32(0)
+    st = lib().kq_device_status(_dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream), ctypes.byref(flags))
+    return st, flags.value
+
+
+def kq_init_codebook(W, sel, C0, ws, stream=None) -> None:
+    _check("kq_init_codebook", lib().kq_init_codebook(
+        _dev(W, "W", torch.float32), _rows(W), _dev(sel, "sel", torch.int64), sel.numel(),
+        _dev(C0, "C0", torch.float32), _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+
+
+def kq_assign(W, C, idx, dist, ws, stream=None) -> None:
+    _check("kq_assign", lib().kq_assign(
+        _dev(W, "W", torch.float32), _rows(W), _dev(C, "C", torch.float32), _rows(C),
+        _dev(idx, "idx", torch.int32), _dev(dist, "dist", torch.float32),
+        _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+
+
+def kq_update_centroids(W, idx, C_prev, C_next, counts, ws, stream=None) -> None:
+    _check("kq_update_centroids", lib().kq_update_centroids(
+        _dev(W, "W", torch.float32), _rows(W), _dev(idx, "idx", torch.int32), _rows(C_prev),
+        _dev(C_prev, "C_prev", torch.float32), _dev(C_next, "C_next", torch.float32),
+        _dev(counts, "counts", torch.int32), _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+
+
+def kq_fit_codebook(W, C_init, iters, C_out, idx, counts, objective, ws, stream=None, flags: int = 0) -> None:
+    _check("kq_fit_codebook", lib().kq_fit_codebook(
+        _dev(W, "W", torch.float32), _rows(W), _rows(C_init), _dev(C_init, "C_init", torch.float32), iters, flags,
+        _dev(C_out, "C_out", torch.float32), _dev(idx, "idx", torch.int32), _dev(counts, "counts", torch.int32),
+        _dev(objective, "objective", torch.float64), _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+
+
+def kq_quantize_codebook_6bit(C, counts, max_iters, levels, codes, iters_run, ws, stream=None) -> None:
+    _check("kq_quantize_codebook_6bit", lib().kq_quantize_codebook_6bit(
+        _dev(C, "C", torch.float32), _rows(C), _dev(counts, "counts", torch.int32), max_iters,
+        _dev(levels, "levels", torch.float32), _dev(codes, "codes", torch.uint8),
+        _dev(iters_run, "iters_run", torch.int32), _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+
+
+def kq_reconstruct(idx, C, codes, levels, W_out, ws, K: Optional[int] = None, stream=None) -> None:
+    K = _rows(C) if C is not None else codes.numel() // 9 if K is None else K
+    _check("kq_reconstruct", lib().kq_reconstruct(
+        _dev(idx, "idx", torch.int32), idx.numel(), _dev(C, "C", torch.float32), K,
+        _dev(codes, "codes", torch.uint8), _dev(levels, "levels", torch.float32),
+        _dev(W_out, "W_out", torch.float32), _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+
+
+def kq_compression_report(n: int, k: int, omega: int = 3, b_c: int = 32) -> dict:
+    r = Report()
+    _check("kq_compression_report", lib().kq_compression_report(n, k, omega, b_c, ctypes.byref(r)))
+    return {f: getattr(r, f) for f, _ in Report._fields_}
+
+
+def kq_conventional_ratio(n: int, omega: int, u: int, b_1: int, b_fp: int = 32) -> float:
+    out = ctypes.c_double(0.0)
+    _check("kq_conventional_ratio", lib().kq_conventional_ratio(n, omega, u, b_1, b_fp, ctypes.byref(out)))
+    return out.value

@@ -1,0 +1,107 @@
+"""The C ABI without a GPU: the library loads, exports what include/kq.h declares,
+validates arguments on the host, and its storage report matches the oracle and
+the paper's tables."""
+import ctypes
+import os
+import re
+from fractions import Fraction
+
+import pytest
+
+import oracle
+from paper_2003_05148_gb300 import build, kq
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "kq.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return kq.lib()
+
+
+def _declared():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(kq_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = _declared()
+    assert len(names) >= 12
+    for name in names:
+        assert hasattr(lib, name), name
+    assert sorted(kq.EXPORTS) == names
+
+
+def test_status_strings_and_version(lib):
+    assert kq.kq_abi_version() == 1
+    for code, name in kq.STATUS_NAMES.items():
+        assert kq.kq_status_string(code) == name
+    assert kq.kq_status_string(99) == "KQ_ERR_UNKNOWN"
+
+
+def test_workspace_bytes_rules(lib):
+    assert kq.kq_workspace_bytes(0, 1) == 0
+    assert kq.kq_workspace_bytes(10, 11) == 0  # K > n
+    assert kq.kq_workspace_bytes(10, 0) == 0
+    assert kq.kq_workspace_bytes(2 ** 31, 16) == 0
+    a = kq.kq_workspace_bytes(4096, 16)
+    b = kq.kq_workspace_bytes(4194304, 65536)
+    assert 4096 < a < b and a % 256 == 0 and b % 256 == 0
+
+
+def test_host_validation_before_any_device_work(lib):
+    # Bad arguments are rejected on the host; the fake pointers are never touched.
+    L = lib
+    good = ctypes.c_void_p(1 << 20)  # 256-byte aligned dummy address
+    odd = ctypes.c_void_p((1 << 20) + 4)
+    ws_bytes = kq.kq_workspace_bytes(1024, 16)
+    assert L.kq_assign(good, 0, good, 16, good, None, good, ws_bytes, None) == 1  # n = 0
+    assert L.kq_assign(good, 1024, good, 2048, good, None, good, ws_bytes, None) == 1  # K > n
+    assert L.kq_assign(odd, 1024, good, 16, good, None, good, ws_bytes, None) == 2  # W not 16-byte aligned
+    assert L.kq_assign(good, 1024, good, 16, good, None, None, ws_bytes, None) == 6  # no workspace
+    assert L.kq_assign(good, 1024, good, 16, good, None, good, ws_bytes - 1, None) == 6  # too small
+    assert L.kq_assign(good, 1024, good, 16, good, None, odd, ws_bytes, None) == 2  # ws alignment
+    assert L.kq_update_centroids(good, 1024, good, 16, None, good, good, good, ws_bytes, None) == 1
+    assert L.kq_fit_codebook(good, 1024, 16, good, -1, 0, good, good, good, None, good, ws_bytes, None) == 1
+    assert L.kq_fit_codebook(good, 1024, 16, good, 3, 7, good, good, good, None, good, ws_bytes, None) == 1
+    assert L.kq_quantize_codebook_6bit(good, 16, good, -1, good, good, None, good, ws_bytes, None) == 1
+    assert L.kq_quantize_codebook_6bit(good, 16, good, 10, good, good, None, good, 100, None) == 6
+    assert L.kq_reconstruct(good, 1024, None, 16, None, None, good, good, ws_bytes, None) == 1  # nothing to decode
+    assert L.kq_reconstruct(good, 1024, good, 16, good, None, good, good, ws_bytes, None) == 1  # codes w/o levels
+    assert L.kq_reconstruct(good, 1024, good, 16, None, None, odd, good, ws_bytes, None) == 2  # W_out alignment
+    assert L.kq_init_codebook(good, 1024, good, 2000, good, good, ws_bytes, None) == 1
+    assert L.kq_device_status(None, 0, None, None) == 6
+
+
+def _report_rows():
+    rows = []
+    with open(os.path.join(os.path.dirname(__file__), "golden", "paper_tables.txt")) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                p = line.split()
+                rows.append((int(p[2]), int(p[3])))
+    return rows
+
+
+@pytest.mark.parametrize("n,k", _report_rows() + [(1, 1), (7, 3), (2 ** 30, 2), (4194304, 65536), (4096, 4096)])
+@pytest.mark.parametrize("b_c", [32, 6])
+def test_report_matches_oracle(lib, n, k, b_c):
+    got = kq.kq_compression_report(n, k, 3, b_c)
+    ref = oracle.report(n, k, 3, b_c)
+    assert got["index_bits"] == ref.index_bits
+    assert got["codebook_bits"] == ref.codebook_bits
+    assert got["total_bits"] == ref.total_bits
+    assert Fraction(got["beta"]) == pytest.approx(ref.beta, rel=1e-15)
+    assert Fraction(got["ratio_kq"]) == pytest.approx(ref.ratio_kq, rel=1e-15)
+
+
+def test_conventional_ratio_matches_oracle(lib):
+    for n, u, b1 in [(4096, 2, 32), (10 ** 9, 2, 32), (65536, 4, 32), (192, 16, 6)]:
+        assert kq.kq_conventional_ratio(n, 3, u, b1) == pytest.approx(float(oracle.ratio_conventional(n, 3, u, b1)),
+                                                                      rel=1e-15)
+    with pytest.raises(kq.KQError):
+        kq.kq_conventional_ratio(10, 3, 1, 32)
+    with pytest.raises(kq.KQError):
+        kq.kq_compression_report(0, 4)

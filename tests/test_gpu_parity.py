@@ -1,0 +1,278 @@
+"""GPU parity: every CUDA step through the C ABI against the CPU oracle, one step
+at a time from identical inputs (Sec. 3.1 Eq. 1 assign/update, Sec. 3.2 6-bit
+codebook quantisation and recovery).
+
+Bars: indices bit-exact (except oracle fp64 near-ties, gpu_util.TIE_RTOL);
+distances bit-exact; counts exact; centroids within gpu_util.CENTROID_RTOL
+(inf-norm relative per codeword); levels, codes and reconstructed weights
+bit-exact given identical fp32 inputs.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from gpu_util import (bits_equal, check_centroids, check_indices, dev, gpu_assign, gpu_quantize, gpu_reconstruct,
+                      gpu_update, to_dev)
+from paper_2003_05148_gb300 import kq
+
+pytestmark = pytest.mark.gpu
+THREADS = oracle.default_threads()
+
+
+def _layer(cfg, li=0):
+    lay = synth.workload(cfg).layers[li]
+    W, sel = synth.layer_inputs(lay)
+    return lay, W, oracle.gather_rows(W, sel)
+
+
+# --------------------------------------------------------------------------- assign
+
+@pytest.mark.parametrize("cfg,li", [(1, 0), (2, 0), (3, 0), (3, 1), (3, 8), (4, 0), (4, 4), (4, 9)])
+def test_assign_workload_layers(cfg, li):
+    lay, W, C0 = _layer(cfg, li)
+    idx, dist, st, _ = gpu_assign(W, C0)
+    assert st == 0
+    rows = None
+    if lay.n * lay.K > 3e8:  # rows are independent: check a seeded sample on the CPU
+        rows = np.sort(synth.below(synth.stream_key(lay.seed, 9), 8192, lay.n))
+    Wc = W if rows is None else W[rows]
+    idx_ref, dist_ref = oracle.assign(Wc, C0, threads=THREADS)
+    ig = idx if rows is None else idx[rows]
+    dg = dist if rows is None else dist[rows]
+    assert check_indices(W, C0, ig, idx_ref, rows) == 0
+    assert bits_equal(dg, dist_ref)
+
+
+def test_assign_full_size_stress_sampled():
+    # 2048x2048 layer, K = 65536: the launch configuration the benchmark times.
+    lay, W, C0 = _layer(5)
+    idx, dist, st, _ = gpu_assign(W, C0)
+    assert st == 0
+    rows = np.sort(synth.below(synth.stream_key(lay.seed, 9), 4096, lay.n))
+    rows[-1] = lay.n - 1  # include the ragged end of the last CTA
+    idx_ref, dist_ref = oracle.assign(W[rows], C0, threads=THREADS)
+    assert check_indices(W, C0, idx[rows], idx_ref, rows) == 0
+    assert bits_equal(dist[rows], dist_ref)
+    # every selected initial kernel is its own nearest codeword at distance 0
+    sel = synth.init_selection(lay.n, lay.K, lay.seed + 1)
+    assert np.all(dist[sel] == 0)
+
+
+@pytest.mark.parametrize("n,K", [(1, 1), (3, 2), (1023, 16), (1025, 17), (2047, 300), (6000, 5000),
+                                 (300, 300), (5000, 1), (100003, 7)])
+def test_assign_ragged_and_split(n, K):
+    W = synth.random_kernels(n, 9, n + 17, 0.1)
+    C = synth.random_kernels(K, 9, K + 29, 0.1)
+    idx, dist, st, _ = gpu_assign(W, C)
+    assert st == 0
+    idx_ref, dist_ref = oracle.assign(W, C, threads=THREADS)
+    assert check_indices(W, C, idx, idx_ref) == 0
+    assert bits_equal(dist, dist_ref)
+
+
+def test_assign_exact_ties_and_duplicates():
+    rng = np.random.default_rng(5)
+    W = rng.integers(-3, 4, size=(5000, 9)).astype(np.float32)
+    C = rng.integers(-3, 4, size=(700, 9)).astype(np.float32)
+    C[350:] = C[:350]  # every codeword duplicated: the lower index must win
+    idx, dist, st, _ = gpu_assign(W, C)
+    idx_ref, dist_ref = oracle.assign(W, C, threads=THREADS)
+    assert st == 0 and np.array_equal(idx, idx_ref) and bits_equal(dist, dist_ref)
+    assert idx.max() < 350
+
+
+def test_assign_nonfinite_flagged():
+    W = synth.random_kernels(2000, 9, 3)
+    W[1234, 5] = np.nan
+    C = synth.random_kernels(40, 9, 4)
+    idx, dist, st, flags = gpu_assign(W, C)
+    assert st == 3 and flags & kq.FLAG_NONFINITE
+    idx_ref, dist_ref = oracle.assign(W, C)
+    assert np.array_equal(idx, idx_ref) and bits_equal(dist, dist_ref)
+
+
+# --------------------------------------------------------------------------- update
+
+@pytest.mark.parametrize("cfg", [1, 2, 5])
+def test_update_from_identical_indices(cfg):
+    lay, W, C0 = _layer(cfg)
+    if cfg == 5:
+        idx = synth.below(synth.stream_key(lay.seed, 8), lay.n, lay.K).astype(np.int32)
+    else:
+        idx, _ = oracle.assign(W, C0, threads=THREADS)
+    C_g, cnt_g, st, _ = gpu_update(W, idx, C0)
+    C_r, cnt_r = oracle.update(W, idx, C0)
+    assert st == 0
+    assert np.array_equal(cnt_g, cnt_r)
+    check_centroids(C_g, C_r)
+    empty = cnt_r == 0
+    assert bits_equal(C_g[empty], C0[empty])
+
+
+def test_update_empty_clusters_and_bad_index():
+    W = synth.random_kernels(3000, 9, 7, 0.2)
+    C0 = synth.random_kernels(50, 9, 8)
+    idx = synth.below(synth.stream_key(9, 2), 3000, 25).astype(np.int32)  # codewords 25..49 stay empty
+    C_g, cnt_g, st, _ = gpu_update(W, idx, C0)
+    C_r, cnt_r = oracle.update(W, idx, C0)
+    assert st == 0 and np.array_equal(cnt_g, cnt_r)
+    check_centroids(C_g, C_r)
+    assert bits_equal(C_g[25:], C0[25:])
+    idx[17] = 50
+    _, cnt_g, st, flags = gpu_update(W, idx, C0)
+    assert st == 5 and flags & kq.FLAG_INDEX_RANGE and cnt_g.sum() == 2999
+
+
+def test_update_k1_global_mean():
+    W = synth.random_kernels(77777, 9, 11, 0.05)
+    C0 = W[:1].copy()
+    C_g, cnt_g, st, _ = gpu_update(W, np.zeros(77777, np.int32), C0)
+    C_r, _ = oracle.update(W, np.zeros(77777, np.int32), C0)
+    assert st == 0 and cnt_g[0] == 77777
+    check_centroids(C_g, C_r)
+
+
+# --------------------------------------------------------------------------- fit
+
+def _gpu_fit(W, C0, iters):
+    n, K = W.shape[0], C0.shape[0]
+    Wd, Cd = to_dev(W), to_dev(C0)
+    C = torch.empty_like(Cd)
+    idx = torch.empty(n, dtype=torch.int32, device=dev())
+    counts = torch.empty(K, dtype=torch.int32, device=dev())
+    obj = torch.empty(iters + 1, dtype=torch.float64, device=dev())
+    ws = kq.workspace(n, K, dev())
+    kq.kq_fit_codebook(Wd, Cd, iters, C, idx, counts, obj, ws)
+    st, _ = kq.kq_device_status(ws)
+    assert st == 0
+    return C.cpu().numpy(), idx.cpu().numpy(), counts.cpu().numpy(), obj.cpu().numpy()
+
+
+@pytest.mark.parametrize("cfg,li", [(1, 0), (2, 0), (3, 2), (4, 1)])
+def test_fit_stepwise(cfg, li):
+    lay, W, C0 = _layer(cfg, li)
+    T = 3
+    C = C0
+    objs = []
+    for t in range(T):
+        C_next, idx_next, cnt_next, obj = _gpu_fit(W, C, 1)
+        idx_ref, dist_ref = oracle.assign(W, C, threads=THREADS)
+        C_ref, _ = oracle.update(W, idx_ref, C)
+        check_centroids(C_next, C_ref)
+        objs.append(obj[0])
+        assert obj[0] == pytest.approx(oracle.objective(dist_ref), rel=1e-12)
+        # the fit's final assignment and counts are those of its own C_next
+        i2, d2 = oracle.assign(W, C_next, threads=THREADS)
+        assert check_indices(W, C_next, idx_next, i2) == 0
+        assert np.array_equal(cnt_next, np.bincount(idx_next, minlength=lay.K))
+        assert obj[1] == pytest.approx(oracle.objective(d2), rel=1e-12)
+        C = C_next
+    # T iterations in one call == T chained single-iteration calls, bit for bit
+    C_T, idx_T, cnt_T, obj_T = _gpu_fit(W, C0, T)
+    assert bits_equal(C_T, C)
+    assert np.all(obj_T[1:] <= obj_T[:-1] * (1 + 1e-6))
+
+
+def test_fit_end_to_end_against_oracle():
+    lay, W, C0 = _layer(1)
+    C_g, idx_g, cnt_g, obj_g = _gpu_fit(W, C0, 10)
+    C_r, idx_r, cnt_r, obj_r = oracle.fit(W, C0, 10, threads=THREADS)
+    # centroid errors of ~1e-13 could flip an exact near-tie; this seeded input has none
+    assert np.array_equal(idx_g, idx_r) and np.array_equal(cnt_g, cnt_r)
+    check_centroids(C_g, C_r)
+    np.testing.assert_allclose(obj_g, obj_r, rtol=1e-9)
+
+
+def test_fit_zero_iterations_and_identity():
+    W = synth.random_kernels(500, 9, 13)
+    C_g, idx_g, cnt_g, obj_g = _gpu_fit(W, W, 0)
+    assert bits_equal(C_g, W) and np.array_equal(idx_g, np.arange(500)) and np.all(cnt_g == 1)
+    assert obj_g[0] == 0.0
+    C_g, idx_g, cnt_g, obj_g = _gpu_fit(W, W, 2)  # K = n seeded with all kernels is a fixed point
+    assert bits_equal(C_g, W) and np.array_equal(idx_g, np.arange(500)) and np.all(obj_g == 0.0)
+
+
+def test_fit_deterministic():
+    lay, W, C0 = _layer(2)
+    a = _gpu_fit(W, C0, 4)
+    b = _gpu_fit(W, C0, 4)
+    for x, y in zip(a, b):
+        assert bits_equal(x, y)
+
+
+# --------------------------------------------------------------------------- 6-bit quantisation
+
+@pytest.mark.parametrize("K,seed,high", [(1, 1, 5), (16, 2, 300), (256, 3, 600), (5000, 4, 100), (65536, 5, 128)])
+def test_quantize_random_codebooks(K, seed, high):
+    C = synth.random_kernels(K, 9, seed, 0.02)
+    counts = synth.random_counts(K, seed + 100, high)
+    lv_g, cd_g, it_g, st, _ = gpu_quantize(C, counts)
+    lv_r, cd_r, it_r = oracle.level_fit(C, counts)
+    assert st == 0
+    assert bits_equal(lv_g, lv_r) and np.array_equal(cd_g, cd_r) and it_g == it_r
+
+
+def test_quantize_fitted_codebook():
+    lay, W, C0 = _layer(2)
+    C, idx, counts, _ = _gpu_fit(W, C0, 5)
+    lv_g, cd_g, it_g, st, _ = gpu_quantize(C, counts)
+    lv_r, cd_r, it_r = oracle.level_fit(C, counts)
+    assert st == 0 and bits_equal(lv_g, lv_r) and np.array_equal(cd_g, cd_r) and it_g == it_r
+
+
+@pytest.mark.parametrize("case", ["zero_iters", "no_weights", "constant", "few_values", "max_iters_1"])
+def test_quantize_edge_cases(case):
+    C = synth.random_kernels(300, 9, 21, 0.05)
+    counts = synth.random_counts(300, 22, 40)
+    iters = 100
+    if case == "zero_iters":
+        iters = 0
+    elif case == "no_weights":
+        counts[:] = 0
+    elif case == "constant":
+        C[:] = 0.25
+    elif case == "few_values":
+        C = (np.arange(300 * 9) % 5).astype(np.float32).reshape(300, 9)
+    elif case == "max_iters_1":
+        iters = 1
+    lv_g, cd_g, it_g, st, _ = gpu_quantize(C, counts, iters)
+    lv_r, cd_r, it_r = oracle.level_fit(C, counts, iters)
+    assert st == 0 and bits_equal(lv_g, lv_r) and np.array_equal(cd_g, cd_r) and it_g == it_r
+
+
+# --------------------------------------------------------------------------- reconstruction
+
+@pytest.mark.parametrize("n,K", [(1, 1), (31, 5), (4096, 16), (100001, 256), (4194304, 65536)])
+def test_reconstruct(n, K):
+    C = synth.random_kernels(K, 9, K, 0.05)
+    idx = synth.below(synth.stream_key(n, 2), n, K).astype(np.int32)
+    counts = np.bincount(idx, minlength=K).astype(np.int32)
+    Wk, st, _ = gpu_reconstruct(idx, C)
+    assert st == 0 and bits_equal(Wk, oracle.reconstruct(idx, C))
+    lv, cd, _ = oracle.level_fit(C, counts, 20)
+    Wkc, st, _ = gpu_reconstruct(idx, C, cd, lv)
+    assert st == 0 and bits_equal(Wkc, oracle.reconstruct(idx, C, cd, lv))
+
+
+def test_reconstruct_flags_bad_index_and_code():
+    C = synth.random_kernels(10, 9, 1)
+    idx = np.arange(100, dtype=np.int32) % 10
+    idx[7] = 10
+    Wr, st, flags = gpu_reconstruct(idx, C)
+    assert st == 5 and flags & kq.FLAG_INDEX_RANGE and np.all(Wr[7] == 0)
+    codes = np.zeros((10, 9), np.uint8)
+    codes[3, 4] = 64
+    Wr, st, flags = gpu_reconstruct(np.arange(10, dtype=np.int32), C, codes, np.arange(64, dtype=np.float32))
+    assert st == 5 and flags & kq.FLAG_CODE_RANGE and Wr[3, 4] == 0
+
+
+def test_init_codebook():
+    lay = synth.workload(2).layers[0]
+    W, sel = synth.layer_inputs(lay)
+    C0 = torch.empty(lay.K, 9, dtype=torch.float32, device=dev())
+    ws = kq.workspace(lay.n, lay.K, dev())
+    kq.kq_init_codebook(to_dev(W), to_dev(sel), C0, ws)
+    assert kq.kq_device_status(ws)[0] == 0
+    assert bits_equal(C0.cpu().numpy(), oracle.gather_rows(W, sel))
