@@ -339,6 +339,59 @@ def run_kq(args, rank, world, local_rank):
     print(json.dumps(out), flush=True)
 
 
+def run_only(args):
+    """One hot-path step on its own, for profiler captures: synthetic stress-layer
+    inputs with n / K overridden, `reps` launches of the chosen entry point."""
+    import torch
+
+    from paper_2003_05148_gb300 import build, kq
+
+    build.build()
+    dev = torch.device("cuda", 0)
+    base = synth.workload(WORKLOAD_CFG).layers[0]
+    p = base.p if args.n % base.p == 0 else 1
+    lay = synth.Layer("profile", p, args.n // p, args.K, min(4 * args.K, args.n), base.seed)
+    W_h, sel_h = synth.layer_inputs(lay)
+    n, K = W_h.shape[0], args.K
+    W = torch.from_numpy(W_h).to(dev)
+    sel = torch.from_numpy(sel_h).to(dev)
+    ws = kq.workspace(n, K, dev)
+    C = torch.empty(K, 9, dtype=torch.float32, device=dev)
+    C2 = torch.empty_like(C)
+    kq.kq_init_codebook(W, sel, C, ws)
+    idx = torch.empty(n, dtype=torch.int32, device=dev)
+    counts = torch.empty(K, dtype=torch.int32, device=dev)
+    kq.kq_assign(W, C, idx, None, ws)
+    kq.kq_update_centroids(W, idx, C, C2, counts, ws)
+    levels = torch.empty(64, dtype=torch.float32, device=dev)
+    codes = torch.empty(K, 9, dtype=torch.uint8, device=dev)
+    kq.kq_quantize_codebook_6bit(C2, counts, 100, levels, codes, None, ws)
+    Wr = torch.empty_like(W)
+    calls = {
+        "assign": lambda: kq.kq_assign(W, C, idx, None, ws),
+        "update": lambda: kq.kq_update_centroids(W, idx, C, C2, counts, ws),
+        "quantize": lambda: kq.kq_quantize_codebook_6bit(C2, counts, 100, levels, codes, None, ws),
+        "reconstruct": lambda: kq.kq_reconstruct(idx, None, codes, levels, Wr, ws, K=K),
+    }
+    f = calls[args.only]
+    for _ in range(2):
+        f()
+    torch.cuda.synchronize()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.reps)]
+    stream = torch.cuda.current_stream()
+    for a, b in evs:
+        a.record(stream)
+        f()
+        b.record(stream)
+    torch.cuda.synchronize()
+    st, flags = kq.kq_device_status(ws)
+    ms = [a.elapsed_time(b) for a, b in evs]
+    print(json.dumps({"only": args.only, "n": n, "K": K, "reps": args.reps, "ms_mean": statistics.mean(ms),
+                      "ms_min": min(ms), "status": st, "flags": flags}), flush=True)
+    if st != 0:
+        sys.exit(1)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -348,7 +401,15 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--ref-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--only", choices=["assign", "update", "quantize", "reconstruct"],
+                    help="profiling aid: time one entry point on its own (no bench line)")
+    ap.add_argument("--n", type=int, default=4194304)
+    ap.add_argument("--K", type=int, default=65536)
+    ap.add_argument("--reps", type=int, default=3)
     args = ap.parse_args()
+    if args.only:
+        run_only(args)
+        return
     if args.warmup < 3:
         print("warning: fewer than 3 warm-up steps", file=sys.stderr)
     world = int(os.environ.get("WORLD_SIZE", "1"))
