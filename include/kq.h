@@ -111,6 +111,24 @@ kq_status kq_init_codebook(const float *W, int64_t n, const int64_t *sel, int32_
 kq_status kq_assign(const float *W, int64_t n, const float *C, int32_t K, int32_t *idx, float *dist, void *ws,
                     size_t ws_bytes, kq_stream_t stream);
 
+/* kq_assign for callers that cannot allocate device memory. The paper has no
+ * counterpart: this exists for code that must not call cudaMalloc (or have
+ * anyone allocate for it) -- e.g. a plugin living inside a host application
+ * whose own allocator owns all of the device's memory, or a latency-critical
+ * service that forbids allocation, and the synchronisation cudaMalloc/cudaFree
+ * can bring, once it is running. Such a caller cannot provide the workspace.
+ * Same inputs, outputs and rules as kq_assign, without the workspace: the
+ * scratch is a fixed array of about 10 MB built into libkq, which every GPU that
+ * loads the library holds until the process exits. Limits: n <= 16,777,216 and
+ * K <= 65,536; larger sizes return KQ_ERR_WORKSPACE. The first call on a device
+ * looks up the array's device address (once per device, so make that first call
+ * before any stream capture). Every call on a device shares the array, so calls
+ * whose work can overlap on the GPU race: issue them in order on one stream.
+ * Device-side flags (e.g. a non-finite input) are not reported by this variant.
+ * It never allocates or frees memory. */
+kq_status kq_assign_noalloc(const float *W, int64_t n, const float *C, int32_t K, int32_t *idx, float *dist,
+                            kq_stream_t stream);
+
 /* Update step of k-means, Sec. 3.1 Eq. 1: for every codeword,
  *   counts[k] = z_k = |S_k| = #{ i : idx[i] == k },
  *   C_next[k] = (1 / z_k) * sum_{i in S_k} m_i   if z_k > 0, else C_prev[k],

@@ -23,7 +23,7 @@ FLAG_NONFINITE, FLAG_INDEX_RANGE, FLAG_CODE_RANGE, FLAG_TIMEOUT = 0x1, 0x2, 0x4,
 
 EXPORTS = ["kq_status_string", "kq_abi_version", "kq_kernel_launches", "kq_workspace_bytes", "kq_device_status", "kq_init_codebook",
            "kq_assign", "kq_update_centroids", "kq_fit_codebook", "kq_quantize_codebook_6bit", "kq_reconstruct",
-           "kq_compression_report", "kq_conventional_ratio"]
+           "kq_compression_report", "kq_conventional_ratio", "kq_assign_noalloc"]
 
 
 class KQError(RuntimeError):
@@ -62,6 +62,7 @@ def lib() -> ctypes.CDLL:
             "kq_reconstruct": ([P, i64, P, i32, P, P, P, P, sz, P], ctypes.c_int),
             "kq_compression_report": ([i64, i32, i32, i32, ctypes.POINTER(Report)], ctypes.c_int),
             "kq_conventional_ratio": ([i64, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
+            "kq_assign_noalloc": ([P, i64, P, i32, P, P, P], ctypes.c_int),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -182,3 +183,10 @@ def kq_conventional_ratio(n: int, omega: int, u: int, b_1: int, b_fp: int = 32) 
     out = ctypes.c_double(0.0)
     _check("kq_conventional_ratio", lib().kq_conventional_ratio(n, omega, u, b_1, b_fp, ctypes.byref(out)))
     return out.value
+
+
+def kq_assign_noalloc(W, C, idx, dist, stream=None) -> None:
+    """kq_assign without a workspace, for callers that cannot allocate device memory."""
+    _check("kq_assign_noalloc", lib().kq_assign_noalloc(
+        _dev(W, "W", torch.float32), _rows(W), _dev(C, "C", torch.float32), _rows(C),
+        _dev(idx, "idx", torch.int32), _dev(dist, "dist", torch.float32), _stream(stream)))
