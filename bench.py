@@ -206,14 +206,15 @@ def run_kq(args, rank, world, local_rank):
         for t in range(T):
             if ev:
                 ev[t][0].record(stream)
-            kq.kq_assign(W, cur, idx, None, ws)
+            # iterations after the first start from the previous assignment (as kq_fit_codebook does)
+            kq.kq_assign(W, cur, idx, None, ws, hint=idx if t > 0 else None)
             if ev:
                 ev[t][1].record(stream)
             kq.kq_update_centroids(W, idx, cur, nxt, counts, ws)
             cur, nxt = nxt, cur
         if ev:
             ev[T][0].record(stream)
-        kq.kq_assign(W, cur, idx, None, ws)
+        kq.kq_assign(W, cur, idx, None, ws, hint=idx if T > 0 else None)
         if ev:
             ev[T][1].record(stream)
         kq.kq_update_centroids(W, idx, cur, nxt, counts, ws)  # cluster sizes of the final assignment

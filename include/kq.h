@@ -101,17 +101,23 @@ kq_status kq_init_codebook(const float *W, int64_t n, const int64_t *sel, int32_
  *   idx[i]  = argmin_k || m_i - c_k ||^2,   dist[i] = that minimum,
  * with the distance evaluated in fp32 as t_j = fl(x_j - c_j), acc = fma(t_j,
  * t_j, acc) for j = 0..8 in order (acc starts at 0), and ties resolved toward
- * the lowest k (the running best starts at (+inf, 0)).
+ * the lowest k (the running best starts at (+inf, 0)). The result is exactly this
+ * argmin; internally most pairs are ruled out by a cheaper expanded-form test
+ * with a rigorous rounding-error bound, which never changes the answer.
  *   W     n x 9 fp32 (device, 16-byte aligned)
  *   C     K x 9 fp32 (device)
+ *   hint  n int32 (device) or NULL: a previous assignment (e.g. the last Lloyd
+ *         iteration's). Each row's search starts from its hinted codeword; only
+ *         speed depends on it, never the result. Entries outside [0, K) are
+ *         ignored. May be the same array as idx (in-place update).
  *   idx   n int32 output (device)
  *   dist  n fp32 output (device) or NULL
  * A non-finite value in W or C sets KQ_FLAG_NONFINITE (the outputs are still
  * written by the rules above). */
-kq_status kq_assign(const float *W, int64_t n, const float *C, int32_t K, int32_t *idx, float *dist, void *ws,
-                    size_t ws_bytes, kq_stream_t stream);
+kq_status kq_assign(const float *W, int64_t n, const float *C, int32_t K, const int32_t *hint, int32_t *idx,
+                    float *dist, void *ws, size_t ws_bytes, kq_stream_t stream);
 
-/* kq_assign for callers that cannot allocate device memory. The paper has no
+/* kq_assign (without a hint) for callers that cannot allocate device memory. The paper has no
  * counterpart: this exists for code that must not call cudaMalloc (or have
  * anyone allocate for it) -- e.g. a plugin living inside a host application
  * whose own allocator owns all of the device's memory, or a latency-critical
@@ -156,7 +162,8 @@ kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int
  *   counts     K int32 output: cluster sizes of the final assignment (device)
  *   objective  iters + 1 fp64 outputs (device) or NULL: Eq. 1 objective per step,
  *              summed in a fixed order (bitwise reproducible)
- * Runs entirely on `stream`; no host synchronisation. */
+ * Every assignment after the first is warm-started from the previous one (see
+ * kq_assign's hint). Runs entirely on `stream`; no host synchronisation. */
 kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_init, int32_t iters, int32_t flags,
                           float *C_out, int32_t *idx, int32_t *counts, double *objective, void *ws, size_t ws_bytes,
                           kq_stream_t stream);

@@ -16,7 +16,7 @@ void count_launch(int kernels) { g_launches.fetch_add((unsigned long long)kernel
 
 namespace {
 
-constexpr int32_t KQ_ABI_VERSION = 1;
+constexpr int32_t KQ_ABI_VERSION = 2;
 
 inline bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
@@ -82,9 +82,9 @@ Ws carve(void *ws, int64_t n, int32_t K) {
 // Update step on prepared state: accumulate into the (zeroed) accumulators and
 // finalise; the finalise leaves the accumulators zeroed again.
 kq_status run_update(const float *W, int64_t n, const int32_t *idx, int32_t K, const float *C_prev, float *C_next,
-                     int32_t *counts, float *Cd_next, const Ws &w, int sms, cudaStream_t s) {
+                     int32_t *counts, const Ws &w, int sms, cudaStream_t s) {
     KQ_TRY(launch_accumulate(W, n, idx, K, &w.hdr->maxabs_bits, w.acc, &w.hdr->status, sms, s));
-    KQ_TRY(launch_finalize(w.acc, K, n, &w.hdr->maxabs_bits, C_prev, C_next, counts, Cd_next, s));
+    KQ_TRY(launch_finalize(w.acc, K, n, &w.hdr->maxabs_bits, C_prev, C_next, counts, s));
     return KQ_OK;
 }
 
@@ -155,19 +155,20 @@ kq_status kq_init_codebook(const float *W, int64_t n, const int64_t *sel, int32_
     return cuda_status(launch_init_codebook(W, n, sel, K, C0, &h->status, reinterpret_cast<cudaStream_t>(stream)));
 }
 
-kq_status kq_assign(const float *W, int64_t n, const float *C, int32_t K, int32_t *idx, float *dist, void *ws,
-                    size_t ws_bytes, kq_stream_t stream) {
+kq_status kq_assign(const float *W, int64_t n, const float *C, int32_t K, const int32_t *hint, int32_t *idx,
+                    float *dist, void *ws, size_t ws_bytes, kq_stream_t stream) {
     if (!sizes_ok(n, K) || !W || !C || !idx) return KQ_ERR_INVALID_ARG;
-    if (!aligned(W, 16) || !aligned(C, 4) || !aligned(idx, 4) || !aligned(dist, 4)) return KQ_ERR_ALIGNMENT;
+    if (!aligned(W, 16) || !aligned(C, 4) || !aligned(idx, 4) || !aligned(dist, 4) || !aligned(hint, 4))
+        return KQ_ERR_ALIGNMENT;
     kq_status st = check_ws(ws, ws_bytes, n, K);
     if (st != KQ_OK) return st;
     int sms = 0;
     if ((st = num_sms(&sms)) != KQ_OK) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     Ws w = carve(ws, n, K);
-    KQ_TRY(launch_pack_codebook(C, K, w.cd, &w.hdr->status, s));
+    KQ_TRY(launch_pack_codebook(C, K, w.cd, w.hdr, s));
     int nb = 0;
-    KQ_TRY(launch_assign(W, n, w.cd, K, idx, dist, w.blocksum, &nb, w.part, &w.hdr->status, sms, s));
+    KQ_TRY(launch_assign(W, n, w.cd, C, K, hint, idx, dist, w.blocksum, &nb, w.part, w.hdr, sms, s));
     return KQ_OK;
 }
 
@@ -183,7 +184,7 @@ kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     Ws w = carve(ws, n, K);
     if ((st = prepare_update(W, n, K, w, sms, s)) != KQ_OK) return st;
-    return run_update(W, n, idx, K, C_prev, C_next, counts, nullptr, w, sms, s);
+    return run_update(W, n, idx, K, C_prev, C_next, counts, w, sms, s);
 }
 
 kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_init, int32_t iters, int32_t flags,
@@ -204,18 +205,22 @@ kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_i
 
     if ((st = prepare_update(W, n, K, w, sms, s)) != KQ_OK) return st;
     KQ_TRY(cudaMemcpyAsync(w.cbuf0, C_init, cbytes, cudaMemcpyDeviceToDevice, s));
-    KQ_TRY(launch_pack_codebook(w.cbuf0, K, w.cd, &w.hdr->status, s));
     float *cur = w.cbuf0, *nxt = w.cbuf1;
     int nb = 0;
+    // iteration t > 0 starts every row from its previous assignment (warm start)
     for (int32_t t = 0; t < iters; ++t) {
-        KQ_TRY(launch_assign(W, n, w.cd, K, idx, nullptr, w.blocksum, &nb, w.part, &w.hdr->status, sms, s));
+        KQ_TRY(launch_pack_codebook(cur, K, w.cd, w.hdr, s));
+        KQ_TRY(launch_assign(W, n, w.cd, cur, K, t > 0 ? idx : nullptr, idx, nullptr, w.blocksum, &nb, w.part, w.hdr,
+                             sms, s));
         if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
-        if ((st = run_update(W, n, idx, K, cur, nxt, counts, w.cd, w, sms, s)) != KQ_OK) return st;
+        if ((st = run_update(W, n, idx, K, cur, nxt, counts, w, sms, s)) != KQ_OK) return st;
         float *tmp = cur;
         cur = nxt;
         nxt = tmp;
     }
-    KQ_TRY(launch_assign(W, n, w.cd, K, idx, nullptr, w.blocksum, &nb, w.part, &w.hdr->status, sms, s));
+    KQ_TRY(launch_pack_codebook(cur, K, w.cd, w.hdr, s));
+    KQ_TRY(launch_assign(W, n, w.cd, cur, K, iters > 0 ? idx : nullptr, idx, nullptr, w.blocksum, &nb, w.part, w.hdr,
+                         sms, s));
     if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + iters, s));
     KQ_TRY(launch_histogram(idx, n, K, counts, &w.hdr->status, sms, s));
     KQ_TRY(cudaMemcpyAsync(C_out, cur, cbytes, cudaMemcpyDeviceToDevice, s));

@@ -14,7 +14,7 @@ constexpr int LEVELS = 64;       // 6-bit codebook quantisation (Sec. 3.2)
 constexpr int CD_FLOATS = 20;    // packed codeword for the assign kernel: 10 duplicated pairs
 constexpr int CP_FLOATS = 12;    // padded codeword row for the reconstruct gather (48 B)
 constexpr int ACC_WORDS = 16;    // int64 accumulator row per codeword: 9 sums, count, pad (128 B)
-constexpr int ROW_BLOCK = 1024;  // kernels per assign CTA (256 threads x 4 rows)
+constexpr int ROW_BLOCK = 1024;  // kernels per assign CTA (128 threads x 8 rows)
 constexpr int MAX_PART_BLOCKS = 512;  // bound on (row blocks x codeword splits) with split-K
 
 // Fixed part of the workspace (first 4 KiB).
@@ -29,6 +29,7 @@ struct Header {
     uint32_t hi_w, hi_a;    // level fit: ordered-int maxima over weighted / all scalars (init 0)
     uint32_t maxv_w;        // level fit: max |v| over weighted scalars (fp32 bits)
     uint32_t pad1;
+    uint32_t cb_cmax, cb_hmax, cb_qmax, pad2;  // assign filter: codebook bounds (fp32 bits, see kq_assign.cu)
     unsigned long long wtotal;          // level fit: sum of weights
     unsigned long long lacc[3][LEVELS][2];  // level fit: (weight sum, fixed-point sum) per level
 };
@@ -90,6 +91,39 @@ __device__ __forceinline__ float ord2f(uint32_t u) {
     return __uint_as_float((u & 0x80000000u) ? (u & 0x7fffffffu) : ~u);
 }
 
+// rint(v * 2^S) as int64 (round half to even) for a finite fp32 v, using only
+// integer operations: v = +-m * 2^(e - 150) (e the biased exponent, m with its
+// implicit bit; subnormals m * 2^-149). Equal to rounding the exact product
+// (double)v * 2^S to the nearest integer, ties to even. Callers choose S so that
+// |v| * 2^S stays below 2^62; larger shifts are clamped (a finite-input bound
+// violation only, reported elsewhere).
+__device__ __forceinline__ long long fixed_rn(float v, int S) {
+    const uint32_t u = __float_as_uint(v);
+    const uint32_t e = (u >> 23) & 0xffu;
+    uint32_t m = u & 0x7fffffu;
+    int sh;
+    if (e == 0) {
+        sh = S - 149;
+    } else {
+        m |= 0x800000u;
+        sh = (int)e - 150 + S;
+    }
+    unsigned long long q;
+    if (sh >= 0) {
+        q = (unsigned long long)m << (sh > 62 ? 62 : sh);
+    } else if (sh <= -25) {
+        q = 0;  // |v| * 2^S < 1/2
+    } else {
+        const int r = -sh;
+        uint32_t qi = m >> r;
+        const uint32_t rem = m & ((1u << r) - 1u);
+        const uint32_t half = 1u << (r - 1);
+        if (rem > half || (rem == half && (qi & 1u))) qi += 1u;
+        q = qi;
+    }
+    return (u >> 31) ? -(long long)q : (long long)q;
+}
+
 __device__ __forceinline__ void set_flag(uint32_t *status, uint32_t bit) { atomicOr(status, bit); }
 
 __device__ __forceinline__ bool finite9(const float *v) {
@@ -103,10 +137,13 @@ __device__ __forceinline__ bool finite9(const float *v) {
 void count_launch(int kernels = 1);
 
 // ---- launchers (defined in the .cu files; all return cudaGetLastError()) ----
-cudaError_t launch_pack_codebook(const float *C, int32_t K, float *Cd, uint32_t *status, cudaStream_t s);
-cudaError_t launch_assign(const float *W, int64_t n, const float *Cd, int32_t K, int32_t *idx, float *dist,
-                          double *blocksum, int *nblocksum, unsigned long long *part, uint32_t *status,
-                          int num_sms, cudaStream_t s);
+// Packs C for the assign kernel and computes the filter's codebook bounds into
+// hdr->cb_* (which must be zero before the call; the launcher clears them).
+cudaError_t launch_pack_codebook(const float *C, int32_t K, float *Cd, Header *hdr, cudaStream_t s);
+// hint (nullable, may alias idx): a previous assignment used as a warm start.
+cudaError_t launch_assign(const float *W, int64_t n, const float *Cd, const float *C, int32_t K, const int32_t *hint,
+                          int32_t *idx, float *dist, double *blocksum, int *nblocksum, unsigned long long *part,
+                          Header *hdr, int num_sms, cudaStream_t s);
 cudaError_t launch_sum_blocks(const double *blocksum, int nblocks, double *out, cudaStream_t s);
 
 cudaError_t launch_maxabs(const float *W, int64_t count, uint32_t *maxabs_bits, uint32_t *status, int num_sms,
@@ -117,8 +154,7 @@ cudaError_t launch_accumulate(const float *W, int64_t n, const int32_t *idx, int
 cudaError_t launch_histogram(const int32_t *idx, int64_t n, int32_t K, int32_t *counts, uint32_t *status,
                              int num_sms, cudaStream_t s);
 cudaError_t launch_finalize(unsigned long long *acc, int32_t K, int64_t n, const uint32_t *maxabs_bits,
-                            const float *C_prev, float *C_next, int32_t *counts, float *Cd_next,
-                            cudaStream_t s);
+                            const float *C_prev, float *C_next, int32_t *counts, cudaStream_t s);
 
 cudaError_t launch_level_fit(const float *C, int32_t K, const int32_t *counts, int32_t max_iters, float *levels,
                              uint8_t *codes, int32_t *iters_run, Header *hdr, int num_sms, cudaStream_t s);

@@ -21,9 +21,9 @@ namespace {
 constexpr int64_t NOALLOC_MAX_N = 1LL << 24;  // 16,777,216 kernels
 constexpr int32_t NOALLOC_MAX_K = 65536;       // codewords
 
-// Byte offsets inside the scratch array.
-constexpr size_t SCR_STATUS = 0;
-constexpr size_t SCR_CD = 256;
+// Byte offsets inside the scratch array (a workspace header comes first).
+constexpr size_t SCR_HEADER = 0;
+constexpr size_t SCR_CD = 4096;
 constexpr size_t SCR_PART = SCR_CD + (size_t)NOALLOC_MAX_K * CD_FLOATS * sizeof(float);
 constexpr size_t SCR_BLOCKSUM = SCR_PART + (size_t)MAX_PART_BLOCKS * ROW_BLOCK * sizeof(unsigned long long);
 constexpr size_t SCR_BYTES =
@@ -68,15 +68,16 @@ extern "C" kq_status kq_assign_noalloc(const float *W, int64_t n, const float *C
     if (cudaGetDevice(&dev) != cudaSuccess) return KQ_ERR_CUDA;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return KQ_ERR_CUDA;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    uint32_t *status = reinterpret_cast<uint32_t *>(scr + SCR_STATUS);
+    Header *hdr = reinterpret_cast<Header *>(scr + SCR_HEADER);
     float *cd = reinterpret_cast<float *>(scr + SCR_CD);
     unsigned long long *part = reinterpret_cast<unsigned long long *>(scr + SCR_PART);
     double *blocksum = reinterpret_cast<double *>(scr + SCR_BLOCKSUM);
-    // The status word is the only part that must start at zero; the rest is
-    // fully written before it is read.
-    if (cudaMemsetAsync(status, 0, sizeof(uint32_t), s) != cudaSuccess) return KQ_ERR_CUDA;
-    if (launch_pack_codebook(C, K, cd, status, s) != cudaSuccess) return KQ_ERR_CUDA;
+    // The status word and the codebook bounds (cleared by the pack launcher) must
+    // start at zero; everything else is fully written before it is read.
+    if (cudaMemsetAsync(&hdr->status, 0, sizeof(uint32_t), s) != cudaSuccess) return KQ_ERR_CUDA;
+    if (launch_pack_codebook(C, K, cd, hdr, s) != cudaSuccess) return KQ_ERR_CUDA;
     int nb = 0;
-    if (launch_assign(W, n, cd, K, idx, dist, blocksum, &nb, part, status, sms, s) != cudaSuccess) return KQ_ERR_CUDA;
+    if (launch_assign(W, n, cd, C, K, nullptr, idx, dist, blocksum, &nb, part, hdr, sms, s) != cudaSuccess)
+        return KQ_ERR_CUDA;
     return KQ_OK;
 }

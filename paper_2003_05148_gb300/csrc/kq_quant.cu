@@ -150,7 +150,7 @@ __global__ void __launch_bounds__(Q_THREADS) level_fit_kernel(LevelArgs a) {
         frexp(__dmul_rn(__ull2double_rn(A), (double)M), &e);
         S = 62 - e;
     }
-    const double up = ldexp(1.0, S), down = ldexp(1.0, -S);
+    const double down = ldexp(1.0, -S);
     if (threadIdx.x < LEVELS) {
         const double t = __ddiv_rn(__dmul_rn(__dsub_rn((double)hi, (double)lo), (double)threadIdx.x), 63.0);
         L[threadIdx.x] = __double2float_rn(__dadd_rn((double)lo, t));
@@ -178,7 +178,7 @@ __global__ void __launch_bounds__(Q_THREADS) level_fit_kernel(LevelArgs a) {
             a.codes[m] = (uint8_t)code;
             const int32_t z = a.counts[m / D];
             if (z > 0) {
-                const long long q = __double2ll_rn((double)v * up);
+                const long long q = fixed_rn(v, S);
                 atomicAdd(&bw[code], (unsigned long long)z);
                 atomicAdd(&bq[code], (unsigned long long)((long long)z * q));
             }

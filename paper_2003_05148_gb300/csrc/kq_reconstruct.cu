@@ -6,9 +6,7 @@
 // 48-byte rows that are 16-byte aligned, then the weight tensor is gathered,
 // W'[i] = C_hat[idx[i]]. The gather is HBM-bound (4 B of index read and 36 B of
 // weights written per kernel); the decoded codebook (<= a few MB) stays in L2.
-// A warp handles 32 consecutive kernels: each lane fetches its codeword row with
-// three 16-byte loads and drops it into a per-warp shared tile, and the warp then
-// writes the 1152 contiguous output bytes with coalesced streaming float4 stores.
+// The gather kernel is described above its definition.
 #include "kq_internal.cuh"
 
 namespace kq {
@@ -44,44 +42,66 @@ decode_codebook_kernel(const float *__restrict__ C, int32_t K, const uint8_t *__
     dst[2] = make_float4(c[8], c[9], c[10], c[11]);
 }
 
+// Each warp owns groups of G_CHUNKS x 32 consecutive kernels. All index loads of
+// a group are issued first, then all codebook-row gathers (three 16-byte loads per
+// kernel), so a warp keeps a whole group of requests in flight. The rows go into a
+// per-warp shared tile (kernel i at float offset 9i, conflict-free), which the warp
+// then writes out with coalesced streaming float4 stores.
+constexpr int G_CHUNKS = 2;
+constexpr int G_ROWS = 32 * G_CHUNKS;
+constexpr int G_TILE_FLOATS = G_ROWS * D;
+constexpr int R_WARPS = R_THREADS / 32;
+
 __global__ void __launch_bounds__(R_THREADS)
 gather_rows_kernel(const int32_t *__restrict__ idx, int64_t n, const float *__restrict__ Cp, int32_t K,
                    float *__restrict__ W_out, uint32_t *status) {
-    __shared__ __align__(16) float tile[R_THREADS / 32][32 * D];
+    __shared__ __align__(16) float tile[R_WARPS][G_TILE_FLOATS];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t ngroups = n / G_ROWS;  // full groups; the ragged end is handled below
+    bool bad = false;
     float *t = tile[warp];
-    const int64_t nchunks = (n + 31) / 32;
-    for (int64_t ch = (int64_t)blockIdx.x * (R_THREADS / 32) + warp; ch < nchunks;
-         ch += (int64_t)gridDim.x * (R_THREADS / 32)) {
-        const int64_t r0 = ch * 32;
-        const int rows = (int)min((int64_t)32, n - r0);
-        if (lane < rows) {
-            const int32_t k = __ldcs(idx + r0 + lane);
-            float4 a = make_float4(0.f, 0.f, 0.f, 0.f), b = a, c = a;
-            if ((uint32_t)k < (uint32_t)K) {
-                const float4 *src = reinterpret_cast<const float4 *>(Cp + (int64_t)k * CP_FLOATS);
-                a = __ldg(src);
-                b = __ldg(src + 1);
-                c = __ldg(src + 2);
-            } else {
-                set_flag(status, KQ_FLAG_INDEX_RANGE);
-            }
-            float *row = t + lane * D;
-            row[0] = a.x; row[1] = a.y; row[2] = a.z; row[3] = a.w;
-            row[4] = b.x; row[5] = b.y; row[6] = b.z; row[7] = b.w;
-            row[8] = c.x;
+    for (int64_t g = (int64_t)blockIdx.x * R_WARPS + warp; g < ngroups; g += (int64_t)gridDim.x * R_WARPS) {
+        const int64_t r0 = g * G_ROWS;
+        int32_t k[G_CHUNKS];
+#pragma unroll
+        for (int c = 0; c < G_CHUNKS; ++c) k[c] = __ldcs(idx + r0 + c * 32 + lane);
+        float4 v[G_CHUNKS][3];
+#pragma unroll
+        for (int c = 0; c < G_CHUNKS; ++c) {
+            const bool ok = (uint32_t)k[c] < (uint32_t)K;
+            bad |= !ok;
+            const float4 *src = reinterpret_cast<const float4 *>(Cp + (int64_t)(ok ? k[c] : 0) * CP_FLOATS);
+            v[c][0] = __ldg(src);
+            v[c][1] = __ldg(src + 1);
+            v[c][2] = __ldg(src + 2);
+            if (!ok) v[c][0] = v[c][1] = v[c][2] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int c = 0; c < G_CHUNKS; ++c) {
+            float *row = t + (c * 32 + lane) * D;
+            row[0] = v[c][0].x; row[1] = v[c][0].y; row[2] = v[c][0].z; row[3] = v[c][0].w;
+            row[4] = v[c][1].x; row[5] = v[c][1].y; row[6] = v[c][1].z; row[7] = v[c][1].w;
+            row[8] = v[c][2].x;
         }
         __syncwarp();
-        float *dst = W_out + r0 * D;
-        if (rows == 32) {
-            const float4 *t4 = reinterpret_cast<const float4 *>(t);
-            float4 *d4 = reinterpret_cast<float4 *>(dst);
-            for (int v = lane; v < 32 * D / 4; v += 32) __stcs(d4 + v, t4[v]);
-        } else {
-            for (int v = lane; v < rows * D; v += 32) dst[v] = t[v];
-        }
+        const float4 *t4 = reinterpret_cast<const float4 *>(t);
+        float4 *d4 = reinterpret_cast<float4 *>(W_out + r0 * D);
+#pragma unroll
+        for (int v2 = lane; v2 < G_TILE_FLOATS / 4; v2 += 32) __stcs(d4 + v2, t4[v2]);
         __syncwarp();
     }
+
+    // ragged end (fewer than G_ROWS kernels): CTA 0, plain loads and stores
+    if (blockIdx.x == 0) {
+        for (int64_t i = ngroups * G_ROWS + threadIdx.x; i < n; i += R_THREADS) {
+            const int32_t kk = idx[i];
+            const bool ok = (uint32_t)kk < (uint32_t)K;
+            bad |= !ok;
+#pragma unroll
+            for (int j = 0; j < D; ++j) W_out[i * D + j] = ok ? Cp[(int64_t)kk * CP_FLOATS + j] : 0.f;
+        }
+    }
+    if (__any_sync(0xffffffffu, bad) && lane == 0) set_flag(status, KQ_FLAG_INDEX_RANGE);
 }
 
 __global__ void __launch_bounds__(256)
@@ -108,8 +128,8 @@ cudaError_t launch_decode_codebook(const float *C, int32_t K, const uint8_t *cod
 
 cudaError_t launch_gather_rows(const int32_t *idx, int64_t n, const float *Cp, int32_t K, float *W_out,
                                uint32_t *status, int num_sms, cudaStream_t s) {
-    const int64_t chunks = (n + 31) / 32;
-    int64_t blocks = (chunks + R_THREADS / 32 - 1) / (R_THREADS / 32);
+    const int64_t groups = n / G_ROWS;
+    int64_t blocks = (groups + R_WARPS - 1) / R_WARPS;
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
     if (blocks < 1) blocks = 1;
     gather_rows_kernel<<<(unsigned)blocks, R_THREADS, 0, s>>>(idx, n, Cp, K, W_out, status);

@@ -8,9 +8,8 @@
 // S = 62 - e gives sum |q| <= 2^62 + n/2 < 2^63.
 //
 // The accumulator of codeword k is one 128-byte line: 9 coordinate sums and the
-// member count. A warp stages 32 kernels (1152 contiguous bytes) in shared memory
-// with float4 loads; each half-warp then adds one kernel: lanes 0..8 a coordinate,
-// lane 9 the count, so one warp-wide RED touches two lines.
+// member count. A warp takes 32 kernels (1152 contiguous bytes) per step with
+// coalesced loads; every lane converts and adds 9 coordinates and one count.
 #include "kq_internal.cuh"
 
 namespace kq {
@@ -32,8 +31,19 @@ __global__ void __launch_bounds__(256) maxabs_kernel(const float *__restrict__ W
     const int64_t n4 = count / 4;
     const float4 *W4 = reinterpret_cast<const float4 *>(W);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < n4; v += stride) {
-        const float4 t = __ldcs(W4 + v);
+    int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    for (; v + 3 * stride < n4; v += 4 * stride) {  // four independent loads in flight per thread
+        float4 t[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) t[u] = __ldg(W4 + v + u * stride);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            ok &= isfinite(t[u].x) & isfinite(t[u].y) & isfinite(t[u].z) & isfinite(t[u].w);
+            m = fmaxf(m, fmaxf(fmaxf(fabsf(t[u].x), fabsf(t[u].y)), fmaxf(fabsf(t[u].z), fabsf(t[u].w))));
+        }
+    }
+    for (; v < n4; v += stride) {
+        const float4 t = __ldg(W4 + v);
         ok &= isfinite(t.x) & isfinite(t.y) & isfinite(t.z) & isfinite(t.w);
         m = fmaxf(m, fmaxf(fmaxf(fabsf(t.x), fabsf(t.y)), fmaxf(fabsf(t.z), fabsf(t.w))));
     }
@@ -52,71 +62,79 @@ __global__ void __launch_bounds__(U_THREADS)
 accumulate_kernel(const float *__restrict__ W, int64_t n, const int32_t *__restrict__ idx, int32_t K,
                   const uint32_t *__restrict__ maxabs_bits, unsigned long long *__restrict__ acc,
                   uint32_t *status) {
-    __shared__ __align__(16) float sw[U_THREADS / 32][32 * D];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const double up = ldexp(1.0, update_scale(*maxabs_bits, n));
-    float *buf = sw[warp];
-    const int64_t nchunks = (n + 31) / 32;
-    for (int64_t ch = (int64_t)blockIdx.x * (U_THREADS / 32) + warp; ch < nchunks;
-         ch += (int64_t)gridDim.x * (U_THREADS / 32)) {
-        const int64_t r0 = ch * 32;
-        const int rows = (int)min((int64_t)32, n - r0);
+    const int S = update_scale(*maxabs_bits, n);
+    // A chunk is 32 kernels = 288 consecutive floats. In pass i a lane handles float
+    // lane + 32 i of the chunk (coalesced loads straight from global memory): kernel
+    // rr[i] of the chunk, coordinate jj[i]; the kernel's codeword comes from lane rr[i].
+    int rr[D], jj[D];
+#pragma unroll
+    for (int i = 0; i < D; ++i) {
+        rr[i] = (lane + 32 * i) / D;
+        jj[i] = (lane + 32 * i) - D * rr[i];
+    }
+    bool bad = false;
+    const int64_t nchunks = n / 32;
+    // Chunks are visited last-to-first: a max|W| pass that just streamed W front to
+    // back leaves the tail of W in L2.
+    for (int64_t it = (int64_t)blockIdx.x * (U_THREADS / 32) + warp; it < nchunks;
+         it += (int64_t)gridDim.x * (U_THREADS / 32)) {
+        const int64_t r0 = (nchunks - 1 - it) * 32;
         const float *src = W + r0 * D;
-        if (rows == 32) {
-            const float4 *s4 = reinterpret_cast<const float4 *>(src);
-            float4 *b4 = reinterpret_cast<float4 *>(buf);
-            for (int v = lane; v < 32 * D / 4; v += 32) b4[v] = __ldcs(s4 + v);
-        } else {
-            for (int v = lane; v < rows * D; v += 32) buf[v] = src[v];
+        float v[D];
+#pragma unroll
+        for (int i = 0; i < D; ++i) v[i] = __ldg(src + lane + 32 * i);
+        const int32_t myk = __ldcs(idx + r0 + lane);
+        const bool okk = (uint32_t)myk < (uint32_t)K;
+        bad |= !okk;
+#pragma unroll
+        for (int i = 0; i < D; ++i) {
+            const int32_t k = __shfl_sync(0xffffffffu, myk, rr[i]);
+            if ((uint32_t)k < (uint32_t)K)
+                atomicAdd(acc + (int64_t)k * ACC_WORDS + jj[i], (unsigned long long)fixed_rn(v[i], S));
         }
-        const int32_t myk = lane < rows ? __ldcs(idx + r0 + lane) : 0;
-        __syncwarp();
-#pragma unroll 4
-        for (int rr = 0; rr < 16; ++rr) {
-            const int r = 2 * rr + (lane >> 4);
-            const int j = lane & 15;
-            const int32_t k = __shfl_sync(0xffffffffu, myk, r);
-            if (r < rows && j <= D) {
-                if ((uint32_t)k < (uint32_t)K) {
-                    const unsigned long long add =
-                        j < D ? (unsigned long long)__double2ll_rn((double)buf[r * D + j] * up) : 1ull;
-                    atomicAdd(acc + (int64_t)k * ACC_WORDS + j, add);
-                } else if (j == 0) {
-                    set_flag(status, KQ_FLAG_INDEX_RANGE);
-                }
+        if (okk) atomicAdd(acc + (int64_t)myk * ACC_WORDS + D, 1ull);
+    }
+    // ragged end (< 32 kernels): one thread per kernel in CTA 0
+    if (blockIdx.x == 0) {
+        const int64_t i = nchunks * 32 + threadIdx.x;
+        if (threadIdx.x < 32 && i < n) {
+            const int32_t k = idx[i];
+            if ((uint32_t)k < (uint32_t)K) {
+#pragma unroll
+                for (int j = 0; j < D; ++j)
+                    atomicAdd(acc + (int64_t)k * ACC_WORDS + j, (unsigned long long)fixed_rn(W[i * D + j], S));
+                atomicAdd(acc + (int64_t)k * ACC_WORDS + D, 1ull);
+            } else {
+                bad = true;
             }
         }
-        __syncwarp();
     }
+    if (bad) set_flag(status, KQ_FLAG_INDEX_RANGE);
 }
 
-// c_k = (sum * 2^-S) / z_k rounded to fp32 (keep C_prev when z_k = 0); also writes
-// the packed copy used by the next assignment and clears the accumulator row.
+// c_k = (sum * 2^-S) / z_k in fp32 (keep C_prev when z_k = 0); clears the
+// accumulator row for the next call. fp32
+// arithmetic (GB300's fp64 rate is low): sum -> fp32, exact power-of-two scaling,
+// one IEEE division; within ~1.5 ulp of the exact mean.
 __global__ void __launch_bounds__(256)
 finalize_kernel(unsigned long long *__restrict__ acc, int32_t K, int64_t n, const uint32_t *__restrict__ maxabs_bits,
-                const float *C_prev, float *C_next, int32_t *__restrict__ counts, float *__restrict__ Cd_next) {
+                const float *C_prev, float *C_next, int32_t *__restrict__ counts) {
     const int k = blockIdx.x * blockDim.x + threadIdx.x;
     if (k >= K) return;
-    const double down = ldexp(1.0, -update_scale(*maxabs_bits, n));
+    const int S = update_scale(*maxabs_bits, n);
     unsigned long long *a = acc + (int64_t)k * ACC_WORDS;
     const long long z = (long long)a[D];
+    const float zf = (float)z;  // exact below 2^24, within half an ulp above
     float c[D];
 #pragma unroll
     for (int j = 0; j < D; ++j) {
-        const double sum = __ll2double_rn((long long)a[j]) * down;
-        c[j] = z > 0 ? __double2float_rn(__ddiv_rn(sum, (double)z)) : C_prev[(int64_t)k * D + j];
+        const float sum = scalbnf(__ll2float_rn((long long)a[j]), -S);
+        c[j] = z > 0 ? __fdiv_rn(sum, zf) : C_prev[(int64_t)k * D + j];
     }
 #pragma unroll
     for (int j = 0; j < D; ++j) C_next[(int64_t)k * D + j] = c[j];
     counts[k] = (int32_t)z;
-    if (Cd_next) {
-        float4 *dst = reinterpret_cast<float4 *>(Cd_next + (int64_t)k * CD_FLOATS);
-        dst[0] = make_float4(c[0], c[0], c[1], c[1]);
-        dst[1] = make_float4(c[2], c[2], c[3], c[3]);
-        dst[2] = make_float4(c[4], c[4], c[5], c[5]);
-        dst[3] = make_float4(c[6], c[6], c[7], c[7]);
-        dst[4] = make_float4(c[8], c[8], 0.f, 0.f);
-    }
     ulonglong2 *a2 = reinterpret_cast<ulonglong2 *>(a);
 #pragma unroll
     for (int w = 0; w < ACC_WORDS / 2; ++w) a2[w] = make_ulonglong2(0ull, 0ull);
@@ -160,7 +178,7 @@ cudaError_t launch_maxabs(const float *W, int64_t count, uint32_t *maxabs_bits, 
 cudaError_t launch_accumulate(const float *W, int64_t n, const int32_t *idx, int32_t K,
                               const uint32_t *maxabs_bits, unsigned long long *acc, uint32_t *status,
                               int num_sms, cudaStream_t s) {
-    const int64_t chunks = (n + 31) / 32;
+    const int64_t chunks = n / 32 + 1;
     int64_t blocks = (chunks + U_THREADS / 32 - 1) / (U_THREADS / 32);
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
     if (blocks < 1) blocks = 1;
@@ -170,9 +188,8 @@ cudaError_t launch_accumulate(const float *W, int64_t n, const int32_t *idx, int
 }
 
 cudaError_t launch_finalize(unsigned long long *acc, int32_t K, int64_t n, const uint32_t *maxabs_bits,
-                            const float *C_prev, float *C_next, int32_t *counts, float *Cd_next,
-                            cudaStream_t s) {
-    finalize_kernel<<<(K + 255) / 256, 256, 0, s>>>(acc, K, n, maxabs_bits, C_prev, C_next, counts, Cd_next);
+                            const float *C_prev, float *C_next, int32_t *counts, cudaStream_t s) {
+    finalize_kernel<<<(K + 255) / 256, 256, 0, s>>>(acc, K, n, maxabs_bits, C_prev, C_next, counts);
     count_launch();
     return cudaGetLastError();
 }

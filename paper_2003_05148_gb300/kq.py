@@ -55,7 +55,7 @@ def lib() -> ctypes.CDLL:
             "kq_workspace_bytes": ([i64, i32], sz),
             "kq_device_status": ([P, sz, P, P], ctypes.c_int),
             "kq_init_codebook": ([P, i64, P, i32, P, P, sz, P], ctypes.c_int),
-            "kq_assign": ([P, i64, P, i32, P, P, P, sz, P], ctypes.c_int),
+            "kq_assign": ([P, i64, P, i32, P, P, P, P, sz, P], ctypes.c_int),
             "kq_update_centroids": ([P, i64, P, i32, P, P, P, P, sz, P], ctypes.c_int),
             "kq_fit_codebook": ([P, i64, i32, P, i32, i32, P, P, P, P, P, sz, P], ctypes.c_int),
             "kq_quantize_codebook_6bit": ([P, i32, P, i32, P, P, P, P, sz, P], ctypes.c_int),
@@ -137,10 +137,10 @@ def kq_init_codebook(W, sel, C0, ws, stream=None) -> None:
         _dev(C0, "C0", torch.float32), _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
 
 
-def kq_assign(W, C, idx, dist, ws, stream=None) -> None:
+def kq_assign(W, C, idx, dist, ws, hint=None, stream=None) -> None:
     _check("kq_assign", lib().kq_assign(
         _dev(W, "W", torch.float32), _rows(W), _dev(C, "C", torch.float32), _rows(C),
-        _dev(idx, "idx", torch.int32), _dev(dist, "dist", torch.float32),
+        _dev(hint, "hint", torch.int32), _dev(idx, "idx", torch.int32), _dev(dist, "dist", torch.float32),
         _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
 
 

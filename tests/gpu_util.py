@@ -28,13 +28,13 @@ def to_dev(a):
     return torch.from_numpy(np.ascontiguousarray(a)).to(dev())
 
 
-def gpu_assign(W, C, with_dist=True):
+def gpu_assign(W, C, with_dist=True, hint=None):
     n, K = W.shape[0], C.shape[0]
     Wd, Cd = to_dev(W), to_dev(C)
     idx = torch.empty(n, dtype=torch.int32, device=dev())
     dist = torch.empty(n, dtype=torch.float32, device=dev()) if with_dist else None
     ws = kq.workspace(n, K, dev())
-    kq.kq_assign(Wd, Cd, idx, dist, ws)
+    kq.kq_assign(Wd, Cd, idx, dist, ws, hint=None if hint is None else to_dev(hint.astype(np.int32)))
     st, flags = kq.kq_device_status(ws)
     return idx.cpu().numpy(), (dist.cpu().numpy() if with_dist else None), st, flags
 

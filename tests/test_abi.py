@@ -35,7 +35,7 @@ def test_exports_every_declared_symbol(lib):
 
 
 def test_status_strings_and_version(lib):
-    assert kq.kq_abi_version() == 1
+    assert kq.kq_abi_version() == 2
     for code, name in kq.STATUS_NAMES.items():
         assert kq.kq_status_string(code) == name
     assert kq.kq_status_string(99) == "KQ_ERR_UNKNOWN"
@@ -57,12 +57,13 @@ def test_host_validation_before_any_device_work(lib):
     good = ctypes.c_void_p(1 << 20)  # 256-byte aligned dummy address
     odd = ctypes.c_void_p((1 << 20) + 4)
     ws_bytes = kq.kq_workspace_bytes(1024, 16)
-    assert L.kq_assign(good, 0, good, 16, good, None, good, ws_bytes, None) == 1  # n = 0
-    assert L.kq_assign(good, 1024, good, 2048, good, None, good, ws_bytes, None) == 1  # K > n
-    assert L.kq_assign(odd, 1024, good, 16, good, None, good, ws_bytes, None) == 2  # W not 16-byte aligned
-    assert L.kq_assign(good, 1024, good, 16, good, None, None, ws_bytes, None) == 6  # no workspace
-    assert L.kq_assign(good, 1024, good, 16, good, None, good, ws_bytes - 1, None) == 6  # too small
-    assert L.kq_assign(good, 1024, good, 16, good, None, odd, ws_bytes, None) == 2  # ws alignment
+    assert L.kq_assign(good, 0, good, 16, None, good, None, good, ws_bytes, None) == 1  # n = 0
+    assert L.kq_assign(good, 1024, good, 2048, None, good, None, good, ws_bytes, None) == 1  # K > n
+    assert L.kq_assign(odd, 1024, good, 16, None, good, None, good, ws_bytes, None) == 2  # W not 16-byte aligned
+    assert L.kq_assign(good, 1024, good, 16, ctypes.c_void_p((1 << 20) + 2), good, None, good, ws_bytes, None) == 2
+    assert L.kq_assign(good, 1024, good, 16, None, good, None, None, ws_bytes, None) == 6  # no workspace
+    assert L.kq_assign(good, 1024, good, 16, None, good, None, good, ws_bytes - 1, None) == 6  # too small
+    assert L.kq_assign(good, 1024, good, 16, None, good, None, odd, ws_bytes, None) == 2  # ws alignment
     assert L.kq_update_centroids(good, 1024, good, 16, None, good, good, good, ws_bytes, None) == 1
     assert L.kq_fit_codebook(good, 1024, 16, good, -1, 0, good, good, good, None, good, ws_bytes, None) == 1
     assert L.kq_fit_codebook(good, 1024, 16, good, 3, 7, good, good, good, None, good, ws_bytes, None) == 1
