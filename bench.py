@@ -38,7 +38,8 @@ METRIC = "kernel x codeword distance evals/s per Lloyd iteration"
 UNIT = "evals/s"
 SM_COUNT_NOMINAL = 152
 FP32_LANES_PER_SM = 128
-OPS_PER_PAIR = 18  # 9 FSUB + 9 FFMA on the FP32 pipe
+OPS_PER_PAIR = 9  # FP32-pipe lane ops per pair executed by the assign kernel: the 9 FFMA of its certified test
+DIRECT_OPS_PER_PAIR = 18  # the fp32 direct form: 9 FSUB + 9 FFMA
 WORKLOAD_CFG = 5
 
 
@@ -103,6 +104,20 @@ class ClockSampler:
         if not sm:
             return None
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def _ncu_traffic():
+    """Per-launch DRAM bytes (read + write) from the committed ncu summary, or {}."""
+    out = {}
+    try:
+        with open(os.path.join(ROOT, "profiles", "ncu_traffic.txt")) as f:
+            for line in f:
+                p = line.split()
+                if len(p) >= 2 and not line.startswith("#"):
+                    out[p[0]] = int(p[1])
+    except (OSError, ValueError):
+        return {}
+    return out
 
 
 def _smi_id(dev) -> str:
@@ -196,30 +211,33 @@ def run_kq(args, rank, world, local_rank):
     Wr = torch.empty_like(W)
     n_assign = T + 1
 
+    def pair():
+        return (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+
     def new_events():
-        return [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_assign)]
+        return {"assign": [pair() for _ in range(n_assign)], "update": [pair() for _ in range(n_assign)],
+                "reconstruct": [pair()]}
+
+    def timed(ev, name, i, fn):
+        if ev:
+            ev[name][i][0].record(stream)
+        fn()
+        if ev:
+            ev[name][i][1].record(stream)
 
     def step(ev=None):
-        """One pass of the hot path through the public entry points; `ev` brackets each assign."""
+        """One pass of the hot path through the public entry points; `ev` brackets the calls."""
         kq.kq_init_codebook(W, sel, Ca, ws)
         cur, nxt = Ca, Cb
-        for t in range(T):
-            if ev:
-                ev[t][0].record(stream)
+        for t in range(T + 1):
             # iterations after the first start from the previous assignment (as kq_fit_codebook does)
-            kq.kq_assign(W, cur, idx, None, ws, hint=idx if t > 0 else None)
-            if ev:
-                ev[t][1].record(stream)
-            kq.kq_update_centroids(W, idx, cur, nxt, counts, ws)
-            cur, nxt = nxt, cur
-        if ev:
-            ev[T][0].record(stream)
-        kq.kq_assign(W, cur, idx, None, ws, hint=idx if T > 0 else None)
-        if ev:
-            ev[T][1].record(stream)
-        kq.kq_update_centroids(W, idx, cur, nxt, counts, ws)  # cluster sizes of the final assignment
+            timed(ev, "assign", t, lambda: kq.kq_assign(W, cur, idx, None, ws, hint=idx if t > 0 else None))
+            # after the last assignment the update gives the cluster sizes the quantiser weighs by
+            timed(ev, "update", t, lambda: kq.kq_update_centroids(W, idx, cur, nxt, counts, ws))
+            if t < T:
+                cur, nxt = nxt, cur
         kq.kq_quantize_codebook_6bit(cur, counts, 100, levels, codes, None, ws)
-        kq.kq_reconstruct(idx, None, codes, levels, Wr, ws, K=K)
+        timed(ev, "reconstruct", 0, lambda: kq.kq_reconstruct(idx, None, codes, levels, Wr, ws, K=K))
 
     for _ in range(args.warmup):
         step()
@@ -244,7 +262,8 @@ def run_kq(args, rank, world, local_rank):
         barrier()
     launches = kq.kq_kernel_launches() - launches0
     ms_total = e0.elapsed_time(e1)
-    assign_ms = [a.elapsed_time(b) for ev in evs for a, b in ev]
+    call_ms = {name: [a.elapsed_time(b) for ev in evs for a, b in ev[name]] for name in evs[0]}
+    assign_ms = call_ms["assign"]
     t_local = torch.tensor([ms_total], dtype=torch.float64, device=dev)
     if world > 1:
         dist.all_reduce(t_local, op=dist.ReduceOp.MAX)
@@ -305,13 +324,33 @@ def run_kq(args, rank, world, local_rank):
     peak_tops = sms * FP32_LANES_PER_SM * max_mhz * 1e6 / 1e12
     t_assign = statistics.mean(assign_ms) / 1e3
     achieved = OPS_PER_PAIR * n * K / t_assign / 1e12
+    traffic = _ncu_traffic()
     roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s", "frac": achieved / peak_tops,
-                "traffic": None, "kernel": "assign_kernel",
+                "traffic": traffic.get("assign_kernel"), "kernel": "assign_kernel",
                 "peak_basis": f"{sms} SMs x {FP32_LANES_PER_SM} FP32 lanes x {max_mhz:.0f} MHz (max SM clock); "
-                              f"op = one FP32-pipe lane op, {OPS_PER_PAIR} per pair (9 FSUB + 9 FFMA)",
+                              f"op = one FP32-pipe lane op; {OPS_PER_PAIR} per pair (the FFMA of the certified "
+                              f"expanded-form test every pair gets; the exact re-evaluations of the few candidate "
+                              f"pairs are not counted)",
+                "direct_form_equivalent": {"achieved": DIRECT_OPS_PER_PAIR * n * K / t_assign / 1e12,
+                                           "note": "18 ops/pair: the rate a direct-form kernel would need"},
                 "assign_ms_mean": 1e3 * t_assign, "assign_launches": len(assign_ms)}
     if clk:
         roofline["frac_at_sampled_clock"] = achieved / (sms * FP32_LANES_PER_SM * clk["sm_mhz"] * 1e6 / 1e12)
+    hbm = float(peaks.get("hbm_gbs", 6776.3))
+
+    def hbm_roofline(name, bytes_per_call, ms_list, note):
+        t = statistics.mean(ms_list) / 1e3
+        a = bytes_per_call / t / 1e9
+        return {"bound": "hbm", "achieved": a, "peak": hbm, "unit": "GB/s", "frac": a / hbm,
+                "traffic": traffic.get(name), "calls": len(ms_list), "us_mean": 1e6 * t,
+                "algorithmic_bytes": int(bytes_per_call), "note": note}
+
+    upd_bytes = n * (36 + 4) + K * (36 + 36 + 4)
+    rec_bytes = n * (4 + 36) + 9 * K + 256
+    roofline_update = hbm_roofline("kq_update_centroids", upd_bytes, call_ms["update"],
+                                   "whole kq_update_centroids call (prepare + accumulate + fallback check + finalize)")
+    roofline_reconstruct = hbm_roofline("kq_reconstruct", rec_bytes, call_ms["reconstruct"],
+                                        "whole kq_reconstruct call, K+C (decode codes + gather)")
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms_max / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
@@ -321,6 +360,8 @@ def run_kq(args, rank, world, local_rank):
                    "l2": "inputs larger than L2 (W is 151 MB, L2 129 MB): no flush",
                    "parallelism": f"replicas x{world}"},
         "roofline": roofline,
+        "roofline_update": roofline_update,
+        "roofline_reconstruct": roofline_reconstruct,
         "gpu_launches": int(launches),
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                 "steps": e2e_steps, "api": "kq_init_codebook + kq_fit_codebook + kq_quantize_codebook_6bit + "
@@ -368,8 +409,11 @@ def run_only(args):
     codes = torch.empty(K, 9, dtype=torch.uint8, device=dev)
     kq.kq_quantize_codebook_6bit(C2, counts, 100, levels, codes, None, ws)
     Wr = torch.empty_like(W)
+    idx2 = torch.empty_like(idx)
     calls = {
-        "assign": lambda: kq.kq_assign(W, C, idx, None, ws),
+        # --hint: one Lloyd step later, warm-started from the previous assignment (as in a fit)
+        "assign": (lambda: kq.kq_assign(W, C2, idx2, None, ws, hint=idx)) if args.hint
+        else (lambda: kq.kq_assign(W, C, idx, None, ws)),
         "update": lambda: kq.kq_update_centroids(W, idx, C, C2, counts, ws),
         "quantize": lambda: kq.kq_quantize_codebook_6bit(C2, counts, 100, levels, codes, None, ws),
         "reconstruct": lambda: kq.kq_reconstruct(idx, None, codes, levels, Wr, ws, K=K),
@@ -407,6 +451,7 @@ def main():
     ap.add_argument("--n", type=int, default=4194304)
     ap.add_argument("--K", type=int, default=65536)
     ap.add_argument("--reps", type=int, default=3)
+    ap.add_argument("--hint", action="store_true", help="with --only assign: warm start as in a fit")
     args = ap.parse_args()
     if args.only:
         run_only(args)

@@ -62,6 +62,7 @@ struct Ws {
     unsigned long long *part;
     double *blocksum;
     float *cbuf0, *cbuf1, *cp;
+    unsigned long long *cq;
 };
 
 Ws carve(void *ws, int64_t n, int32_t K) {
@@ -76,22 +77,16 @@ Ws carve(void *ws, int64_t n, int32_t K) {
     w.cbuf0 = reinterpret_cast<float *>(b + L.cbuf0);
     w.cbuf1 = reinterpret_cast<float *>(b + L.cbuf1);
     w.cp = reinterpret_cast<float *>(b + L.cp);
+    w.cq = reinterpret_cast<unsigned long long *>(b + L.cq);
     return w;
 }
 
-// Update step on prepared state: accumulate into the (zeroed) accumulators and
-// finalise; the finalise leaves the accumulators zeroed again.
-kq_status run_update(const float *W, int64_t n, const int32_t *idx, int32_t K, const float *C_prev, float *C_next,
-                     int32_t *counts, const Ws &w, int sms, cudaStream_t s) {
-    KQ_TRY(launch_accumulate(W, n, idx, K, &w.hdr->maxabs_bits, w.acc, &w.hdr->status, sms, s));
-    KQ_TRY(launch_finalize(w.acc, K, n, &w.hdr->maxabs_bits, C_prev, C_next, counts, s));
-    return KQ_OK;
-}
-
-kq_status prepare_update(const float *W, int64_t n, int32_t K, const Ws &w, int sms, cudaStream_t s) {
-    KQ_TRY(cudaMemsetAsync(&w.hdr->maxabs_bits, 0, sizeof(uint32_t), s));
-    KQ_TRY(launch_maxabs(W, n * D, &w.hdr->maxabs_bits, &w.hdr->status, sms, s));
-    KQ_TRY(cudaMemsetAsync(w.acc, 0, (size_t)K * ACC_WORDS * sizeof(unsigned long long), s));
+// Update step with the scale chosen once per fit from max|W| (exact mode); the
+// finalise leaves the accumulators zeroed again.
+kq_status run_update_exact(const float *W, int64_t n, const int32_t *idx, int32_t K, const float *C_prev,
+                           float *C_next, int32_t *counts, const Ws &w, int sms, cudaStream_t s) {
+    KQ_TRY(launch_accumulate(W, n, idx, K, w.hdr, w.acc, false, sms, s));
+    KQ_TRY(launch_finalize(w.acc, K, w.hdr, C_prev, C_next, counts, s));
     return KQ_OK;
 }
 
@@ -183,8 +178,12 @@ kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int
     if ((st = num_sms(&sms)) != KQ_OK) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     Ws w = carve(ws, n, K);
-    if ((st = prepare_update(W, n, K, w, sms, s)) != KQ_OK) return st;
-    return run_update(W, n, idx, K, C_prev, C_next, counts, w, sms, s);
+    // scale guessed from C_prev, checked on every value, exact fallback if violated
+    KQ_TRY(launch_update_prepare(C_prev, K, w.acc, w.hdr, true, s));
+    KQ_TRY(launch_accumulate(W, n, idx, K, w.hdr, w.acc, true, sms, s));
+    KQ_TRY(launch_update_fallback(W, n, idx, K, w.hdr, w.acc, sms, s));
+    KQ_TRY(launch_finalize(w.acc, K, w.hdr, C_prev, C_next, counts, s));
+    return KQ_OK;
 }
 
 kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_init, int32_t iters, int32_t flags,
@@ -203,7 +202,8 @@ kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_i
     Ws w = carve(ws, n, K);
     const size_t cbytes = (size_t)K * D * sizeof(float);
 
-    if ((st = prepare_update(W, n, K, w, sms, s)) != KQ_OK) return st;
+    KQ_TRY(launch_update_prepare(nullptr, K, w.acc, w.hdr, false, s));
+    KQ_TRY(launch_maxabs(W, n * D, &w.hdr->maxabs_bits, &w.hdr->status, sms, s));  // the scale, once per fit
     KQ_TRY(cudaMemcpyAsync(w.cbuf0, C_init, cbytes, cudaMemcpyDeviceToDevice, s));
     float *cur = w.cbuf0, *nxt = w.cbuf1;
     int nb = 0;
@@ -213,7 +213,7 @@ kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_i
         KQ_TRY(launch_assign(W, n, w.cd, cur, K, t > 0 ? idx : nullptr, idx, nullptr, w.blocksum, &nb, w.part, w.hdr,
                              sms, s));
         if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
-        if ((st = run_update(W, n, idx, K, cur, nxt, counts, w, sms, s)) != KQ_OK) return st;
+        if ((st = run_update_exact(W, n, idx, K, cur, nxt, counts, w, sms, s)) != KQ_OK) return st;
         float *tmp = cur;
         cur = nxt;
         nxt = tmp;
@@ -255,8 +255,9 @@ kq_status kq_reconstruct(const int32_t *idx, int64_t n, const float *C, int32_t 
     if ((st = num_sms(&sms)) != KQ_OK) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     Ws w = carve(ws, n, K);
-    KQ_TRY(launch_decode_codebook(C, K, codes, levels, w.cp, &w.hdr->status, s));
-    KQ_TRY(launch_gather_rows(idx, n, w.cp, K, W_out, &w.hdr->status, sms, s));
+    KQ_TRY(launch_decode_codebook(C, K, codes, w.cp, w.cq, &w.hdr->status, s));
+    KQ_TRY(launch_gather_rows(idx, n, codes ? nullptr : w.cp, codes ? w.cq : nullptr, levels, K, W_out,
+                              &w.hdr->status, sms, s));
     return KQ_OK;
 }
 

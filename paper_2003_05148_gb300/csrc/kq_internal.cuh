@@ -30,13 +30,17 @@ struct Header {
     uint32_t maxv_w;        // level fit: max |v| over weighted scalars (fp32 bits)
     uint32_t pad1;
     uint32_t cb_cmax, cb_hmax, cb_qmax, pad2;  // assign filter: codebook bounds (fp32 bits, see kq_assign.cu)
+    uint32_t upd_bound;     // update: bound B on |W| the fixed-point scale was chosen for (fp32 bits)
+    uint32_t upd_violation; // update: a |w| > B was seen (the exact fallback must run)
+    int32_t upd_scale;      // update: the scale exponent S the accumulators hold
+    uint32_t pad3;
     unsigned long long wtotal;          // level fit: sum of weights
     unsigned long long lacc[3][LEVELS][2];  // level fit: (weight sum, fixed-point sum) per level
 };
 static_assert(sizeof(Header) <= 4096, "header too large");
 
 struct WsLayout {
-    size_t cd, acc, part, blocksum, cbuf0, cbuf1, cp, total;
+    size_t cd, acc, part, blocksum, cbuf0, cbuf1, cp, cq, total;
 };
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -52,6 +56,7 @@ inline WsLayout ws_layout(int64_t n, int32_t K) {
     L.cbuf0 = off;    off = align_up(off + (size_t)K * D * 4, 256);
     L.cbuf1 = off;    off = align_up(off + (size_t)K * D * 4, 256);
     L.cp = off;       off = align_up(off + (size_t)K * CP_FLOATS * 4, 256);
+    L.cq = off;       off = align_up(off + (size_t)K * 8, 256);
     L.total = off;
     return L;
 }
@@ -133,6 +138,41 @@ __device__ __forceinline__ bool finite9(const float *v) {
     return ok;
 }
 
+// Bounded grid barrier for cooperative launches (all CTAs co-resident). The
+// arrival counter hdr->barrier only grows (it must be zero at launch); barrier
+// number `epoch` completes at epoch * nblocks arrivals. A wait that runs ~2 s sets
+// KQ_FLAG_TIMEOUT and hdr->abort; every CTA then returns false and exits.
+constexpr long long BARRIER_SPIN_LIMIT = 20000000;  // ~2 s of 100 ns naps
+__device__ __forceinline__ bool grid_barrier(Header *h, unsigned nblocks, unsigned &epoch) {
+    __shared__ int s_ok;
+    __syncthreads();
+    ++epoch;
+    if (threadIdx.x == 0) {
+        __threadfence();
+        atomicAdd(&h->barrier, 1u);
+        const unsigned target = epoch * nblocks;
+        int ok = 1;
+        for (long long spin = 0;; ++spin) {
+            if (*(volatile unsigned *)&h->barrier >= target) break;
+            if (*(volatile unsigned *)&h->abort) {
+                ok = 0;
+                break;
+            }
+            if (spin > BARRIER_SPIN_LIMIT) {
+                atomicExch(&h->abort, 1u);
+                set_flag(&h->status, KQ_FLAG_TIMEOUT);
+                ok = 0;
+                break;
+            }
+            __nanosleep(100);
+        }
+        __threadfence();
+        s_ok = ok;
+    }
+    __syncthreads();
+    return s_ok != 0;
+}
+
 // Process-wide count of kernels libkq has launched (kq_kernel_launches()).
 void count_launch(int kernels = 1);
 
@@ -146,23 +186,32 @@ cudaError_t launch_assign(const float *W, int64_t n, const float *Cd, const floa
                           Header *hdr, int num_sms, cudaStream_t s);
 cudaError_t launch_sum_blocks(const double *blocksum, int nblocks, double *out, cudaStream_t s);
 
+// Update step. Two ways to pick the fixed-point scale: `exact` takes B = max|W|
+// (launch_maxabs first, as the fit does once); otherwise B is a guess from
+// max|C_prev| checked against every value, with an exact fallback pass.
 cudaError_t launch_maxabs(const float *W, int64_t count, uint32_t *maxabs_bits, uint32_t *status, int num_sms,
                           cudaStream_t s);
-cudaError_t launch_accumulate(const float *W, int64_t n, const int32_t *idx, int32_t K,
-                              const uint32_t *maxabs_bits, unsigned long long *acc, uint32_t *status,
-                              int num_sms, cudaStream_t s);
+cudaError_t launch_update_prepare(const float *C_prev, int32_t K, unsigned long long *acc, Header *hdr,
+                                  bool guess_from_codebook, cudaStream_t s);
+cudaError_t launch_accumulate(const float *W, int64_t n, const int32_t *idx, int32_t K, Header *hdr,
+                              unsigned long long *acc, bool guess, int num_sms, cudaStream_t s);
+cudaError_t launch_update_fallback(const float *W, int64_t n, const int32_t *idx, int32_t K, Header *hdr,
+                                   unsigned long long *acc, int num_sms, cudaStream_t s);
 cudaError_t launch_histogram(const int32_t *idx, int64_t n, int32_t K, int32_t *counts, uint32_t *status,
                              int num_sms, cudaStream_t s);
-cudaError_t launch_finalize(unsigned long long *acc, int32_t K, int64_t n, const uint32_t *maxabs_bits,
-                            const float *C_prev, float *C_next, int32_t *counts, cudaStream_t s);
+cudaError_t launch_finalize(unsigned long long *acc, int32_t K, const Header *hdr, const float *C_prev,
+                            float *C_next, int32_t *counts, cudaStream_t s);
 
 cudaError_t launch_level_fit(const float *C, int32_t K, const int32_t *counts, int32_t max_iters, float *levels,
                              uint8_t *codes, int32_t *iters_run, Header *hdr, int num_sms, cudaStream_t s);
 
-cudaError_t launch_decode_codebook(const float *C, int32_t K, const uint8_t *codes, const float *levels,
-                                   float *Cp, uint32_t *status, cudaStream_t s);
-cudaError_t launch_gather_rows(const int32_t *idx, int64_t n, const float *Cp, int32_t K, float *W_out,
-                               uint32_t *status, int num_sms, cudaStream_t s);
+// Recovery. K only: C is re-laid as 48-byte rows (Cp) and gathered. K+C: the
+// codes are packed 9 x 6 bits per codeword (Cq, 8 bytes) and decoded on the fly.
+cudaError_t launch_decode_codebook(const float *C, int32_t K, const uint8_t *codes, float *Cp,
+                                   unsigned long long *Cq, uint32_t *status, cudaStream_t s);
+cudaError_t launch_gather_rows(const int32_t *idx, int64_t n, const float *Cp, const unsigned long long *Cq,
+                               const float *levels, int32_t K, float *W_out, uint32_t *status, int num_sms,
+                               cudaStream_t s);
 cudaError_t launch_init_codebook(const float *W, int64_t n, const int64_t *sel, int32_t K, float *C0,
                                  uint32_t *status, cudaStream_t s);
 

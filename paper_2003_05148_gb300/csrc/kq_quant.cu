@@ -18,8 +18,6 @@
 namespace kq {
 
 constexpr int Q_THREADS = 512;
-constexpr long long SPIN_LIMIT = 20000000;  // ~2 s of 100 ns naps, then give up
-
 struct LevelArgs {
     const float *C;
     int32_t K;
@@ -30,39 +28,6 @@ struct LevelArgs {
     int32_t *iters_run;
     Header *hdr;
 };
-
-// Bounded grid barrier for a cooperative launch (all CTAs co-resident). The
-// arrival counter only grows; barrier number `epoch` completes at epoch*nblocks.
-// Returns false when some CTA gave up (timeout): every CTA then exits.
-__device__ bool grid_barrier(Header *h, unsigned nblocks, unsigned &epoch) {
-    __shared__ int s_ok;
-    __syncthreads();
-    ++epoch;
-    if (threadIdx.x == 0) {
-        __threadfence();
-        atomicAdd(&h->barrier, 1u);
-        const unsigned target = epoch * nblocks;
-        int ok = 1;
-        for (long long spin = 0;; ++spin) {
-            if (*(volatile unsigned *)&h->barrier >= target) break;
-            if (*(volatile unsigned *)&h->abort) {
-                ok = 0;
-                break;
-            }
-            if (spin > SPIN_LIMIT) {
-                atomicExch(&h->abort, 1u);
-                set_flag(&h->status, KQ_FLAG_TIMEOUT);
-                ok = 0;
-                break;
-            }
-            __nanosleep(100);
-        }
-        __threadfence();
-        s_ok = ok;
-    }
-    __syncthreads();
-    return s_ok != 0;
-}
 
 // Nearest of the 64 levels by fp32 |v - level|, lower index on ties (Sec. 3.2 encode).
 __device__ __forceinline__ int nearest_level(float v, const float *L) {

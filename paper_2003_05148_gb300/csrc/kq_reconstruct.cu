@@ -13,29 +13,32 @@ namespace kq {
 
 constexpr int R_THREADS = 256;
 
+// K only: C into 48-byte rows (Cp). K+C: the 9 codes of a codeword into one
+// 64-bit word (Cq), 7 bits each so an out-of-range code (>= 64) stays visible and
+// decodes to 0.
 __global__ void __launch_bounds__(256)
 decode_codebook_kernel(const float *__restrict__ C, int32_t K, const uint8_t *__restrict__ codes,
-                       const float *__restrict__ levels, float *__restrict__ Cp, uint32_t *status) {
-    __shared__ float sl[LEVELS];
-    if (codes && threadIdx.x < LEVELS) sl[threadIdx.x] = levels[threadIdx.x];
-    __syncthreads();
+                       float *__restrict__ Cp, unsigned long long *__restrict__ Cq, uint32_t *status) {
     const int k = blockIdx.x * blockDim.x + threadIdx.x;
     if (k >= K) return;
-    float c[CP_FLOATS];
-    bool bad = false;
+    if (codes) {
+        unsigned long long q = 0;
+        bool bad = false;
 #pragma unroll
-    for (int j = 0; j < D; ++j) {
-        if (codes) {
-            const uint8_t q = codes[(int64_t)k * D + j];
-            bad |= q >= LEVELS;
-            c[j] = q < LEVELS ? sl[q] : 0.f;
-        } else {
-            c[j] = C[(int64_t)k * D + j];
+        for (int j = 0; j < D; ++j) {
+            const uint32_t c = codes[(int64_t)k * D + j];
+            bad |= c >= LEVELS;
+            q |= (unsigned long long)(c < LEVELS ? c : LEVELS) << (7 * j);
         }
+        if (bad) set_flag(status, KQ_FLAG_CODE_RANGE);
+        Cq[k] = q;
+        return;
     }
+    float c[CP_FLOATS];
+#pragma unroll
+    for (int j = 0; j < D; ++j) c[j] = C[(int64_t)k * D + j];
 #pragma unroll
     for (int j = D; j < CP_FLOATS; ++j) c[j] = 0.f;
-    if (bad) set_flag(status, KQ_FLAG_CODE_RANGE);
     float4 *dst = reinterpret_cast<float4 *>(Cp + (int64_t)k * CP_FLOATS);
     dst[0] = make_float4(c[0], c[1], c[2], c[3]);
     dst[1] = make_float4(c[4], c[5], c[6], c[7]);
@@ -48,6 +51,7 @@ decode_codebook_kernel(const float *__restrict__ C, int32_t K, const uint8_t *__
 // per-warp shared tile (kernel i at float offset 9i, conflict-free), which the warp
 // then writes out with coalesced streaming float4 stores.
 constexpr int G_CHUNKS = 2;
+constexpr unsigned long long ALL_CODES_OUT_OF_RANGE = 0x4081020408102040ull;  // nine 7-bit fields = 64
 constexpr int G_ROWS = 32 * G_CHUNKS;
 constexpr int G_TILE_FLOATS = G_ROWS * D;
 constexpr int R_WARPS = R_THREADS / 32;
@@ -104,6 +108,72 @@ gather_rows_kernel(const int32_t *__restrict__ idx, int64_t n, const float *__re
     if (__any_sync(0xffffffffu, bad) && lane == 0) set_flag(status, KQ_FLAG_INDEX_RANGE);
 }
 
+// K+C recovery. A warp owns 32 consecutive kernels (1152 output bytes = 72 float4).
+// Each lane fetches the packed codes of its own kernel (one 8-byte word, instead of
+// a 36-byte row), then produces output float4 number lane, lane + 32 and (lanes
+// 0-7) lane + 64 directly: the at most two kernels a float4 spans send their code
+// words by shuffle, and every code is looked up in a level table replicated across
+// the 32 shared-memory banks (level l for lane L at [l][L]: no bank conflicts). No
+// staging tile; the stores are coalesced streaming float4 stores.
+__global__ void __launch_bounds__(R_THREADS)
+gather_codes_kernel(const int32_t *__restrict__ idx, int64_t n, const unsigned long long *__restrict__ Cq,
+                    const float *__restrict__ levels, int32_t K, float *__restrict__ W_out, uint32_t *status) {
+    __shared__ float lv[LEVELS + 1][32];  // row LEVELS decodes out-of-range codes to 0
+    for (int e = threadIdx.x; e < (LEVELS + 1) * 32; e += R_THREADS)
+        lv[e / 32][e % 32] = e / 32 < LEVELS ? levels[e / 32] : 0.f;
+    __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // slot s: float4 v = lane + 32 s of the chunk; its first element is coordinate
+    // j0 of kernel ra, elements e < split belong to ra, the rest to ra + 1
+    int ra[3], j0[3], split[3];
+#pragma unroll
+    for (int s = 0; s < 3; ++s) {
+        const int v = min(lane + 32 * s, 32 * D / 4 - 1);
+        ra[s] = (4 * v) / D;
+        j0[s] = 4 * v - D * ra[s];
+        split[s] = D - j0[s];
+    }
+    bool bad = false;
+    const int64_t nch = n / 32;
+    for (int64_t ch = (int64_t)blockIdx.x * R_WARPS + warp; ch < nch; ch += (int64_t)gridDim.x * R_WARPS) {
+        const int64_t r0 = ch * 32;
+        const int32_t k = __ldcs(idx + r0 + lane);
+        const bool ok = (uint32_t)k < (uint32_t)K;
+        bad |= !ok;
+        const unsigned long long q = ok ? __ldg(Cq + k) : ALL_CODES_OUT_OF_RANGE;
+        const uint32_t qlo = (uint32_t)q, qhi = (uint32_t)(q >> 32);
+        float4 *d4 = reinterpret_cast<float4 *>(W_out + r0 * D);
+#pragma unroll
+        for (int s = 0; s < 3; ++s) {
+            const int rb = min(ra[s] + 1, 31);
+            const unsigned long long qa = ((unsigned long long)__shfl_sync(0xffffffffu, qhi, ra[s]) << 32) |
+                                          __shfl_sync(0xffffffffu, qlo, ra[s]);
+            const unsigned long long qb = ((unsigned long long)__shfl_sync(0xffffffffu, qhi, rb) << 32) |
+                                          __shfl_sync(0xffffffffu, qlo, rb);
+            float r[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const bool first = e < split[s];
+                const int j = first ? j0[s] + e : e - split[s];
+                r[e] = lv[((first ? qa : qb) >> (7 * j)) & 127u][lane];
+            }
+            if (s < 2 || lane < 32 * D / 4 - 64) __stcs(d4 + lane + 32 * s, make_float4(r[0], r[1], r[2], r[3]));
+        }
+    }
+    // ragged end (< 32 kernels): CTA 0, plain loads and stores
+    if (blockIdx.x == 0) {
+        for (int64_t i = nch * 32 + threadIdx.x; i < n; i += R_THREADS) {
+            const int32_t kk = idx[i];
+            const bool ok = (uint32_t)kk < (uint32_t)K;
+            bad |= !ok;
+            const unsigned long long q = ok ? Cq[kk] : ALL_CODES_OUT_OF_RANGE;
+#pragma unroll
+            for (int j = 0; j < D; ++j) W_out[i * D + j] = lv[(q >> (7 * j)) & 127u][0];
+        }
+    }
+    if (__any_sync(0xffffffffu, bad) && lane == 0) set_flag(status, KQ_FLAG_INDEX_RANGE);
+}
+
 __global__ void __launch_bounds__(256)
 init_codebook_kernel(const float *__restrict__ W, int64_t n, const int64_t *__restrict__ sel, int32_t K,
                      float *__restrict__ C0, uint32_t *status) {
@@ -119,15 +189,24 @@ init_codebook_kernel(const float *__restrict__ W, int64_t n, const int64_t *__re
     }
 }
 
-cudaError_t launch_decode_codebook(const float *C, int32_t K, const uint8_t *codes, const float *levels,
-                                   float *Cp, uint32_t *status, cudaStream_t s) {
-    decode_codebook_kernel<<<(K + 255) / 256, 256, 0, s>>>(C, K, codes, levels, Cp, status);
+cudaError_t launch_decode_codebook(const float *C, int32_t K, const uint8_t *codes, float *Cp,
+                                   unsigned long long *Cq, uint32_t *status, cudaStream_t s) {
+    decode_codebook_kernel<<<(K + 255) / 256, 256, 0, s>>>(C, K, codes, Cp, Cq, status);
     count_launch();
     return cudaGetLastError();
 }
 
-cudaError_t launch_gather_rows(const int32_t *idx, int64_t n, const float *Cp, int32_t K, float *W_out,
-                               uint32_t *status, int num_sms, cudaStream_t s) {
+cudaError_t launch_gather_rows(const int32_t *idx, int64_t n, const float *Cp, const unsigned long long *Cq,
+                               const float *levels, int32_t K, float *W_out, uint32_t *status, int num_sms,
+                               cudaStream_t s) {
+    if (Cq) {
+        int64_t blocks = (n / 32 + R_WARPS - 1) / R_WARPS;
+        if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
+        if (blocks < 1) blocks = 1;
+        gather_codes_kernel<<<(unsigned)blocks, R_THREADS, 0, s>>>(idx, n, Cq, levels, K, W_out, status);
+        count_launch();
+        return cudaGetLastError();
+    }
     const int64_t groups = n / G_ROWS;
     int64_t blocks = (groups + R_WARPS - 1) / R_WARPS;
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;

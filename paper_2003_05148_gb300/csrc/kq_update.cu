@@ -1,27 +1,106 @@
 // kq_update.cu -- update step of KQ's k-means (Sec. 3.1, Eq. 1): c_k = mean of S_k.
 //
 // Deterministic without floating-point atomics: every coordinate of every kernel
-// is converted to an int64 fixed-point number q = rint(v * 2^S) and added with
-// integer atomics (red.global.add.u64), which are associative, so the sums do not
-// depend on the order the hardware applies them in. S is chosen from max |W| and
-// n so that no sum can overflow: with n*max|W| = f * 2^e (f in [0.5, 1)),
-// S = 62 - e gives sum |q| <= 2^62 + n/2 < 2^63.
+// is converted to an int64 fixed-point number q = rint(v * 2^S) (integer
+// operations only, see fixed_rn) and added with integer atomics
+// (red.global.add.u64), which are associative, so the sums do not depend on the
+// order the hardware applies them in. With a bound B >= |v| for every value and
+// n * B = f * 2^e (f in [0.5, 1)), S = 62 - e keeps every sum below 2^63.
+//
+// Where B comes from:
+//  - exact: B = max|W| from a pass over W (kq_fit_codebook does this once per fit);
+//  - guess (kq_update_centroids): B = 256 * max|C_prev|, read from the small
+//    codebook instead of W. Every value is checked against B while it is added; if
+//    any finite |w| > B, a cooperative fallback pass clears the sums, takes max|W|
+//    and accumulates again with that exact bound. Either way the sums are exact
+//    fixed-point sums at the scale recorded in the workspace header.
 //
 // The accumulator of codeword k is one 128-byte line: 9 coordinate sums and the
-// member count. A warp takes 32 kernels (1152 contiguous bytes) per step with
-// coalesced loads; every lane converts and adds 9 coordinates and one count.
+// member count (layout of the adds: see accumulate_rows). The throughput limit is
+// the L2's integer-atomic units (about three 32-byte sector operations per kernel)
+// and the L1's handling of the RED requests, not HBM.
 #include "kq_internal.cuh"
 
 namespace kq {
 
 constexpr int U_THREADS = 256;
+constexpr int SCALE_INVALID = -100000;
+constexpr float GUESS_FACTOR = 256.f;
+constexpr float F32_MAX = 3.402823466e38f;
 
-__device__ __forceinline__ int update_scale(uint32_t maxabs_bits, int64_t n) {
-    const float M = __uint_as_float(maxabs_bits);
-    if (!(M > 0.f) || isinf(M)) return 0;
+// Scale exponent for n values bounded by B; SCALE_INVALID when B is zero,
+// negative, infinite or NaN.
+__device__ __forceinline__ int update_scale(float B, int64_t n) {
+    if (!(B > 0.f) || !(B <= F32_MAX)) return SCALE_INVALID;
     int e;
-    frexp((double)n * (double)M, &e);
+    frexp((double)n * (double)B, &e);
     return 62 - e;
+}
+
+// Adds the kernels of 32-kernel chunks it0, it0 + step, ... into the accumulators
+// at scale S. In pass i a lane handles float lane + 32 i of the chunk (coalesced
+// loads straight from global memory): kernel rr[i] of the chunk, coordinate jj[i];
+// that kernel's codeword comes from lane rr[i] by shuffle. All 32 lanes add in
+// every pass; each lane also adds one count.
+// With `check`, a finite value above B sets the violation flag (the exact fallback
+// pass then redoes the sums).
+__device__ __forceinline__ void accumulate_rows(const float *__restrict__ W, int64_t n, const int32_t *__restrict__ idx,
+                                                int32_t K, int S, float B, bool check, unsigned long long *acc,
+                                                Header *hdr, int64_t it0, int64_t step, bool do_tail) {
+    const int lane = threadIdx.x & 31;
+    int rr[D], jj[D];
+#pragma unroll
+    for (int i = 0; i < D; ++i) {
+        rr[i] = (lane + 32 * i) / D;
+        jj[i] = (lane + 32 * i) - D * rr[i];
+    }
+    bool bad_idx = false, too_big = false, nonfinite = false;
+    const int64_t nchunks = n / 32;
+    // Chunks are visited last-to-first: a max|W| pass that just streamed W front to
+    // back leaves the tail of W in L2.
+    for (int64_t it = it0; it < nchunks; it += step) {
+        const int64_t r0 = (nchunks - 1 - it) * 32;
+        const float *src = W + r0 * D;
+        float v[D];
+#pragma unroll
+        for (int i = 0; i < D; ++i) v[i] = __ldg(src + lane + 32 * i);
+        const int32_t myk = __ldcs(idx + r0 + lane);
+        const bool okk = (uint32_t)myk < (uint32_t)K;
+        bad_idx |= !okk;
+#pragma unroll
+        for (int i = 0; i < D; ++i) {
+            const float a = fabsf(v[i]);
+            nonfinite |= !(a <= F32_MAX);
+            too_big |= check && a > B && a <= F32_MAX;
+            const int32_t k = __shfl_sync(0xffffffffu, myk, rr[i]);
+            if ((uint32_t)k < (uint32_t)K)
+                atomicAdd(acc + (int64_t)k * ACC_WORDS + jj[i], (unsigned long long)fixed_rn(v[i], S));
+        }
+        if (okk) atomicAdd(acc + (int64_t)myk * ACC_WORDS + D, 1ull);
+    }
+    // ragged end (< 32 kernels): one thread per kernel
+    if (do_tail) {
+        const int64_t i = nchunks * 32 + threadIdx.x;
+        if (threadIdx.x < 32 && i < n) {
+            const int32_t k = idx[i];
+            if ((uint32_t)k < (uint32_t)K) {
+#pragma unroll
+                for (int j = 0; j < D; ++j) {
+                    const float x = W[i * D + j];
+                    const float a = fabsf(x);
+                    nonfinite |= !(a <= F32_MAX);
+                    too_big |= check && a > B && a <= F32_MAX;
+                    atomicAdd(acc + (int64_t)k * ACC_WORDS + j, (unsigned long long)fixed_rn(x, S));
+                }
+                atomicAdd(acc + (int64_t)k * ACC_WORDS + D, 1ull);
+            } else {
+                bad_idx = true;
+            }
+        }
+    }
+    if (bad_idx) set_flag(&hdr->status, KQ_FLAG_INDEX_RANGE);
+    if (nonfinite) set_flag(&hdr->status, KQ_FLAG_NONFINITE);
+    if (too_big) atomicExch(&hdr->upd_violation, 1u);
 }
 
 __global__ void __launch_bounds__(256) maxabs_kernel(const float *__restrict__ W, int64_t count,
@@ -47,8 +126,8 @@ __global__ void __launch_bounds__(256) maxabs_kernel(const float *__restrict__ W
         ok &= isfinite(t.x) & isfinite(t.y) & isfinite(t.z) & isfinite(t.w);
         m = fmaxf(m, fmaxf(fmaxf(fabsf(t.x), fabsf(t.y)), fmaxf(fabsf(t.z), fabsf(t.w))));
     }
-    for (int64_t v = n4 * 4 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < count; v += stride) {
-        const float t = W[v];
+    for (int64_t u = n4 * 4 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < count; u += stride) {
+        const float t = W[u];
         ok &= isfinite(t);
         m = fmaxf(m, fabsf(t));
     }
@@ -58,71 +137,82 @@ __global__ void __launch_bounds__(256) maxabs_kernel(const float *__restrict__ W
     if ((threadIdx.x & 31) == 0) atomicMax(maxabs_bits, __float_as_uint(m));  // m >= +0: bits order as values
 }
 
+// Clears the accumulators; in guess mode also reduces max|C_prev| into upd_bound.
+__global__ void __launch_bounds__(256) update_prepare_kernel(const float *__restrict__ C_prev, int32_t K,
+                                                             unsigned long long *__restrict__ acc, Header *hdr,
+                                                             bool guess) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    ulonglong2 *a2 = reinterpret_cast<ulonglong2 *>(acc);
+    for (int64_t w = t0; w < (int64_t)K * ACC_WORDS / 2; w += stride) a2[w] = make_ulonglong2(0ull, 0ull);
+    if (!guess) return;
+    float m = 0.f;
+    for (int64_t e = t0; e < (int64_t)K * D; e += stride) {
+        const float a = fabsf(C_prev[e]);
+        m = a <= F32_MAX ? fmaxf(m, a) : __int_as_float(0x7f800000);  // non-finite: no usable guess
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    if ((threadIdx.x & 31) == 0) atomicMax(&hdr->upd_bound, __float_as_uint(m));
+}
+
 __global__ void __launch_bounds__(U_THREADS)
-accumulate_kernel(const float *__restrict__ W, int64_t n, const int32_t *__restrict__ idx, int32_t K,
-                  const uint32_t *__restrict__ maxabs_bits, unsigned long long *__restrict__ acc,
-                  uint32_t *status) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int S = update_scale(*maxabs_bits, n);
-    // A chunk is 32 kernels = 288 consecutive floats. In pass i a lane handles float
-    // lane + 32 i of the chunk (coalesced loads straight from global memory): kernel
-    // rr[i] of the chunk, coordinate jj[i]; the kernel's codeword comes from lane rr[i].
-    int rr[D], jj[D];
-#pragma unroll
-    for (int i = 0; i < D; ++i) {
-        rr[i] = (lane + 32 * i) / D;
-        jj[i] = (lane + 32 * i) - D * rr[i];
-    }
-    bool bad = false;
-    const int64_t nchunks = n / 32;
-    // Chunks are visited last-to-first: a max|W| pass that just streamed W front to
-    // back leaves the tail of W in L2.
-    for (int64_t it = (int64_t)blockIdx.x * (U_THREADS / 32) + warp; it < nchunks;
-         it += (int64_t)gridDim.x * (U_THREADS / 32)) {
-        const int64_t r0 = (nchunks - 1 - it) * 32;
-        const float *src = W + r0 * D;
-        float v[D];
-#pragma unroll
-        for (int i = 0; i < D; ++i) v[i] = __ldg(src + lane + 32 * i);
-        const int32_t myk = __ldcs(idx + r0 + lane);
-        const bool okk = (uint32_t)myk < (uint32_t)K;
-        bad |= !okk;
-#pragma unroll
-        for (int i = 0; i < D; ++i) {
-            const int32_t k = __shfl_sync(0xffffffffu, myk, rr[i]);
-            if ((uint32_t)k < (uint32_t)K)
-                atomicAdd(acc + (int64_t)k * ACC_WORDS + jj[i], (unsigned long long)fixed_rn(v[i], S));
+accumulate_kernel(const float *__restrict__ W, int64_t n, const int32_t *__restrict__ idx, int32_t K, Header *hdr,
+                  unsigned long long *__restrict__ acc, bool guess) {
+    const float B = guess ? __uint_as_float(__ldcg(&hdr->upd_bound)) * GUESS_FACTOR  // power-of-two scaling
+                          : __uint_as_float(__ldcg(&hdr->maxabs_bits));
+    int S = update_scale(B, n);
+    if (S == SCALE_INVALID) {
+        if (guess) {  // no usable guess: leave everything to the exact pass
+            if (blockIdx.x == 0 && threadIdx.x == 0) atomicExch(&hdr->upd_violation, 1u);
+            return;
         }
-        if (okk) atomicAdd(acc + (int64_t)myk * ACC_WORDS + D, 1ull);
+        S = 0;  // all-zero W (nothing to scale) or non-finite W (flagged)
     }
-    // ragged end (< 32 kernels): one thread per kernel in CTA 0
-    if (blockIdx.x == 0) {
-        const int64_t i = nchunks * 32 + threadIdx.x;
-        if (threadIdx.x < 32 && i < n) {
-            const int32_t k = idx[i];
-            if ((uint32_t)k < (uint32_t)K) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) hdr->upd_scale = S;
+    accumulate_rows(W, n, idx, K, S, B, guess, acc, hdr, (int64_t)blockIdx.x * (U_THREADS / 32) + (threadIdx.x >> 5),
+                    (int64_t)gridDim.x * (U_THREADS / 32), blockIdx.x == 0);
+}
+
+// Runs only when the guessed bound was violated (the flag is final: the accumulate
+// kernel has completed). Cooperative launch: all CTAs are resident, so they can
+// meet at the bounded grid barrier between clearing/measuring and re-adding.
+__global__ void __launch_bounds__(U_THREADS)
+update_fallback_kernel(const float *__restrict__ W, int64_t n, const int32_t *__restrict__ idx, int32_t K,
+                       Header *hdr, unsigned long long *__restrict__ acc) {
+    if (__ldcg(&hdr->upd_violation) == 0u) return;  // the common case: nothing to do
+    unsigned epoch = 0;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    ulonglong2 *a2 = reinterpret_cast<ulonglong2 *>(acc);
+    for (int64_t w = t0; w < (int64_t)K * ACC_WORDS / 2; w += stride) a2[w] = make_ulonglong2(0ull, 0ull);
+    float m = 0.f;
+    for (int64_t e = t0; e < n * D; e += stride) {
+        const float a = fabsf(W[e]);
+        m = a <= F32_MAX ? fmaxf(m, a) : m;
+    }
 #pragma unroll
-                for (int j = 0; j < D; ++j)
-                    atomicAdd(acc + (int64_t)k * ACC_WORDS + j, (unsigned long long)fixed_rn(W[i * D + j], S));
-                atomicAdd(acc + (int64_t)k * ACC_WORDS + D, 1ull);
-            } else {
-                bad = true;
-            }
-        }
-    }
-    if (bad) set_flag(status, KQ_FLAG_INDEX_RANGE);
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    if ((threadIdx.x & 31) == 0) atomicMax(&hdr->maxabs_bits, __float_as_uint(m));
+    if (!grid_barrier(hdr, gridDim.x, epoch)) return;
+    const float B = __uint_as_float(__ldcg(&hdr->maxabs_bits));
+    int S = update_scale(B, n);
+    if (S == SCALE_INVALID) S = 0;
+    if (blockIdx.x == 0 && threadIdx.x == 0) hdr->upd_scale = S;
+    accumulate_rows(W, n, idx, K, S, B, false, acc, hdr, (int64_t)blockIdx.x * (U_THREADS / 32) + (threadIdx.x >> 5),
+                    (int64_t)gridDim.x * (U_THREADS / 32), blockIdx.x == 0);
 }
 
 // c_k = (sum * 2^-S) / z_k in fp32 (keep C_prev when z_k = 0); clears the
-// accumulator row for the next call. fp32
-// arithmetic (GB300's fp64 rate is low): sum -> fp32, exact power-of-two scaling,
-// one IEEE division; within ~1.5 ulp of the exact mean.
+// accumulator row for the next call. fp32 arithmetic (GB300's fp64 rate is low):
+// sum -> fp32, exact power-of-two scaling, one IEEE division; within ~1.5 ulp of
+// the exact mean.
 __global__ void __launch_bounds__(256)
-finalize_kernel(unsigned long long *__restrict__ acc, int32_t K, int64_t n, const uint32_t *__restrict__ maxabs_bits,
-                const float *C_prev, float *C_next, int32_t *__restrict__ counts) {
+finalize_kernel(unsigned long long *__restrict__ acc, int32_t K, const Header *hdr, const float *C_prev,
+                float *C_next, int32_t *__restrict__ counts) {
     const int k = blockIdx.x * blockDim.x + threadIdx.x;
     if (k >= K) return;
-    const int S = update_scale(*maxabs_bits, n);
+    const int S = __ldcg(&hdr->upd_scale);
     unsigned long long *a = acc + (int64_t)k * ACC_WORDS;
     const long long z = (long long)a[D];
     const float zf = (float)z;  // exact below 2^24, within half an ulp above
@@ -167,6 +257,8 @@ cudaError_t launch_histogram(const int32_t *idx, int64_t n, int32_t K, int32_t *
 
 cudaError_t launch_maxabs(const float *W, int64_t count, uint32_t *maxabs_bits, uint32_t *status, int num_sms,
                           cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(maxabs_bits, 0, sizeof(uint32_t), s);
+    if (e != cudaSuccess) return e;
     int64_t blocks = (count / 4 + 255) / 256;
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
     if (blocks < 1) blocks = 1;
@@ -175,21 +267,53 @@ cudaError_t launch_maxabs(const float *W, int64_t count, uint32_t *maxabs_bits, 
     return cudaGetLastError();
 }
 
-cudaError_t launch_accumulate(const float *W, int64_t n, const int32_t *idx, int32_t K,
-                              const uint32_t *maxabs_bits, unsigned long long *acc, uint32_t *status,
-                              int num_sms, cudaStream_t s) {
-    const int64_t chunks = n / 32 + 1;
-    int64_t blocks = (chunks + U_THREADS / 32 - 1) / (U_THREADS / 32);
-    if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
+cudaError_t launch_update_prepare(const float *C_prev, int32_t K, unsigned long long *acc, Header *hdr,
+                                  bool guess_from_codebook, cudaStream_t s) {
+    // scale state (bound, violation flag, scale) and the fallback's barrier words
+    cudaError_t e = cudaMemsetAsync(&hdr->upd_bound, 0, 3 * sizeof(uint32_t), s);
+    if (e != cudaSuccess) return e;
+    e = cudaMemsetAsync(&hdr->barrier, 0, 2 * sizeof(uint32_t), s);
+    if (e != cudaSuccess) return e;
+    if (guess_from_codebook) {
+        e = cudaMemsetAsync(&hdr->maxabs_bits, 0, sizeof(uint32_t), s);
+        if (e != cudaSuccess) return e;
+    }
+    int64_t blocks = ((int64_t)K * ACC_WORDS / 2 + 255) / 256;
+    if (blocks > 1024) blocks = 1024;
     if (blocks < 1) blocks = 1;
-    accumulate_kernel<<<(unsigned)blocks, U_THREADS, 0, s>>>(W, n, idx, K, maxabs_bits, acc, status);
+    update_prepare_kernel<<<(unsigned)blocks, 256, 0, s>>>(C_prev, K, acc, hdr, guess_from_codebook);
     count_launch();
     return cudaGetLastError();
 }
 
-cudaError_t launch_finalize(unsigned long long *acc, int32_t K, int64_t n, const uint32_t *maxabs_bits,
-                            const float *C_prev, float *C_next, int32_t *counts, cudaStream_t s) {
-    finalize_kernel<<<(K + 255) / 256, 256, 0, s>>>(acc, K, n, maxabs_bits, C_prev, C_next, counts);
+cudaError_t launch_accumulate(const float *W, int64_t n, const int32_t *idx, int32_t K, Header *hdr,
+                              unsigned long long *acc, bool guess, int num_sms, cudaStream_t s) {
+    const int64_t chunks = n / 32 + 1;
+    int64_t blocks = (chunks + U_THREADS / 32 - 1) / (U_THREADS / 32);
+    if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
+    if (blocks < 1) blocks = 1;
+    accumulate_kernel<<<(unsigned)blocks, U_THREADS, 0, s>>>(W, n, idx, K, hdr, acc, guess);
+    count_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_update_fallback(const float *W, int64_t n, const int32_t *idx, int32_t K, Header *hdr,
+                                   unsigned long long *acc, int num_sms, cudaStream_t s) {
+    int per_sm = 0;
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, update_fallback_kernel, U_THREADS, 0);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    const unsigned blocks = (unsigned)num_sms;  // one CTA per SM: co-resident by construction
+    void *params[] = {(void *)&W, (void *)&n, (void *)&idx, (void *)&K, (void *)&hdr, (void *)&acc};
+    e = cudaLaunchCooperativeKernel((const void *)update_fallback_kernel, dim3(blocks), dim3(U_THREADS), params, 0, s);
+    if (e != cudaSuccess) return e;
+    count_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_finalize(unsigned long long *acc, int32_t K, const Header *hdr, const float *C_prev,
+                            float *C_next, int32_t *counts, cudaStream_t s) {
+    finalize_kernel<<<(K + 255) / 256, 256, 0, s>>>(acc, K, hdr, C_prev, C_next, counts);
     count_launch();
     return cudaGetLastError();
 }

@@ -188,6 +188,30 @@ def test_update_empty_clusters_and_bad_index():
     assert st == 5 and flags & kq.FLAG_INDEX_RANGE and cnt_g.sum() == 2999
 
 
+@pytest.mark.parametrize("case", ["zero_prev", "tiny_prev", "outlier", "nonfinite_prev"])
+def test_update_scale_fallback(case):
+    # kq_update_centroids guesses its fixed-point scale from max|C_prev|; inputs that
+    # break the guess take the exact fallback pass and must give the same answer.
+    n, K = 50000, 700
+    W = synth.random_kernels(n, 9, 5, 0.05)
+    C0 = synth.random_kernels(K, 9, 6, 0.05)
+    idx = synth.below(synth.stream_key(7, 2), n, K).astype(np.int32)
+    if case == "zero_prev":
+        C0[:] = 0
+    elif case == "tiny_prev":
+        C0 *= 1e-6
+    elif case == "outlier":
+        W[123, 4] = 1e4
+    elif case == "nonfinite_prev":
+        C0[5, 5] = np.inf
+    C_g, cnt_g, st, _ = gpu_update(W, idx, C0)
+    C_r, cnt_r = oracle.update(W, idx, C0)
+    assert st == 0 and np.array_equal(cnt_g, cnt_r)
+    check_centroids(C_g, C_r)
+    C_g2, _, _, _ = gpu_update(W, idx, C0)
+    assert bits_equal(C_g, C_g2)
+
+
 def test_update_k1_global_mean():
     W = synth.random_kernels(77777, 9, 11, 0.05)
     C0 = W[:1].copy()
