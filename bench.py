@@ -139,7 +139,7 @@ def _cpu_sample(W, C, seconds: float, threads: int):
     """Time the oracle's assignment on a seeded row sample sized for ~`seconds`."""
     import oracle
 
-    rows_all = synth.below(synth.stream_key(4242, 9), 1 << 16, W.shape[0])
+    rows_all = synth.below(synth.stream_key(4242, 9), 1 << 20, W.shape[0])
     probe = 64
     t0 = time.perf_counter()
     oracle.assign(W[rows_all[:probe]], C, threads=threads)
@@ -338,18 +338,18 @@ def run_kq(args, rank, world, local_rank):
         roofline["frac_at_sampled_clock"] = achieved / (sms * FP32_LANES_PER_SM * clk["sm_mhz"] * 1e6 / 1e12)
     hbm = float(peaks.get("hbm_gbs", 6776.3))
 
-    def hbm_roofline(name, bytes_per_call, ms_list, note):
+    def hbm_roofline(kernel, bytes_per_call, ms_list, note):
         t = statistics.mean(ms_list) / 1e3
         a = bytes_per_call / t / 1e9
         return {"bound": "hbm", "achieved": a, "peak": hbm, "unit": "GB/s", "frac": a / hbm,
-                "traffic": traffic.get(name), "calls": len(ms_list), "us_mean": 1e6 * t,
+                "traffic": traffic.get(kernel), "traffic_kernel": kernel, "calls": len(ms_list), "us_mean": 1e6 * t,
                 "algorithmic_bytes": int(bytes_per_call), "note": note}
 
     upd_bytes = n * (36 + 4) + K * (36 + 36 + 4)
     rec_bytes = n * (4 + 36) + 9 * K + 256
-    roofline_update = hbm_roofline("kq_update_centroids", upd_bytes, call_ms["update"],
+    roofline_update = hbm_roofline("accumulate_kernel", upd_bytes, call_ms["update"],
                                    "whole kq_update_centroids call (prepare + accumulate + fallback check + finalize)")
-    roofline_reconstruct = hbm_roofline("kq_reconstruct", rec_bytes, call_ms["reconstruct"],
+    roofline_reconstruct = hbm_roofline("gather_codes_kernel", rec_bytes, call_ms["reconstruct"],
                                         "whole kq_reconstruct call, K+C (decode codes + gather)")
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
