@@ -135,29 +135,44 @@ gather_codes_kernel(const int32_t *__restrict__ idx, int64_t n, const unsigned l
     }
     bool bad = false;
     const int64_t nch = n / 32;
-    for (int64_t ch = (int64_t)blockIdx.x * R_WARPS + warp; ch < nch; ch += (int64_t)gridDim.x * R_WARPS) {
-        const int64_t r0 = ch * 32;
-        const int32_t k = __ldcs(idx + r0 + lane);
-        const bool ok = (uint32_t)k < (uint32_t)K;
-        bad |= !ok;
-        const unsigned long long q = ok ? __ldg(Cq + k) : ALL_CODES_OUT_OF_RANGE;
-        const uint32_t qlo = (uint32_t)q, qhi = (uint32_t)(q >> 32);
-        float4 *d4 = reinterpret_cast<float4 *>(W_out + r0 * D);
+    // two chunks per warp step: both index loads, then both code gathers are in
+    // flight before any decoding
+    const int64_t nch2 = nch / 2;
+    for (int64_t c2 = (int64_t)blockIdx.x * R_WARPS + warp; c2 < nch2 + (nch & 1); c2 += (int64_t)gridDim.x * R_WARPS) {
+        const int64_t ch0 = 2 * c2;
+        const bool two = ch0 + 1 < nch;
+        int32_t k[2];
+        k[0] = __ldcs(idx + ch0 * 32 + lane);
+        k[1] = two ? __ldcs(idx + (ch0 + 1) * 32 + lane) : 0;
+        unsigned long long q[2];
 #pragma unroll
-        for (int s = 0; s < 3; ++s) {
-            const int rb = min(ra[s] + 1, 31);
-            const unsigned long long qa = ((unsigned long long)__shfl_sync(0xffffffffu, qhi, ra[s]) << 32) |
-                                          __shfl_sync(0xffffffffu, qlo, ra[s]);
-            const unsigned long long qb = ((unsigned long long)__shfl_sync(0xffffffffu, qhi, rb) << 32) |
-                                          __shfl_sync(0xffffffffu, qlo, rb);
-            float r[4];
+        for (int h = 0; h < 2; ++h) {
+            const bool ok = (uint32_t)k[h] < (uint32_t)K;
+            bad |= !ok && (h == 0 || two);
+            q[h] = ok ? __ldg(Cq + k[h]) : ALL_CODES_OUT_OF_RANGE;
+        }
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const bool first = e < split[s];
-                const int j = first ? j0[s] + e : e - split[s];
-                r[e] = lv[((first ? qa : qb) >> (7 * j)) & 127u][lane];
+        for (int h = 0; h < 2; ++h) {
+            if (h == 1 && !two) break;
+            const int64_t r0 = (ch0 + h) * 32;
+            const uint32_t qlo = (uint32_t)q[h], qhi = (uint32_t)(q[h] >> 32);
+            float4 *d4 = reinterpret_cast<float4 *>(W_out + r0 * D);
+#pragma unroll
+            for (int s = 0; s < 3; ++s) {
+                const int rb = min(ra[s] + 1, 31);
+                const unsigned long long qa = ((unsigned long long)__shfl_sync(0xffffffffu, qhi, ra[s]) << 32) |
+                                              __shfl_sync(0xffffffffu, qlo, ra[s]);
+                const unsigned long long qb = ((unsigned long long)__shfl_sync(0xffffffffu, qhi, rb) << 32) |
+                                              __shfl_sync(0xffffffffu, qlo, rb);
+                float r[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const bool first = e < split[s];
+                    const int j = first ? j0[s] + e : e - split[s];
+                    r[e] = lv[((first ? qa : qb) >> (7 * j)) & 127u][lane];
+                }
+                if (s < 2 || lane < 32 * D / 4 - 64) __stcs(d4 + lane + 32 * s, make_float4(r[0], r[1], r[2], r[3]));
             }
-            if (s < 2 || lane < 32 * D / 4 - 64) __stcs(d4 + lane + 32 * s, make_float4(r[0], r[1], r[2], r[3]));
         }
     }
     // ragged end (< 32 kernels): CTA 0, plain loads and stores
@@ -200,7 +215,7 @@ cudaError_t launch_gather_rows(const int32_t *idx, int64_t n, const float *Cp, c
                                const float *levels, int32_t K, float *W_out, uint32_t *status, int num_sms,
                                cudaStream_t s) {
     if (Cq) {
-        int64_t blocks = (n / 32 + R_WARPS - 1) / R_WARPS;
+        int64_t blocks = ((n / 32 + 1) / 2 + R_WARPS - 1) / R_WARPS;
         if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
         if (blocks < 1) blocks = 1;
         gather_codes_kernel<<<(unsigned)blocks, R_THREADS, 0, s>>>(idx, n, Cq, levels, K, W_out, status);
