@@ -106,6 +106,20 @@ class ClockSampler:
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def replica_throughput(local_ms: float, units_per_step: float, steps: int, world: int, device):
+    """Weak scaling of independent replicas: (all ranks' units / max-over-ranks
+    seconds, max-over-ranks ms). Needs an initialised process group when world > 1
+    (NCCL with a CUDA device, or gloo with the CPU)."""
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([local_ms], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms_max = float(t.item())
+    return world * steps * units_per_step / (ms_max / 1e3), ms_max
+
+
 def _ncu_traffic():
     """Per-launch DRAM bytes (read + write) from the committed ncu summary, or {}."""
     out = {}
@@ -264,12 +278,8 @@ def run_kq(args, rank, world, local_rank):
     ms_total = e0.elapsed_time(e1)
     call_ms = {name: [a.elapsed_time(b) for ev in evs for a, b in ev[name]] for name in evs[0]}
     assign_ms = call_ms["assign"]
-    t_local = torch.tensor([ms_total], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t_local, op=dist.ReduceOp.MAX)
-    ms_max = float(t_local.item())
     pairs_per_step = n_assign * n * K
-    value = world * args.steps * pairs_per_step / (ms_max / 1e3)
+    value, ms_max = replica_throughput(ms_total, pairs_per_step, args.steps, world, dev)
 
     st, flags = kq.kq_device_status(ws)
     if st != 0:
@@ -308,10 +318,7 @@ def run_kq(args, rank, world, local_rank):
         e2e_step()
     torch.cuda.synchronize()
     e2e_s = time.perf_counter() - t0
-    t_e2e = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t_e2e, op=dist.ReduceOp.MAX)
-    e2e_value = world * e2e_steps * pairs_per_step / float(t_e2e.item())
+    e2e_value, _ = replica_throughput(1e3 * e2e_s, pairs_per_step, e2e_steps, world, dev)
     h2d = W_pin.numel() * 4 + sel_pin.numel() * 8
     d2h = sum(t.numel() * t.element_size() for t in outs.values())
 

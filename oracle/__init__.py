@@ -37,7 +37,7 @@ def build(force: bool = False) -> str:
     os.makedirs(_BUILD, exist_ok=True)
     if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
         tmp = _LIB_PATH + f".tmp{os.getpid()}"
-        subprocess.run(["gcc", *_CFLAGS, _SRC, "-o", tmp, "-lm"], check=True)
+        compile_library(_SRC, tmp)
         os.replace(tmp, _LIB_PATH)
     return _LIB_PATH
 
@@ -45,10 +45,9 @@ def build(force: bool = False) -> str:
 _lib = None
 
 
-def _load():
-    global _lib
-    if _lib is None:
-        lib = ctypes.CDLL(build())
+def _bind(lib):
+    """Declare the C signatures on a loaded oracle library and return it."""
+    if True:
         P = ctypes.c_void_p
         i64, i32, f64 = ctypes.c_int64, ctypes.c_int32, ctypes.c_double
         lib.kqo_assign.argtypes = [P, i64, P, i32, P, P, P, P, i32]
@@ -69,7 +68,19 @@ def _load():
         lib.kqo_encode.restype = None
         lib.kqo_gather_rows.argtypes = [P, P, i32, P]
         lib.kqo_gather_rows.restype = None
-        _lib = lib
+    return lib
+
+
+def compile_library(src: str, out: str) -> str:
+    """Compile an oracle C source (this one, or a test's modified copy) to `out`."""
+    subprocess.run(["gcc", *_CFLAGS, src, "-o", out, "-lm"], check=True)
+    return out
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        _lib = _bind(ctypes.CDLL(build()))
     return _lib
 
 

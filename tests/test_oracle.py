@@ -110,11 +110,15 @@ def test_assign_brute_force_integers(n, K, seed):
     C[K // 2] = C[0]  # duplicate codeword: the lower index must win
     W[0] = C[K - 1]
     idx, dist = oracle.assign(W, C)
+    total = Fraction(0)
     for i in range(n):
         ds = [_exact_d(W[i], C[k]) for k in range(K)]
         m = min(ds)
         assert idx[i] == ds.index(m)
         assert Fraction(float(dist[i])) == m
+        total += m
+    # Eq. 1 objective: the sum of the minimal squared distances (exact here)
+    assert Fraction(oracle.objective(dist)) == total
     first = next(k for k in range(K) if np.array_equal(C[k], C[K - 1]))
     assert idx[0] == first and dist[0] == 0
 
@@ -312,6 +316,19 @@ def test_level_fit_codes_round_trip():
     assert np.array_equal(oracle.encode(C.reshape(-1), levels), codes.reshape(-1))
     # decoding then re-encoding is the identity on codes
     assert np.array_equal(oracle.encode(levels[codes].reshape(-1), levels), codes.reshape(-1))
+
+
+def test_encode_ties_go_to_the_lower_level():
+    # Exact ties by construction: midpoints between levels and duplicated levels.
+    levels = np.arange(64, dtype=np.float32) * 2.0  # 0, 2, 4, ...
+    levels[10] = levels[9]  # a duplicate pair
+    # small integers: every fp32 difference is exact, so exact arithmetic decides
+    v = np.concatenate([np.arange(1, 127, 2), [18.0, 19.0, 20.0, -5.0, 500.0]]).astype(np.float32)
+    codes = oracle.encode(v, levels)
+    for x, c in zip(v, codes):
+        d = [abs(Fraction(float(x)) - Fraction(float(L))) for L in levels]
+        assert c == d.index(min(d)), (x, c)
+    assert oracle.encode(np.float32([1.0]), levels)[0] == 0  # equidistant from levels 0 and 1
 
 
 def test_level_scale_bounds():
