@@ -63,6 +63,7 @@ struct Ws {
     double *blocksum;
     float *cbuf0, *cbuf1, *cp;
     unsigned long long *cq;
+    float *cpk;
 };
 
 Ws carve(void *ws, int64_t n, int32_t K) {
@@ -78,6 +79,7 @@ Ws carve(void *ws, int64_t n, int32_t K) {
     w.cbuf1 = reinterpret_cast<float *>(b + L.cbuf1);
     w.cp = reinterpret_cast<float *>(b + L.cp);
     w.cq = reinterpret_cast<unsigned long long *>(b + L.cq);
+    w.cpk = reinterpret_cast<float *>(b + L.cpk);
     return w;
 }
 
@@ -87,6 +89,19 @@ kq_status run_update_exact(const float *W, int64_t n, const int32_t *idx, int32_
                            float *C_next, int32_t *counts, const Ws &w, int sms, cudaStream_t s) {
     KQ_TRY(launch_accumulate(W, n, idx, K, w.hdr, w.acc, false, sms, s));
     KQ_TRY(launch_finalize(w.acc, K, w.hdr, C_prev, C_next, counts, s));
+    return KQ_OK;
+}
+
+// One assignment: tensor-core path when n fills every SM, CUDA-core path otherwise.
+kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const int32_t *hint, int32_t *idx,
+                     float *dist, int *nb, const Ws &w, int sms, cudaStream_t s) {
+    if (tc_eligible(n, sms)) {
+        KQ_TRY(launch_pack_codebook_tc(C, K, w.cpk, w.hdr, s));
+        KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K, hint, idx, dist, w.blocksum, nb, w.hdr, s));
+    } else {
+        KQ_TRY(launch_pack_codebook(C, K, w.cd, w.hdr, s));
+        KQ_TRY(launch_assign(W, n, w.cd, C, K, hint, idx, dist, w.blocksum, nb, w.part, w.hdr, sms, s));
+    }
     return KQ_OK;
 }
 
@@ -161,10 +176,8 @@ kq_status kq_assign(const float *W, int64_t n, const float *C, int32_t K, const 
     if ((st = num_sms(&sms)) != KQ_OK) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     Ws w = carve(ws, n, K);
-    KQ_TRY(launch_pack_codebook(C, K, w.cd, w.hdr, s));
     int nb = 0;
-    KQ_TRY(launch_assign(W, n, w.cd, C, K, hint, idx, dist, w.blocksum, &nb, w.part, w.hdr, sms, s));
-    return KQ_OK;
+    return run_assign(W, n, C, K, hint, idx, dist, &nb, w, sms, s);
 }
 
 kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int32_t K, const float *C_prev,
@@ -209,18 +222,14 @@ kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_i
     int nb = 0;
     // iteration t > 0 starts every row from its previous assignment (warm start)
     for (int32_t t = 0; t < iters; ++t) {
-        KQ_TRY(launch_pack_codebook(cur, K, w.cd, w.hdr, s));
-        KQ_TRY(launch_assign(W, n, w.cd, cur, K, t > 0 ? idx : nullptr, idx, nullptr, w.blocksum, &nb, w.part, w.hdr,
-                             sms, s));
+        if ((st = run_assign(W, n, cur, K, t > 0 ? idx : nullptr, idx, nullptr, &nb, w, sms, s)) != KQ_OK) return st;
         if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
         if ((st = run_update_exact(W, n, idx, K, cur, nxt, counts, w, sms, s)) != KQ_OK) return st;
         float *tmp = cur;
         cur = nxt;
         nxt = tmp;
     }
-    KQ_TRY(launch_pack_codebook(cur, K, w.cd, w.hdr, s));
-    KQ_TRY(launch_assign(W, n, w.cd, cur, K, iters > 0 ? idx : nullptr, idx, nullptr, w.blocksum, &nb, w.part, w.hdr,
-                         sms, s));
+    if ((st = run_assign(W, n, cur, K, iters > 0 ? idx : nullptr, idx, nullptr, &nb, w, sms, s)) != KQ_OK) return st;
     if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + iters, s));
     KQ_TRY(launch_histogram(idx, n, K, counts, &w.hdr->status, sms, s));
     KQ_TRY(cudaMemcpyAsync(C_out, cur, cbytes, cudaMemcpyDeviceToDevice, s));

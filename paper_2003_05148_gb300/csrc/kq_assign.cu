@@ -9,6 +9,7 @@
 //   error bounds    fl(e) is within g9 (|h| + |x||c|) of e (recursive FMA sum of 10
 //                   terms, g9 >= 9u/(1-9u), u = 2^-24), and the fp32 direct form
 //                   D_dir >= D (1 - g11) (nine non-negative terms, g11 >= 11u/(1-11u)).
+//   (plus an absolute 2^-126 for underflowing intermediate results),
 //   so with Cmax >= |c|, Hmax >= |h|, Qmax >= ||c|^2 - 2h| over the codebook and
 //   X2lo <= |x|^2, fl(e) < thr := (X2lo - Qmax - 2 g9 (Hmax + |x| Cmax) - best/(1-g11)) / 2
 //   implies D_dir > best: the codeword cannot improve (or tie) the running best and
@@ -157,6 +158,7 @@ assign_kernel(const float *__restrict__ W, int64_t n, const float *__restrict__ 
         }
         x2lo[r] = lo;
         slack[r] = __fadd_ru(qmax, __fmul_ru(2.f * G9, __fadd_ru(hmax, __fmul_ru(__fsqrt_ru(hi), cmax))));
+        slack[r] = __fadd_ru(slack[r], 1.1754944e-38f);  // absolute part: underflow of the 9 FMAs, < 20 * 2^-150
         best[r] = __int_as_float(0x7f800000);  // +inf
         bi[r] = kb;
         thr[r] = __int_as_float(0xff800000);   // -inf: nothing is skipped

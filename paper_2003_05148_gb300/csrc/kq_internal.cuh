@@ -40,7 +40,7 @@ struct Header {
 static_assert(sizeof(Header) <= 4096, "header too large");
 
 struct WsLayout {
-    size_t cd, acc, part, blocksum, cbuf0, cbuf1, cp, cq, total;
+    size_t cd, acc, part, blocksum, cbuf0, cbuf1, cp, cq, cpk, total;
 };
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -57,6 +57,7 @@ inline WsLayout ws_layout(int64_t n, int32_t K) {
     L.cbuf1 = off;    off = align_up(off + (size_t)K * D * 4, 256);
     L.cp = off;       off = align_up(off + (size_t)K * CP_FLOATS * 4, 256);
     L.cq = off;       off = align_up(off + (size_t)K * 8, 256);
+    L.cpk = off;      off = align_up(off + (size_t)((K + 127) / 128 * 128) * 128, 256);  // tensor-core codeword tiles
     L.total = off;
     return L;
 }
@@ -184,6 +185,12 @@ cudaError_t launch_pack_codebook(const float *C, int32_t K, float *Cd, Header *h
 cudaError_t launch_assign(const float *W, int64_t n, const float *Cd, const float *C, int32_t K, const int32_t *hint,
                           int32_t *idx, float *dist, double *blocksum, int *nblocksum, unsigned long long *part,
                           Header *hdr, int num_sms, cudaStream_t s);
+// Tensor-core assignment (kq_assign_tc.cu): used when n fills every SM.
+bool tc_eligible(int64_t n, int num_sms);
+cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Header *hdr, cudaStream_t s);
+cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const float *Cpk, int32_t K,
+                             const int32_t *hint, int32_t *idx, float *dist, double *blocksum, int *nblocksum,
+                             Header *hdr, cudaStream_t s);
 cudaError_t launch_sum_blocks(const double *blocksum, int nblocks, double *out, cudaStream_t s);
 
 // Update step. Two ways to pick the fixed-point scale: `exact` takes B = max|W|

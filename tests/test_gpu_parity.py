@@ -116,6 +116,49 @@ def test_assign_filter_extreme_scales(case):
     _oracle_check(W, C, idx, dist)
 
 
+TC_MIN_N = 256 * 152  # from this many kernels on, the assignment runs on the tensor cores
+
+
+@pytest.mark.parametrize("case", ["plain", "offset", "mixed", "large", "near_dup", "ragged"])
+def test_assign_tensor_core_path(case):
+    # n large enough for the tensor-core path; K = 1000 is not a multiple of the
+    # 128-codeword tile, so padding codewords are exercised too.
+    n, K = TC_MIN_N + 1000, 1000
+    if case == "ragged":
+        n = TC_MIN_N + 77
+    W = synth.random_kernels(n, 9, 201, 0.05)
+    C = synth.random_kernels(K, 9, 202, 0.05)
+    if case == "offset":
+        W, C = W * 1e-3 + 1000.0, C * 1e-3 + 1000.0
+    elif case == "mixed":
+        W[::2] *= 1e6
+        C[::3] *= 1e-6
+    elif case == "large":
+        W, C = W * 1e15, C * 1e15
+    elif case == "near_dup":
+        C[1::2] = np.nextafter(C[0::2], np.float32(np.inf))[: C[1::2].shape[0]]
+        W[:K] = C
+    W, C = W.astype(np.float32), C.astype(np.float32)
+    idx, dist, st, _ = gpu_assign(W, C)
+    assert st == 0
+    rows = np.sort(synth.below(synth.stream_key(203, 9), 6000, n))
+    rows[-1] = n - 1
+    idx_ref, dist_ref = oracle.assign(W[rows], C, threads=THREADS)
+    assert check_indices(W, C, idx[rows], idx_ref, rows) == 0
+    assert bits_equal(dist[rows], dist_ref)
+
+
+def test_assign_paths_agree():
+    # the same kernels through the tensor-core path (large n) and the CUDA-core
+    # path (small n) give bit-identical results
+    W = synth.random_kernels(TC_MIN_N + 5000, 9, 211, 0.05)
+    C = synth.random_kernels(2000, 9, 212, 0.05)
+    i_tc, d_tc, st1, _ = gpu_assign(W, C)
+    i_cc, d_cc, st2, _ = gpu_assign(W[:20000], C)
+    assert st1 == 0 and st2 == 0
+    assert np.array_equal(i_tc[:20000], i_cc) and bits_equal(d_tc[:20000], d_cc)
+
+
 def test_assign_hint_never_changes_result():
     lay, W, C0 = _layer(2)
     idx0, dist0, _, _ = gpu_assign(W, C0)
