@@ -40,6 +40,11 @@ SM_COUNT_NOMINAL = 152
 FP32_LANES_PER_SM = 128
 OPS_PER_PAIR = 9  # FP32-pipe lane ops per pair executed by the assign kernel: the 9 FFMA of its certified test
 DIRECT_OPS_PER_PAIR = 18  # the fp32 direct form: 9 FSUB + 9 FFMA
+# Tensor-core assign: the certified test is an (n x 32) . (32 x K) split-TF32 GEMM, 2 * 32 flops per pair.
+TC_FLOPS_PER_PAIR = 64
+TC_ROWS_PER_CTA = 256  # the library takes the tensor-core kernel when n >= 256 * SMs
+TF32_PER_BF16 = 1.1 / 2.25  # nominal dense tf32 : bf16 tensor rate
+TF32_FLOPS_PER_CLK_SM = 4096  # nominal dense tf32 rate per SM per clock
 WORKLOAD_CFG = 5
 
 
@@ -330,19 +335,37 @@ def run_kq(args, rank, world, local_rank):
     max_mhz = float(peaks.get("sm_max_mhz", 2070.0))
     peak_tops = sms * FP32_LANES_PER_SM * max_mhz * 1e6 / 1e12
     t_assign = statistics.mean(assign_ms) / 1e3
-    achieved = OPS_PER_PAIR * n * K / t_assign / 1e12
     traffic = _ncu_traffic()
-    roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s", "frac": achieved / peak_tops,
-                "traffic": traffic.get("assign_kernel"), "kernel": "assign_kernel",
-                "peak_basis": f"{sms} SMs x {FP32_LANES_PER_SM} FP32 lanes x {max_mhz:.0f} MHz (max SM clock); "
-                              f"op = one FP32-pipe lane op; {OPS_PER_PAIR} per pair (the FFMA of the certified "
-                              f"expanded-form test every pair gets; the exact re-evaluations of the few candidate "
-                              f"pairs are not counted)",
-                "direct_form_equivalent": {"achieved": DIRECT_OPS_PER_PAIR * n * K / t_assign / 1e12,
-                                           "note": "18 ops/pair: the rate a direct-form kernel would need"},
-                "assign_ms_mean": 1e3 * t_assign, "assign_launches": len(assign_ms)}
-    if clk:
-        roofline["frac_at_sampled_clock"] = achieved / (sms * FP32_LANES_PER_SM * clk["sm_mhz"] * 1e6 / 1e12)
+    if n >= TC_ROWS_PER_CTA * sms:
+        # kernel timed inside a long step: the sustained bf16 figure, scaled to tf32
+        bf16 = float(peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops", 1700.0)))
+        peak = bf16 * TF32_PER_BF16
+        achieved = TC_FLOPS_PER_PAIR * n * K / t_assign / 1e12
+        roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                    "traffic": traffic.get("assign_tc_kernel"), "kernel": "assign_tc_kernel",
+                    "peak_basis": f"measured cuBLAS bf16 sustained {bf16:.1f} TFLOP/s x {TF32_PER_BF16:.4f} "
+                                  f"(nominal tf32:bf16); flops = {TC_FLOPS_PER_PAIR} per pair (the split-TF32 "
+                                  f"GEMM of the certified test, K = 32); the exact fp32 re-evaluations of the "
+                                  f"few candidate pairs run on the CUDA cores and are not counted",
+                    "frac_of_burst": achieved / (float(peaks.get("bf16_tflops", bf16)) * TF32_PER_BF16),
+                    "peak_at_max_clock": sms * TF32_FLOPS_PER_CLK_SM * max_mhz * 1e6 / 1e12,
+                    "assign_ms_mean": 1e3 * t_assign, "assign_launches": len(assign_ms)}
+        roofline["frac_of_peak_at_max_clock"] = achieved / roofline["peak_at_max_clock"]
+    else:
+        achieved = OPS_PER_PAIR * n * K / t_assign / 1e12
+        roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s",
+                    "frac": achieved / peak_tops, "traffic": traffic.get("assign_kernel"), "kernel": "assign_kernel",
+                    "peak_basis": f"{sms} SMs x {FP32_LANES_PER_SM} FP32 lanes x {max_mhz:.0f} MHz (max SM clock); "
+                                  f"op = one FP32-pipe lane op; {OPS_PER_PAIR} per pair (the FFMA of the certified "
+                                  f"expanded-form test every pair gets; the exact re-evaluations of the few "
+                                  f"candidate pairs are not counted)",
+                    "assign_ms_mean": 1e3 * t_assign, "assign_launches": len(assign_ms)}
+        if clk:
+            roofline["frac_at_sampled_clock"] = achieved / (sms * FP32_LANES_PER_SM * clk["sm_mhz"] * 1e6 / 1e12)
+    roofline["direct_form_equivalent"] = {"achieved_tops": DIRECT_OPS_PER_PAIR * n * K / t_assign / 1e12,
+                                          "frac_of_fp32_peak": DIRECT_OPS_PER_PAIR * n * K / t_assign / 1e12 / peak_tops,
+                                          "note": "18 FP32 ops/pair: the rate a direct-form CUDA-core kernel "
+                                                  "would need for the same time"}
     hbm = float(peaks.get("hbm_gbs", 6776.3))
 
     def hbm_roofline(kernel, bytes_per_call, ms_list, note):

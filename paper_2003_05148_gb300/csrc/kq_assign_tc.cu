@@ -2,57 +2,92 @@
 // the 5th-generation tensor cores (tcgen05, sm_103a).
 //
 // Same answer as kq_assign.cu (the fp32 direct-form argmin, lowest index on ties);
-// only the cheap test that rules codewords out moves to the tensor cores:
+// only the cheap test that rules codewords out moves to the tensor cores, and the
+// row's threshold moves into the GEMM so that the test is one sign bit:
 //
-//   e = x . c - h for a 128-row x 128-codeword tile is one GEMM, kind::tf32. The
-//   tensor core truncates fp32 operands to tf32 (relative error < 2^-10 each;
-//   measured: products match truncated inputs to fp32 accumulation error). To keep
-//   fp32-like accuracy every value is split exactly into v = v_hi + v_lo with v_hi
-//   = v truncated to tf32, and the three significant cross terms go side by side
-//   along the GEMM's K dimension (K = 32, two MMAs per 16-column half):
-//     A[i] = ( x_hi,  1,     x_hi,  1,     x_lo, 0, 0, 0 )
-//     B[k] = ( c_hi, -h_hi,  c_lo, -h_lo,  c_hi, 0, 0, 0 )     (9 + 1 + 9 + 1 + 9 + 3)
-//   so e_tc = x.c - h - x_lo.c_lo + (truncation of the lo parts) + (fp32 accumulation):
-//   |e_tc - e| <= (3 * 2^-20 + 29 * 2^-23) (sum |x_j c_j| + |h|) < 2^-16 (|x| Cmax + Hmax),
-//   plus an absolute 2^-120 (Cmax + |x| + 1) for subnormal inputs flushed to zero.
-//   With that bound in place of the fp32 one, the threshold test of kq_assign.cu
-//   is unchanged: e_tc < thr proves D_dir > best. Codewords that pass get the exact
-//   fp32 direct form on the CUDA cores, reading c = c_hi + c_lo (exact) from the
-//   shared tile.
+//   g = x . c - h - R - T' for a 128-row x 256-codeword tile is one GEMM,
+//   kind::tf32. The tensor core truncates fp32 operands to tf32 (relative error
+//   < 2^-10 each; measured: products match truncated inputs to fp32 accumulation
+//   error). To keep fp32-like accuracy every value is split exactly into
+//   v = v_hi + v_lo with v_hi = v truncated to tf32, and the three significant
+//   cross terms go side by side along the GEMM's K dimension (K = 32):
+//     A[i] = ( x_hi,  1,     x_hi,  1,     x_lo,  -T'0, -R, -T'1 )
+//     B[k] = ( c_hi, -h_hi,  c_lo, -h_lo,  c_hi,  s0,    1,  s1  )   (9 + 1 + 9 + 1 + 9 + 3)
+//   where (s0, s1) = (1, 0) for the first 128 codewords of a tile and (0, 1) for
+//   the other 128, so each half of a tile row sees its own T' (each half is tested
+//   by its own thread, with its own running best). R (tf32, fixed per row, about
+//   |x|^2 / 2) and T' (tf32) are exact; the other half's T' meets an exact 0.
+//   Dropping x_lo.c_lo, truncating the lo parts to tf32 and accumulating 31 terms
+//   in fp32 give
+//     |g - (e - R - T')| <= E = 2^-16 (|x| Cmax + Hmax + |R| + |T'|) + 2^-120 (Cmax + |x| + 1)
+//   (3 * 2^-20 + 31 * 2^-23 (1 + 2^-8) < 2^-16 on the first group, 31 * 2^-23 on R
+//   and T'; the absolute part covers subnormal inputs the tensor core may flush).
+//   The kernel keeps R + T' + E < thr0, where e < thr0 proves D_dir > best (the
+//   test of kq_assign.cu without its arithmetic slack), so a negative g (sign bit
+//   set, -0 included since E > 0) rules the codeword out. The TMEM load reduces as
+//   it reads (tcgen05.ld.red.max, sm_103a): a 32-codeword chunk whose maximum g has
+//   its sign bit set is ruled out with no further work (NaN test values, which the
+//   maximum skips, only arise in rows whose thread tests every codeword anyway: see
+//   T' = -2^100 below). Only a chunk with a non-negative maximum sends the row to
+//   the exact fp32 direct form on the CUDA cores, which reads c = c_hi + c_lo
+//   (exact) from the shared tile. When a row's best improves, its thread rewrites
+//   its T' (one 4-byte shared store). MMAs already issued, or issued before the
+//   store is seen, use the older T', which satisfied the inequality for the older,
+//   larger best, and so for the current one: the test stays sound at every moment.
+//   A half row without a usable T' (no running best yet, non-finite inputs) holds
+//   T' = -2^100: its g is then huge and positive (and no infinity meets the other
+//   half's 0), and its thread tests every codeword exactly anyway.
 //
-// Warp roles in a CTA of 320 threads that owns 256 kernels (two 128-row MMA tiles):
-//   warp 0      producer: streams packed codeword tiles (128 codewords x 128 B,
+// Warp roles in a CTA of 352 threads that owns 256 kernels (two 128-row tiles):
+//   warp 0      producer: streams packed codeword tiles (256 codewords x 128 B,
 //               already in the tensor-core layout) into a 4-stage shared ring with
 //               one bulk asynchronous copy per tile (TMA engine), mbarrier tx counts;
-//   warp 1      owns TMEM (all 512 columns: two buffers x two row tiles x 128
-//               columns) and issues the MMAs from one thread; tcgen05.commit
-//               publishes the TMEM buffer;
-//   warps 2-9   epilogue: one kernel (row) per thread; per tile, tcgen05.ld 32
-//               columns at a time, max, compare with the row's threshold, exact
-//               pass for the rare candidates from the shared tile, then release
-//               the TMEM buffer and the shared stage.
+//   warps 1-2   MMA issuers, one per row tile (warp 1 also owns TMEM: 512 columns,
+//               one 256-column accumulator per row tile): from one thread, the 4
+//               MMAs (M = 128, N = 256, K = 8 each) of its row tile for a codeword
+//               tile, then tcgen05.commit. The epilogue drains one accumulator
+//               while the tensor core fills the other. Two issuers, because the
+//               first shared-memory access (a barrier wait) of a thread after its
+//               MMAs waits until they have executed: with one issuer the tensor
+//               core would idle at every such wait, with two the other's MMAs run;
+//   warps 3-10  epilogue: a thread owns one kernel in each row tile and one
+//               128-codeword half of every tile: four reducing tcgen05.ld of 32
+//               columns and one wait, the accumulator goes back at once, then the
+//               sign test of the chunk maxima and the exact pass for the rare
+//               candidates; the shared stage goes back when both row tiles are done.
+//               The halves merge at the end.
+// The producer and MMA loops run in lane 0 of their warps while lanes 1-31 wait at
+// the CTA barrier that opens the teardown: a lone lane waits on a completed
+// mbarrier phase in ~20 cycles, a whole warp (or a lane whose partners wait at a
+// warp-level sync) in ~100-300, all of it idle time for the tensor core when it is
+// the MMA issuer's. (N = 256 MMAs keep the tensor core fully busy from one thread;
+// N = 128 ones lose ~20%.)
 // Every wait is bounded; a wait that runs out sets KQ_FLAG_TIMEOUT and an abort
 // word, every role then drains out, and warp 1 frees TMEM before the CTA exits.
 #include "kq_internal.cuh"
 
 namespace kq {
 
-constexpr int TC_M = 128;                  // rows per MMA tile
+constexpr int TC_M = 128;                  // rows per MMA (row tile)
 constexpr int TC_RT = 2;                   // row tiles per CTA
 constexpr int TC_ROWS = TC_M * TC_RT;      // kernels per CTA
-constexpr int TC_N = 128;                  // codewords per tile
+constexpr int TC_N = 256;                  // codewords per tile (N of every MMA)
+constexpr int TC_HALF = TC_N / 2;          // codewords of a tile one epilogue thread tests
 constexpr int TC_KD = 32;                  // K of the GEMM (hi/lo split, see top of file)
 constexpr int TC_STAGES = 4;
-constexpr int TC_TILE_BYTES = TC_N * TC_KD * 4;  // 16 KiB per codeword tile
+constexpr int TC_TILE_BYTES = TC_N * TC_KD * 4;  // 32 KiB per codeword tile
 constexpr int TC_A_BYTES = TC_M * TC_KD * 4;     // 16 KiB per row tile
-constexpr int TC_THREADS = 320;
+constexpr int TC_THREADS = 352;
+constexpr int TC_EPI_WARP0 = 3;            // first epilogue warp (0: producer, 1-2: MMA issuers)
 constexpr int TC_EPI_WARPS = 8;
-constexpr uint32_t TC_COLS = 512;          // TMEM columns allocated (2 buffers x 2 row tiles x 128)
+constexpr uint32_t TC_COLS = 512;          // TMEM columns allocated (2 row tiles x 256)
 constexpr uint32_t TC_LBO = 128;           // K-adjacent core matrices (8 rows x 16 B each)
 constexpr uint32_t TC_SBO = TC_KD / 4 * 128; // next 8-row group (8 core matrices along K)
 constexpr long long TC_WAIT_LIMIT = 4000000;
-constexpr float G_TC = 1.52587890625e-5f;  // 2^-16 (see top of file)
-constexpr float ONE_M_G11_TC = 0.9999993f; // <= 1 - gamma_11 (direct-form bound)
+constexpr float TWO_G_TC = 3.0517578125e-5f;  // 2 x 2^-16 (see top of file)
+constexpr float INV_ONE_M_G11_TC = 1.0000008344650269f;  // 1 + 7 * 2^-23 >= 1 / (1 - gamma_11) (direct-form bound)
+constexpr int TC_SLOT_T0 = 29, TC_SLOT_R = 30, TC_SLOT_T1 = 31;  // K slots of -T'0, -R, -T'1
+constexpr float TC_T_EVERY = 1.2676506002282294e30f;  // 2^100: -T' of a half row tested exactly
 
 // Byte offset of element (row, k) in a K-major, no-swizzle core-matrix tile.
 __host__ __device__ __forceinline__ uint32_t tc_offset(int row, int k) {
@@ -94,28 +129,47 @@ __device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, volatile 
     return false;
 }
 
-// 32 consecutive TMEM columns of this warp's 32 lanes (one row per thread).
-__device__ __forceinline__ void tc_ld32(uint32_t taddr, float (&v)[32]) {
-    uint32_t r[32];
+// Starts loading 32 consecutive TMEM columns of this warp's 32 lanes (one row per
+// thread) into r, and their maximum (NaN skipped, as fmaxf) into m; both are valid
+// only after tcgen05.wait::ld.
+__device__ __forceinline__ void tc_ld32_max(uint32_t taddr, uint32_t (&r)[32], float &m) {
     asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        "tcgen05.ld.red.sync.aligned.32x32b.x32.max.f32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, %32, [%33];"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
           "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
           "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]),
+          "=f"(m)
         : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+}
+
+// Orders every later use of r and m after the tcgen05.wait::ld that precedes it
+// (volatile asm statements keep their order; the "+" operands make the uses depend
+// on this one).
+__device__ __forceinline__ void tc_regs_ready(uint32_t (&r)[32], float &m) {
+    asm volatile(""
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                   "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                   "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+                   "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]),
+                   "+r"(r[29]), "+r"(r[30]), "+r"(r[31]), "+f"(m));
 }
 
 // v = hi + lo exactly, hi = v truncated to tf32 (10 explicit mantissa bits).
 __device__ __forceinline__ float tf32_hi(float v) { return __uint_as_float(__float_as_uint(v) & 0xFFFFE000u); }
 
-// Slot s of the K = 32 row layout for one operand (see top of file). `a_side`
-// selects the A pattern (x_hi, 1, x_hi, 1, x_lo) or the B pattern (c_hi, -h_hi,
-// c_lo, -h_lo, c_hi); v holds the 9 values, extra the 10th (1 for A, -h for B).
+// v rounded toward -inf to tf32 (finite v).
+__device__ __forceinline__ float tf32_rd(float v) {
+    const uint32_t u = __float_as_uint(v);
+    if ((u & 0x1FFFu) == 0u) return v;
+    return __uint_as_float(v > 0.f ? (u & 0xFFFFE000u) : (u & 0xFFFFE000u) + 0x2000u);
+}
+
+// The first 29 slots of the K = 32 row layout for one operand (see top of file).
+// `a_side` selects the A pattern (x_hi, 1, x_hi, 1, x_lo) or the B pattern (c_hi,
+// -h_hi, c_lo, -h_lo, c_hi); v holds the 9 values, extra the 10th (1 for A, -h for
+// B). The caller fills slots 29-31.
 __device__ __forceinline__ void tc_row(const float (&v)[D], float extra, bool a_side, float (&out)[TC_KD]) {
 #pragma unroll
     for (int j = 0; j < D; ++j) {
@@ -127,12 +181,11 @@ __device__ __forceinline__ void tc_row(const float (&v)[D], float extra, bool a_
     const float ehi = tf32_hi(extra);
     out[D] = a_side ? 1.f : ehi;
     out[19] = a_side ? 1.f : extra - ehi;
-    out[29] = out[30] = out[31] = 0.f;
 }
 
 // Packs C into tensor-core tiles (Kpad codewords, Kpad a multiple of TC_N) and
 // reduces the same codebook bounds as pack_codebook_kernel into hdr->cb_*.
-// Padding codewords get c = 0 and -h = -inf, so their e is -inf.
+// Padding codewords get c = 0 and -h = -inf, so their g is -inf.
 __global__ void __launch_bounds__(256) pack_codebook_tc_kernel(const float *__restrict__ C, int32_t K, int32_t Kpad,
                                                                float *__restrict__ Cpk, Header *hdr) {
     const int k = blockIdx.x * blockDim.x + threadIdx.x;
@@ -164,11 +217,14 @@ __global__ void __launch_bounds__(256) pack_codebook_tc_kernel(const float *__re
                 cmax = hmax = qmax = __int_as_float(0x7fc00000);  // NaN: disables the test
             }
         }
+        const int kl = k % TC_N;
         float v[TC_KD];
         tc_row(c, mh, false, v);
         if (!(mh >= -3.402823466e38f)) v[19] = 0.f;  // padding: -inf already sits in the hi slot
+        v[TC_SLOT_T0] = kl < TC_HALF ? 1.f : 0.f;
+        v[TC_SLOT_R] = 1.f;
+        v[TC_SLOT_T1] = kl < TC_HALF ? 0.f : 1.f;
         unsigned char *tile = reinterpret_cast<unsigned char *>(Cpk) + (int64_t)(k / TC_N) * TC_TILE_BYTES;
-        const int kl = k % TC_N;
 #pragma unroll
         for (int q = 0; q < TC_KD / 4; ++q)
             *reinterpret_cast<float4 *>(tile + tc_offset(kl, 4 * q)) =
@@ -187,9 +243,25 @@ __global__ void __launch_bounds__(256) pack_codebook_tc_kernel(const float *__re
     }
 }
 
-__device__ __forceinline__ float tc_threshold(float x2lo, float slack, float b) {
-    const float t = __fmul_rd(__fsub_rd(__fsub_rd(x2lo, slack), __fdiv_ru(b, ONE_M_G11_TC)), 0.5f);
-    return t == t ? t : __int_as_float(0xff800000);
+// Per-row constants of the test: k0 = X2lo - Qmax (rounded down), k1 = |x| Cmax +
+// Hmax + |R| (rounded up), k2 = 2 x the absolute part of E (rounded up), and R.
+struct RowConst {
+    float k0, k1, k2, R;
+};
+
+// T' for a running best b: with thr0 = (k0 - b / (1 - gamma_11)) / 2 (rounded down)
+// and dT = thr0 - R (rounded down), T' = dT - 2^-15 (k1 + |dT|) - k2 rounded down
+// to tf32. Then E(T') < thr0 - R - T' (|T'| <= (1 + 2^-9)(|dT| + margin) and
+// 2^-16 (k1 + that) stays below the margin), so R + T' + E < thr0. Returns false
+// (test every codeword) when any of it is not finite or |T'| would reach 2^100.
+__device__ __forceinline__ bool tc_shift(const RowConst &rc, float b, float &tp) {
+    const float thr0 = __fmul_rd(__fsub_rd(rc.k0, __fmul_ru(b, INV_ONE_M_G11_TC)), 0.5f);
+    const float dT = __fsub_rd(thr0, rc.R);
+    const float margin = __fadd_ru(__fmul_ru(TWO_G_TC, __fadd_ru(rc.k1, fabsf(dT))), rc.k2);
+    const float pre = __fsub_rd(dT, margin);
+    if (!(fabsf(pre) < 1.0e30f)) return false;
+    tp = tf32_rd(pre);
+    return true;
 }
 
 __device__ __forceinline__ float direct_distance(const float (&x)[D], const float *__restrict__ c) {
@@ -205,10 +277,14 @@ __device__ __forceinline__ float direct_distance(const float (&x)[D], const floa
 struct TcShared {
     unsigned char a[TC_RT][TC_A_BYTES];             // row tiles (tensor-core layout)
     unsigned char b[TC_STAGES][TC_TILE_BYTES];      // codeword tiles
-    unsigned long long full[TC_STAGES], empty[TC_STAGES], tfull[2], tempty[2], done;
+    unsigned long long full[TC_STAGES], empty[TC_STAGES], tfull[TC_RT], tempty[TC_RT], done;
     uint32_t tmem_base;
     uint32_t abort_flag;
-    double wsum[TC_EPI_WARPS];
+    float xs[TC_ROWS][D];    // the CTA's kernels and test constants, read on the
+    RowConst rc[TC_ROWS];    // rare exact path only (registers go to the tile values)
+    float pbest[TC_ROWS];    // second half's result per row, merged at the end
+    int32_t pidx[TC_ROWS];
+    double wsum[TC_EPI_WARPS / 2][TC_RT];
 };
 
 __global__ void __launch_bounds__(TC_THREADS, 1)
@@ -221,53 +297,76 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
     volatile uint32_t *abort_flag = &S.abort_flag;
     uint32_t *status = &hdr->status;
 
-    // ---- epilogue threads: own one kernel each; load it, bounds, warm start, A tile row
-    const bool epi = warp >= 2;
+    // ---- epilogue threads: one kernel in each row tile, one half of every tile
+    const bool epi = warp >= TC_EPI_WARP0;
     const int q = warp & 3;                           // TMEM lane quarter this warp may access
-    const int half = epi ? (warp - 2) / 4 : 0;        // row tile
-    const int rloc = half * TC_M + q * 32 + lane;     // row within the CTA
-    const int64_t row = (int64_t)blockIdx.x * TC_ROWS + rloc;
-    float x[D];
-    float x2lo = 0.f, slack = 0.f, best = __int_as_float(0x7f800000), thr = __int_as_float(0xff800000);
-    int32_t bi = 0;
+    const int hsel = epi ? (warp - TC_EPI_WARP0) >> 2 : 0;  // codeword half (warps 3-6: first, 7-10: second)
+    const int r = q * 32 + lane;                      // row within a row tile
+    float best[TC_RT];
+    int32_t bi[TC_RT], known[TC_RT];  // known: codeword whose exact distance is best[] (-1: none)
+    uint32_t every = 0;               // bit t: half row in row tile t tests every codeword exactly
+#pragma unroll
+    for (int t = 0; t < TC_RT; ++t) {
+        best[t] = __int_as_float(0x7f800000);
+        bi[t] = 0;
+        known[t] = -1;
+    }
     if (epi) {
 #pragma unroll
-        for (int j = 0; j < D; ++j) x[j] = row < n ? W[row * D + j] : 0.f;
-        bool ok = true;
+        for (int t = 0; t < TC_RT; ++t) {
+            const int rloc = t * TC_M + r;
+            const int64_t row = (int64_t)blockIdx.x * TC_ROWS + rloc;
+            float x[D];
 #pragma unroll
-        for (int j = 0; j < D; ++j) ok &= isfinite(x[j]);
-        if (row < n && !ok) set_flag(status, KQ_FLAG_NONFINITE);
-        const float cmax = __uint_as_float(__ldcg(&hdr->cb_cmax));
-        const float hmax = __uint_as_float(__ldcg(&hdr->cb_hmax));
-        const float qmax = __uint_as_float(__ldcg(&hdr->cb_qmax));
-        float hi = 0.f;
+            for (int j = 0; j < D; ++j) x[j] = row < n ? W[row * D + j] : 0.f;
+            bool ok = true;
 #pragma unroll
-        for (int j = 0; j < D; ++j) {
-            x2lo = __fadd_rd(x2lo, __fmul_rd(x[j], x[j]));
-            hi = __fadd_ru(hi, __fmul_ru(x[j], x[j]));
-        }
-        const float xn = __fsqrt_ru(hi);
-        slack = __fadd_ru(qmax, __fmul_ru(2.f * G_TC, __fadd_ru(hmax, __fmul_ru(xn, cmax))));
-        // absolute part: tf32 inputs below 2^-126 may be flushed to zero; each such
-        // term is below 2^-126 times the other factor
-        slack = __fadd_ru(slack, __fmul_ru(7.52316384526264e-37f /* 2^-120 */, __fadd_ru(__fadd_ru(cmax, xn), 1.f)));
-        if (hint != nullptr && row < n) {
-            const int32_t h = hint[row];
-            if ((uint32_t)h < (uint32_t)K) {
-                const float d = direct_distance(x, C + (int64_t)h * D);
-                if (d < best) {
-                    best = d;
-                    bi = h;
-                    thr = tc_threshold(x2lo, slack, d);
+            for (int j = 0; j < D; ++j) ok &= isfinite(x[j]);
+            if (row < n && !ok && hsel == 0) set_flag(status, KQ_FLAG_NONFINITE);
+            const float cmax = __uint_as_float(__ldcg(&hdr->cb_cmax));
+            const float hmax = __uint_as_float(__ldcg(&hdr->cb_hmax));
+            const float qmax = __uint_as_float(__ldcg(&hdr->cb_qmax));
+            float x2lo = 0.f, x2hi = 0.f;
+#pragma unroll
+            for (int j = 0; j < D; ++j) {
+                x2lo = __fadd_rd(x2lo, __fmul_rd(x[j], x[j]));
+                x2hi = __fadd_ru(x2hi, __fmul_ru(x[j], x[j]));
+            }
+            const float xn = __fsqrt_ru(x2hi);
+            RowConst rc;
+            rc.R = tf32_hi(0.5f * x2lo);
+            if (!(fabsf(rc.R) <= 3.402823466e38f)) rc.R = 0.f;  // any tf32 value is valid
+            rc.k0 = __fsub_rd(x2lo, qmax);
+            rc.k1 = __fadd_ru(__fadd_ru(hmax, __fmul_ru(xn, cmax)), fabsf(rc.R));
+            rc.k2 = __fmul_ru(1.504632769052528e-36f /* 2 x 2^-120 */, __fadd_ru(__fadd_ru(cmax, xn), 1.f));
+            bool ev = true;
+            float tp = 0.f;
+            if (hint != nullptr && row < n) {
+                const int32_t h = hint[row];
+                if ((uint32_t)h < (uint32_t)K) {
+                    const float d = direct_distance(x, C + (int64_t)h * D);
+                    if (d < best[t]) {
+                        best[t] = d;
+                        bi[t] = known[t] = h;
+                        ev = !tc_shift(rc, d, tp);
+                    }
                 }
             }
-        }
-        float a[TC_KD];
-        tc_row(x, 1.f, true, a);
-        const int r = q * 32 + lane;
+            every |= (ev ? 1u : 0u) << t;
+            if (hsel == 0) {  // both halves start from the same state; one writes it
 #pragma unroll
-        for (int u = 0; u < TC_KD / 4; ++u)
-            *reinterpret_cast<float4 *>(&S.a[half][tc_offset(r, 4 * u)]) = make_float4(a[4 * u], a[4 * u + 1], a[4 * u + 2], a[4 * u + 3]);
+                for (int j = 0; j < D; ++j) S.xs[rloc][j] = x[j];
+                S.rc[rloc] = rc;
+                float a[TC_KD];
+                tc_row(x, 1.f, true, a);
+                a[TC_SLOT_T0] = a[TC_SLOT_T1] = ev ? TC_T_EVERY : -tp;
+                a[TC_SLOT_R] = -rc.R;
+#pragma unroll
+                for (int u = 0; u < TC_KD / 4; ++u)
+                    *reinterpret_cast<float4 *>(&S.a[t][tc_offset(r, 4 * u)]) =
+                        make_float4(a[4 * u], a[4 * u + 1], a[4 * u + 2], a[4 * u + 3]);
+            }
+        }
     }
 
     // ---- barriers and TMEM
@@ -276,11 +375,11 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
             mbar_init((uint32_t)__cvta_generic_to_shared(&S.full[s]), 1);
             mbar_init((uint32_t)__cvta_generic_to_shared(&S.empty[s]), TC_EPI_WARPS);
         }
-        for (int b = 0; b < 2; ++b) {
-            mbar_init((uint32_t)__cvta_generic_to_shared(&S.tfull[b]), 1);
-            mbar_init((uint32_t)__cvta_generic_to_shared(&S.tempty[b]), TC_EPI_WARPS);
+        for (int t = 0; t < TC_RT; ++t) {
+            mbar_init((uint32_t)__cvta_generic_to_shared(&S.tfull[t]), 1);
+            mbar_init((uint32_t)__cvta_generic_to_shared(&S.tempty[t]), TC_EPI_WARPS);
         }
-        mbar_init((uint32_t)__cvta_generic_to_shared(&S.done), 1);
+        mbar_init((uint32_t)__cvta_generic_to_shared(&S.done), TC_RT);
         S.abort_flag = 0u;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -298,7 +397,7 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
     const uint32_t tmem = S.tmem_base;
 
     if (warp == 0) {
-        // ---- producer
+        // ---- producer (lane 0)
         if (lane == 0) {
             for (int i = 0; i < ntiles; ++i) {
                 const int s = i % TC_STAGES;
@@ -317,124 +416,179 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                     : "memory");
             }
         }
-    } else if (warp == 1) {
-        // ---- MMA issuer
+    } else if (warp <= TC_RT) {
+        // ---- MMA issuer of row tile t = warp - 1 (lane 0)
+        const int t = warp - 1;
         if (lane == 0) {
             constexpr uint32_t idesc = tc_idesc(TC_M, TC_N);
-            const uint32_t a0 = (uint32_t)__cvta_generic_to_shared(S.a[0]);
+            const uint32_t a0 = (uint32_t)__cvta_generic_to_shared(S.a[t]);
+            const uint32_t dcol = tmem + (uint32_t)(t * TC_N);
             for (int i = 0; i < ntiles; ++i) {
-                const int s = i % TC_STAGES, b = i & 1;
+                const int s = i % TC_STAGES;
                 if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.full[s]), (i / TC_STAGES) & 1, abort_flag, status))
                     break;
-                if (i >= 2 && !mbar_wait((uint32_t)__cvta_generic_to_shared(&S.tempty[b]), ((i / 2) - 1) & 1,
-                                         abort_flag, status))
+                // the accumulator is free once the epilogue read tile i - 1
+                if (i >= 1 &&
+                    !mbar_wait((uint32_t)__cvta_generic_to_shared(&S.tempty[t]), (i - 1) & 1, abort_flag, status))
                     break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t b0 = (uint32_t)__cvta_generic_to_shared(S.b[s]);
 #pragma unroll
-                for (int r = 0; r < TC_RT; ++r) {
-                    const uint32_t dcol = tmem + (uint32_t)(b * TC_RT * TC_N + r * TC_N);
-#pragma unroll
-                    for (int kb = 0; kb < TC_KD / 8; ++kb) {
-                        const uint64_t ad = tc_smem_desc(a0 + r * TC_A_BYTES + kb * 2 * TC_LBO);
-                        const uint64_t bd = tc_smem_desc(b0 + kb * 2 * TC_LBO);  // 8 tf32 of K per MMA
-                        asm volatile(
-                            "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-                            " tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}" ::"r"(dcol),
-                            "l"(ad), "l"(bd), "r"(idesc), "r"((uint32_t)kb)
-                            : "memory");
-                    }
+                for (int kb = 0; kb < TC_KD / 8; ++kb) {
+                    const uint64_t ad = tc_smem_desc(a0 + kb * 2 * TC_LBO);
+                    const uint64_t bd = tc_smem_desc(b0 + kb * 2 * TC_LBO);  // 8 tf32 of K per MMA
+                    asm volatile(
+                        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+                        " tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}" ::"r"(dcol),
+                        "l"(ad), "l"(bd), "r"(idesc), "r"((uint32_t)kb)
+                        : "memory");
                 }
+                // row tile t's values are in TMEM once these MMAs complete (the epilogue
+                // warps, which wait for that, also free the shared stage)
                 asm volatile(
                     "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                        (uint32_t)__cvta_generic_to_shared(&S.tfull[b]))
+                        (uint32_t)__cvta_generic_to_shared(&S.tfull[t]))
                     : "memory");
             }
-            // every MMA this thread issued has finished before TMEM can be freed
+            // every MMA of both issuers has finished before TMEM can be freed (warp 1
+            // frees it)
             const uint32_t db = (uint32_t)__cvta_generic_to_shared(&S.done);
             asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(db)
                          : "memory");
-            for (long long it = 0; it < TC_WAIT_LIMIT; ++it) {
-                uint32_t ok;
-                asm volatile(
-                    "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n selp.u32 %0, 1, 0, p;\n}"
-                    : "=r"(ok)
-                    : "r"(db)
-                    : "memory");
-                if (ok) break;
-                if (it + 1 == TC_WAIT_LIMIT) set_flag(status, KQ_FLAG_TIMEOUT);
+            if (t == 0) {
+                for (long long it = 0; it < TC_WAIT_LIMIT; ++it) {
+                    uint32_t ok;
+                    asm volatile(
+                        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n selp.u32 %0, 1, 0, p;\n}"
+                        : "=r"(ok)
+                        : "r"(db)
+                        : "memory");
+                    if (ok) break;
+                    if (it + 1 == TC_WAIT_LIMIT) set_flag(status, KQ_FLAG_TIMEOUT);
+                }
             }
         }
     } else {
-        // ---- epilogue: one row per thread
+        // ---- epilogue: per tile, for each row tile: load this thread's 128 values
+        // with their chunk maxima (one wait), hand the accumulator back; a chunk
+        // maximum without its sign bit means some codeword of that chunk may improve
+        // or tie the running best.
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-        for (int i = 0; i < ntiles; ++i) {
-            const int b = i & 1, st = i % TC_STAGES;
-            if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.tfull[b]), (i / 2) & 1, abort_flag, status)) break;
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            const uint32_t col0 = (uint32_t)(b * TC_RT * TC_N + half * TC_N);
-            const unsigned char *tile = S.b[st];
-#pragma unroll 1
-            for (int c = 0; c < TC_N; c += 32) {
-                float v[32];
-                tc_ld32(tmem + lane_base + col0 + (uint32_t)c, v);
-                float m0 = fmaxf(fmaxf(fmaxf(v[0], v[1]), fmaxf(v[2], v[3])), fmaxf(fmaxf(v[4], v[5]), fmaxf(v[6], v[7])));
-                float m1 = fmaxf(fmaxf(fmaxf(v[8], v[9]), fmaxf(v[10], v[11])), fmaxf(fmaxf(v[12], v[13]), fmaxf(v[14], v[15])));
-                float m2 = fmaxf(fmaxf(fmaxf(v[16], v[17]), fmaxf(v[18], v[19])), fmaxf(fmaxf(v[20], v[21]), fmaxf(v[22], v[23])));
-                float m3 = fmaxf(fmaxf(fmaxf(v[24], v[25]), fmaxf(v[26], v[27])), fmaxf(fmaxf(v[28], v[29]), fmaxf(v[30], v[31])));
-                const float m = fmaxf(fmaxf(m0, m1), fmaxf(m2, m3));
-                // A NaN test value only arises when the row's threshold is already -inf
-                // (non-finite or overflowing inputs), where every chunk takes this path.
-                if (!(m < thr)) {  // rare: some codeword of these 32 may improve or tie
-                    // candidate mask with static indexing, so v stays in registers
-                    uint32_t mask = 0u;
+        bool go = true;
+        for (int i = 0; i < ntiles && go; ++i) {
+            const int st = i % TC_STAGES;
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) mask |= (v[j] < thr) ? 0u : (1u << j);
-                    while (mask) {
-                        const int j = __ffs(mask) - 1;
-                        mask &= mask - 1u;
-                        const int kl = c + j;
-                        const int32_t k = i * TC_N + kl;
-                        if (k >= K) break;
-                        float cw[D];
+            for (int t = 0; t < TC_RT; ++t) {
+                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.tfull[t]), i & 1, abort_flag, status)) {
+                    go = false;
+                    break;
+                }
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t taddr = tmem + lane_base + (uint32_t)(t * TC_N + hsel * TC_HALF);
+                uint32_t v[4][32];
+                float cm[4];
 #pragma unroll
-                        for (int u = 0; u < D; ++u)
-                            cw[u] = *reinterpret_cast<const float *>(tile + tc_offset(kl, u)) +
-                                    *reinterpret_cast<const float *>(tile + tc_offset(kl, 10 + u));  // c_hi + c_lo = c
-                        const float d = direct_distance(x, cw);
-                        if (d < best || (d == best && k < bi)) {
-                            best = d;
-                            bi = k;
-                            thr = tc_threshold(x2lo, slack, d);
+                for (int c = 0; c < 4; ++c) tc_ld32_max(taddr + 32u * c, v[c], cm[c]);
+                asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+                for (int c = 0; c < 4; ++c) tc_regs_ready(v[c], cm[c]);
+                asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                __syncwarp();
+                if (lane == 0)
+                    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(
+                                     (uint32_t)__cvta_generic_to_shared(&S.tempty[t]))
+                                 : "memory");
+                const bool ev = (every >> t) & 1u;
+                const float m = fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3]));
+                if (!(__float_as_uint(m) >> 31) || ev) {  // rare
+                    const int rloc = t * TC_M + r;
+                    const unsigned char *tile = S.b[st];
+                    float xr[D];
+#pragma unroll
+                    for (int j = 0; j < D; ++j) xr[j] = S.xs[rloc][j];
+                    bool moved = false;
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        if ((__float_as_uint(cm[c]) >> 31) && !ev) continue;  // the whole chunk is ruled out
+                        // candidate mask with static indexing, so v stays in registers
+                        uint32_t mask = ev ? 0xffffffffu : 0u;
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) mask |= (~v[c][j] >> 31) << j;
+                        while (mask) {
+                            const int j = __ffs(mask) - 1;
+                            mask &= mask - 1u;
+                            const int kl = hsel * TC_HALF + 32 * c + j;
+                            const int32_t k = i * TC_N + kl;
+                            if (k >= K) break;
+                            if (k == known[t]) continue;  // the running best itself: nothing to decide
+                            float cw[D];
+#pragma unroll
+                            for (int u = 0; u < D; ++u)
+                                cw[u] = *reinterpret_cast<const float *>(tile + tc_offset(kl, u)) +
+                                        *reinterpret_cast<const float *>(tile + tc_offset(kl, 10 + u));  // c_hi + c_lo = c
+                            const float d = direct_distance(xr, cw);
+                            if (d < best[t] || (d == best[t] && k < bi[t])) {
+                                best[t] = d;
+                                bi[t] = known[t] = k;
+                                moved = true;
+                            }
                         }
+                    }
+                    if (moved) {
+                        float tp = 0.f;
+                        const bool e2 = !tc_shift(S.rc[rloc], best[t], tp);
+                        every = (every & ~(1u << t)) | ((e2 ? 1u : 0u) << t);
+                        *reinterpret_cast<float *>(&S.a[t][tc_offset(r, hsel ? TC_SLOT_T1 : TC_SLOT_T0)]) =
+                            e2 ? TC_T_EVERY : -tp;
+                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // for later MMAs
                     }
                 }
             }
-            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
-            if (lane == 0) {
-                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"((uint32_t)__cvta_generic_to_shared(&S.tempty[b]))
-                             : "memory");
+            if (lane == 0)
                 asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"((uint32_t)__cvta_generic_to_shared(&S.empty[st]))
                              : "memory");
-            }
         }
-        if (row < n) {
-            idx[row] = bi;
-            if (dist) dist[row] = best;
+        if (hsel == 1) {
+#pragma unroll
+            for (int t = 0; t < TC_RT; ++t) {
+                S.pbest[t * TC_M + r] = best[t];
+                S.pidx[t * TC_M + r] = bi[t];
+            }
         }
     }
 
-    // ---- objective partial sum (fixed order) and teardown
-    double sum = (epi && row < n) ? (double)best : 0.0;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    if (epi && lane == 0) S.wsum[warp - 2] = sum;
+    // ---- teardown (a CTA barrier first: see above); merge the halves (lowest index
+    // on equal distances); objective partial sum in a fixed order
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (epi && hsel == 0) {
+#pragma unroll
+        for (int t = 0; t < TC_RT; ++t) {
+            const int rloc = t * TC_M + r;
+            const int64_t row = (int64_t)blockIdx.x * TC_ROWS + rloc;
+            const float ob = S.pbest[rloc];
+            const int32_t oi = S.pidx[rloc];
+            if (ob < best[t] || (ob == best[t] && oi < bi[t])) {
+                best[t] = ob;
+                bi[t] = oi;
+            }
+            double sum = 0.0;
+            if (row < n) {
+                idx[row] = bi[t];
+                if (dist) dist[row] = best[t];
+                sum = (double)best[t];
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+            if (lane == 0) S.wsum[warp - TC_EPI_WARP0][t] = sum;
+        }
+    }
     __syncthreads();
     if (tid == 0) {
         double s = 0.0;
-        for (int w = 0; w < TC_EPI_WARPS; ++w) s += S.wsum[w];
+        for (int t = 0; t < TC_RT; ++t)
+            for (int w = 0; w < TC_EPI_WARPS / 2; ++w) s += S.wsum[w][t];
         blocksum[blockIdx.x] = s;
     }
     if (warp == 1) {
@@ -459,9 +613,10 @@ cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Heade
 cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const float *Cpk, int32_t K,
                              const int32_t *hint, int32_t *idx, float *dist, double *blocksum, int *nblocksum,
                              Header *hdr, cudaStream_t s) {
-    // More shared memory than two CTAs can share, so one CTA per SM owns all of TMEM.
-    const int smem = 120 * 1024;
-    static_assert(sizeof(TcShared) + 1024 <= 120 * 1024, "shared layout too large");
+    // One CTA per SM (it owns all of TMEM); the shared layout alone rules out a second.
+    const int smem = (int)sizeof(TcShared) + 1024;  // + alignment slack of the dynamic base
+    static_assert(sizeof(TcShared) + 1024 <= 227 * 1024, "shared layout too large");
+    static_assert(sizeof(TcShared) + 1024 > 114 * 1024, "two CTAs per SM would share TMEM");
     cudaError_t e = cudaFuncSetAttribute(assign_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const int64_t blocks = (n + TC_ROWS - 1) / TC_ROWS;

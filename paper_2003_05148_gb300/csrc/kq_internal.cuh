@@ -57,7 +57,7 @@ inline WsLayout ws_layout(int64_t n, int32_t K) {
     L.cbuf1 = off;    off = align_up(off + (size_t)K * D * 4, 256);
     L.cp = off;       off = align_up(off + (size_t)K * CP_FLOATS * 4, 256);
     L.cq = off;       off = align_up(off + (size_t)K * 8, 256);
-    L.cpk = off;      off = align_up(off + (size_t)((K + 127) / 128 * 128) * 128, 256);  // tensor-core codeword tiles
+    L.cpk = off;      off = align_up(off + (size_t)((K + 255) / 256 * 256) * 128, 256);  // tensor-core codeword tiles
     L.total = off;
     return L;
 }
