@@ -156,6 +156,19 @@ __device__ __forceinline__ void tc_regs_ready(uint32_t (&r)[32], float &m) {
                    "+r"(r[29]), "+r"(r[30]), "+r"(r[31]), "+f"(m));
 }
 
+// Bit j = sign bit of r[j]: 32 shifts, then a 5-level tree of multiply-adds (FMA
+// pipe) instead of a chain of 32 dependent ORs.
+__device__ __forceinline__ uint32_t sign_mask32(const uint32_t (&r)[32]) {
+    uint32_t s[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) s[j] = r[j] >> 31;
+#pragma unroll
+    for (int w = 1; w < 32; w *= 2)
+#pragma unroll
+        for (int j = 0; j < 32; j += 2 * w) s[j] = s[j + w] * (1u << w) + s[j];
+    return s[0];
+}
+
 // v = hi + lo exactly, hi = v truncated to tf32 (10 explicit mantissa bits).
 __device__ __forceinline__ float tf32_hi(float v) { return __uint_as_float(__float_as_uint(v) & 0xFFFFE000u); }
 
@@ -503,29 +516,29 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                 if (!(__float_as_uint(m) >> 31) || ev) {  // rare
                     const int rloc = t * TC_M + r;
                     const unsigned char *tile = S.b[st];
-                    float xr[D];
-#pragma unroll
-                    for (int j = 0; j < D; ++j) xr[j] = S.xs[rloc][j];
                     bool moved = false;
 #pragma unroll
                     for (int c = 0; c < 4; ++c) {
                         if ((__float_as_uint(cm[c]) >> 31) && !ev) continue;  // the whole chunk is ruled out
-                        // candidate mask with static indexing, so v stays in registers
-                        uint32_t mask = ev ? 0xffffffffu : 0u;
-#pragma unroll
-                        for (int j = 0; j < 32; ++j) mask |= (~v[c][j] >> 31) << j;
+                        // candidate mask with static indexing, so v stays in registers;
+                        // the running best itself needs no decision (in a warm start it
+                        // is almost always the only codeword that passes)
+                        uint32_t mask = ev ? 0xffffffffu : ~sign_mask32(v[c]);
+                        const int kloc = known[t] - (i * TC_N + hsel * TC_HALF + 32 * c);
+                        if ((uint32_t)kloc < 32u) mask &= ~(1u << kloc);
                         while (mask) {
                             const int j = __ffs(mask) - 1;
                             mask &= mask - 1u;
                             const int kl = hsel * TC_HALF + 32 * c + j;
                             const int32_t k = i * TC_N + kl;
                             if (k >= K) break;
-                            if (k == known[t]) continue;  // the running best itself: nothing to decide
-                            float cw[D];
+                            float xr[D], cw[D];
 #pragma unroll
-                            for (int u = 0; u < D; ++u)
+                            for (int u = 0; u < D; ++u) {
+                                xr[u] = S.xs[rloc][u];
                                 cw[u] = *reinterpret_cast<const float *>(tile + tc_offset(kl, u)) +
                                         *reinterpret_cast<const float *>(tile + tc_offset(kl, 10 + u));  // c_hi + c_lo = c
+                            }
                             const float d = direct_distance(xr, cw);
                             if (d < best[t] || (d == best[t] && k < bi[t])) {
                                 best[t] = d;
