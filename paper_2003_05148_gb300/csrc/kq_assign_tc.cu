@@ -513,17 +513,21 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                                  : "memory");
                 const bool ev = (every >> t) & 1u;
                 const float m = fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3]));
-                if (!(__float_as_uint(m) >> 31) || ev) {  // rare
+                // Warp-uniform branches (votes) around the rare work: a lane-divergent
+                // condition lets the compiler predicate all four chunks' mask builds
+                // into every entry.
+                if (__any_sync(0xffffffffu, !(__float_as_uint(m) >> 31) || ev)) {  // rare
                     const int rloc = t * TC_M + r;
                     const unsigned char *tile = S.b[st];
                     bool moved = false;
 #pragma unroll
                     for (int c = 0; c < 4; ++c) {
-                        if ((__float_as_uint(cm[c]) >> 31) && !ev) continue;  // the whole chunk is ruled out
+                        const bool need = ev || !(__float_as_uint(cm[c]) >> 31);
+                        if (!__any_sync(0xffffffffu, need)) continue;  // the whole chunk is ruled out in every lane
                         // candidate mask with static indexing, so v stays in registers;
                         // the running best itself needs no decision (in a warm start it
                         // is almost always the only codeword that passes)
-                        uint32_t mask = ev ? 0xffffffffu : ~sign_mask32(v[c]);
+                        uint32_t mask = !need ? 0u : (ev ? 0xffffffffu : ~sign_mask32(v[c]));
                         const int kloc = known[t] - (i * TC_N + hsel * TC_HALF + 32 * c);
                         if ((uint32_t)kloc < 32u) mask &= ~(1u << kloc);
                         while (mask) {
