@@ -467,6 +467,67 @@ def run_only(args):
         sys.exit(1)
 
 
+def run_configs(args):
+    """Every configuration (the five seeded workloads) through the public API on one
+    GPU: per layer kq_init_codebook + kq_fit_codebook (the workload's iteration
+    count) + kq_quantize_codebook_6bit + K+C kq_reconstruct, inputs resident in HBM,
+    CUDA events around `reps` runs of the whole workload after one untimed run.
+    Prints one JSON line per configuration (a report, not the bench line)."""
+    import torch
+
+    from paper_2003_05148_gb300 import build, kq
+
+    build.build()
+    dev = torch.device("cuda", 0)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    for cfg in [int(c) for c in args.configs.split(",")]:
+        wl = synth.workload(cfg)
+        T = wl.iters
+        layers = []
+        for lay in wl.layers:
+            W_h, sel_h = synth.layer_inputs(lay)
+            n, K = W_h.shape[0], lay.K
+            layers.append({
+                "n": n, "K": K,
+                "W": torch.from_numpy(W_h).to(dev), "sel": torch.from_numpy(sel_h).to(dev),
+                "ws": kq.workspace(n, K, dev),
+                "Ca": torch.empty(K, 9, dtype=torch.float32, device=dev),
+                "Cb": torch.empty(K, 9, dtype=torch.float32, device=dev),
+                "idx": torch.empty(n, dtype=torch.int32, device=dev),
+                "counts": torch.empty(K, dtype=torch.int32, device=dev),
+                "obj": torch.empty(T + 1, dtype=torch.float64, device=dev),
+                "levels": torch.empty(64, dtype=torch.float32, device=dev),
+                "codes": torch.empty(K, 9, dtype=torch.uint8, device=dev),
+                "Wr": torch.empty(n, 9, dtype=torch.float32, device=dev)})
+
+        def run_all():
+            for L in layers:
+                kq.kq_init_codebook(L["W"], L["sel"], L["Ca"], L["ws"])
+                kq.kq_fit_codebook(L["W"], L["Ca"], T, L["Cb"], L["idx"], L["counts"], L["obj"], L["ws"])
+                kq.kq_quantize_codebook_6bit(L["Cb"], L["counts"], 100, L["levels"], L["codes"], None, L["ws"])
+                kq.kq_reconstruct(L["idx"], None, L["codes"], L["levels"], L["Wr"], L["ws"], K=L["K"])
+
+        run_all()
+        torch.cuda.synchronize()
+        stream = torch.cuda.current_stream()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        launches0 = kq.kq_kernel_launches()
+        e0.record(stream)
+        for _ in range(args.reps):
+            run_all()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / args.reps
+        statuses = [kq.kq_device_status(L["ws"]) for L in layers]
+        evals = sum((T + 1) * L["n"] * L["K"] for L in layers)
+        print(json.dumps({
+            "config": wl.name, "layers": len(layers), "kernels": sum(L["n"] for L in layers),
+            "codewords": sum(L["K"] for L in layers), "iters": T, "evals": evals, "ms_per_run": ms,
+            "evals_per_s": evals / (ms / 1e3), "tensor_core_assign_layers": sum(L["n"] >= 256 * sms for L in layers),
+            "gpu_launches_per_run": (kq.kq_kernel_launches() - launches0) // args.reps,
+            "status": max(st for st, _ in statuses), "reps": args.reps}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -482,9 +543,14 @@ def main():
     ap.add_argument("--K", type=int, default=65536)
     ap.add_argument("--reps", type=int, default=3)
     ap.add_argument("--hint", action="store_true", help="with --only assign: warm start as in a fit")
+    ap.add_argument("--configs", default=None,
+                    help="report aid: fit the listed workloads (e.g. 1,2,3,4,5) end to end, one line each")
     args = ap.parse_args()
     if args.only:
         run_only(args)
+        return
+    if args.configs:
+        run_configs(args)
         return
     if args.warmup < 3:
         print("warning: fewer than 3 warm-up steps", file=sys.stderr)
