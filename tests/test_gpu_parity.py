@@ -150,13 +150,22 @@ def test_assign_tensor_core_path(case):
 
 def test_assign_paths_agree():
     # the same kernels through the tensor-core path (large n) and the CUDA-core
-    # path (small n) give bit-identical results
-    W = synth.random_kernels(TC_MIN_N + 5000, 9, 211, 0.05)
+    # path (small n) give bit-identical results; n spans several row blocks per
+    # SM and a ragged last block, cold and warm-started
+    n = 5 * TC_MIN_N + 333
+    W = synth.random_kernels(n, 9, 211, 0.05)
     C = synth.random_kernels(2000, 9, 212, 0.05)
     i_tc, d_tc, st1, _ = gpu_assign(W, C)
-    i_cc, d_cc, st2, _ = gpu_assign(W[:20000], C)
-    assert st1 == 0 and st2 == 0
-    assert np.array_equal(i_tc[:20000], i_cc) and bits_equal(d_tc[:20000], d_cc)
+    assert st1 == 0
+    for sl in (slice(0, 20000), slice(n - 20000, n)):
+        i_cc, d_cc, st2, _ = gpu_assign(W[sl], C)
+        assert st2 == 0
+        assert np.array_equal(i_tc[sl], i_cc) and bits_equal(d_tc[sl], d_cc)
+    hint = synth.below(synth.stream_key(213, 9), n, 2000).astype(np.int32)
+    hint[::3] = i_tc[::3]
+    i_w, d_w, st3, _ = gpu_assign(W, C, hint=hint)
+    assert st3 == 0
+    assert np.array_equal(i_w, i_tc) and bits_equal(d_w, d_tc)
 
 
 def test_assign_hint_never_changes_result():
