@@ -68,6 +68,12 @@ def _bind(lib):
         lib.kqo_encode.restype = None
         lib.kqo_gather_rows.argtypes = [P, P, i32, P]
         lib.kqo_gather_rows.restype = None
+        lib.kqo_level_fit_scalars.argtypes = [P, i64, i32, P, P]
+        lib.kqo_level_fit_scalars.restype = i32
+        lib.kqo_codebook_grad_step.argtypes = [P, i64, P, i32, ctypes.c_float, P, P, P]
+        lib.kqo_codebook_grad_step.restype = None
+        lib.kqo_levels_grad_step.argtypes = [P, i64, P, i32, P, ctypes.c_float, P, P, P]
+        lib.kqo_levels_grad_step.restype = None
     return lib
 
 
@@ -165,6 +171,40 @@ def level_fit(C, counts, max_iters: int = 100):
     codes = np.empty((K, D), np.uint8)
     it = _load().kqo_level_fit(_ptr(C), K, _ptr(counts), max_iters, _ptr(levels), _ptr(codes))
     return levels, codes, int(it)
+
+
+def level_fit_scalars(values, max_iters: int = 100):
+    """Sec. 3.2 6-bit quantisation of a fully-connected layer (every scalar weighted 1).
+
+    Returns (levels fp32 (64,), codes uint8 (m,), updates)."""
+    v = _f32(values).reshape(-1)
+    levels = np.empty(LEVELS, np.float32)
+    codes = np.empty(v.shape[0], np.uint8)
+    it = _load().kqo_level_fit_scalars(_ptr(v), v.shape[0], max_iters, _ptr(levels), _ptr(codes))
+    return levels, codes, int(it)
+
+
+def codebook_grad_step(G, idx, C, lr: float):
+    """Eq. 2 (Sec. 3.1): c_k - lr * mean of the gradients of S_k. Returns (C_next, counts)."""
+    G, C, idx = _f32(G).reshape(-1, D), _f32(C).reshape(-1, D), _i32(idx)
+    K = C.shape[0]
+    C_next = np.empty_like(C)
+    counts = np.empty(K, np.int32)
+    _load().kqo_codebook_grad_step(_ptr(G), G.shape[0], _ptr(idx), K, float(lr), _ptr(C), _ptr(C_next), _ptr(counts))
+    return C_next, counts
+
+
+def levels_grad_step(G, idx, codes, levels, lr: float):
+    """Sec. 3.2 retraining of the 6-bit levels with averaged gradients.
+
+    Returns (levels_next fp32 (64,), counts int64 (64,))."""
+    G, idx, levels = _f32(G).reshape(-1, D), _i32(idx), _f32(levels)
+    codes = np.ascontiguousarray(codes, dtype=np.uint8).reshape(-1, D)
+    nxt = np.empty(LEVELS, np.float32)
+    counts = np.empty(LEVELS, np.int64)
+    _load().kqo_levels_grad_step(_ptr(G), G.shape[0], _ptr(idx), codes.shape[0], _ptr(codes), float(lr),
+                                 _ptr(levels), _ptr(nxt), _ptr(counts))
+    return nxt, counts
 
 
 def encode(values, levels):

@@ -17,6 +17,15 @@
  *                       appearance count z_k; then the 6-bit code of every scalar.
  *   - kqo_reconstruct   Sec. 3.2 (testing phase): recover the codebook from the
  *                       codes, then W from the kernel indices.
+ *   - kqo_codebook_grad_step  Sec. 3.1, Eq. 2: retraining step of the codebook
+ *                       with the element-wise average of the gradients of the
+ *                       kernels mapped to each entry.
+ *   - kqo_levels_grad_step    Sec. 3.2: the same averaged-gradient step for the
+ *                       64 levels of the quantised codebook (average over every
+ *                       weight whose value is that level).
+ *   - kqo_level_fit_scalars   Sec. 3.2 (last step): 6-bit quantisation of a
+ *                       fully-connected layer, the same k-means with weight 1 per
+ *                       scalar.
  *
  * Readings where the paper is silent (each is also listed in the design notes):
  *   - Distance arithmetic: fp32, t_j = fl(x_j - c_j), acc = fmaf(t_j, t_j, acc)
@@ -35,6 +44,13 @@
  *     where A*M = f * 2^e, f in [0.5, 1), A = total weight, M = max |v| over
  *     weighted scalars); an empty level keeps its value; stop when no code
  *     changes or after max_iters updates.
+ *   - Averaged-gradient steps (Eq. 2): the mean gradient is the fp64 sum in
+ *     ascending element order divided by the member count in fp64, rounded once
+ *     to fp32; then step = fl32(lr * mean) and the new value = fl32(old - step).
+ *     An entry (codeword or level) with no members keeps its value. A kernel
+ *     whose index is outside [0, K) contributes nothing.
+ *   - Fully-connected 6-bit quantisation: the level fit above with every scalar
+ *     weighted 1.
  *
  * Build: gcc -O2 -ffp-contract=off -fno-fast-math -fPIC -shared -pthread
  *        kq_oracle.c -o libkq_oracle.so -lm
@@ -218,15 +234,19 @@ static int nearest_level(float v, const float *levels) {
     return bl;
 }
 
-/* Fixed-point scale exponent S for the exact weighted sums (see header). */
-int32_t kqo_level_scale(const float *C, int32_t K, const int32_t *counts) {
+/* Weight of scalar m in a level fit: w[m / group] when weights are given, else 1. */
+static int64_t scalar_weight(const int32_t *w, int64_t group, int64_t m) { return w ? (int64_t)w[m / group] : 1; }
+
+/* Fixed-point scale exponent S for the exact weighted sums (see header): N scalars,
+ * weight of scalar m from scalar_weight. */
+static int32_t level_scale_w(const float *v, int64_t N, const int32_t *w, int64_t group) {
     int64_t A = 0;
     float M = 0.0f;
-    for (int64_t m = 0; m < (int64_t)K * KQO_D; ++m) {
-        int32_t z = counts[m / KQO_D];
+    for (int64_t m = 0; m < N; ++m) {
+        int64_t z = scalar_weight(w, group, m);
         if (z > 0) {
             A += z;
-            float a = fabsf(C[m]);
+            float a = fabsf(v[m]);
             if (a > M) M = a;
         }
     }
@@ -236,37 +256,40 @@ int32_t kqo_level_scale(const float *C, int32_t K, const int32_t *counts) {
     return 62 - e;
 }
 
-/* Weighted 64-level k-means over the K*9 codebook scalars; writes the 64 levels
- * and the 6-bit code of each scalar. Returns the number of level updates made. */
-int32_t kqo_level_fit(const float *C, int32_t K, const int32_t *counts, int32_t max_iters, float *levels,
-                      uint8_t *codes) {
-    const int64_t N = (int64_t)K * KQO_D;
+int32_t kqo_level_scale(const float *C, int32_t K, const int32_t *counts) {
+    return level_scale_w(C, (int64_t)K * KQO_D, counts, KQO_D);
+}
+
+/* Weighted 64-level k-means over N scalars (Sec. 3.2); writes the 64 levels and
+ * the 6-bit code of each scalar. Returns the number of level updates made. */
+static int32_t level_fit_w(const float *v, int64_t N, const int32_t *w, int64_t group, int32_t max_iters,
+                           float *levels, uint8_t *codes) {
     /* initial levels: linspace(min, max, 64) over weighted scalars */
     int any = 0;
-    for (int64_t m = 0; m < N; ++m) any |= counts[m / KQO_D] > 0;
+    for (int64_t m = 0; m < N; ++m) any |= scalar_weight(w, group, m) > 0;
     float lo = INFINITY, hi = -INFINITY;
     for (int64_t m = 0; m < N; ++m) {
-        if (any && counts[m / KQO_D] <= 0) continue;
-        if (C[m] < lo) lo = C[m];
-        if (C[m] > hi) hi = C[m];
+        if (any && scalar_weight(w, group, m) <= 0) continue;
+        if (v[m] < lo) lo = v[m];
+        if (v[m] > hi) hi = v[m];
     }
     for (int l = 0; l < KQO_LEVELS; ++l)
         levels[l] = (float)((double)lo + ((double)hi - (double)lo) * (double)l / 63.0);
 
-    const int32_t S = kqo_level_scale(C, K, counts);
+    const int32_t S = level_scale_w(v, N, w, group);
     const double up = ldexp(1.0, S), down = ldexp(1.0, -S);
     int64_t *q = (int64_t *)malloc((size_t)(N > 0 ? N : 1) * sizeof(int64_t));
-    for (int64_t m = 0; m < N; ++m) q[m] = llrint((double)C[m] * up);
+    for (int64_t m = 0; m < N; ++m) q[m] = llrint((double)v[m] * up);
 
     uint8_t *prev = (uint8_t *)malloc((size_t)(N > 0 ? N : 1));
     uint8_t *cur = (uint8_t *)malloc((size_t)(N > 0 ? N : 1));
     int32_t updates = 0;
     for (int32_t it = 0; it < max_iters; ++it) {
-        for (int64_t m = 0; m < N; ++m) cur[m] = (uint8_t)nearest_level(C[m], levels);
+        for (int64_t m = 0; m < N; ++m) cur[m] = (uint8_t)nearest_level(v[m], levels);
         if (it > 0 && memcmp(cur, prev, (size_t)N) == 0) break;
         int64_t wsum[KQO_LEVELS] = {0}, qsum[KQO_LEVELS] = {0};
         for (int64_t m = 0; m < N; ++m) {
-            int64_t z = counts[m / KQO_D];
+            int64_t z = scalar_weight(w, group, m);
             if (z <= 0) continue;
             wsum[cur[m]] += z;
             qsum[cur[m]] += z * q[m];
@@ -276,11 +299,23 @@ int32_t kqo_level_fit(const float *C, int32_t K, const int32_t *counts, int32_t 
         memcpy(prev, cur, (size_t)N);
         ++updates;
     }
-    for (int64_t m = 0; m < N; ++m) codes[m] = (uint8_t)nearest_level(C[m], levels);
+    for (int64_t m = 0; m < N; ++m) codes[m] = (uint8_t)nearest_level(v[m], levels);
     free(q);
     free(prev);
     free(cur);
     return updates;
+}
+
+/* Sec. 3.2 codebook quantisation: the K*9 codebook scalars, each weighted by its
+ * entry's appearance count z_k. */
+int32_t kqo_level_fit(const float *C, int32_t K, const int32_t *counts, int32_t max_iters, float *levels,
+                      uint8_t *codes) {
+    return level_fit_w(C, (int64_t)K * KQO_D, counts, KQO_D, max_iters, levels, codes);
+}
+
+/* Sec. 3.2 fully-connected layers: m scalars, each weighted 1. */
+int32_t kqo_level_fit_scalars(const float *v, int64_t m, int32_t max_iters, float *levels, uint8_t *codes) {
+    return level_fit_w(v, m, NULL, 1, max_iters, levels, codes);
 }
 
 /* Sec. 3.2 testing phase: W'_i = decoded codebook row idx_i. With codes == NULL
@@ -302,4 +337,72 @@ void kqo_gather_rows(const float *W, const int64_t *sel, int32_t K, float *C0) {
 /* Sec. 3.2 encode: the 6-bit code (nearest level) of each of m values. */
 void kqo_encode(const float *v, int64_t m, const float *levels, uint8_t *codes) {
     for (int64_t i = 0; i < m; ++i) codes[i] = (uint8_t)nearest_level(v[i], levels);
+}
+
+/* ---------------------------------------------------------------------------
+ * Retraining with averaged gradients: Sec. 3.1 Eq. 2 and its use for the
+ * quantised codebook in Sec. 3.2.
+ * ------------------------------------------------------------------------- */
+
+/* Eq. 2: every kernel i mapped to entry k (idx[i] == k, the set S_k) has a loss
+ * gradient g_i = dL/dm_i (9 floats, row i of G); the entry moves against their
+ * element-wise average:  c_k <- c_k - lr * (1 / z_k) * sum_{i in S_k} g_i,  z_k = |S_k|.
+ * counts[k] receives z_k; an entry with z_k = 0 keeps its value. */
+void kqo_codebook_grad_step(const float *G, int64_t n, const int32_t *idx, int32_t K, float lr, const float *C,
+                            float *C_next, int32_t *counts) {
+    double *sum = (double *)calloc((size_t)K * KQO_D, sizeof(double));
+    int64_t *z = (int64_t *)calloc((size_t)K, sizeof(int64_t));
+    for (int64_t i = 0; i < n; ++i) {
+        int32_t k = idx[i];
+        if (k < 0 || k >= K) continue;
+        z[k] += 1;
+        for (int j = 0; j < KQO_D; ++j) sum[(int64_t)k * KQO_D + j] += (double)G[i * KQO_D + j];
+    }
+    for (int32_t k = 0; k < K; ++k) {
+        for (int j = 0; j < KQO_D; ++j) {
+            int64_t e = (int64_t)k * KQO_D + j;
+            if (z[k] > 0) {
+                float mean = (float)(sum[e] / (double)z[k]);
+                float step = lr * mean;
+                C_next[e] = C[e] - step;
+            } else {
+                C_next[e] = C[e];
+            }
+        }
+        counts[k] = (int32_t)z[k];
+    }
+    free(sum);
+    free(z);
+}
+
+/* Sec. 3.2 retraining of the quantised codebook: the weights of the network are
+ * W'_ij = levels[codes[idx_i][j]], so level l moves against the average gradient
+ * of every weight whose value it is:
+ *   levels[l] <- levels[l] - lr * mean{ G_ij : codes[idx_i * 9 + j] == l }.
+ * counts[l] receives the number of such weights; a level with none keeps its value.
+ * A kernel whose index is outside [0, K) contributes nothing. */
+void kqo_levels_grad_step(const float *G, int64_t n, const int32_t *idx, int32_t K, const uint8_t *codes, float lr,
+                          const float *levels, float *levels_next, int64_t *counts) {
+    double sum[KQO_LEVELS] = {0};
+    int64_t z[KQO_LEVELS] = {0};
+    for (int64_t i = 0; i < n; ++i) {
+        int32_t k = idx[i];
+        if (k < 0 || k >= K) continue;
+        for (int j = 0; j < KQO_D; ++j) {
+            int l = codes[(int64_t)k * KQO_D + j];
+            if (l >= KQO_LEVELS) continue;
+            z[l] += 1;
+            sum[l] += (double)G[i * KQO_D + j];
+        }
+    }
+    for (int l = 0; l < KQO_LEVELS; ++l) {
+        if (z[l] > 0) {
+            float mean = (float)(sum[l] / (double)z[l]);
+            float step = lr * mean;
+            levels_next[l] = levels[l] - step;
+        } else {
+            levels_next[l] = levels[l];
+        }
+        counts[l] = z[l];
+    }
 }

@@ -341,6 +341,132 @@ def test_level_scale_bounds():
 
 
 # ---------------------------------------------------------------------------
+# Sec. 3.2 (last step): 6-bit quantisation of a fully-connected layer.
+# ---------------------------------------------------------------------------
+
+def test_level_fit_scalars_equally_spaced_is_fixed_point():
+    # 64 distinct integers plus repeats, m not a multiple of 9: linspace init hits
+    # every value, nothing moves and every scalar keeps its own level.
+    v = np.concatenate([np.arange(64), [5, 5, 63, 0, 17]]).astype(np.float32)
+    levels, codes, it = oracle.level_fit_scalars(v)
+    assert np.array_equal(levels, np.arange(64, dtype=np.float32))
+    assert np.array_equal(codes, v.astype(np.uint8))
+    assert it == 1
+
+
+def test_level_fit_scalars_converged_levels_are_means():
+    # unit weights: every converged level is the exact (unweighted) mean of its
+    # scalars, and every scalar sits at its nearest level.
+    rng = np.random.default_rng(17)
+    v = (rng.standard_normal(1001) * 512).round().astype(np.float32) / np.float32(4096)
+    levels, codes, it = oracle.level_fit_scalars(v, max_iters=200)
+    assert it < 200
+    assert np.all(np.diff(levels) >= 0)
+    for l in np.unique(codes):
+        m = codes == l
+        exact = sum(Fraction(float(a)) for a in v[m]) / int(m.sum())
+        assert _f32_ulps(levels[l], np.float32(float(exact))) <= 1
+    for x, c in zip(v, codes):
+        d = [abs(Fraction(float(x)) - Fraction(float(L))) for L in levels]
+        assert c == d.index(min(d))
+
+
+def test_level_fit_scalars_is_unit_weight_codebook_fit():
+    # the same scalars as a K x 9 codebook with every count 1 give the same fit
+    v = synth.random_kernels(70, 9, 81, 0.05).reshape(-1)
+    lv1, cd1, it1 = oracle.level_fit_scalars(v)
+    lv2, cd2, it2 = oracle.level_fit(v.reshape(-1, 9), np.ones(70, np.int32))
+    assert np.array_equal(lv1.view(np.int32), lv2.view(np.int32)) and it1 == it2
+    assert np.array_equal(cd1, cd2.reshape(-1))
+
+
+# ---------------------------------------------------------------------------
+# Retraining with averaged gradients: Eq. 2 (Sec. 3.1) and Sec. 3.2.
+# ---------------------------------------------------------------------------
+
+def test_codebook_grad_step_dyadic_bit_exact():
+    # Values on a 2^-10 grid: the fp64 member sums are exact, so the mean rounds
+    # once (as the exact rational rounded to fp32); then step = fl32(lr * mean)
+    # and c - step in fp32. lr = 0.375 is not a power of two.
+    rng = np.random.default_rng(5)
+    n, K = 301, 7
+    G = (rng.integers(-2048, 2048, size=(n, 9)) / 1024.0).astype(np.float32)
+    C = (rng.integers(-512, 512, size=(K, 9)) / 256.0).astype(np.float32)
+    idx = rng.integers(0, K - 1, size=n).astype(np.int32)  # codeword K-1 stays empty
+    idx[:3] = [-1, K, 2 ** 30]  # out of range: contribute nothing
+    lr = np.float32(0.375)
+    C_next, counts = oracle.codebook_grad_step(G, idx, C, lr)
+    for k in range(K):
+        m = idx == k
+        assert counts[k] == int(m.sum())
+        if not m.any():
+            assert np.array_equal(C_next[k].view(np.int32), C[k].view(np.int32))
+            continue
+        for j in range(9):
+            exact = sum(Fraction(float(g)) for g in G[m, j]) / int(m.sum())
+            mean = np.float32(float(exact))
+            assert C_next[k, j] == np.float32(C[k, j] - np.float32(lr * mean))
+
+
+def test_codebook_grad_step_quadratic_loss_gives_the_centroid():
+    # With L = 1/2 sum_i ||W'_i - W_i||^2 and W'_i = c_{idx_i}, dL/dW'_i = c_{idx_i} - W_i;
+    # one Eq. 2 step with lr = 1 then lands on the mean of S_k: the Eq. 1 update.
+    W = synth.random_kernels(400, 9, 91, 0.1)
+    C = synth.random_kernels(12, 9, 92, 0.1)
+    idx, _ = oracle.assign(W, C)
+    G = (C[idx] - W).astype(np.float32)
+    C_next, counts = oracle.codebook_grad_step(G, idx, C, 1.0)
+    C_upd, counts_upd = oracle.update(W, idx, C)
+    assert np.array_equal(counts, counts_upd)
+    scale = np.abs(C).max() + np.abs(W).max()
+    assert np.abs(C_next - C_upd).max() <= 4 * scale * 2.0 ** -24
+    # lr = 0 leaves the codebook unchanged, bit for bit
+    C0, _ = oracle.codebook_grad_step(G, idx, C, 0.0)
+    assert np.array_equal(C0.view(np.int32), C.view(np.int32))
+
+
+def test_levels_grad_step_dyadic_bit_exact():
+    rng = np.random.default_rng(6)
+    n, K = 211, 13
+    G = (rng.integers(-4096, 4096, size=(n, 9)) / 2048.0).astype(np.float32)
+    idx = rng.integers(0, K, size=n).astype(np.int32)
+    idx[5] = -3
+    codes = rng.integers(0, 40, size=(K, 9)).astype(np.uint8)  # levels 40..63 stay empty
+    levels = (np.arange(64) / 8.0 - 3.0).astype(np.float32)
+    lr = np.float32(0.625)
+    nxt, counts = oracle.levels_grad_step(G, idx, codes, levels, lr)
+    sums = [Fraction(0)] * 64
+    z = [0] * 64
+    for i in range(n):
+        if not 0 <= idx[i] < K:
+            continue
+        for j in range(9):
+            l = int(codes[idx[i], j])
+            sums[l] += Fraction(float(G[i, j]))
+            z[l] += 1
+    for l in range(64):
+        assert counts[l] == z[l]
+        if z[l] == 0:
+            assert nxt[l] == levels[l]
+        else:
+            mean = np.float32(float(sums[l] / z[l]))
+            assert nxt[l] == np.float32(levels[l] - np.float32(lr * mean))
+    assert counts.sum() == 9 * int(((idx >= 0) & (idx < K)).sum())
+
+
+def test_levels_grad_step_constant_gradient_shifts_every_used_level():
+    W = synth.random_kernels(500, 9, 93, 0.05)
+    C = synth.random_kernels(40, 9, 94, 0.05)
+    idx, _ = oracle.assign(W, C)
+    levels, codes, _ = oracle.level_fit(C, np.bincount(idx, minlength=40).astype(np.int32))
+    G = np.full((500, 9), np.float32(0.0390625), np.float32)
+    nxt, counts = oracle.levels_grad_step(G, idx, codes, levels, 2.0)
+    used = counts > 0
+    assert np.array_equal(nxt[used], (levels[used] - np.float32(0.078125)).astype(np.float32))
+    assert np.array_equal(nxt[~used], levels[~used])
+
+
+# ---------------------------------------------------------------------------
 # Sec. 3.2 testing phase: reconstruction.
 # ---------------------------------------------------------------------------
 
