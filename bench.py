@@ -448,6 +448,24 @@ def run_only(args):
         "quantize": lambda: kq.kq_quantize_codebook_6bit(C2, counts, 100, levels, codes, None, ws),
         "reconstruct": lambda: kq.kq_reconstruct(idx, None, codes, levels, Wr, ws, K=K),
     }
+    # retraining steps (Eq. 2; Sec. 3.2): the kernels themselves stand in for the
+    # gradients (the timing depends on sizes and the code distribution only)
+    lv_next = torch.empty(64, dtype=torch.float32, device=dev)
+    lv_counts = torch.empty(64, dtype=torch.int64, device=dev)
+    calls["gradstep"] = lambda: kq.kq_codebook_grad_step(W, idx, 0.01, C2, C, counts, ws)
+    calls["levelgrad"] = lambda: kq.kq_levels_grad_step(W, idx, codes, 0.01, levels, lv_next, lv_counts, ws)
+    alg_bytes = {"update": 40 * n + 76 * K, "gradstep": 40 * n + 76 * K, "levelgrad": 40 * n + 9 * K,
+                 "reconstruct": 40 * n + 9 * K + 256}
+    if args.only == "fcquant":
+        # 6-bit quantisation of a fully-connected weight of m scalars (He-scaled
+        # Gaussian, seeded), 100 iterations at most
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(WORKLOAD_CFG * 1000 + 7)
+        v = torch.randn(args.m, generator=gen, device=dev) * float(np.sqrt(2.0 / 4096))
+        fc_codes = torch.empty(args.m, dtype=torch.uint8, device=dev)
+        fc_it = torch.zeros(1, dtype=torch.int32, device=dev)
+        calls["fcquant"] = lambda: kq.kq_quantize_scalars_6bit(v, 100, levels, fc_codes, fc_it, ws)
+        n, K = args.m, 64
     f = calls[args.only]
     for _ in range(2):
         f()
@@ -461,8 +479,16 @@ def run_only(args):
     torch.cuda.synchronize()
     st, flags = kq.kq_device_status(ws)
     ms = [a.elapsed_time(b) for a, b in evs]
-    print(json.dumps({"only": args.only, "n": n, "K": K, "reps": args.reps, "ms_mean": statistics.mean(ms),
-                      "ms_min": min(ms), "status": st, "flags": flags}), flush=True)
+    out = {"only": args.only, "n": n, "K": K, "reps": args.reps, "ms_mean": statistics.mean(ms),
+           "ms_min": min(ms), "status": st, "flags": flags}
+    if args.only in alg_bytes:
+        out["alg_bytes"] = alg_bytes[args.only]
+        out["GB_s_at_min"] = alg_bytes[args.only] / (min(ms) * 1e-3) / 1e9
+    if args.only == "fcquant":
+        it = int(fc_it.item())
+        out["iters_run"] = it
+        out["ms_per_iter"] = min(ms) / max(it, 1)
+    print(json.dumps(out), flush=True)
     if st != 0:
         sys.exit(1)
 
@@ -537,10 +563,12 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--ref-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--only", choices=["assign", "update", "quantize", "reconstruct"],
+    ap.add_argument("--only", choices=["assign", "update", "quantize", "reconstruct", "gradstep", "levelgrad",
+                                       "fcquant"],
                     help="profiling aid: time one entry point on its own (no bench line)")
     ap.add_argument("--n", type=int, default=4194304)
     ap.add_argument("--K", type=int, default=65536)
+    ap.add_argument("--m", type=int, default=25088 * 4096, help="with --only fcquant: scalars (VGG-16 fc6)")
     ap.add_argument("--reps", type=int, default=3)
     ap.add_argument("--hint", action="store_true", help="with --only assign: warm start as in a fit")
     ap.add_argument("--configs", default=None,

@@ -192,6 +192,55 @@ kq_status kq_quantize_codebook_6bit(const float *C, int32_t K, const int32_t *co
                                     float *levels, uint8_t *codes, int32_t *iters_run, void *ws, size_t ws_bytes,
                                     kq_stream_t stream);
 
+/* 6-bit quantisation of a fully-connected layer, Sec. 3.2 (last step: after the
+ * codebooks, the fully-connected layers get the same layer-by-layer k-means):
+ * the rules of kq_quantize_codebook_6bit over m scalars with every weight 1.
+ *   v          m fp32 (device; e.g. the flattened FC weight), 1 <= m <= 2^40
+ *   max_iters  0 .. 100000
+ *   levels     64 fp32 output (device);  codes m uint8 output (device)
+ *   iters_run  1 int32 output (device) or NULL
+ * Uses only the first 4096 bytes of the workspace (ws_bytes >= 4096). Bounded
+ * grid barriers as in kq_quantize_codebook_6bit. */
+kq_status kq_quantize_scalars_6bit(const float *v, int64_t m, int32_t max_iters, float *levels, uint8_t *codes,
+                                   int32_t *iters_run, void *ws, size_t ws_bytes, kq_stream_t stream);
+
+/* Codebook retraining step, Sec. 3.1 Eq. 2: with G the loss gradients of the
+ * (reconstructed) kernels, G_i = dL/dm_i, every entry moves against the
+ * element-wise average gradient of the kernels mapped to it:
+ *   counts[k] = z_k = #{ i : idx[i] == k },
+ *   C_next[k] = C[k] - lr * (1 / z_k) * sum_{i in S_k} G_i   if z_k > 0, else C[k].
+ * The sums are the exact int64 fixed-point sums of kq_update_centroids (scale
+ * from max|G|); mean -> fp32 as there, then step = fl(lr * mean) and
+ * C_next = fl(C - step).
+ *   G       n x 9 fp32 (device, 16-byte aligned);  idx  n int32 (device)
+ *   lr      finite learning rate (the paper's gamma)
+ *   C       K x 9 fp32 (device);  C_next K x 9 fp32 output (device, may equal C)
+ *   counts  K int32 output (device)
+ * An index outside [0, K) is skipped and sets KQ_FLAG_INDEX_RANGE; a non-finite
+ * gradient sets KQ_FLAG_NONFINITE. Needs the full workspace of (n, K). */
+kq_status kq_codebook_grad_step(const float *G, int64_t n, const int32_t *idx, int32_t K, float lr, const float *C,
+                                float *C_next, int32_t *counts, void *ws, size_t ws_bytes, kq_stream_t stream);
+
+/* Retraining step of the quantised codebook, Sec. 3.2 ("Retraining of codebook
+ * quantization follows the same scheme"): a network weight is
+ * W'_ij = levels[codes[idx_i * 9 + j]], so level l moves against the average
+ * gradient of every weight whose value it is:
+ *   counts[l]      = #{ (i, j) : codes[idx_i * 9 + j] == l },
+ *   levels_next[l] = levels[l] - lr * (1 / counts[l]) * sum of those G_ij,
+ *                    or levels[l] when counts[l] == 0.
+ * Exact int64 fixed-point sums (scale from max|G| and 9n values); mean, step and
+ * result rounded as in kq_codebook_grad_step.
+ *   G      n x 9 fp32 (device, 16-byte aligned);  idx n int32 (device)
+ *   codes  K x 9 uint8 (device), values 0..63;  lr finite
+ *   levels 64 fp32 (device);  levels_next 64 fp32 output (device, may equal levels)
+ *   counts 64 int64 output (device, 8-byte aligned) or NULL
+ * 1 <= n < 2^31, 1 <= K, K*9 < 2^31. An index outside [0, K) is skipped
+ * (KQ_FLAG_INDEX_RANGE); a code above 63 is skipped (KQ_FLAG_CODE_RANGE). Uses
+ * only the first 4096 bytes of the workspace (ws_bytes >= 4096). */
+kq_status kq_levels_grad_step(const float *G, int64_t n, const int32_t *idx, int32_t K, const uint8_t *codes,
+                              float lr, const float *levels, float *levels_next, int64_t *counts, void *ws,
+                              size_t ws_bytes, kq_stream_t stream);
+
 /* Test-time recovery, Sec. 3.2 (last paragraph): first the kernel codebook is
  * recovered (C_hat[k][j] = levels[codes[k][j]]), then the weight tensor:
  *   W_out[i] = C_hat[idx[i]]   (K+C: codes and levels given), or

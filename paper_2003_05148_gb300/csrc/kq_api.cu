@@ -16,7 +16,7 @@ void count_launch(int kernels) { g_launches.fetch_add((unsigned long long)kernel
 
 namespace {
 
-constexpr int32_t KQ_ABI_VERSION = 2;
+constexpr int32_t KQ_ABI_VERSION = 3;
 
 inline bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
@@ -248,8 +248,62 @@ kq_status kq_quantize_codebook_6bit(const float *C, int32_t K, const int32_t *co
     int sms = 0;
     if ((st = num_sms(&sms)) != KQ_OK) return st;
     Header *h = static_cast<Header *>(ws);
-    return cuda_status(launch_level_fit(C, K, counts, max_iters, levels, codes, iters_run, h, sms,
+    return cuda_status(launch_level_fit(C, (int64_t)K * D, counts, max_iters, levels, codes, iters_run, h, sms,
                                         reinterpret_cast<cudaStream_t>(stream)));
+}
+
+kq_status kq_quantize_scalars_6bit(const float *v, int64_t m, int32_t max_iters, float *levels, uint8_t *codes,
+                                   int32_t *iters_run, void *ws, size_t ws_bytes, kq_stream_t stream) {
+    if (m < 1 || m > (1LL << 40) || !v || !levels || !codes) return KQ_ERR_INVALID_ARG;
+    if (max_iters < 0 || max_iters > 100000) return KQ_ERR_INVALID_ARG;
+    if (!aligned(v, 4) || !aligned(levels, 4) || !aligned(iters_run, 4)) return KQ_ERR_ALIGNMENT;
+    kq_status st = check_ws_header(ws, ws_bytes);
+    if (st != KQ_OK) return st;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != KQ_OK) return st;
+    Header *h = static_cast<Header *>(ws);
+    return cuda_status(launch_level_fit(v, m, nullptr, max_iters, levels, codes, iters_run, h, sms,
+                                        reinterpret_cast<cudaStream_t>(stream)));
+}
+
+kq_status kq_codebook_grad_step(const float *G, int64_t n, const int32_t *idx, int32_t K, float lr, const float *C,
+                                float *C_next, int32_t *counts, void *ws, size_t ws_bytes, kq_stream_t stream) {
+    if (!sizes_ok(n, K) || !G || !idx || !C || !C_next || !counts) return KQ_ERR_INVALID_ARG;
+    if (!(lr == lr) || lr > 3.402823466e38f || lr < -3.402823466e38f) return KQ_ERR_INVALID_ARG;
+    if (!aligned(G, 16) || !aligned(idx, 4) || !aligned(C, 4) || !aligned(C_next, 4) || !aligned(counts, 4))
+        return KQ_ERR_ALIGNMENT;
+    kq_status st = check_ws(ws, ws_bytes, n, K);
+    if (st != KQ_OK) return st;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != KQ_OK) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    Ws w = carve(ws, n, K);
+    // exact mode of the update: the scale from max|G|, the sums of the gradients
+    KQ_TRY(launch_update_prepare(nullptr, K, w.acc, w.hdr, false, s));
+    KQ_TRY(launch_maxabs(G, n * D, &w.hdr->maxabs_bits, &w.hdr->status, sms, s));
+    KQ_TRY(launch_accumulate(G, n, idx, K, w.hdr, w.acc, false, sms, s));
+    KQ_TRY(launch_grad_finalize(w.acc, K, w.hdr, lr, C, C_next, counts, s));
+    return KQ_OK;
+}
+
+kq_status kq_levels_grad_step(const float *G, int64_t n, const int32_t *idx, int32_t K, const uint8_t *codes,
+                              float lr, const float *levels, float *levels_next, int64_t *counts, void *ws,
+                              size_t ws_bytes, kq_stream_t stream) {
+    if (n < 1 || n >= (1LL << 31) || K < 1 || (int64_t)K * D >= (1LL << 31)) return KQ_ERR_INVALID_ARG;
+    if (!G || !idx || !codes || !levels || !levels_next) return KQ_ERR_INVALID_ARG;
+    if (!(lr == lr) || lr > 3.402823466e38f || lr < -3.402823466e38f) return KQ_ERR_INVALID_ARG;
+    if (!aligned(G, 16) || !aligned(idx, 4) || !aligned(levels, 4) || !aligned(levels_next, 4) ||
+        !aligned(counts, 8))
+        return KQ_ERR_ALIGNMENT;
+    kq_status st = check_ws_header(ws, ws_bytes);
+    if (st != KQ_OK) return st;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != KQ_OK) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    Header *h = static_cast<Header *>(ws);
+    KQ_TRY(launch_maxabs(G, n * D, &h->maxabs_bits, &h->status, sms, s));
+    KQ_TRY(launch_level_grad(G, n, idx, K, codes, lr, levels, levels_next, counts, h, sms, s));
+    return KQ_OK;
 }
 
 kq_status kq_reconstruct(const int32_t *idx, int64_t n, const float *C, int32_t K, const uint8_t *codes,

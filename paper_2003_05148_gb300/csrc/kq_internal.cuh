@@ -209,8 +209,16 @@ cudaError_t launch_histogram(const int32_t *idx, int64_t n, int32_t K, int32_t *
 cudaError_t launch_finalize(unsigned long long *acc, int32_t K, const Header *hdr, const float *C_prev,
                             float *C_next, int32_t *counts, cudaStream_t s);
 
-cudaError_t launch_level_fit(const float *C, int32_t K, const int32_t *counts, int32_t max_iters, float *levels,
+cudaError_t launch_level_fit(const float *C, int64_t N, const int32_t *counts, int32_t max_iters, float *levels,
                              uint8_t *codes, int32_t *iters_run, Header *hdr, int num_sms, cudaStream_t s);
+
+// Retraining with averaged gradients (Eq. 2): codebook finalise over the update's
+// accumulators, and the 64-level segment mean of the quantised codebook.
+cudaError_t launch_grad_finalize(unsigned long long *acc, int32_t K, const Header *hdr, float lr, const float *C,
+                                 float *C_next, int32_t *counts, cudaStream_t s);
+cudaError_t launch_level_grad(const float *G, int64_t n, const int32_t *idx, int32_t K, const uint8_t *codes,
+                              float lr, const float *levels, float *levels_next, int64_t *counts, Header *hdr,
+                              int num_sms, cudaStream_t s);
 
 // Recovery. K only: C is re-laid as 48-byte rows (Cp) and gathered. K+C: the
 // codes are packed 9 x 6 bits per codeword (Cq, 8 bytes) and decoded on the fly.

@@ -23,7 +23,8 @@ FLAG_NONFINITE, FLAG_INDEX_RANGE, FLAG_CODE_RANGE, FLAG_TIMEOUT = 0x1, 0x2, 0x4,
 
 EXPORTS = ["kq_status_string", "kq_abi_version", "kq_kernel_launches", "kq_workspace_bytes", "kq_device_status", "kq_init_codebook",
            "kq_assign", "kq_update_centroids", "kq_fit_codebook", "kq_quantize_codebook_6bit", "kq_reconstruct",
-           "kq_compression_report", "kq_conventional_ratio", "kq_assign_noalloc"]
+           "kq_compression_report", "kq_conventional_ratio", "kq_assign_noalloc", "kq_quantize_scalars_6bit",
+           "kq_codebook_grad_step", "kq_levels_grad_step"]
 
 
 class KQError(RuntimeError):
@@ -63,6 +64,9 @@ def lib() -> ctypes.CDLL:
             "kq_compression_report": ([i64, i32, i32, i32, ctypes.POINTER(Report)], ctypes.c_int),
             "kq_conventional_ratio": ([i64, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
             "kq_assign_noalloc": ([P, i64, P, i32, P, P, P], ctypes.c_int),
+            "kq_quantize_scalars_6bit": ([P, i64, i32, P, P, P, P, sz, P], ctypes.c_int),
+            "kq_codebook_grad_step": ([P, i64, P, i32, ctypes.c_float, P, P, P, P, sz, P], ctypes.c_int),
+            "kq_levels_grad_step": ([P, i64, P, i32, P, ctypes.c_float, P, P, P, P, sz, P], ctypes.c_int),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -163,6 +167,28 @@ def kq_quantize_codebook_6bit(C, counts, max_iters, levels, codes, iters_run, ws
         _dev(C, "C", torch.float32), _rows(C), _dev(counts, "counts", torch.int32), max_iters,
         _dev(levels, "levels", torch.float32), _dev(codes, "codes", torch.uint8),
         _dev(iters_run, "iters_run", torch.int32), _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+
+
+def kq_quantize_scalars_6bit(v, max_iters, levels, codes, iters_run, ws, stream=None) -> None:
+    _check("kq_quantize_scalars_6bit", lib().kq_quantize_scalars_6bit(
+        _dev(v, "v", torch.float32), v.numel(), max_iters, _dev(levels, "levels", torch.float32),
+        _dev(codes, "codes", torch.uint8), _dev(iters_run, "iters_run", torch.int32), _dev(ws, "ws", torch.uint8),
+        ws.numel(), _stream(stream)))
+
+
+def kq_codebook_grad_step(G, idx, lr: float, C, C_next, counts, ws, stream=None) -> None:
+    _check("kq_codebook_grad_step", lib().kq_codebook_grad_step(
+        _dev(G, "G", torch.float32), _rows(G), _dev(idx, "idx", torch.int32), _rows(C), float(lr),
+        _dev(C, "C", torch.float32), _dev(C_next, "C_next", torch.float32), _dev(counts, "counts", torch.int32),
+        _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+
+
+def kq_levels_grad_step(G, idx, codes, lr: float, levels, levels_next, counts, ws, stream=None) -> None:
+    _check("kq_levels_grad_step", lib().kq_levels_grad_step(
+        _dev(G, "G", torch.float32), _rows(G), _dev(idx, "idx", torch.int32), codes.numel() // 9,
+        _dev(codes, "codes", torch.uint8), float(lr), _dev(levels, "levels", torch.float32),
+        _dev(levels_next, "levels_next", torch.float32), _dev(counts, "counts", torch.int64),
+        _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
 
 
 def kq_reconstruct(idx, C, codes, levels, W_out, ws, K: Optional[int] = None, stream=None) -> None:

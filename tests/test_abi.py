@@ -35,7 +35,7 @@ def test_exports_every_declared_symbol(lib):
 
 
 def test_status_strings_and_version(lib):
-    assert kq.kq_abi_version() == 2
+    assert kq.kq_abi_version() == 3
     for code, name in kq.STATUS_NAMES.items():
         assert kq.kq_status_string(code) == name
     assert kq.kq_status_string(99) == "KQ_ERR_UNKNOWN"
@@ -74,6 +74,21 @@ def test_host_validation_before_any_device_work(lib):
     assert L.kq_reconstruct(good, 1024, good, 16, None, None, odd, good, ws_bytes, None) == 2  # W_out alignment
     assert L.kq_init_codebook(good, 1024, good, 2000, good, good, ws_bytes, None) == 1
     assert L.kq_device_status(None, 0, None, None) == 6
+    nan = float("nan")
+    assert L.kq_quantize_scalars_6bit(good, 0, 10, good, good, None, good, 4096, None) == 1  # m = 0
+    assert L.kq_quantize_scalars_6bit(good, 100, 100001, good, good, None, good, 4096, None) == 1
+    assert L.kq_quantize_scalars_6bit(good, 100, 10, good, good, None, good, 4095, None) == 6
+    assert L.kq_codebook_grad_step(good, 1024, good, 16, nan, good, good, good, good, ws_bytes, None) == 1  # lr NaN
+    assert L.kq_codebook_grad_step(good, 1024, good, 16, float("inf"), good, good, good, good, ws_bytes, None) == 1
+    assert L.kq_codebook_grad_step(odd, 1024, good, 16, 0.1, good, good, good, good, ws_bytes, None) == 2
+    assert L.kq_codebook_grad_step(good, 1024, good, 16, 0.1, good, good, good, good, ws_bytes - 1, None) == 6
+    assert L.kq_levels_grad_step(good, 0, good, 16, good, 0.1, good, good, None, good, 4096, None) == 1
+    assert L.kq_levels_grad_step(good, 1024, good, 16, None, 0.1, good, good, None, good, 4096, None) == 1
+    assert L.kq_levels_grad_step(good, 1024, good, 16, good, nan, good, good, None, good, 4096, None) == 1
+    assert L.kq_levels_grad_step(odd, 1024, good, 16, good, 0.1, good, good, None, good, 4096, None) == 2
+    assert L.kq_levels_grad_step(good, 1024, good, 16, good, 0.1, good, good, ctypes.c_void_p((1 << 20) + 4),
+                                 good, 4096, None) == 2  # counts not 8-byte aligned
+    assert L.kq_levels_grad_step(good, 1024, good, 16, good, 0.1, good, good, None, good, 4095, None) == 6
 
 
 def _report_rows():

@@ -18,7 +18,7 @@ MUTANTS = {
     "distance_drops_last_term": ("    for (int j = 0; j < KQO_D; ++j) {\n        float t = x[j] - c[j];",
                                  "    for (int j = 0; j < KQO_D - 1; ++j) {\n        float t = x[j] - c[j];"),
     "distance_sign_error": ("float t = x[j] - c[j];", "float t = x[j] + c[j];"),
-    "mean_divides_by_z_plus_1": ("(float)(sum[e] / (double)z[k])", "(float)(sum[e] / (double)(z[k] + 1))"),
+    "mean_divides_by_z_plus_1": ("z[k] > 0 ? (float)(sum[e] / (double)z[k])", "z[k] > 0 ? (float)(sum[e] / (double)(z[k] + 1))"),
     "empty_cluster_zeroed": (": C_prev[e];", ": 0.0f;"),
     "update_wrong_coordinate": ("+= (double)W[i * KQO_D + j];", "+= (double)W[i * KQO_D + (j + 1) % KQO_D];"),
     "levels_ignore_weights": ("wsum[cur[m]] += z;\n            qsum[cur[m]] += z * q[m];",
@@ -29,6 +29,16 @@ MUTANTS = {
     "level_fit_never_converges": ("if (it > 0 && memcmp(cur, prev, (size_t)N) == 0) break;", "if (0) break;"),
     "reconstruct_reversed_row": ("C[k * KQO_D + j];", "C[k * KQO_D + (KQO_D - 1 - j)];"),
     "objective_squares": ("J += (double)dist[i];", "J += (double)dist[i] * (double)dist[i];"),
+    "grad_step_sign_error": ("C_next[e] = C[e] - step;", "C_next[e] = C[e] + step;"),
+    "grad_step_divides_by_z_plus_1": ("float mean = (float)(sum[e] / (double)z[k]);",
+                                      "float mean = (float)(sum[e] / (double)(z[k] + 1));"),
+    "grad_step_empty_zeroed": ("C_next[e] = C[e];\n            }", "C_next[e] = 0.0f;\n            }"),
+    "grad_step_skips_lr": ("float step = lr * mean;\n                C_next", "float step = mean;\n                C_next"),
+    "levels_grad_wrong_coordinate": ("int l = codes[(int64_t)k * KQO_D + j];",
+                                     "int l = codes[(int64_t)k * KQO_D + (j + 1) % KQO_D];"),
+    "levels_grad_sign_error": ("levels_next[l] = levels[l] - step;", "levels_next[l] = levels[l] + step;"),
+    "levels_grad_counts_kernels": ("z[l] += 1;\n            sum[l]", "z[l] += (j == 0);\n            sum[l]"),
+    "scalar_fit_zero_weight": ("return w ? (int64_t)w[m / group] : 1;", "return w ? (int64_t)w[m / group] : 0;"),
 }
 
 PINS = [
@@ -48,6 +58,13 @@ PINS = [
     pins.test_encode_ties_go_to_the_lower_level,
     pins.test_reconstruct_round_trip,
     pins.test_reconstruct_with_codes_uses_levels,
+    pins.test_level_fit_scalars_equally_spaced_is_fixed_point,
+    pins.test_level_fit_scalars_converged_levels_are_means,
+    pins.test_level_fit_scalars_is_unit_weight_codebook_fit,
+    pins.test_codebook_grad_step_dyadic_bit_exact,
+    pins.test_codebook_grad_step_quadratic_loss_gives_the_centroid,
+    pins.test_levels_grad_step_dyadic_bit_exact,
+    pins.test_levels_grad_step_constant_gradient_shifts_every_used_level,
 ]
 
 
