@@ -14,12 +14,12 @@
 // Per-iteration global state is triple buffered (iteration it accumulates into
 // slot it%3 while CTA 0 clears slot (it+1)%3, last read two barriers earlier),
 // so one grid barrier per iteration suffices.
+#include <type_traits>
+
 #include "kq_internal.cuh"
 
 namespace kq {
 
-constexpr int Q_THREADS = 512;
-constexpr int Q_WARPS = Q_THREADS / 32;
 struct LevelArgs {
     const float *C;  // the N scalars
     int64_t N;
@@ -29,6 +29,7 @@ struct LevelArgs {
     uint8_t *codes;
     int32_t *iters_run;
     Header *hdr;
+    int use_table;  // many scalars per thread: find codes through the bucket table
 };
 
 // Nearest of the 64 levels by fp32 |v - level|, lower index on ties (Sec. 3.2 encode).
@@ -52,13 +53,8 @@ __device__ __forceinline__ int nearest_level(float v, const float *L) {
 // d_p or d_{p+1}; the first index holding it (the scan's tie rule) is p + 1 when
 // d_{p+1} < d_p, else the start of the run of levels <= p whose distance equals
 // d_p, which is a suffix of [0, p]. A minimum of +inf gives 0, as in the scan.
-__device__ __forceinline__ int nearest_level_sorted(float v, const float *L) {
-    if (v != v) return 0;  // NaN: no distance is below +inf
-    int cnt = 0;           // number of levels <= v
-#pragma unroll
-    for (int step = 32; step > 0; step >>= 1)
-        if (L[cnt + step - 1] <= v) cnt += step;
-    cnt += L[cnt] <= v;  // cnt could only reach 63 above
+// The code of v given cnt = #{l : L_l <= v} (levels sorted; see above).
+__device__ __forceinline__ int nearest_from_count(float v, const float *L, int cnt) {
     const int p = cnt - 1;
     if (p < 0) return 0;  // every level is above v: distances grow with l
     const float dp = fabsf(v - L[p]);
@@ -72,6 +68,31 @@ __device__ __forceinline__ int nearest_level_sorted(float v, const float *L) {
     return f;
 }
 
+__device__ __forceinline__ int nearest_level_sorted(float v, const float *L) {
+    if (v != v) return 0;  // NaN: no distance is below +inf
+    int cnt = 0;           // number of levels <= v
+#pragma unroll
+    for (int step = 32; step > 0; step >>= 1)
+        if (L[cnt + step - 1] <= v) cnt += step;
+    cnt += L[cnt] <= v;  // cnt could only reach 63 above
+    return nearest_from_count(v, L, cnt);
+}
+
+// nearest_level_sorted with the count found from a table instead of a binary
+// search: Tb[b] is the number of levels at or below a point of bucket b of a
+// uniform grid over [L_0, L_63] (inv_w buckets per unit), and the two walks make
+// it the exact count for v whatever the guess; in most buckets no level lies,
+// so each walk stops at its first test.
+constexpr int Q_TABLE = 1024;
+__device__ __forceinline__ int nearest_level_table(float v, const float *L, const uint8_t *Tb, float lo, float inv_w) {
+    if (v != v) return 0;
+    const float x = fminf(fmaxf((v - lo) * inv_w, 0.f), (float)(Q_TABLE - 1));
+    int c = Tb[(int)x];
+    while (c < LEVELS && L[c] <= v) ++c;
+    while (c > 0 && L[c - 1] > v) --c;
+    return nearest_from_count(v, L, c);
+}
+
 // Levels in non-decreasing order (and no NaN), so that nearest_level_sorted applies.
 __device__ __forceinline__ bool levels_sorted(const float *L) {
     bool ok = true;
@@ -80,15 +101,63 @@ __device__ __forceinline__ bool levels_sorted(const float *L) {
     return ok;
 }
 
-__global__ void __launch_bounds__(Q_THREADS) level_fit_kernel(LevelArgs a) {
+// Per-lane private accumulators: lane l of warp w adds into column l of its
+// warp's [level][lane] arrays with plain read-modify-writes (no atomics; a 64-bit
+// add would otherwise be a compare-and-swap loop, and lanes of a warp often share
+// a level). Weight sums are 32-bit per lane; one that would overflow is first
+// moved into the 64-bit global total of its level (only with very large counts).
+constexpr int Q_THREADS = 256;
+constexpr int Q_WARPS = Q_THREADS / 32;
+struct LevelBins {
+    unsigned long long q[Q_WARPS][LEVELS][32];  // sum of weight * fixed-point value
+    uint32_t w[Q_WARPS][LEVELS][32];            // sum of weights
+};
+
+constexpr int Q_UNROLL = 4;  // scalars per thread whose loads are in flight together
+
+// After the levels change (all threads): whether they are sorted, and if so the
+// bucket table of nearest_level_table over [L_0, L_63].
+__device__ __forceinline__ void build_table(const float *L, uint8_t *Tb, int &s_sorted, float &s_tlo, float &s_tinv,
+                                            bool use_table) {
+    if (threadIdx.x == 0) {
+        const bool srt = levels_sorted(L);
+        s_sorted = srt;
+        const float lo = L[0], span = L[LEVELS - 1] - L[0];
+        s_tlo = lo;
+        // buckets per unit; 0 (every value in bucket 0) when the span is empty or not finite
+        s_tinv = (srt && span > 0.f && span <= 3.402823466e38f) ? (float)Q_TABLE / span : 0.f;
+    }
+    __syncthreads();
+    if (!use_table) return;
+    const float lo = s_tlo, inv = s_tinv;
+    const float w = inv > 0.f ? 1.f / inv : 0.f;
+    for (int b = threadIdx.x; b < Q_TABLE; b += blockDim.x) {
+        const float x = lo + ((float)b + 0.5f) * w;  // a point of bucket b (any guess is corrected)
+        int cnt = 0;
+#pragma unroll
+        for (int step = 32; step > 0; step >>= 1)
+            if (L[cnt + step - 1] <= x) cnt += step;
+        cnt += L[cnt] <= x;
+        Tb[b] = (uint8_t)cnt;
+    }
+    __syncthreads();
+}
+
+template <bool UNIT>
+__global__ void __launch_bounds__(Q_THREADS, 1) level_fit_kernel(LevelArgs a) {
+    constexpr int NP = Q_THREADS / LEVELS;  // reducer threads per level
+    extern __shared__ __align__(16) unsigned char q_smem[];
+    LevelBins &B = *reinterpret_cast<LevelBins *>(q_smem);
     __shared__ float L[LEVELS];
-    __shared__ unsigned long long bw[Q_WARPS][LEVELS], bq[Q_WARPS][LEVELS];
+    __shared__ uint8_t Tb[Q_TABLE];
+    __shared__ float s_tlo, s_tinv;
+    __shared__ unsigned long long red_q[NP][LEVELS], red_w[NP][LEVELS];
     __shared__ int s_changed;
     __shared__ int s_stop;
     __shared__ int s_sorted;
     Header *h = a.hdr;
     const int64_t N = a.N;
-    const int warp = threadIdx.x >> 5;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t tid0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     unsigned epoch = 0;
@@ -100,7 +169,7 @@ __global__ void __launch_bounds__(Q_THREADS) level_fit_kernel(LevelArgs a) {
         bool ok = true, badc = false;
         for (int64_t m = tid0; m < N; m += stride) {
             const float v = a.C[m];
-            int32_t z = a.counts ? a.counts[m / D] : 1;
+            int32_t z = UNIT ? 1 : a.counts[(uint32_t)m / D];
             if (z < 0) {
                 badc = true;
                 z = 0;
@@ -128,7 +197,7 @@ __global__ void __launch_bounds__(Q_THREADS) level_fit_kernel(LevelArgs a) {
             wt += __shfl_xor_sync(0xffffffffu, wt, o);
         }
         const bool all_ok = __all_sync(0xffffffffu, ok), any_bad = __any_sync(0xffffffffu, badc);
-        if ((threadIdx.x & 31) == 0) {
+        if (lane == 0) {
             atomicMin(&h->lo_w, f2ord(lo_w));
             atomicMax(&h->hi_w, f2ord(hi_w));
             atomicMin(&h->lo_a, f2ord(lo_a));
@@ -138,6 +207,10 @@ __global__ void __launch_bounds__(Q_THREADS) level_fit_kernel(LevelArgs a) {
             if (!all_ok) set_flag(&h->status, KQ_FLAG_NONFINITE);
             if (any_bad) set_flag(&h->status, KQ_FLAG_INDEX_RANGE);
         }
+    }
+    for (int l = 0; l < LEVELS; ++l) {
+        B.q[warp][l][lane] = 0ull;
+        B.w[warp][l][lane] = 0;
     }
     if (!grid_barrier(h, gridDim.x, epoch)) return;
 
@@ -159,15 +232,12 @@ __global__ void __launch_bounds__(Q_THREADS) level_fit_kernel(LevelArgs a) {
         L[threadIdx.x] = __double2float_rn(__dadd_rn((double)lo, t));
     }
     __syncthreads();
-    if (threadIdx.x == 0) s_sorted = levels_sorted(L);
+    const bool use_table = a.use_table;
+    build_table(L, Tb, s_sorted, s_tlo, s_tinv, use_table);
 
     int32_t updates = 0;
     for (int32_t it = 0; it < a.max_iters; ++it) {
         const int buf = it % 3, nxt = (it + 1) % 3;
-        for (int t = threadIdx.x; t < Q_WARPS * LEVELS; t += Q_THREADS) {
-            (&bw[0][0])[t] = 0ull;
-            (&bq[0][0])[t] = 0ull;
-        }
         if (threadIdx.x == 0) s_changed = 0;
         if (blockIdx.x == 0) {
             if (threadIdx.x < 2 * LEVELS) (&h->lacc[nxt][0][0])[threadIdx.x] = 0ull;
@@ -176,26 +246,65 @@ __global__ void __launch_bounds__(Q_THREADS) level_fit_kernel(LevelArgs a) {
         __syncthreads();
         bool changed = false;
         const bool sorted = s_sorted;
-        for (int64_t m = tid0; m < N; m += stride) {
-            const float v = a.C[m];
-            const int code = sorted ? nearest_level_sorted(v, L) : nearest_level(v, L);
-            if (it > 0 && a.codes[m] != (uint8_t)code) changed = true;
-            a.codes[m] = (uint8_t)code;
-            const int32_t z = a.counts ? a.counts[m / D] : 1;
-            if (z > 0) {
-                const long long q = fixed_rn(v, S);
-                atomicAdd(&bw[warp][code], (unsigned long long)z);
-                atomicAdd(&bq[warp][code], (unsigned long long)((long long)z * q));
+        const float tlo = s_tlo, tinv = s_tinv;
+        for (int64_t m0 = tid0; m0 < N; m0 += Q_UNROLL * stride) {
+            float v[Q_UNROLL];
+            int32_t z[Q_UNROLL];
+            uint32_t old[Q_UNROLL];
+#pragma unroll
+            for (int u = 0; u < Q_UNROLL; ++u) {
+                const int64_t m = m0 + u * stride;
+                const bool in = m < N;
+                v[u] = in ? __ldg(a.C + m) : 0.f;
+                z[u] = in ? (UNIT ? 1 : __ldg(a.counts + (uint32_t)m / D)) : 0;
+                old[u] = (in && it > 0) ? a.codes[m] : 0u;
+            }
+#pragma unroll
+            for (int u = 0; u < Q_UNROLL; ++u) {
+                const int64_t m = m0 + u * stride;
+                if (m >= N) break;
+                const int code = !sorted     ? nearest_level(v[u], L)
+                                 : use_table ? nearest_level_table(v[u], L, Tb, tlo, tinv)
+                                             : nearest_level_sorted(v[u], L);
+                changed |= it > 0 && old[u] != (uint32_t)code;
+                a.codes[m] = (uint8_t)code;
+                if (z[u] > 0) {
+                    const long long q = fixed_rn(v[u], S);
+                    B.q[warp][code][lane] += (unsigned long long)((long long)z[u] * q);
+                    const uint32_t w0 = B.w[warp][code][lane];
+                    if (!UNIT && w0 > 0xffffffffu - (uint32_t)z[u]) {  // would overflow: move to the total
+                        atomicAdd(&h->lacc[buf][code][0], (unsigned long long)w0);
+                        B.w[warp][code][lane] = (uint32_t)z[u];
+                    } else {
+                        B.w[warp][code][lane] = w0 + (uint32_t)z[u];
+                    }
+                }
             }
         }
-        if (__any_sync(0xffffffffu, changed) && (threadIdx.x & 31) == 0) s_changed = 1;
+        if (__any_sync(0xffffffffu, changed) && lane == 0) s_changed = 1;
+        __syncthreads();
+        {  // CTA totals per level: NP threads per level, 2 warps' columns each; bins cleared as read
+            const int l = threadIdx.x % LEVELS, part = threadIdx.x / LEVELS;
+            unsigned long long sq = 0ull, sw = 0ull;
+            for (int w = 2 * part; w < 2 * part + 2; ++w)
+#pragma unroll 8
+                for (int j = 0; j < 32; ++j) {
+                    const int ln = (j + l) & 31;  // lanes of a warp read 32 different banks
+                    sq += B.q[w][l][ln];
+                    sw += (unsigned long long)B.w[w][l][ln];
+                    B.q[w][l][ln] = 0ull;
+                    B.w[w][l][ln] = 0u;
+                }
+            red_q[part][l] = sq;
+            red_w[part][l] = sw;
+        }
         __syncthreads();
         if (threadIdx.x < LEVELS) {
-            unsigned long long sw = 0ull, sq = 0ull;
-#pragma unroll 4
-            for (int w = 0; w < Q_WARPS; ++w) {
-                sw += bw[w][threadIdx.x];
-                sq += bq[w][threadIdx.x];
+            unsigned long long sq = 0ull, sw = 0ull;
+#pragma unroll
+            for (int p = 0; p < NP; ++p) {
+                sq += red_q[p][threadIdx.x];
+                sw += red_w[p][threadIdx.x];
             }
             if (sw) {
                 atomicAdd(&h->lacc[buf][threadIdx.x][0], sw);
@@ -215,19 +324,60 @@ __global__ void __launch_bounds__(Q_THREADS) level_fit_kernel(LevelArgs a) {
                     __double2float_rn(__ddiv_rn(__dmul_rn(__ll2double_rn(Ql), down), __ull2double_rn(Wl)));
         }
         __syncthreads();
-        if (threadIdx.x == 0) s_sorted = levels_sorted(L);
+        build_table(L, Tb, s_sorted, s_tlo, s_tinv, use_table);
         ++updates;
     }
 
     // Codes of the final levels.
     __syncthreads();
     const bool sorted = s_sorted;
-    for (int64_t m = tid0; m < N; m += stride)
-        a.codes[m] = (uint8_t)(sorted ? nearest_level_sorted(a.C[m], L) : nearest_level(a.C[m], L));
+    const float tlo = s_tlo, tinv = s_tinv;
+    for (int64_t m0 = tid0; m0 < N; m0 += Q_UNROLL * stride) {
+        float v[Q_UNROLL];
+#pragma unroll
+        for (int u = 0; u < Q_UNROLL; ++u) {
+            const int64_t m = m0 + u * stride;
+            v[u] = m < N ? __ldg(a.C + m) : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < Q_UNROLL; ++u) {
+            const int64_t m = m0 + u * stride;
+            if (m < N)
+                a.codes[m] = (uint8_t)(!sorted     ? nearest_level(v[u], L)
+                                       : use_table ? nearest_level_table(v[u], L, Tb, tlo, tinv)
+                                                   : nearest_level_sorted(v[u], L));
+        }
+    }
     if (blockIdx.x == 0) {
         if (threadIdx.x < LEVELS) a.levels[threadIdx.x] = L[threadIdx.x];
         if (threadIdx.x == 0 && a.iters_run) *a.iters_run = updates;
     }
+}
+
+template <bool UNIT>
+cudaError_t launch_level_fit_t(const LevelArgs &args, int num_sms, cudaStream_t s) {
+    constexpr int T = Q_THREADS;
+    const int smem = (int)sizeof(LevelBins);
+    static_assert(sizeof(LevelBins) <= 200 * 1024, "level bins too large");
+    cudaError_t e = cudaFuncSetAttribute(level_fit_kernel<UNIT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, level_fit_kernel<UNIT>, T, smem);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    int64_t blocks = (args.N + T - 1) / T;
+    if (blocks > (int64_t)num_sms) blocks = num_sms;  // one CTA per SM: co-resident by construction
+    if (blocks < 1) blocks = 1;
+    // a lane's 32-bit count of unit weights stays below 2^31
+    if (UNIT && args.N / (blocks * T) >= (1LL << 31)) return cudaErrorInvalidValue;
+    LevelArgs a = args;
+    a.use_table = args.N / (blocks * T) >= 64;  // the table pays for itself from ~64 scalars per thread
+    void *params[] = {&a};
+    e = cudaLaunchCooperativeKernel((const void *)level_fit_kernel<UNIT>, dim3((unsigned)blocks), dim3(T), params,
+                                    smem, s);
+    if (e != cudaSuccess) return e;
+    count_launch();
+    return cudaGetLastError();
 }
 
 cudaError_t launch_level_fit(const float *C, int64_t N, const int32_t *counts, int32_t max_iters, float *levels,
@@ -237,20 +387,8 @@ cudaError_t launch_level_fit(const float *C, int64_t N, const int32_t *counts, i
     if (e != cudaSuccess) return e;
     e = cudaMemsetAsync(&hdr->lo_w, 0xff, 2 * sizeof(uint32_t), s);
     if (e != cudaSuccess) return e;
-    int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, level_fit_kernel, Q_THREADS, 0);
-    if (e != cudaSuccess) return e;
-    if (per_sm < 1) return cudaErrorInvalidConfiguration;
-    int64_t blocks = (N + Q_THREADS - 1) / Q_THREADS;
-    if (blocks > (int64_t)num_sms) blocks = num_sms;  // one CTA per SM is plenty, and co-resident
-    if (blocks < 1) blocks = 1;
-    LevelArgs args{C, N, counts, max_iters, levels, codes, iters_run, hdr};
-    void *params[] = {&args};
-    e = cudaLaunchCooperativeKernel((const void *)level_fit_kernel, dim3((unsigned)blocks), dim3(Q_THREADS), params,
-                                    0, s);
-    if (e != cudaSuccess) return e;
-    count_launch();
-    return cudaGetLastError();
+    const LevelArgs args{C, N, counts, max_iters, levels, codes, iters_run, hdr, 0};
+    return counts ? launch_level_fit_t<false>(args, num_sms, s) : launch_level_fit_t<true>(args, num_sms, s);
 }
 
 }  // namespace kq
