@@ -14,6 +14,7 @@ Parity pins for every function are in ``tests/test_oracle.py``.
 from __future__ import annotations
 
 import ctypes
+import math
 import dataclasses
 import os
 import subprocess
@@ -233,6 +234,72 @@ def gather_rows(W, sel):
     C0 = np.empty((sel.shape[0], D), np.float32)
     _load().kqo_gather_rows(_ptr(W), _ptr(sel), sel.shape[0], _ptr(C0))
     return C0
+
+
+# ---------------------------------------------------------------------------
+# Algorithm 1 (Sec. 3.1): adaptive codebook size by binary search, Eq. 3.
+# ---------------------------------------------------------------------------
+
+def initial_size(n: int, alpha: float) -> int:
+    """N_init = alpha * n (Algorithm 1), rounded down and kept in [1, n]."""
+    return max(1, min(n, int(math.floor(alpha * n))))
+
+
+def target_accuracy(a_ori: float, a_base: float, r: float) -> float:
+    """Eq. 3: A_target = A_base - (A_ori - A_base) * r."""
+    return a_base - (a_ori - a_base) * r
+
+
+def bisect_codebook_size(n: int, alpha: float, r: float, max_steps: int, accuracy_of, a_ori: float):
+    """Algorithm 1's search for one layer, with the accuracy test supplied by the caller.
+
+    accuracy_of(K) quantises the layer with K entries and returns its accuracy.
+    B_upper starts at N_init, B_lower at 0; each step tests N_curr = floor((B_upper +
+    B_lower) / 2) and moves B_upper there if the accuracy beats A_target (Eq. 3),
+    else B_lower. The search stops after max_steps tests, when the interval cannot
+    be split any more, or when a test lands exactly on A_target. Returns
+    (K, trace): K = B_upper, the smallest tested size that beats the target (N_init
+    when none does), and trace = [(size, accuracy)] starting with (N_init, A_base).
+    """
+    n_init = initial_size(n, alpha)
+    a_base = accuracy_of(n_init)
+    a_target = target_accuracy(a_ori, a_base, r)
+    b_up, b_lo = n_init, 0
+    trace = [(n_init, a_base)]
+    steps = 0
+    while steps < max_steps and b_up - b_lo > 1:
+        steps += 1
+        k = (b_up + b_lo) // 2
+        a = accuracy_of(k)
+        trace.append((k, a))
+        if a > a_target:
+            b_up = k
+        else:
+            b_lo = k
+        if a == a_target:
+            break
+    return b_up, trace
+
+
+def search_codebook_size(W, sel, alpha: float, r: float, max_steps: int, lloyd_iters: int, threads: int = 1):
+    """Algorithm 1 with the reconstruction-error proxy: accuracy A(K) = -e(K), where
+    e(K) = sqrt(J_K / J_0) is the relative l2 error of kernel-level quantisation with K
+    entries (J_K: Eq. 1 objective after `lloyd_iters` updates from C_0 = W[sel[:K]];
+    J_0 = sum of |W_i|^2, the objective against the zero codeword) and A_ori = 0.
+
+    Returns (K, trace [(size, error)])."""
+    W = _f32(W).reshape(-1, D)
+    sel = np.ascontiguousarray(sel, dtype=np.int64)
+    n = W.shape[0]
+    _, d0 = assign(W, np.zeros((1, D), np.float32), threads=threads)
+    J0 = objective(d0)
+
+    def accuracy_of(k):
+        _, _, _, obj = fit(W, gather_rows(W, sel[:k]), lloyd_iters, threads=threads)
+        return -math.sqrt(obj[-1] / J0) if J0 > 0 else 0.0
+
+    k, trace = bisect_codebook_size(n, alpha, r, max_steps, accuracy_of, 0.0)
+    return k, [(size, -a) for size, a in trace]
 
 
 # ---------------------------------------------------------------------------

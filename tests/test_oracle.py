@@ -341,6 +341,75 @@ def test_level_scale_bounds():
 
 
 # ---------------------------------------------------------------------------
+# Algorithm 1 and Eq. 3: adaptive codebook size.
+# ---------------------------------------------------------------------------
+
+def test_target_accuracy_eq3():
+    # A_target = A_base - (A_ori - A_base) * r
+    assert oracle.target_accuracy(0.70, 0.60, 0.5) == pytest.approx(0.55)
+    assert oracle.target_accuracy(0.70, 0.70, 3.0) == pytest.approx(0.70)
+    assert oracle.target_accuracy(0.0, -0.2, 0.25) == pytest.approx(-0.25)
+    assert oracle.initial_size(1000, 0.25) == 250 and oracle.initial_size(10, 0.01) == 1
+    assert oracle.initial_size(7, 5.0) == 7
+
+
+@pytest.mark.parametrize("n,alpha,r", [(1000, 0.5, 0.5), (4096, 0.25, 0.3), (777, 0.6, 0.7), (65536, 0.3, 0.5)])
+def test_bisection_closed_form(n, alpha, r):
+    # accuracy -1/K grows with K; A_target = -(1 + r) / N_init, so the sizes that
+    # beat it are K > N_init / (1 + r) and the search ends on the smallest of them
+    n_init = oracle.initial_size(n, alpha)
+    k, trace = oracle.bisect_codebook_size(n, alpha, r, 64, lambda K: -1.0 / K, 0.0)
+    assert trace[0] == (n_init, -1.0 / n_init)
+    expect = int(Fraction(n_init) / (1 + Fraction(r).limit_denominator(1000))) + 1
+    assert k == min(expect, n_init)
+    # sizes are halved intervals: every tested size lies strictly inside the bounds
+    assert all(0 < size < n_init for size, _ in trace[1:])
+    # no steps: the initial size is kept
+    assert oracle.bisect_codebook_size(n, alpha, r, 0, lambda K: -1.0 / K, 0.0)[0] == n_init
+
+
+def test_bisection_stops_on_the_exact_target():
+    # N_init / (1 + r) = 466 / 2 = 233: the test of 233 lands exactly on A_target
+    # (-1/233 == -2/466 in fp64), which ends the search; 233 itself does not beat it
+    k, trace = oracle.bisect_codebook_size(777, 0.6, 1.0, 64, lambda K: -1.0 / K, 0.0)
+    assert trace[-1][0] == 233 and k > 233
+
+
+def test_bisection_matches_brute_force_on_monotone_accuracies():
+    rng = np.random.default_rng(8)
+    for _ in range(40):
+        n = int(rng.integers(10, 3000))
+        alpha, r = float(rng.uniform(0.05, 1.0)), float(rng.uniform(0.0, 2.0))
+        n_init = oracle.initial_size(n, alpha)
+        acc = np.sort(rng.uniform(0.0, 1.0, n_init + 1))  # non-decreasing in K
+        k, _ = oracle.bisect_codebook_size(n, alpha, r, 64, lambda K: float(acc[K]), 1.0)
+        target = oracle.target_accuracy(1.0, float(acc[n_init]), r)
+        beats = [K for K in range(1, n_init + 1) if acc[K] > target]
+        assert k == (min(beats) if beats else n_init)
+
+
+def test_search_codebook_size_reconstruction_proxy():
+    lay = synth.workload(1).layers[0]
+    W, sel = synth.layer_inputs(lay)
+    sel = synth.init_selection(W.shape[0], oracle.initial_size(W.shape[0], 0.25), lay.seed + 1)
+    k, trace = oracle.search_codebook_size(W, sel, 0.25, 0.5, 8, 3, threads=4)
+    n_init = oracle.initial_size(W.shape[0], 0.25)
+    assert trace[0][0] == n_init and 1 <= k <= n_init
+    e_base = trace[0][1]
+    # the proxy is the relative l2 error of W against its kernel-level reconstruction
+    C, idx, _, _ = oracle.fit(W, oracle.gather_rows(W, sel[:n_init]), 3)
+    W64 = W.astype(np.float64)
+    err = np.sqrt(((W64 - C[idx].astype(np.float64)) ** 2).sum() / (W64 ** 2).sum())
+    assert abs(err - e_base) <= 1e-6 * err
+    # the size returned meets the relaxed target; the size below it (when tested) does not
+    limit = e_base * 1.5
+    tested = dict(trace)
+    assert tested.get(k, e_base) < limit or k == n_init
+    if k - 1 in tested:
+        assert tested[k - 1] >= limit
+
+
+# ---------------------------------------------------------------------------
 # Sec. 3.2 (last step): 6-bit quantisation of a fully-connected layer.
 # ---------------------------------------------------------------------------
 
