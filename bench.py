@@ -456,6 +456,26 @@ def run_only(args):
     calls["levelgrad"] = lambda: kq.kq_levels_grad_step(W, idx, codes, 0.01, levels, lv_next, lv_counts, ws)
     alg_bytes = {"update": 40 * n + 76 * K, "gradstep": 40 * n + 76 * K, "levelgrad": 40 * n + 9 * K,
                  "reconstruct": 40 * n + 9 * K + 256}
+    if args.only == "search":
+        # Algorithm 1 on the VGG-16 conv3_2 layer (workload 2): alpha = 0.25, r = 0.5,
+        # 8 bisection steps, 20 Lloyd updates per trial (the workload's own count)
+        lay2 = synth.workload(2).layers[0]
+        W2_h, _ = synth.layer_inputs(lay2)
+        n2 = W2_h.shape[0]
+        n_init = int(np.floor(0.25 * n2))
+        sel2 = torch.from_numpy(synth.init_selection(n2, n_init, lay2.seed + 1)).to(dev)
+        W2 = torch.from_numpy(W2_h).to(dev)
+        C_s = torch.empty(n_init, 9, dtype=torch.float32, device=dev)
+        idx_s = torch.empty(n2, dtype=torch.int32, device=dev)
+        cnt_s = torch.empty(n_init, dtype=torch.int32, device=dev)
+        ws2 = kq.workspace(n2, n_init, dev)
+        search_out = {}
+
+        def run_search():
+            search_out["r"] = kq.kq_search_codebook_size(W2, sel2, 0.25, 0.5, 8, 20, C_s, idx_s, cnt_s, ws2)
+
+        calls["search"] = run_search
+        n, K = n2, n_init
     if args.only == "fcquant":
         # 6-bit quantisation of a fully-connected weight of m scalars (He-scaled
         # Gaussian, seeded), 100 iterations at most
@@ -484,6 +504,10 @@ def run_only(args):
     if args.only in alg_bytes:
         out["alg_bytes"] = alg_bytes[args.only]
         out["GB_s_at_min"] = alg_bytes[args.only] / (min(ms) * 1e-3) / 1e9
+    if args.only == "search":
+        k_s, e_s, tr_s = search_out["r"]
+        out["K_chosen"], out["error"], out["trials"] = k_s, e_s, len(tr_s)
+        out["trace"] = [[a, round(b, 6)] for a, b in tr_s]
     if args.only == "fcquant":
         it = int(fc_it.item())
         out["iters_run"] = it
@@ -564,7 +588,7 @@ def main():
     ap.add_argument("--ref-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--only", choices=["assign", "update", "quantize", "reconstruct", "gradstep", "levelgrad",
-                                       "fcquant"],
+                                       "fcquant", "search"],
                     help="profiling aid: time one entry point on its own (no bench line)")
     ap.add_argument("--n", type=int, default=4194304)
     ap.add_argument("--K", type=int, default=65536)

@@ -168,6 +168,36 @@ kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_i
                           float *C_out, int32_t *idx, int32_t *counts, double *objective, void *ws, size_t ws_bytes,
                           kq_stream_t stream);
 
+/* Adaptive codebook size, Algorithm 1 with Eq. 3 (Sec. 3.1): a binary search for
+ * the smallest codebook that keeps a layer's quality above a target. The paper's
+ * quality test is validation accuracy; here it is the reconstruction proxy
+ *   A(K) = -e(K),  e(K) = sqrt(J_K / J_0),
+ * J_K the Eq. 1 objective after `lloyd_iters` updates of kq_fit_codebook from
+ * C_0 = W[sel[0..K)], J_0 = sum_i |W_i|^2 (A_ori = 0: the unquantised layer has
+ * no error). N_init = floor(alpha * n) (kept in [1, n]); A_base = A(N_init);
+ * A_target = A_base - (A_ori - A_base) * r (Eq. 3); B_upper = N_init, B_lower = 0;
+ * each step tests N_curr = floor((B_upper + B_lower) / 2) and moves B_upper there
+ * when A(N_curr) > A_target, else B_lower. Stops after max_steps tests, when
+ * B_upper - B_lower <= 1, or when a test equals A_target exactly. The result is
+ * K = B_upper; C_out / idx / counts hold the fit of that size.
+ *   W          n x 9 fp32 (device, 16-byte aligned)
+ *   sel        sel_len >= N_init distinct row numbers in [0, n) (device int64): the
+ *              seeded draw whose prefixes initialise every trial
+ *   alpha      entry ratio, > 0;  r  threshold ratio, >= 0
+ *   max_steps  0 .. 64;  lloyd_iters  0 .. 100000 (updates per trial fit)
+ *   C_out      N_init x 9 fp32 (device);  idx  n int32;  counts  N_init int32 (device)
+ *   K_out      host int32;  err_out  host double e(K) or NULL
+ *   trace_K / trace_err  host arrays of max_steps + 1 entries or NULL: the sizes
+ *              tested (N_init first) and their e
+ *   steps_run  host int32 or NULL: bisection steps made
+ * Needs the workspace of (n, N_init). Synchronises `stream` after every trial fit
+ * (the decisions are taken on the host). */
+kq_status kq_search_codebook_size(const float *W, int64_t n, const int64_t *sel, int32_t sel_len, double alpha,
+                                  double r, int32_t max_steps, int32_t lloyd_iters, float *C_out, int32_t *idx,
+                                  int32_t *counts, int32_t *K_out, double *err_out, int32_t *trace_K,
+                                  double *trace_err, int32_t *steps_run, void *ws, size_t ws_bytes,
+                                  kq_stream_t stream);
+
 /* 6-bit kernel-codebook quantisation, Sec. 3.2: k-means with 64 levels over all
  * K*9 codebook scalars v_kj, each weighted by its entry's appearance count
  * z_k ("entry appearance time"), then the code of every scalar.

@@ -4,6 +4,7 @@
 #include <stddef.h>
 
 #include <atomic>
+#include <cmath>
 
 #include "kq_internal.cuh"
 
@@ -102,6 +103,36 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
         KQ_TRY(launch_pack_codebook(C, K, w.cd, w.hdr, s));
         KQ_TRY(launch_assign(W, n, w.cd, C, K, hint, idx, dist, w.blocksum, nb, w.part, w.hdr, sms, s));
     }
+    return KQ_OK;
+}
+
+// The k-means fit of kq_fit_codebook on carved workspace regions (sized for at
+// least K codewords). objective: iters + 1 device doubles or null; final_obj: one
+// device double receiving the objective of the final assignment, or null.
+kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int32_t iters, float *C_out,
+                  int32_t *idx, int32_t *counts, double *objective, double *final_obj, const Ws &w, int sms,
+                  cudaStream_t s) {
+    const size_t cbytes = (size_t)K * D * sizeof(float);
+    kq_status st;
+    KQ_TRY(launch_update_prepare(nullptr, K, w.acc, w.hdr, false, s));
+    KQ_TRY(launch_maxabs(W, n * D, &w.hdr->maxabs_bits, &w.hdr->status, sms, s));  // the scale, once per fit
+    KQ_TRY(cudaMemcpyAsync(w.cbuf0, C_init, cbytes, cudaMemcpyDeviceToDevice, s));
+    float *cur = w.cbuf0, *nxt = w.cbuf1;
+    int nb = 0;
+    // iteration t > 0 starts every row from its previous assignment (warm start)
+    for (int32_t t = 0; t < iters; ++t) {
+        if ((st = run_assign(W, n, cur, K, t > 0 ? idx : nullptr, idx, nullptr, &nb, w, sms, s)) != KQ_OK) return st;
+        if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
+        if ((st = run_update_exact(W, n, idx, K, cur, nxt, counts, w, sms, s)) != KQ_OK) return st;
+        float *tmp = cur;
+        cur = nxt;
+        nxt = tmp;
+    }
+    if ((st = run_assign(W, n, cur, K, iters > 0 ? idx : nullptr, idx, nullptr, &nb, w, sms, s)) != KQ_OK) return st;
+    if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + iters, s));
+    if (final_obj) KQ_TRY(launch_sum_blocks(w.blocksum, nb, final_obj, s));
+    KQ_TRY(launch_histogram(idx, n, K, counts, &w.hdr->status, sms, s));
+    KQ_TRY(cudaMemcpyAsync(C_out, cur, cbytes, cudaMemcpyDeviceToDevice, s));
     return KQ_OK;
 }
 
@@ -211,28 +242,81 @@ kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_i
     if (st != KQ_OK) return st;
     int sms = 0;
     if ((st = num_sms(&sms)) != KQ_OK) return st;
-    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    Ws w = carve(ws, n, K);
-    const size_t cbytes = (size_t)K * D * sizeof(float);
+    return run_fit(W, n, K, C_init, iters, C_out, idx, counts, objective, nullptr, carve(ws, n, K), sms,
+                   reinterpret_cast<cudaStream_t>(stream));
+}
 
-    KQ_TRY(launch_update_prepare(nullptr, K, w.acc, w.hdr, false, s));
-    KQ_TRY(launch_maxabs(W, n * D, &w.hdr->maxabs_bits, &w.hdr->status, sms, s));  // the scale, once per fit
-    KQ_TRY(cudaMemcpyAsync(w.cbuf0, C_init, cbytes, cudaMemcpyDeviceToDevice, s));
-    float *cur = w.cbuf0, *nxt = w.cbuf1;
-    int nb = 0;
-    // iteration t > 0 starts every row from its previous assignment (warm start)
-    for (int32_t t = 0; t < iters; ++t) {
-        if ((st = run_assign(W, n, cur, K, t > 0 ? idx : nullptr, idx, nullptr, &nb, w, sms, s)) != KQ_OK) return st;
-        if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
-        if ((st = run_update_exact(W, n, idx, K, cur, nxt, counts, w, sms, s)) != KQ_OK) return st;
-        float *tmp = cur;
-        cur = nxt;
-        nxt = tmp;
+kq_status kq_search_codebook_size(const float *W, int64_t n, const int64_t *sel, int32_t sel_len, double alpha,
+                                  double r, int32_t max_steps, int32_t lloyd_iters, float *C_out, int32_t *idx,
+                                  int32_t *counts, int32_t *K_out, double *err_out, int32_t *trace_K,
+                                  double *trace_err, int32_t *steps_run, void *ws, size_t ws_bytes,
+                                  kq_stream_t stream) {
+    if (n < 1 || n >= (1LL << 31) || !W || !sel || !C_out || !idx || !counts || !K_out) return KQ_ERR_INVALID_ARG;
+    if (!(alpha > 0.0) || !(alpha <= 1e9) || !(r >= 0.0) || !(r <= 1e9)) return KQ_ERR_INVALID_ARG;
+    if (max_steps < 0 || max_steps > 64 || lloyd_iters < 0 || lloyd_iters > 100000) return KQ_ERR_INVALID_ARG;
+    int64_t n_init = (int64_t)std::floor(alpha * (double)n);  // Algorithm 1: N_init = alpha * n
+    if (n_init < 1) n_init = 1;
+    if (n_init > n) n_init = n;
+    if (!sizes_ok(n, (int32_t)n_init) || sel_len < n_init) return KQ_ERR_INVALID_ARG;
+    if (!aligned(W, 16) || !aligned(sel, 8) || !aligned(C_out, 4) || !aligned(idx, 4) || !aligned(counts, 4))
+        return KQ_ERR_ALIGNMENT;
+    const int32_t N0 = (int32_t)n_init;
+    kq_status st = check_ws(ws, ws_bytes, n, N0);
+    if (st != KQ_OK) return st;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != KQ_OK) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    const Ws w = carve(ws, n, N0);  // every region sized for the largest codebook tried
+    // J_0 = sum |W_i|^2: the objective against the single zero codeword
+    KQ_TRY(cudaMemsetAsync(C_out, 0, D * sizeof(float), s));
+    if ((st = run_fit(W, n, 1, C_out, 0, C_out, idx, counts, nullptr, &w.hdr->obj, w, sms, s)) != KQ_OK) return st;
+    double J0 = 0.0;
+    KQ_TRY(cudaMemcpyAsync(&J0, &w.hdr->obj, sizeof(double), cudaMemcpyDeviceToHost, s));
+    KQ_TRY(cudaStreamSynchronize(s));
+    int32_t last_fit = 0;
+    // accuracy of a codebook of k entries: -(relative l2 reconstruction error)
+    auto accuracy_of = [&](int32_t k, double *acc) -> kq_status {
+        KQ_TRY(launch_init_codebook(W, n, sel, k, C_out, &w.hdr->status, s));
+        kq_status e = run_fit(W, n, k, C_out, lloyd_iters, C_out, idx, counts, nullptr, &w.hdr->obj, w, sms, s);
+        if (e != KQ_OK) return e;
+        double J = 0.0;
+        KQ_TRY(cudaMemcpyAsync(&J, &w.hdr->obj, sizeof(double), cudaMemcpyDeviceToHost, s));
+        KQ_TRY(cudaStreamSynchronize(s));
+        last_fit = k;
+        *acc = J0 > 0.0 ? -std::sqrt(J / J0) : 0.0;
+        return KQ_OK;
+    };
+    double a_base = 0.0;
+    if ((st = accuracy_of(N0, &a_base)) != KQ_OK) return st;
+    const double a_ori = 0.0;                              // the unquantised layer: no error
+    const double a_target = a_base - (a_ori - a_base) * r;  // Eq. 3
+    if (trace_K) trace_K[0] = N0;
+    if (trace_err) trace_err[0] = -a_base;
+    int32_t b_up = N0, b_lo = 0, steps = 0;
+    double a_up = a_base;  // accuracy at b_up
+    while (steps < max_steps && b_up - b_lo > 1) {
+        ++steps;
+        const int32_t k = (int32_t)(((int64_t)b_up + b_lo) / 2);
+        double a = 0.0;
+        if ((st = accuracy_of(k, &a)) != KQ_OK) return st;
+        if (trace_K) trace_K[steps] = k;
+        if (trace_err) trace_err[steps] = -a;
+        if (a > a_target) {
+            b_up = k;
+            a_up = a;
+        } else {
+            b_lo = k;
+        }
+        if (a == a_target) break;
     }
-    if ((st = run_assign(W, n, cur, K, iters > 0 ? idx : nullptr, idx, nullptr, &nb, w, sms, s)) != KQ_OK) return st;
-    if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + iters, s));
-    KQ_TRY(launch_histogram(idx, n, K, counts, &w.hdr->status, sms, s));
-    KQ_TRY(cudaMemcpyAsync(C_out, cur, cbytes, cudaMemcpyDeviceToDevice, s));
+    // leave the fit of the chosen size in C_out / idx / counts
+    if (last_fit != b_up) {
+        double a = 0.0;
+        if ((st = accuracy_of(b_up, &a)) != KQ_OK) return st;
+    }
+    *K_out = b_up;
+    if (err_out) *err_out = -a_up;
+    if (steps_run) *steps_run = steps;
     return KQ_OK;
 }
 

@@ -36,6 +36,7 @@ struct Header {
     uint32_t pad3;
     unsigned long long wtotal;          // level fit: sum of weights
     unsigned long long lacc[3][LEVELS][2];  // level fit: (weight sum, fixed-point sum) per level
+    double obj;                         // codebook-size search: objective of the last fit
 };
 static_assert(sizeof(Header) <= 4096, "header too large");
 

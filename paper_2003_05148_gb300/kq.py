@@ -24,7 +24,7 @@ FLAG_NONFINITE, FLAG_INDEX_RANGE, FLAG_CODE_RANGE, FLAG_TIMEOUT = 0x1, 0x2, 0x4,
 EXPORTS = ["kq_status_string", "kq_abi_version", "kq_kernel_launches", "kq_workspace_bytes", "kq_device_status", "kq_init_codebook",
            "kq_assign", "kq_update_centroids", "kq_fit_codebook", "kq_quantize_codebook_6bit", "kq_reconstruct",
            "kq_compression_report", "kq_conventional_ratio", "kq_assign_noalloc", "kq_quantize_scalars_6bit",
-           "kq_codebook_grad_step", "kq_levels_grad_step"]
+           "kq_codebook_grad_step", "kq_levels_grad_step", "kq_search_codebook_size"]
 
 
 class KQError(RuntimeError):
@@ -67,6 +67,8 @@ def lib() -> ctypes.CDLL:
             "kq_quantize_scalars_6bit": ([P, i64, i32, P, P, P, P, sz, P], ctypes.c_int),
             "kq_codebook_grad_step": ([P, i64, P, i32, ctypes.c_float, P, P, P, P, sz, P], ctypes.c_int),
             "kq_levels_grad_step": ([P, i64, P, i32, P, ctypes.c_float, P, P, P, P, sz, P], ctypes.c_int),
+            "kq_search_codebook_size": ([P, i64, P, i32, ctypes.c_double, ctypes.c_double, i32, i32, P, P, P,
+                                         P, P, P, P, P, P, sz, P], ctypes.c_int),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -189,6 +191,22 @@ def kq_levels_grad_step(G, idx, codes, lr: float, levels, levels_next, counts, w
         _dev(codes, "codes", torch.uint8), float(lr), _dev(levels, "levels", torch.float32),
         _dev(levels_next, "levels_next", torch.float32), _dev(counts, "counts", torch.int64),
         _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+
+
+def kq_search_codebook_size(W, sel, alpha: float, r: float, max_steps: int, lloyd_iters: int, C_out, idx, counts,
+                            ws, stream=None):
+    """Returns (K, e(K), trace [(size, e)]); C_out / idx / counts hold the fit of size K."""
+    k = ctypes.c_int32(0)
+    err = ctypes.c_double(0.0)
+    steps = ctypes.c_int32(0)
+    tK = (ctypes.c_int32 * (max_steps + 1))()
+    tE = (ctypes.c_double * (max_steps + 1))()
+    _check("kq_search_codebook_size", lib().kq_search_codebook_size(
+        _dev(W, "W", torch.float32), _rows(W), _dev(sel, "sel", torch.int64), sel.numel(), float(alpha), float(r),
+        max_steps, lloyd_iters, _dev(C_out, "C_out", torch.float32), _dev(idx, "idx", torch.int32),
+        _dev(counts, "counts", torch.int32), ctypes.byref(k), ctypes.byref(err), tK, tE, ctypes.byref(steps),
+        _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+    return k.value, err.value, [(tK[i], tE[i]) for i in range(steps.value + 1)]
 
 
 def kq_reconstruct(idx, C, codes, levels, W_out, ws, K: Optional[int] = None, stream=None) -> None:

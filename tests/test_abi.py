@@ -89,6 +89,22 @@ def test_host_validation_before_any_device_work(lib):
     assert L.kq_levels_grad_step(good, 1024, good, 16, good, 0.1, good, good, ctypes.c_void_p((1 << 20) + 4),
                                  good, 4096, None) == 2  # counts not 8-byte aligned
     assert L.kq_levels_grad_step(good, 1024, good, 16, good, 0.1, good, good, None, good, 4095, None) == 6
+    ws_s = kq.kq_workspace_bytes(1024, 256)
+    S = L.kq_search_codebook_size
+    assert S(good, 1024, good, 256, 0.0, 0.5, 8, 3, good, good, good, ctypes.byref(ctypes.c_int32()), None, None, None,
+             None, good, ws_s, None) == 1  # alpha = 0
+    assert S(good, 1024, good, 256, 0.25, -0.5, 8, 3, good, good, good, ctypes.byref(ctypes.c_int32()), None, None,
+             None, None, good, ws_s, None) == 1  # r < 0
+    assert S(good, 1024, good, 256, 0.25, 0.5, 65, 3, good, good, good, ctypes.byref(ctypes.c_int32()), None, None,
+             None, None, good, ws_s, None) == 1  # too many steps
+    assert S(good, 1024, good, 255, 0.25, 0.5, 8, 3, good, good, good, ctypes.byref(ctypes.c_int32()), None, None,
+             None, None, good, ws_s, None) == 1  # sel shorter than N_init = 256
+    assert S(good, 1024, good, 256, 0.25, 0.5, 8, 3, good, good, good, None, None, None, None, None, good, ws_s,
+             None) == 1  # no K output
+    assert S(odd, 1024, good, 256, 0.25, 0.5, 8, 3, good, good, good, ctypes.byref(ctypes.c_int32()), None, None,
+             None, None, good, ws_s, None) == 2
+    assert S(good, 1024, good, 256, 0.25, 0.5, 8, 3, good, good, good, ctypes.byref(ctypes.c_int32()), None, None,
+             None, None, good, ws_s - 1, None) == 6
 
 
 def _report_rows():
