@@ -447,6 +447,7 @@ def run_only(args):
         "update": lambda: kq.kq_update_centroids(W, idx, C, C2, counts, ws),
         "quantize": lambda: kq.kq_quantize_codebook_6bit(C2, counts, 100, levels, codes, None, ws),
         "reconstruct": lambda: kq.kq_reconstruct(idx, None, codes, levels, Wr, ws, K=K),
+        "fusedrecon": lambda: kq.kq_quantize_reconstruct(idx, C2, levels, codes, Wr, ws),
     }
     # retraining steps (Eq. 2; Sec. 3.2): the kernels themselves stand in for the
     # gradients (the timing depends on sizes and the code distribution only)
@@ -455,7 +456,7 @@ def run_only(args):
     calls["gradstep"] = lambda: kq.kq_codebook_grad_step(W, idx, 0.01, C2, C, counts, ws)
     calls["levelgrad"] = lambda: kq.kq_levels_grad_step(W, idx, codes, 0.01, levels, lv_next, lv_counts, ws)
     alg_bytes = {"update": 40 * n + 76 * K, "gradstep": 40 * n + 76 * K, "levelgrad": 40 * n + 9 * K,
-                 "reconstruct": 40 * n + 9 * K + 256}
+                 "reconstruct": 40 * n + 9 * K + 256, "fusedrecon": 40 * n + 45 * K + 256}
     if args.only == "search":
         # Algorithm 1 on the VGG-16 conv3_2 layer (workload 2): alpha = 0.25, r = 0.5,
         # 8 bisection steps, 20 Lloyd updates per trial (the workload's own count)
@@ -588,7 +589,7 @@ def main():
     ap.add_argument("--ref-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--only", choices=["assign", "update", "quantize", "reconstruct", "gradstep", "levelgrad",
-                                       "fcquant", "search"],
+                                       "fcquant", "search", "fusedrecon"],
                     help="profiling aid: time one entry point on its own (no bench line)")
     ap.add_argument("--n", type=int, default=4194304)
     ap.add_argument("--K", type=int, default=65536)

@@ -283,6 +283,20 @@ kq_status kq_levels_grad_step(const float *G, int64_t n, const int32_t *idx, int
 kq_status kq_reconstruct(const int32_t *idx, int64_t n, const float *C, int32_t K, const uint8_t *codes,
                          const float *levels, float *W_out, void *ws, size_t ws_bytes, kq_stream_t stream);
 
+/* Fused 6-bit encode + recovery, Sec. 3.2: the codebook scalars are encoded to
+ * their nearest levels (the encode rule of kq_quantize_codebook_6bit: fp32
+ * |v - level|, lower index on ties) and the weights rebuilt from the encoded
+ * codebook, in one launch:
+ *   codes[k][j] = argmin_l |C[k][j] - levels[l]|,   W_out[i][j] = levels[codes[idx[i]][j]].
+ *   idx    n int32 (device);  C  K x 9 fp32 (device);  levels 64 fp32 (device)
+ *   codes  K x 9 uint8 output (device) or NULL (not stored)
+ *   W_out  n x 9 fp32 output (device, 16-byte aligned)
+ * An index outside [0, K) writes a zero row and sets KQ_FLAG_INDEX_RANGE; a
+ * non-finite codebook value sets KQ_FLAG_NONFINITE (it encodes to level 0). The
+ * CTAs meet at a bounded grid barrier (~2 s; KQ_FLAG_TIMEOUT if it runs out). */
+kq_status kq_quantize_reconstruct(const int32_t *idx, int64_t n, const float *C, int32_t K, const float *levels,
+                                  uint8_t *codes, float *W_out, void *ws, size_t ws_bytes, kq_stream_t stream);
+
 /* Storage accounting of one layer (host only, no device work), Sec. 3.2-3.3 and
  * Sec. 4.1:
  *   Eq. 4  total_bits B = k * omega^2 * b_c + n * ceil(log2 k)

@@ -408,6 +408,19 @@ kq_status kq_reconstruct(const int32_t *idx, int64_t n, const float *C, int32_t 
     return KQ_OK;
 }
 
+kq_status kq_quantize_reconstruct(const int32_t *idx, int64_t n, const float *C, int32_t K, const float *levels,
+                                  uint8_t *codes, float *W_out, void *ws, size_t ws_bytes, kq_stream_t stream) {
+    if (!sizes_ok(n, K) || !idx || !C || !levels || !W_out) return KQ_ERR_INVALID_ARG;
+    if (!aligned(idx, 4) || !aligned(C, 4) || !aligned(levels, 4) || !aligned(W_out, 16)) return KQ_ERR_ALIGNMENT;
+    kq_status st = check_ws(ws, ws_bytes, n, K);
+    if (st != KQ_OK) return st;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != KQ_OK) return st;
+    Ws w = carve(ws, n, K);
+    return cuda_status(launch_encode_gather(C, K, levels, codes, w.cq, idx, n, W_out, w.hdr, sms,
+                                            reinterpret_cast<cudaStream_t>(stream)));
+}
+
 kq_status kq_compression_report(int64_t n, int32_t k, int32_t omega, int32_t b_c, kq_report *out) {
     if (n < 1 || k < 1 || omega < 1 || b_c < 1 || !out) return KQ_ERR_INVALID_ARG;
     const int64_t w2 = (int64_t)omega * omega;

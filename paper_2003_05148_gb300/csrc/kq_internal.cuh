@@ -133,6 +133,64 @@ __device__ __forceinline__ long long fixed_rn(float v, int S) {
 
 __device__ __forceinline__ void set_flag(uint32_t *status, uint32_t bit) { atomicOr(status, bit); }
 
+// ---- 6-bit encode (Sec. 3.2): nearest of 64 levels (used by the level fit and by
+// the fused encode + recovery kernel)
+
+// Nearest of the 64 levels by fp32 |v - level|, lower index on ties (Sec. 3.2 encode).
+__device__ __forceinline__ int nearest_level(float v, const float *L) {
+    float best = __int_as_float(0x7f800000);
+    int bl = 0;
+#pragma unroll 16
+    for (int l = 0; l < LEVELS; ++l) {
+        const float d = fabsf(v - L[l]);
+        if (d < best) {
+            best = d;
+            bl = l;
+        }
+    }
+    return bl;
+}
+
+// nearest_level for levels in non-decreasing order, by binary search; the same
+// code. With p the last level <= v, d_l = |fl(v - L_l)| is non-increasing on
+// [0, p] and non-decreasing on [p, 63] (rounding is monotone), so the minimum is
+// d_p or d_{p+1}; the first index holding it (the scan's tie rule) is p + 1 when
+// d_{p+1} < d_p, else the start of the run of levels <= p whose distance equals
+// d_p, which is a suffix of [0, p]. A minimum of +inf gives 0, as in the scan.
+// The code of v given cnt = #{l : L_l <= v} (levels sorted; see above).
+__device__ __forceinline__ int nearest_from_count(float v, const float *L, int cnt) {
+    const int p = cnt - 1;
+    if (p < 0) return 0;  // every level is above v: distances grow with l
+    const float dp = fabsf(v - L[p]);
+    if (p < LEVELS - 1 && fabsf(v - L[p + 1]) < dp) return p + 1;
+    if (!(dp < __int_as_float(0x7f800000))) return 0;  // the minimum distance is +inf
+    if (p == 0 || fabsf(v - L[p - 1]) > dp) return p;
+    int f = 0;  // number of levels l < p with d_l > d_p (a prefix)
+#pragma unroll
+    for (int step = 32; step > 0; step >>= 1)
+        if (f + step - 1 < p && fabsf(v - L[f + step - 1]) > dp) f += step;
+    return f;
+}
+
+__device__ __forceinline__ int nearest_level_sorted(float v, const float *L) {
+    if (v != v) return 0;  // NaN: no distance is below +inf
+    int cnt = 0;           // number of levels <= v
+#pragma unroll
+    for (int step = 32; step > 0; step >>= 1)
+        if (L[cnt + step - 1] <= v) cnt += step;
+    cnt += L[cnt] <= v;  // cnt could only reach 63 above
+    return nearest_from_count(v, L, cnt);
+}
+
+// Levels in non-decreasing order (and no NaN), so that nearest_level_sorted applies.
+__device__ __forceinline__ bool levels_sorted(const float *L) {
+    bool ok = true;
+#pragma unroll 8
+    for (int l = 0; l < LEVELS - 1; ++l) ok &= L[l] <= L[l + 1];
+    return ok;
+}
+
+
 __device__ __forceinline__ bool finite9(const float *v) {
     bool ok = true;
 #pragma unroll
@@ -230,5 +288,10 @@ cudaError_t launch_gather_rows(const int32_t *idx, int64_t n, const float *Cp, c
                                cudaStream_t s);
 cudaError_t launch_init_codebook(const float *W, int64_t n, const int64_t *sel, int32_t K, float *C0,
                                  uint32_t *status, cudaStream_t s);
+// Fused 6-bit encode of the codebook against given levels + K+C recovery (one
+// cooperative launch with a bounded grid barrier).
+cudaError_t launch_encode_gather(const float *C, int32_t K, const float *levels, uint8_t *codes,
+                                 unsigned long long *Cq, const int32_t *idx, int64_t n, float *W_out, Header *hdr,
+                                 int num_sms, cudaStream_t s);
 
 }  // namespace kq

@@ -111,42 +111,20 @@ gather_rows_kernel(const int32_t *__restrict__ idx, int64_t n, const float *__re
     if (__any_sync(0xffffffffu, bad) && lane == 0) set_flag(status, KQ_FLAG_INDEX_RANGE);
 }
 
-// K+C recovery. A warp owns 32 consecutive kernels (1152 output bytes = 72 float4).
-// Each lane fetches the packed codes of its own kernel (one 8-byte word, instead of
-// a 36-byte row), then produces output float4 number lane, lane + 32 and (lanes
-// 0-7) lane + 64 directly: the at most two kernels a float4 spans send their code
-// words by shuffle, and every code is looked up in a level table replicated across
-// the 32 shared-memory banks (level l for lane L at [l][L]: no bank conflicts). No
-// staging tile; the stores are coalesced streaming float4 stores. Launched as a
-// programmatic dependent of decode_codebook_kernel (the launch and the level table
-// overlap the decode; Cq is read after griddepcontrol.wait): 47.3 -> 44.0 us per
-// call on the stress layer. (Prefetching the next step's indices, and 4 instead
-// of 8 CTAs per SM, measured faster alone but slower inside the fit's step.)
-__global__ void __launch_bounds__(R_THREADS)
-gather_codes_kernel(const int32_t *__restrict__ idx, int64_t n, const unsigned long long *__restrict__ Cq,
-                    const float *__restrict__ levels, int32_t K, float *__restrict__ W_out, uint32_t *status) {
-    __shared__ float lv[LEVELS + 1][32];  // row LEVELS decodes out-of-range codes to 0
-    for (int e = threadIdx.x; e < (LEVELS + 1) * 32; e += R_THREADS)
-        lv[e / 32][e % 32] = e / 32 < LEVELS ? levels[e / 32] : 0.f;
-    __syncthreads();
+// The loop of gather_codes_kernel over the chunks of CTA `cta` of `ncta` (and the
+// ragged end in CTA 0); lv is the replicated level table, ra/j0/split the lane's
+// float4 slots. Returns whether this thread saw an index outside [0, K).
+__device__ __forceinline__ bool gather_codes_rows(const int32_t *__restrict__ idx, int64_t n,
+                                                  const unsigned long long *__restrict__ Cq, int32_t K,
+                                                  float *__restrict__ W_out, const float (*lv)[32], const int *ra,
+                                                  const int *j0, const int *split, int64_t cta, int64_t ncta) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // slot s: float4 v = lane + 32 s of the chunk; its first element is coordinate
-    // j0 of kernel ra, elements e < split belong to ra, the rest to ra + 1
-    int ra[3], j0[3], split[3];
-#pragma unroll
-    for (int s = 0; s < 3; ++s) {
-        const int v = min(lane + 32 * s, 32 * D / 4 - 1);
-        ra[s] = (4 * v) / D;
-        j0[s] = 4 * v - D * ra[s];
-        split[s] = D - j0[s];
-    }
-    asm volatile("griddepcontrol.wait;" ::: "memory");  // Cq is written by the decode kernel
     bool bad = false;
     const int64_t nch = n / 32;
     // two chunks per warp step: both index loads, then both code gathers are in
     // flight before any decoding
     const int64_t nch2 = nch / 2;
-    for (int64_t c2 = (int64_t)blockIdx.x * R_WARPS + warp; c2 < nch2 + (nch & 1); c2 += (int64_t)gridDim.x * R_WARPS) {
+    for (int64_t c2 = cta * R_WARPS + warp; c2 < nch2 + (nch & 1); c2 += ncta * R_WARPS) {
         const int64_t ch0 = 2 * c2;
         const bool two = ch0 + 1 < nch;
         int32_t k[2];
@@ -184,7 +162,7 @@ gather_codes_kernel(const int32_t *__restrict__ idx, int64_t n, const unsigned l
         }
     }
     // ragged end (< 32 kernels): CTA 0, plain loads and stores
-    if (blockIdx.x == 0) {
+    if (cta == 0) {
         for (int64_t i = nch * 32 + threadIdx.x; i < n; i += R_THREADS) {
             const int32_t kk = idx[i];
             const bool ok = (uint32_t)kk < (uint32_t)K;
@@ -194,7 +172,91 @@ gather_codes_kernel(const int32_t *__restrict__ idx, int64_t n, const unsigned l
             for (int j = 0; j < D; ++j) W_out[i * D + j] = lv[(q >> (7 * j)) & 127u][0];
         }
     }
+    return bad;
+}
+
+// K+C recovery. A warp owns 32 consecutive kernels (1152 output bytes = 72 float4).
+// Each lane fetches the packed codes of its own kernel (one 8-byte word, instead of
+// a 36-byte row), then produces output float4 number lane, lane + 32 and (lanes
+// 0-7) lane + 64 directly: the at most two kernels a float4 spans send their code
+// words by shuffle, and every code is looked up in a level table replicated across
+// the 32 shared-memory banks (level l for lane L at [l][L]: no bank conflicts). No
+// staging tile; the stores are coalesced streaming float4 stores. Launched as a
+// programmatic dependent of decode_codebook_kernel (the launch and the level table
+// overlap the decode; Cq is read after griddepcontrol.wait): 47.3 -> 44.0 us per
+// call on the stress layer. (Prefetching the next step's indices, and 4 instead
+// of 8 CTAs per SM, measured faster alone but slower inside the fit's step.)
+__global__ void __launch_bounds__(R_THREADS)
+gather_codes_kernel(const int32_t *__restrict__ idx, int64_t n, const unsigned long long *__restrict__ Cq,
+                    const float *__restrict__ levels, int32_t K, float *__restrict__ W_out, uint32_t *status) {
+    __shared__ float lv[LEVELS + 1][32];  // row LEVELS decodes out-of-range codes to 0
+    for (int e = threadIdx.x; e < (LEVELS + 1) * 32; e += R_THREADS)
+        lv[e / 32][e % 32] = e / 32 < LEVELS ? levels[e / 32] : 0.f;
+    __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // slot s: float4 v = lane + 32 s of the chunk; its first element is coordinate
+    // j0 of kernel ra, elements e < split belong to ra, the rest to ra + 1
+    int ra[3], j0[3], split[3];
+#pragma unroll
+    for (int s = 0; s < 3; ++s) {
+        const int v = min(lane + 32 * s, 32 * D / 4 - 1);
+        ra[s] = (4 * v) / D;
+        j0[s] = 4 * v - D * ra[s];
+        split[s] = D - j0[s];
+    }
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // Cq is written by the decode kernel
+    const bool bad = gather_codes_rows(idx, n, Cq, K, W_out, lv, ra, j0, split, blockIdx.x, gridDim.x);
     if (__any_sync(0xffffffffu, bad) && lane == 0) set_flag(status, KQ_FLAG_INDEX_RANGE);
+}
+
+// Fused 6-bit encode + K+C recovery (Sec. 3.2: the codebook scalars are encoded
+// to their nearest levels, and the weights are the decoded codebook rows at the
+// kernel indices), one cooperative launch: every CTA encodes a grid-stride share of
+// the codewords into the packed code words of gather_codes_kernel (and the code
+// bytes, when asked for), all CTAs meet at a bounded grid barrier, then gather.
+__global__ void __launch_bounds__(R_THREADS)
+encode_gather_kernel(const float *__restrict__ C, int32_t K, const float *__restrict__ levels,
+                     uint8_t *__restrict__ codes, unsigned long long *__restrict__ Cq, const int32_t *__restrict__ idx,
+                     int64_t n, float *__restrict__ W_out, Header *hdr) {
+    __shared__ float L[LEVELS];
+    __shared__ float lv[LEVELS + 1][32];
+    __shared__ int s_sorted;
+    for (int e = threadIdx.x; e < (LEVELS + 1) * 32; e += R_THREADS)
+        lv[e / 32][e % 32] = e / 32 < LEVELS ? levels[e / 32] : 0.f;
+    if (threadIdx.x < LEVELS) L[threadIdx.x] = levels[threadIdx.x];
+    __syncthreads();
+    if (threadIdx.x == 0) s_sorted = levels_sorted(L);
+    __syncthreads();
+    const bool sorted = s_sorted;
+    bool nonfinite = false;
+    for (int64_t k = (int64_t)blockIdx.x * R_THREADS + threadIdx.x; k < K; k += (int64_t)gridDim.x * R_THREADS) {
+        float v[D];
+#pragma unroll
+        for (int j = 0; j < D; ++j) v[j] = __ldg(C + k * D + j);
+        unsigned long long q = 0;
+#pragma unroll
+        for (int j = 0; j < D; ++j) {
+            nonfinite |= !isfinite(v[j]);
+            const int c = sorted ? nearest_level_sorted(v[j], L) : nearest_level(v[j], L);
+            q |= (unsigned long long)c << (7 * j);
+            if (codes) codes[k * D + j] = (uint8_t)c;
+        }
+        Cq[k] = q;
+    }
+    if (nonfinite) set_flag(&hdr->status, KQ_FLAG_NONFINITE);
+    unsigned epoch = 0;
+    if (!grid_barrier(hdr, gridDim.x, epoch)) return;
+    const int lane = threadIdx.x & 31;
+    int ra[3], j0[3], split[3];
+#pragma unroll
+    for (int s = 0; s < 3; ++s) {
+        const int v = min(lane + 32 * s, 32 * D / 4 - 1);
+        ra[s] = (4 * v) / D;
+        j0[s] = 4 * v - D * ra[s];
+        split[s] = D - j0[s];
+    }
+    const bool bad = gather_codes_rows(idx, n, Cq, K, W_out, lv, ra, j0, split, blockIdx.x, gridDim.x);
+    if (__any_sync(0xffffffffu, bad) && lane == 0) set_flag(&hdr->status, KQ_FLAG_INDEX_RANGE);
 }
 
 __global__ void __launch_bounds__(256)
@@ -244,6 +306,29 @@ cudaError_t launch_gather_rows(const int32_t *idx, int64_t n, const float *Cp, c
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
     if (blocks < 1) blocks = 1;
     gather_rows_kernel<<<(unsigned)blocks, R_THREADS, 0, s>>>(idx, n, Cp, K, W_out, status);
+    count_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_encode_gather(const float *C, int32_t K, const float *levels, uint8_t *codes,
+                                 unsigned long long *Cq, const int32_t *idx, int64_t n, float *W_out, Header *hdr,
+                                 int num_sms, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(&hdr->barrier, 0, 2 * sizeof(uint32_t), s);  // barrier counter, abort word
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, encode_gather_kernel, R_THREADS, 0);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    int64_t blocks = ((n / 32 + 1) / 2 + R_WARPS - 1) / R_WARPS;
+    const int64_t enc_blocks = ((int64_t)K + R_THREADS - 1) / R_THREADS;
+    if (blocks < enc_blocks) blocks = enc_blocks;
+    if (blocks > (int64_t)per_sm * num_sms) blocks = (int64_t)per_sm * num_sms;  // co-resident by construction
+    if (blocks < 1) blocks = 1;
+    void *params[] = {(void *)&C, (void *)&K, (void *)&levels, (void *)&codes, (void *)&Cq,
+                      (void *)&idx, (void *)&n, (void *)&W_out, (void *)&hdr};
+    e = cudaLaunchCooperativeKernel((const void *)encode_gather_kernel, dim3((unsigned)blocks), dim3(R_THREADS),
+                                    params, 0, s);
+    if (e != cudaSuccess) return e;
     count_launch();
     return cudaGetLastError();
 }

@@ -24,7 +24,7 @@ FLAG_NONFINITE, FLAG_INDEX_RANGE, FLAG_CODE_RANGE, FLAG_TIMEOUT = 0x1, 0x2, 0x4,
 EXPORTS = ["kq_status_string", "kq_abi_version", "kq_kernel_launches", "kq_workspace_bytes", "kq_device_status", "kq_init_codebook",
            "kq_assign", "kq_update_centroids", "kq_fit_codebook", "kq_quantize_codebook_6bit", "kq_reconstruct",
            "kq_compression_report", "kq_conventional_ratio", "kq_assign_noalloc", "kq_quantize_scalars_6bit",
-           "kq_codebook_grad_step", "kq_levels_grad_step", "kq_search_codebook_size"]
+           "kq_codebook_grad_step", "kq_levels_grad_step", "kq_search_codebook_size", "kq_quantize_reconstruct"]
 
 
 class KQError(RuntimeError):
@@ -67,6 +67,7 @@ def lib() -> ctypes.CDLL:
             "kq_quantize_scalars_6bit": ([P, i64, i32, P, P, P, P, sz, P], ctypes.c_int),
             "kq_codebook_grad_step": ([P, i64, P, i32, ctypes.c_float, P, P, P, P, sz, P], ctypes.c_int),
             "kq_levels_grad_step": ([P, i64, P, i32, P, ctypes.c_float, P, P, P, P, sz, P], ctypes.c_int),
+            "kq_quantize_reconstruct": ([P, i64, P, i32, P, P, P, P, sz, P], ctypes.c_int),
             "kq_search_codebook_size": ([P, i64, P, i32, ctypes.c_double, ctypes.c_double, i32, i32, P, P, P,
                                          P, P, P, P, P, P, sz, P], ctypes.c_int),
         }
@@ -207,6 +208,13 @@ def kq_search_codebook_size(W, sel, alpha: float, r: float, max_steps: int, lloy
         _dev(counts, "counts", torch.int32), ctypes.byref(k), ctypes.byref(err), tK, tE, ctypes.byref(steps),
         _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
     return k.value, err.value, [(tK[i], tE[i]) for i in range(steps.value + 1)]
+
+
+def kq_quantize_reconstruct(idx, C, levels, codes, W_out, ws, stream=None) -> None:
+    _check("kq_quantize_reconstruct", lib().kq_quantize_reconstruct(
+        _dev(idx, "idx", torch.int32), idx.numel(), _dev(C, "C", torch.float32), _rows(C),
+        _dev(levels, "levels", torch.float32), _dev(codes, "codes", torch.uint8), _dev(W_out, "W_out", torch.float32),
+        _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
 
 
 def kq_reconstruct(idx, C, codes, levels, W_out, ws, K: Optional[int] = None, stream=None) -> None:

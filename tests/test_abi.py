@@ -89,6 +89,11 @@ def test_host_validation_before_any_device_work(lib):
     assert L.kq_levels_grad_step(good, 1024, good, 16, good, 0.1, good, good, ctypes.c_void_p((1 << 20) + 4),
                                  good, 4096, None) == 2  # counts not 8-byte aligned
     assert L.kq_levels_grad_step(good, 1024, good, 16, good, 0.1, good, good, None, good, 4095, None) == 6
+    QR = L.kq_quantize_reconstruct
+    assert QR(good, 1024, good, 16, None, None, good, good, ws_bytes, None) == 1  # no levels
+    assert QR(good, 1024, good, 2048, good, None, good, good, ws_bytes, None) == 1  # K > n
+    assert QR(good, 1024, good, 16, good, None, odd, good, ws_bytes, None) == 2  # W_out alignment
+    assert QR(good, 1024, good, 16, good, None, good, good, ws_bytes - 1, None) == 6
     ws_s = kq.kq_workspace_bytes(1024, 256)
     S = L.kq_search_codebook_size
     assert S(good, 1024, good, 256, 0.0, 0.5, 8, 3, good, good, good, ctypes.byref(ctypes.c_int32()), None, None, None,

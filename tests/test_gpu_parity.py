@@ -400,6 +400,50 @@ def test_reconstruct(n, K):
     assert st == 0 and bits_equal(Wkc, oracle.reconstruct(idx, C, cd, lv))
 
 
+def gpu_quantize_reconstruct(idx, C, levels, want_codes=True):
+    n, K = idx.shape[0], C.shape[0]
+    Wr = torch.empty(n, 9, dtype=torch.float32, device=dev())
+    codes = torch.empty(K, 9, dtype=torch.uint8, device=dev()) if want_codes else None
+    ws = kq.workspace(n, K, dev())
+    kq.kq_quantize_reconstruct(to_dev(idx.astype(np.int32)), to_dev(C), to_dev(levels), codes, Wr, ws)
+    st, flags = kq.kq_device_status(ws)
+    return Wr.cpu().numpy(), (codes.cpu().numpy() if want_codes else None), st, flags
+
+
+@pytest.mark.parametrize("n,K,case", [(1, 1, "fit"), (31, 5, "fit"), (4096, 16, "fit"), (100001, 256, "fit"),
+                                      (4194304, 65536, "fit"), (50000, 3000, "shuffled"), (50000, 3000, "duplicates"),
+                                      (50000, 3000, "no_codes")])
+def test_quantize_reconstruct_fused(n, K, case):
+    # one launch: encode the float codebook against the levels, then gather; equal to
+    # encoding with the oracle and reconstructing from those codes
+    C = synth.random_kernels(K, 9, K + 7, 0.05)
+    idx = synth.below(synth.stream_key(n + 9, 2), n, K).astype(np.int32)
+    counts = np.bincount(idx, minlength=K).astype(np.int32)
+    levels, _, _ = oracle.level_fit(C, counts, 20)
+    if case == "shuffled":  # unsorted levels: the 64-way scan
+        levels = levels[synth.below(synth.stream_key(11, 2), 64, 64).argsort(kind="stable")]
+    elif case == "duplicates":  # ties between equal levels go to the lower index
+        levels = np.repeat(levels[::4], 4).astype(np.float32)
+    codes_ref = oracle.encode(C.reshape(-1), levels).reshape(K, 9)
+    Wr, codes, st, _ = gpu_quantize_reconstruct(idx, C, levels, want_codes=case != "no_codes")
+    assert st == 0
+    assert bits_equal(Wr, oracle.reconstruct(idx, C, codes_ref, levels))
+    if case != "no_codes":
+        assert np.array_equal(codes, codes_ref)
+
+
+def test_quantize_reconstruct_flags():
+    C = synth.random_kernels(10, 9, 3)
+    idx = np.arange(100, dtype=np.int32) % 10
+    idx[7] = 10
+    levels = np.linspace(-1, 1, 64).astype(np.float32)
+    Wr, _, st, flags = gpu_quantize_reconstruct(idx, C, levels)
+    assert st == 5 and flags & kq.FLAG_INDEX_RANGE and np.all(Wr[7] == 0)
+    C[2, 2] = np.nan
+    Wr, codes, st, flags = gpu_quantize_reconstruct(np.arange(10, dtype=np.int32), C, levels)
+    assert st == 3 and flags & kq.FLAG_NONFINITE and codes[2, 2] == 0
+
+
 def test_reconstruct_flags_bad_index_and_code():
     C = synth.random_kernels(10, 9, 1)
     idx = np.arange(100, dtype=np.int32) % 10
