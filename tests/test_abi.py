@@ -142,3 +142,22 @@ def test_conventional_ratio_matches_oracle(lib):
         kq.kq_conventional_ratio(10, 3, 1, 32)
     with pytest.raises(kq.KQError):
         kq.kq_compression_report(0, 4)
+
+
+def test_cuda_failure_returns_status_without_device(lib):
+    # Every argument valid, no CUDA device: the first CUDA runtime call fails, and the
+    # entry point returns KQ_ERR_CUDA (4) before anything is enqueued. (Skipped where a
+    # GPU exists: the placeholder pointers below must never reach a kernel.)
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a CUDA device is present")
+    L = lib
+    good = ctypes.c_void_p(1 << 20)
+    ws_bytes = kq.kq_workspace_bytes(1024, 16)
+    assert L.kq_assign(good, 1024, good, 16, None, good, None, good, ws_bytes, None) == 4
+    assert L.kq_update_centroids(good, 1024, good, 16, good, good, good, good, ws_bytes, None) == 4
+    assert L.kq_fit_codebook(good, 1024, 16, good, 3, 0, good, good, good, None, good, ws_bytes, None) == 4
+    assert L.kq_quantize_codebook_6bit(good, 16, good, 10, good, good, None, good, ws_bytes, None) == 4
+    assert L.kq_reconstruct(good, 1024, good, 16, None, None, good, good, ws_bytes, None) == 4
+    assert L.kq_quantize_reconstruct(good, 1024, good, 16, good, None, good, good, ws_bytes, None) == 4
+    assert L.kq_device_status(good, ws_bytes, None, None) == 4
