@@ -65,6 +65,8 @@ struct Ws {
     float *cbuf0, *cbuf1, *cp;
     unsigned long long *cq;
     float *cpk;
+    float *dist;
+    int32_t *perm, *pcnt;
 };
 
 Ws carve(void *ws, int64_t n, int32_t K) {
@@ -81,6 +83,9 @@ Ws carve(void *ws, int64_t n, int32_t K) {
     w.cp = reinterpret_cast<float *>(b + L.cp);
     w.cq = reinterpret_cast<unsigned long long *>(b + L.cq);
     w.cpk = reinterpret_cast<float *>(b + L.cpk);
+    w.dist = reinterpret_cast<float *>(b + L.dist);
+    w.perm = reinterpret_cast<int32_t *>(b + L.perm);
+    w.pcnt = reinterpret_cast<int32_t *>(b + L.pcnt);
     return w;
 }
 
@@ -98,7 +103,16 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
                      float *dist, int *nb, const Ws &w, int sms, cudaStream_t s) {
     if (tc_eligible(n, sms)) {
         KQ_TRY(launch_pack_codebook_tc(C, K, w.cpk, w.hdr, s));
-        KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K, hint, idx, dist, w.blocksum, nb, w.hdr, s));
+        // warm start: rows grouped by hint (see kq_assign_tc.cu); the objective's block
+        // sums are then taken over the distances in row order, whatever the grouping
+        const int32_t *perm = nullptr;
+        if (hint) {
+            KQ_TRY(launch_hint_permutation(hint, n, K, w.pcnt, w.perm, sms, s));
+            perm = w.perm;
+        }
+        float *d = dist ? dist : w.dist;
+        KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K, hint, perm, idx, d, nullptr, nb, w.hdr, s));
+        KQ_TRY(launch_dist_block_sums(d, n, w.blocksum, nb, s));
     } else {
         KQ_TRY(launch_pack_codebook(C, K, w.cd, w.hdr, s));
         KQ_TRY(launch_assign(W, n, w.cd, C, K, hint, idx, dist, w.blocksum, nb, w.part, w.hdr, sms, s));

@@ -302,8 +302,8 @@ struct TcShared {
 
 __global__ void __launch_bounds__(TC_THREADS, 1)
 assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict__ C, const float *__restrict__ Cpk,
-                 int32_t K, int32_t ntiles, const int32_t *hint, int32_t *idx, float *__restrict__ dist,
-                 double *__restrict__ blocksum, Header *hdr) {
+                 int32_t K, int32_t ntiles, const int32_t *hint, const int32_t *__restrict__ perm, int32_t *idx,
+                 float *__restrict__ dist, double *__restrict__ blocksum, Header *hdr) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     TcShared &S = *reinterpret_cast<TcShared *>(smem_raw);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -328,7 +328,9 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
 #pragma unroll
         for (int t = 0; t < TC_RT; ++t) {
             const int rloc = t * TC_M + r;
-            const int64_t row = (int64_t)blockIdx.x * TC_ROWS + rloc;
+            // slot -> kernel row (rows in the order of a permutation, when given)
+            const int64_t slot = (int64_t)blockIdx.x * TC_ROWS + rloc;
+            const int64_t row = slot < n ? (perm ? (int64_t)__ldg(perm + slot) : slot) : n;
             float x[D];
 #pragma unroll
             for (int j = 0; j < D; ++j) x[j] = row < n ? W[row * D + j] : 0.f;
@@ -583,7 +585,8 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
 #pragma unroll
         for (int t = 0; t < TC_RT; ++t) {
             const int rloc = t * TC_M + r;
-            const int64_t row = (int64_t)blockIdx.x * TC_ROWS + rloc;
+            const int64_t slot = (int64_t)blockIdx.x * TC_ROWS + rloc;
+            const int64_t row = slot < n ? (perm ? (int64_t)__ldg(perm + slot) : slot) : n;
             const float ob = S.pbest[rloc];
             const int32_t oi = S.pidx[rloc];
             if (ob < best[t] || (ob == best[t] && oi < bi[t])) {
@@ -606,7 +609,7 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
         double s = 0.0;
         for (int t = 0; t < TC_RT; ++t)
             for (int w = 0; w < TC_EPI_WARPS / 2; ++w) s += S.wsum[w][t];
-        blocksum[blockIdx.x] = s;
+        if (blocksum) blocksum[blockIdx.x] = s;
     }
     if (warp == 1) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -627,9 +630,111 @@ cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Heade
     return cudaGetLastError();
 }
 
+// ---- Warm starts: rows in the order of their hinted codeword. A warp's rows then
+// share one hint, so the exact path that every row takes once (in the tile of its
+// own running best, whose column the test cannot rule out) is entered once per warp
+// instead of once per distinct hint. Results do not depend on the order.
+
+// cnt[h] = rows hinted to codeword h; cnt[K] = rows without a usable hint.
+__global__ void __launch_bounds__(256) hint_histogram_kernel(const int32_t *__restrict__ hint, int64_t n, int32_t K,
+                                                             int32_t *cnt) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        const int32_t h = __ldcs(hint + i);
+        atomicAdd(cnt + ((uint32_t)h < (uint32_t)K ? h : K), 1);
+    }
+}
+
+// cursor = exclusive prefix sum of cnt[0..m) (one CTA).
+constexpr int SCAN_THREADS = 1024;
+__global__ void __launch_bounds__(SCAN_THREADS) scan_counts_kernel(const int32_t *cnt, int32_t m, int32_t *cursor) {
+    __shared__ int32_t wsum[SCAN_THREADS / 32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int32_t seg = (m + SCAN_THREADS - 1) / SCAN_THREADS;
+    const int32_t b0 = min(tid * seg, m), b1 = min(b0 + seg, m);
+    int32_t local = 0;
+    for (int32_t k = b0; k < b1; ++k) local += cnt[k];
+    int32_t incl = local;  // inclusive scan over the warp
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        int32_t w = lane < SCAN_THREADS / 32 ? wsum[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int32_t y = __shfl_up_sync(0xffffffffu, w, o);
+            if (lane >= o) w += y;
+        }
+        if (lane < SCAN_THREADS / 32) wsum[lane] = w;
+    }
+    __syncthreads();
+    int32_t run = incl - local + (warp > 0 ? wsum[warp - 1] : 0);
+    for (int32_t k = b0; k < b1; ++k) {
+        const int32_t c = cnt[k];  // read before the write: cursor may be cnt itself
+        cursor[k] = run;
+        run += c;
+    }
+}
+
+// perm = the rows grouped by hint (any order within a group).
+__global__ void __launch_bounds__(256) hint_scatter_kernel(const int32_t *__restrict__ hint, int64_t n, int32_t K,
+                                                           int32_t *cursor, int32_t *__restrict__ perm) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        const int32_t h = __ldcs(hint + i);
+        const int32_t pos = atomicAdd(cursor + ((uint32_t)h < (uint32_t)K ? h : K), 1);
+        perm[pos] = (int32_t)i;
+    }
+}
+
+// blocksum[b] = sum of dist over rows [256 b, 256 b + 256) in a fixed order (fp64).
+__global__ void __launch_bounds__(256) dist_block_sums_kernel(const float *__restrict__ dist, int64_t n,
+                                                              double *__restrict__ blocksum) {
+    __shared__ double ws[8];
+    const int64_t i = (int64_t)blockIdx.x * 256 + threadIdx.x;
+    double v = i < n ? (double)__ldcs(dist + i) : 0.0;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if ((threadIdx.x & 31) == 0) ws[threadIdx.x >> 5] = v;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < 8; ++w) t += ws[w];
+        blocksum[blockIdx.x] = t;
+    }
+}
+
+cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, int32_t *cnt, int32_t *perm,
+                                    int num_sms, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(cnt, 0, (size_t)(K + 1) * sizeof(int32_t), s);
+    if (e != cudaSuccess) return e;
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
+    hint_histogram_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cnt);
+    count_launch();
+    // the scan turns cnt into start offsets in place (each entry is read before it is written)
+    scan_counts_kernel<<<1, SCAN_THREADS, 0, s>>>(cnt, K + 1, cnt);
+    count_launch();
+    hint_scatter_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cnt, perm);
+    count_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_dist_block_sums(const float *dist, int64_t n, double *blocksum, int *nblocksum, cudaStream_t s) {
+    const int64_t blocks = (n + 255) / 256;
+    dist_block_sums_kernel<<<(unsigned)blocks, 256, 0, s>>>(dist, n, blocksum);
+    count_launch();
+    *nblocksum = (int)blocks;
+    return cudaGetLastError();
+}
+
 cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const float *Cpk, int32_t K,
-                             const int32_t *hint, int32_t *idx, float *dist, double *blocksum, int *nblocksum,
-                             Header *hdr, cudaStream_t s) {
+                             const int32_t *hint, const int32_t *perm, int32_t *idx, float *dist, double *blocksum,
+                             int *nblocksum, Header *hdr, cudaStream_t s) {
     // One CTA per SM (it owns all of TMEM); the shared layout alone rules out a second.
     const int smem = (int)sizeof(TcShared) + 1024;  // + alignment slack of the dynamic base
     static_assert(sizeof(TcShared) + 1024 <= 227 * 1024, "shared layout too large");
@@ -638,7 +743,8 @@ cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const fl
     if (e != cudaSuccess) return e;
     const int64_t blocks = (n + TC_ROWS - 1) / TC_ROWS;
     const int32_t ntiles = tc_kpad(K) / TC_N;
-    assign_tc_kernel<<<(unsigned)blocks, TC_THREADS, smem, s>>>(W, n, C, Cpk, K, ntiles, hint, idx, dist, blocksum, hdr);
+    assign_tc_kernel<<<(unsigned)blocks, TC_THREADS, smem, s>>>(W, n, C, Cpk, K, ntiles, hint, perm, idx, dist,
+                                                                blocksum, hdr);
     count_launch();
     *nblocksum = (int)blocks;
     return cudaGetLastError();

@@ -41,7 +41,7 @@ struct Header {
 static_assert(sizeof(Header) <= 4096, "header too large");
 
 struct WsLayout {
-    size_t cd, acc, part, blocksum, cbuf0, cbuf1, cp, cq, cpk, total;
+    size_t cd, acc, part, blocksum, cbuf0, cbuf1, cp, cq, cpk, dist, perm, pcnt, total;
 };
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -59,6 +59,9 @@ inline WsLayout ws_layout(int64_t n, int32_t K) {
     L.cp = off;       off = align_up(off + (size_t)K * CP_FLOATS * 4, 256);
     L.cq = off;       off = align_up(off + (size_t)K * 8, 256);
     L.cpk = off;      off = align_up(off + (size_t)((K + 255) / 256 * 256) * 128, 256);  // tensor-core codeword tiles
+    L.dist = off;     off = align_up(off + (size_t)n * 4, 256);          // distances when the caller keeps none
+    L.perm = off;     off = align_up(off + (size_t)n * 4, 256);          // rows in hint order
+    L.pcnt = off;     off = align_up(off + (size_t)(K + 1) * 4, 256);    // per-hint counts / cursors
     L.total = off;
     return L;
 }
@@ -248,8 +251,13 @@ cudaError_t launch_assign(const float *W, int64_t n, const float *Cd, const floa
 bool tc_eligible(int64_t n, int num_sms);
 cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Header *hdr, cudaStream_t s);
 cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const float *Cpk, int32_t K,
-                             const int32_t *hint, int32_t *idx, float *dist, double *blocksum, int *nblocksum,
-                             Header *hdr, cudaStream_t s);
+                             const int32_t *hint, const int32_t *perm, int32_t *idx, float *dist, double *blocksum,
+                             int *nblocksum, Header *hdr, cudaStream_t s);
+// Rows grouped by their hinted codeword (cnt: K + 1 ints of scratch, perm: n ints).
+cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, int32_t *cnt, int32_t *perm,
+                                    int num_sms, cudaStream_t s);
+// blocksum[b] = fp64 sum of dist over rows [256 b, 256 b + 256), in row order.
+cudaError_t launch_dist_block_sums(const float *dist, int64_t n, double *blocksum, int *nblocksum, cudaStream_t s);
 cudaError_t launch_sum_blocks(const double *blocksum, int nblocks, double *out, cudaStream_t s);
 
 // Update step. Two ways to pick the fixed-point scale: `exact` takes B = max|W|
