@@ -18,6 +18,7 @@ void count_launch(int kernels) { g_launches.fetch_add((unsigned long long)kernel
 namespace {
 
 constexpr int32_t KQ_ABI_VERSION = 3;
+constexpr int32_t HINT_ORDER_MIN_K = 4096;  // warm starts in hint order from 16 codeword tiles on
 
 inline bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
@@ -103,16 +104,18 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
                      float *dist, int *nb, const Ws &w, int sms, cudaStream_t s) {
     if (tc_eligible(n, sms)) {
         KQ_TRY(launch_pack_codebook_tc(C, K, w.cpk, w.hdr, s));
-        // warm start: rows grouped by hint (see kq_assign_tc.cu); the objective's block
-        // sums are then taken over the distances in row order, whatever the grouping
-        const int32_t *perm = nullptr;
-        if (hint) {
+        // Warm start with many codeword tiles: rows grouped by hint (see
+        // kq_assign_tc.cu); the objective's block sums are then taken over the
+        // distances in row order, whatever the grouping. With few tiles the four extra
+        // launches cost more than they save, and rows stay in order.
+        if (hint && K >= HINT_ORDER_MIN_K) {
             KQ_TRY(launch_hint_permutation(hint, n, K, w.pcnt, w.perm, sms, s));
-            perm = w.perm;
+            float *d = dist ? dist : w.dist;
+            KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K, hint, w.perm, idx, d, nullptr, nb, w.hdr, s));
+            KQ_TRY(launch_dist_block_sums(d, n, w.blocksum, nb, s));
+        } else {
+            KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K, hint, nullptr, idx, dist, w.blocksum, nb, w.hdr, s));
         }
-        float *d = dist ? dist : w.dist;
-        KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K, hint, perm, idx, d, nullptr, nb, w.hdr, s));
-        KQ_TRY(launch_dist_block_sums(d, n, w.blocksum, nb, s));
     } else {
         KQ_TRY(launch_pack_codebook(C, K, w.cd, w.hdr, s));
         KQ_TRY(launch_assign(W, n, w.cd, C, K, hint, idx, dist, w.blocksum, nb, w.part, w.hdr, sms, s));

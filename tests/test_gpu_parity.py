@@ -168,6 +168,42 @@ def test_assign_paths_agree():
     assert np.array_equal(i_w, i_tc) and bits_equal(d_w, d_tc)
 
 
+def test_assign_hint_order_path():
+    # K >= 4096 on the tensor-core path: warm-started rows are processed grouped by
+    # hint; the result must be the cold result, whatever the hints (exact, random,
+    # out of range), and the cold result matches the oracle on sampled rows
+    n, K = 5 * TC_MIN_N + 333, 5000
+    W = synth.random_kernels(n, 9, 221, 0.05)
+    C = synth.random_kernels(K, 9, 222, 0.05)
+    i0, d0, st, _ = gpu_assign(W, C)
+    assert st == 0
+    rows = np.sort(synth.below(synth.stream_key(223, 9), 3000, n))
+    idx_ref, dist_ref = oracle.assign(W[rows], C, threads=THREADS)
+    assert check_indices(W, C, i0[rows], idx_ref, rows) == 0
+    assert bits_equal(d0[rows], dist_ref)
+    rand = synth.below(synth.stream_key(224, 2), n, K).astype(np.int32)
+    rand[::7] = -1
+    rand[3::11] = K + 5
+    for h in (i0, rand, np.where(np.arange(n) % 3 == 0, i0, rand).astype(np.int32)):
+        i1, d1, st, _ = gpu_assign(W, C, hint=h)
+        assert st == 0 and np.array_equal(i1, i0) and bits_equal(d1, d0)
+
+
+def test_fit_hint_order_deterministic_and_chained():
+    n, K = TC_MIN_N + 21000, 4500
+    W = synth.random_kernels(n, 9, 231, 0.05)
+    C0 = W[synth.init_selection(n, K, 232)]
+    a = _gpu_fit(W, C0, 3)
+    b = _gpu_fit(W, C0, 3)
+    for x, y in zip(a, b):
+        assert bits_equal(x, y)
+    C = C0
+    for _ in range(3):
+        C = _gpu_fit(W, C, 1)[0]
+    assert bits_equal(a[0], C)
+    assert np.all(a[3][1:] <= a[3][:-1] * (1 + 1e-6))
+
+
 def test_assign_hint_never_changes_result():
     lay, W, C0 = _layer(2)
     idx0, dist0, _, _ = gpu_assign(W, C0)
