@@ -259,8 +259,14 @@ kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_i
     if (st != KQ_OK) return st;
     int sms = 0;
     if ((st = num_sms(&sms)) != KQ_OK) return st;
-    return run_fit(W, n, K, C_init, iters, C_out, idx, counts, objective, nullptr, carve(ws, n, K), sms,
-                   reinterpret_cast<cudaStream_t>(stream));
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    const Ws w = carve(ws, n, K);
+    if (small_fit_eligible(n, K)) {  // the whole fit in one cooperative launch
+        const int nblk = (int)((n + 255) / 256) + MAX_PART_BLOCKS;
+        return cuda_status(launch_small_fit(W, n, C_init, K, iters, C_out, idx, counts, objective, w.acc, w.cbuf0,
+                                            w.cbuf1, w.blocksum, nblk, w.hdr, sms, s));
+    }
+    return run_fit(W, n, K, C_init, iters, C_out, idx, counts, objective, nullptr, w, sms, s);
 }
 
 kq_status kq_search_codebook_size(const float *W, int64_t n, const int64_t *sel, int32_t sel_len, double alpha,

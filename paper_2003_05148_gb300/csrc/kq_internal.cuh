@@ -276,6 +276,13 @@ cudaError_t launch_histogram(const int32_t *idx, int64_t n, int32_t K, int32_t *
 cudaError_t launch_finalize(unsigned long long *acc, int32_t K, const Header *hdr, const float *C_prev,
                             float *C_next, int32_t *counts, cudaStream_t s);
 
+// The whole k-means fit in one cooperative launch, for small codebooks (K <= 512).
+bool small_fit_eligible(int64_t n, int32_t K);
+cudaError_t launch_small_fit(const float *W, int64_t n, const float *C0, int32_t K, int32_t iters, float *C_out,
+                             int32_t *idx, int32_t *counts, double *objective, unsigned long long *acc, float *cbuf0,
+                             float *cbuf1, double *blocksum, int max_blocksum, Header *hdr, int num_sms,
+                             cudaStream_t s);
+
 cudaError_t launch_level_fit(const float *C, int64_t N, const int32_t *counts, int32_t max_iters, float *levels,
                              uint8_t *codes, int32_t *iters_run, Header *hdr, int num_sms, cudaStream_t s);
 
