@@ -38,6 +38,14 @@
 //   T' = -2^100: its g is then huge and positive (and no infinity meets the other
 //   half's 0), and its thread tests every codeword exactly anyway.
 //
+// Warm starts (a hint per kernel): a row's own hinted codeword always passes the
+// test (its distance is the best, which the test cannot rule out), so every row
+// takes the exact path once per pass. With K >= 4096 the caller hands the kernel a
+// permutation that groups rows by hint (hint_histogram / scan_counts /
+// hint_scatter below); a warp's rows then share that tile and the warp takes the
+// exact path once instead of once per distinct hint. The kernel's slot s works on
+// row perm[s]; results do not depend on the order.
+//
 // Warp roles in a CTA of 352 threads that owns 256 kernels (two 128-row tiles):
 //   warp 0      producer: streams packed codeword tiles (256 codewords x 128 B,
 //               already in the tensor-core layout) into a 4-stage shared ring with
