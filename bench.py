@@ -530,7 +530,6 @@ def run_configs(args):
 
     build.build()
     dev = torch.device("cuda", 0)
-    sms = torch.cuda.get_device_properties(dev).multi_processor_count
     for cfg in [int(c) for c in args.configs.split(",")]:
         wl = synth.workload(cfg)
         T = wl.iters
@@ -574,7 +573,7 @@ def run_configs(args):
         print(json.dumps({
             "config": wl.name, "layers": len(layers), "kernels": sum(L["n"] for L in layers),
             "codewords": sum(L["K"] for L in layers), "iters": T, "evals": evals, "ms_per_run": ms,
-            "evals_per_s": evals / (ms / 1e3), "tensor_core_assign_layers": sum(L["n"] >= 256 * sms for L in layers),
+            "evals_per_s": evals / (ms / 1e3),
             "gpu_launches_per_run": (kq.kq_kernel_launches() - launches0) // args.reps,
             "status": max(st for st, _ in statuses), "reps": args.reps}), flush=True)
 

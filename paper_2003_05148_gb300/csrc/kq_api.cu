@@ -102,7 +102,7 @@ kq_status run_update_exact(const float *W, int64_t n, const int32_t *idx, int32_
 // One assignment: tensor-core path when n fills every SM, CUDA-core path otherwise.
 kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const int32_t *hint, int32_t *idx,
                      float *dist, int *nb, const Ws &w, int sms, cudaStream_t s) {
-    if (tc_eligible(n, sms)) {
+    if (tc_eligible(n, K, sms)) {
         KQ_TRY(launch_pack_codebook_tc(C, K, w.cpk, w.hdr, s));
         // Warm start with many codeword tiles: rows grouped by hint (see
         // kq_assign_tc.cu); the objective's block sums are then taken over the

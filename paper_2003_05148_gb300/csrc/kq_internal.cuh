@@ -248,7 +248,7 @@ cudaError_t launch_assign(const float *W, int64_t n, const float *Cd, const floa
                           int32_t *idx, float *dist, double *blocksum, int *nblocksum, unsigned long long *part,
                           Header *hdr, int num_sms, cudaStream_t s);
 // Tensor-core assignment (kq_assign_tc.cu): used when n fills every SM.
-bool tc_eligible(int64_t n, int num_sms);
+bool tc_eligible(int64_t n, int32_t K, int num_sms);
 cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Header *hdr, cudaStream_t s);
 cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const float *Cpk, int32_t K,
                              const int32_t *hint, const int32_t *perm, int32_t *idx, float *dist, double *blocksum,

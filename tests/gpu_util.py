@@ -39,6 +39,17 @@ def gpu_assign(W, C, with_dist=True, hint=None):
     return idx.cpu().numpy(), (dist.cpu().numpy() if with_dist else None), st, flags
 
 
+def gpu_assign_cuda_cores(W, C):
+    """The same assignment through kq_assign_noalloc, which always runs the
+    CUDA-core kernel (kq_assign picks the kernel by size)."""
+    n = W.shape[0]
+    idx = torch.empty(n, dtype=torch.int32, device=dev())
+    dist = torch.empty(n, dtype=torch.float32, device=dev())
+    kq.kq_assign_noalloc(to_dev(W), to_dev(C), idx, dist)
+    torch.cuda.synchronize()
+    return idx.cpu().numpy(), dist.cpu().numpy()
+
+
 def gpu_update(W, idx, C_prev):
     n, K = W.shape[0], C_prev.shape[0]
     Wd, idxd, Cp = to_dev(W), to_dev(idx.astype(np.int32)), to_dev(C_prev)

@@ -13,7 +13,8 @@ import torch
 
 import oracle
 import synth
-from gpu_util import (bits_equal, check_centroids, check_indices, dev, gpu_assign, gpu_quantize, gpu_reconstruct,
+from gpu_util import (bits_equal, check_centroids, check_indices, dev, gpu_assign, gpu_assign_cuda_cores, gpu_quantize,
+                      gpu_reconstruct,
                       gpu_update, to_dev)
 from paper_2003_05148_gb300 import kq
 
@@ -114,9 +115,12 @@ def test_assign_filter_extreme_scales(case):
     idx, dist, st, _ = gpu_assign(W, C)
     assert st == 0
     _oracle_check(W, C, idx, dist)
+    # the CUDA-core kernel (kq_assign takes the tensor cores at this size) as well
+    idx2, dist2 = gpu_assign_cuda_cores(W, C)
+    _oracle_check(W, C, idx2, dist2)
 
 
-TC_MIN_N = 256 * 152  # from this many kernels on, the assignment runs on the tensor cores
+TC_MIN_N = 256 * 152  # one row block per SM (from about 256 kernels on the tensor cores run)
 
 
 @pytest.mark.parametrize("case", ["plain", "offset", "mixed", "large", "near_dup", "ragged"])
@@ -149,18 +153,20 @@ def test_assign_tensor_core_path(case):
 
 
 def test_assign_paths_agree():
-    # the same kernels through the tensor-core path (large n) and the CUDA-core
-    # path (small n) give bit-identical results; n spans several row blocks per
+    # the tensor-core kernel (kq_assign) and the CUDA-core kernel (kq_assign_noalloc)
+    # give bit-identical results on the same kernels; n spans several row blocks per
     # SM and a ragged last block, cold and warm-started
     n = 5 * TC_MIN_N + 333
     W = synth.random_kernels(n, 9, 211, 0.05)
     C = synth.random_kernels(2000, 9, 212, 0.05)
     i_tc, d_tc, st1, _ = gpu_assign(W, C)
     assert st1 == 0
+    i_cc, d_cc = gpu_assign_cuda_cores(W, C)
+    assert np.array_equal(i_tc, i_cc) and bits_equal(d_tc, d_cc)
     for sl in (slice(0, 20000), slice(n - 20000, n)):
-        i_cc, d_cc, st2, _ = gpu_assign(W[sl], C)
+        i_s, d_s, st2, _ = gpu_assign(W[sl], C)  # a smaller n: fewer CTAs than SMs
         assert st2 == 0
-        assert np.array_equal(i_tc[sl], i_cc) and bits_equal(d_tc[sl], d_cc)
+        assert np.array_equal(i_tc[sl], i_s) and bits_equal(d_tc[sl], d_s)
     hint = synth.below(synth.stream_key(213, 9), n, 2000).astype(np.int32)
     hint[::3] = i_tc[::3]
     i_w, d_w, st3, _ = gpu_assign(W, C, hint=hint)
