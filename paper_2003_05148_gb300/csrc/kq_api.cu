@@ -99,9 +99,10 @@ kq_status run_update_exact(const float *W, int64_t n, const int32_t *idx, int32_
     return KQ_OK;
 }
 
-// One assignment: tensor-core path when n fills every SM, CUDA-core path otherwise.
+// One assignment, on the kernel tc_eligible picks. hint_counts: rows per hinted
+// codeword, when known (the fit's previous update counted them), or null.
 kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const int32_t *hint, int32_t *idx,
-                     float *dist, int *nb, const Ws &w, int sms, cudaStream_t s) {
+                     float *dist, int *nb, const Ws &w, int sms, cudaStream_t s, const int32_t *hint_counts = nullptr) {
     if (tc_eligible(n, K, sms)) {
         KQ_TRY(launch_pack_codebook_tc(C, K, w.cpk, w.hdr, s));
         // Warm start with many codeword tiles: rows grouped by hint (see
@@ -109,7 +110,7 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
         // distances in row order, whatever the grouping. With few tiles the four extra
         // launches cost more than they save, and rows stay in order.
         if (hint && K >= HINT_ORDER_MIN_K) {
-            KQ_TRY(launch_hint_permutation(hint, n, K, w.pcnt, w.perm, sms, s));
+            KQ_TRY(launch_hint_permutation(hint, n, K, hint_counts, w.pcnt, w.perm, sms, s));
             float *d = dist ? dist : w.dist;
             KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K, hint, w.perm, idx, d, nullptr, nb, w.hdr, s));
             KQ_TRY(launch_dist_block_sums(d, n, w.blocksum, nb, s));
@@ -138,14 +139,19 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
     int nb = 0;
     // iteration t > 0 starts every row from its previous assignment (warm start)
     for (int32_t t = 0; t < iters; ++t) {
-        if ((st = run_assign(W, n, cur, K, t > 0 ? idx : nullptr, idx, nullptr, &nb, w, sms, s)) != KQ_OK) return st;
+        // from t > 0 the hint is the last assignment, whose counts the update wrote
+        if ((st = run_assign(W, n, cur, K, t > 0 ? idx : nullptr, idx, nullptr, &nb, w, sms, s,
+                             t > 0 ? counts : nullptr)) != KQ_OK)
+            return st;
         if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
         if ((st = run_update_exact(W, n, idx, K, cur, nxt, counts, w, sms, s)) != KQ_OK) return st;
         float *tmp = cur;
         cur = nxt;
         nxt = tmp;
     }
-    if ((st = run_assign(W, n, cur, K, iters > 0 ? idx : nullptr, idx, nullptr, &nb, w, sms, s)) != KQ_OK) return st;
+    if ((st = run_assign(W, n, cur, K, iters > 0 ? idx : nullptr, idx, nullptr, &nb, w, sms, s,
+                         iters > 0 ? counts : nullptr)) != KQ_OK)
+        return st;
     if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + iters, s));
     if (final_obj) KQ_TRY(launch_sum_blocks(w.blocksum, nb, final_obj, s));
     KQ_TRY(launch_histogram(idx, n, K, counts, &w.hdr->status, sms, s));

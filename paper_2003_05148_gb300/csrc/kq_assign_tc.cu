@@ -663,38 +663,66 @@ __global__ void __launch_bounds__(256) hint_histogram_kernel(const int32_t *__re
     }
 }
 
-// cursor = exclusive prefix sum of cnt[0..m) (one CTA).
+// cursor[0..m) = exclusive prefix sum of cnt[0..m) (one CTA), where entries past
+// mc read as 0 (so a K-entry count array can stand for K + 1 entries). Rounds of
+// 4096 entries: coalesced 16-byte loads, a scan over the CTA, 16-byte stores, the
+// round's total carried into the next. cursor may be cnt itself: each round reads
+// all its entries before any are written.
 constexpr int SCAN_THREADS = 1024;
-__global__ void __launch_bounds__(SCAN_THREADS) scan_counts_kernel(const int32_t *cnt, int32_t m, int32_t *cursor) {
+__global__ void __launch_bounds__(SCAN_THREADS) scan_counts_kernel(const int32_t *cnt, int32_t mc, int32_t m,
+                                                                   int32_t *cursor) {
     __shared__ int32_t wsum[SCAN_THREADS / 32];
+    __shared__ int32_t s_carry;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int32_t seg = (m + SCAN_THREADS - 1) / SCAN_THREADS;
-    const int32_t b0 = min(tid * seg, m), b1 = min(b0 + seg, m);
-    int32_t local = 0;
-    for (int32_t k = b0; k < b1; ++k) local += cnt[k];
-    int32_t incl = local;  // inclusive scan over the warp
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const int32_t y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += y;
-    }
-    if (lane == 31) wsum[warp] = incl;
+    if (tid == 0) s_carry = 0;
     __syncthreads();
-    if (warp == 0) {
-        int32_t w = lane < SCAN_THREADS / 32 ? wsum[lane] : 0;
+    for (int32_t base = 0; base < m; base += 4 * SCAN_THREADS) {
+        const int32_t k0 = base + 4 * tid;
+        int32_t c[4];
+        if (k0 + 3 < mc && ((reinterpret_cast<uintptr_t>(cnt + k0) & 15) == 0)) {
+            const int4 v = *reinterpret_cast<const int4 *>(cnt + k0);
+            c[0] = v.x; c[1] = v.y; c[2] = v.z; c[3] = v.w;
+        } else {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) c[u] = k0 + u < mc ? cnt[k0 + u] : 0;
+        }
+        const int32_t local = c[0] + c[1] + c[2] + c[3];
+        int32_t incl = local;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-            const int32_t y = __shfl_up_sync(0xffffffffu, w, o);
-            if (lane >= o) w += y;
+            const int32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += y;
         }
-        if (lane < SCAN_THREADS / 32) wsum[lane] = w;
-    }
-    __syncthreads();
-    int32_t run = incl - local + (warp > 0 ? wsum[warp - 1] : 0);
-    for (int32_t k = b0; k < b1; ++k) {
-        const int32_t c = cnt[k];  // read before the write: cursor may be cnt itself
-        cursor[k] = run;
-        run += c;
+        if (lane == 31) wsum[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            int32_t w = wsum[lane];
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int32_t y = __shfl_up_sync(0xffffffffu, w, o);
+                if (lane >= o) w += y;
+            }
+            wsum[lane] = w;  // inclusive over the warps
+        }
+        __syncthreads();
+        const int32_t carry = s_carry;
+        int32_t run = carry + incl - local + (warp > 0 ? wsum[warp - 1] : 0);
+        int32_t out[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            out[u] = run;
+            run += c[u];
+        }
+        if (k0 + 3 < m && ((reinterpret_cast<uintptr_t>(cursor + k0) & 15) == 0)) {
+            *reinterpret_cast<int4 *>(cursor + k0) = make_int4(out[0], out[1], out[2], out[3]);
+        } else {
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                if (k0 + u < m) cursor[k0 + u] = out[u];
+        }
+        __syncthreads();  // every thread has read s_carry and wsum
+        if (tid == SCAN_THREADS - 1) s_carry = run;
+        __syncthreads();
     }
 }
 
@@ -705,7 +733,7 @@ __global__ void __launch_bounds__(256) hint_scatter_kernel(const int32_t *__rest
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
         const int32_t h = __ldcs(hint + i);
         const int32_t pos = atomicAdd(cursor + ((uint32_t)h < (uint32_t)K ? h : K), 1);
-        perm[pos] = (int32_t)i;
+        if ((uint32_t)pos < (uint32_t)n) perm[pos] = (int32_t)i;  // counts that do not match the hints: no stray write
     }
 }
 
@@ -726,17 +754,24 @@ __global__ void __launch_bounds__(256) dist_block_sums_kernel(const float *__res
     }
 }
 
-cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, int32_t *cnt, int32_t *perm,
-                                    int num_sms, cudaStream_t s) {
-    cudaError_t e = cudaMemsetAsync(cnt, 0, (size_t)(K + 1) * sizeof(int32_t), s);
-    if (e != cudaSuccess) return e;
+cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, const int32_t *hint_counts,
+                                    int32_t *cnt, int32_t *perm, int num_sms, cudaStream_t s) {
     int64_t blocks = (n + 255) / 256;
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
-    hint_histogram_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cnt);
-    count_launch();
-    // the scan turns cnt into start offsets in place (each entry is read before it is written)
-    scan_counts_kernel<<<1, SCAN_THREADS, 0, s>>>(cnt, K + 1, cnt);
-    count_launch();
+    if (hint_counts) {
+        // the rows per hinted codeword are known (all hints valid): start offsets
+        // straight from them, K + 1 entries with the last count 0
+        scan_counts_kernel<<<1, SCAN_THREADS, 0, s>>>(hint_counts, K, K + 1, cnt);
+        count_launch();
+    } else {
+        cudaError_t e = cudaMemsetAsync(cnt, 0, (size_t)(K + 1) * sizeof(int32_t), s);
+        if (e != cudaSuccess) return e;
+        hint_histogram_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cnt);
+        count_launch();
+        // the scan turns cnt into start offsets in place
+        scan_counts_kernel<<<1, SCAN_THREADS, 0, s>>>(cnt, K + 1, K + 1, cnt);
+        count_launch();
+    }
     hint_scatter_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cnt, perm);
     count_launch();
     return cudaGetLastError();

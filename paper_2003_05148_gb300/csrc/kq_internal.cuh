@@ -254,8 +254,10 @@ cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const fl
                              const int32_t *hint, const int32_t *perm, int32_t *idx, float *dist, double *blocksum,
                              int *nblocksum, Header *hdr, cudaStream_t s);
 // Rows grouped by their hinted codeword (cnt: K + 1 ints of scratch, perm: n ints).
-cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, int32_t *cnt, int32_t *perm,
-                                    int num_sms, cudaStream_t s);
+// hint_counts: the number of rows per hinted codeword when the caller knows it (every
+// hint then valid), else null (counted here).
+cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, const int32_t *hint_counts,
+                                    int32_t *cnt, int32_t *perm, int num_sms, cudaStream_t s);
 // blocksum[b] = fp64 sum of dist over rows [256 b, 256 b + 256), in row order.
 cudaError_t launch_dist_block_sums(const float *dist, int64_t n, double *blocksum, int *nblocksum, cudaStream_t s);
 cudaError_t launch_sum_blocks(const double *blocksum, int nblocks, double *out, cudaStream_t s);
