@@ -101,6 +101,17 @@ __device__ __forceinline__ float ord2f(uint32_t u) {
     return __uint_as_float((u & 0x80000000u) ? (u & 0x7fffffffu) : ~u);
 }
 
+// Scale exponent of exact fixed-point sums of n values bounded by B (B = max|W| of
+// the fit): S = 62 - e with n B = f 2^e, f in [0.5, 1), so no sum reaches 2^62;
+// 0 when B is zero or not finite (all-zero W: nothing to scale; non-finite W is
+// flagged by the callers).
+__device__ __forceinline__ int fit_sum_scale(float B, int64_t n) {
+    if (!(B > 0.f) || !(B <= 3.402823466e38f)) return 0;
+    int e;
+    frexp((double)n * (double)B, &e);
+    return 62 - e;
+}
+
 // rint(v * 2^S) as int64 (round half to even) for a finite fp32 v, using only
 // integer operations: v = +-m * 2^(e - 150) (e the biased exponent, m with its
 // implicit bit; subnormals m * 2^-149). Equal to rounding the exact product
@@ -247,7 +258,7 @@ cudaError_t launch_pack_codebook(const float *C, int32_t K, float *Cd, Header *h
 cudaError_t launch_assign(const float *W, int64_t n, const float *Cd, const float *C, int32_t K, const int32_t *hint,
                           int32_t *idx, float *dist, double *blocksum, int *nblocksum, unsigned long long *part,
                           Header *hdr, int num_sms, cudaStream_t s);
-// Tensor-core assignment (kq_assign_tc.cu): used when n fills every SM.
+// Tensor-core assignment (kq_assign_tc.cu): used where tc_eligible's cost estimate favours it.
 bool tc_eligible(int64_t n, int32_t K, int num_sms);
 cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Header *hdr, cudaStream_t s);
 cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const float *Cpk, int32_t K,

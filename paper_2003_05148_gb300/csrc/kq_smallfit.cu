@@ -38,15 +38,6 @@ struct SmallFitArgs {
     Header *hdr;
 };
 
-// Scale exponent of the fixed-point sums for n values bounded by B (as the update's:
-// S = 62 - e with n B = f 2^e; 0 when B is zero or not finite).
-__device__ __forceinline__ int small_fit_scale(float B, int64_t n) {
-    if (!(B > 0.f) || !(B <= 3.402823466e38f)) return 0;
-    int e;
-    frexp((double)n * (double)B, &e);
-    return 62 - e;
-}
-
 // One pass of the assignment against the codebook pairs in shared memory; adds the
 // kernels to the sums (accumulate) or only to the counts (final pass), and returns
 // this thread's share of the objective (its distances in row order, fp64).
@@ -137,7 +128,7 @@ __global__ void __launch_bounds__(SF_THREADS) small_fit_kernel(SmallFitArgs a) {
         for (int64_t e = gtid; e < (int64_t)a.K * D; e += nthr) a.cbuf0[e] = a.C0[e];
     }
     if (!grid_barrier(h, gridDim.x, epoch)) return;
-    const int S = small_fit_scale(__uint_as_float(__ldcg(&h->maxabs_bits)), a.n);
+    const int S = fit_sum_scale(__uint_as_float(__ldcg(&h->maxabs_bits)), a.n);
 
     for (int32_t t = 0; t <= a.iters; ++t) {
         const bool last = t == a.iters;

@@ -210,6 +210,26 @@ def test_fit_hint_order_deterministic_and_chained():
     assert np.all(a[3][1:] <= a[3][:-1] * (1 + 1e-6))
 
 
+def test_fit_second_iteration_against_oracle():
+    """The second iteration of a fit with K >= 4096 (a hint-ordered warm start, the
+    counts of the first update reused as the grouping's histogram): its centroids are
+    the oracle's update of the oracle's assignment against the first iteration's
+    centroids, and bit-identical to a one-iteration fit started there. Kernel norms
+    spread over a factor of ~100 (log-normal) exercise the fixed-point scale."""
+    n, K = TC_MIN_N + 9001, 4200
+    rng = np.random.default_rng(244)
+    W = (synth.random_kernels(n, 9, 241, 0.05) * np.exp(rng.normal(0.0, 1.0, size=(n, 1)))).astype(np.float32)
+    C0 = W[synth.init_selection(n, K, 243)]
+    C1 = _gpu_fit(W, C0, 1)[0]
+    C2, idx2, cnt2, obj2 = _gpu_fit(W, C0, 2)
+    idx1_ref, _ = oracle.assign(W, C1, threads=THREADS)
+    C2_ref, _ = oracle.update(W, idx1_ref, C1)
+    check_centroids(C2, C2_ref)
+    C2b, idx2b, cnt2b, _ = _gpu_fit(W, C1, 1)
+    assert bits_equal(C2, C2b) and np.array_equal(idx2, idx2b) and np.array_equal(cnt2, cnt2b)
+    assert np.array_equal(cnt2, np.bincount(idx2, minlength=K))
+
+
 def test_assign_hint_never_changes_result():
     lay, W, C0 = _layer(2)
     idx0, dist0, _, _ = gpu_assign(W, C0)
