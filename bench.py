@@ -40,11 +40,10 @@ SM_COUNT_NOMINAL = 152
 FP32_LANES_PER_SM = 128
 OPS_PER_PAIR = 9  # FP32-pipe lane ops per pair executed by the assign kernel: the 9 FFMA of its certified test
 DIRECT_OPS_PER_PAIR = 18  # the fp32 direct form: 9 FSUB + 9 FFMA
-# Tensor-core assign: the certified test is an (n x 32) . (32 x K) split-TF32 GEMM, 2 * 32 flops per pair.
+# Tensor-core assign: the certified test is an (n x 32) . (32 x K) split-fp16 GEMM, 2 * 32 flops per pair.
 TC_FLOPS_PER_PAIR = 64
 TC_ROWS_PER_CTA = 256  # the library takes the tensor-core kernel when n >= 256 * SMs
-TF32_PER_BF16 = 1.1 / 2.25  # nominal dense tf32 : bf16 tensor rate
-TF32_FLOPS_PER_CLK_SM = 4096  # nominal dense tf32 rate per SM per clock
+F16_FLOPS_PER_CLK_SM = 8192  # dense fp16 / bf16 tensor rate per SM per clock
 WORKLOAD_CFG = 5
 
 
@@ -337,18 +336,18 @@ def run_kq(args, rank, world, local_rank):
     t_assign = statistics.mean(assign_ms) / 1e3
     traffic = _ncu_traffic()
     if n >= TC_ROWS_PER_CTA * sms:
-        # kernel timed inside a long step: the sustained bf16 figure, scaled to tf32
+        # kernel timed inside a long step: the sustained bf16 figure (fp16 runs at the bf16 rate)
         bf16 = float(peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops", 1700.0)))
-        peak = bf16 * TF32_PER_BF16
+        peak = bf16
         achieved = TC_FLOPS_PER_PAIR * n * K / t_assign / 1e12
         roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                     "traffic": traffic.get("assign_tc_kernel"), "kernel": "assign_tc_kernel",
-                    "peak_basis": f"measured cuBLAS bf16 sustained {bf16:.1f} TFLOP/s x {TF32_PER_BF16:.4f} "
-                                  f"(nominal tf32:bf16); flops = {TC_FLOPS_PER_PAIR} per pair (the split-TF32 "
-                                  f"GEMM of the certified test, K = 32); the exact fp32 re-evaluations of the "
-                                  f"few candidate pairs run on the CUDA cores and are not counted",
-                    "frac_of_burst": achieved / (float(peaks.get("bf16_tflops", bf16)) * TF32_PER_BF16),
-                    "peak_at_max_clock": sms * TF32_FLOPS_PER_CLK_SM * max_mhz * 1e6 / 1e12,
+                    "peak_basis": f"measured cuBLAS bf16 sustained {bf16:.1f} TFLOP/s (dense fp16 and bf16 share "
+                                  f"one rate); flops = {TC_FLOPS_PER_PAIR} per pair (the split-fp16 GEMM of the "
+                                  f"certified test, K = 32 fp16 per row, fp32 accumulation); the exact fp32 "
+                                  f"re-evaluations of the few candidate pairs run on the CUDA cores and are not counted",
+                    "frac_of_burst": achieved / float(peaks.get("bf16_tflops", bf16)),
+                    "peak_at_max_clock": sms * F16_FLOPS_PER_CLK_SM * max_mhz * 1e6 / 1e12,
                     "assign_ms_mean": 1e3 * t_assign, "assign_launches": len(assign_ms)}
         roofline["frac_of_peak_at_max_clock"] = achieved / roofline["peak_at_max_clock"]
     else:

@@ -6,22 +6,31 @@
 // row's threshold moves into the GEMM so that the test is one sign bit:
 //
 //   g = x . c - h - R - T' for a 128-row x 256-codeword tile is one GEMM,
-//   kind::tf32. The tensor core truncates fp32 operands to tf32 (relative error
-//   < 2^-10 each; measured: products match truncated inputs to fp32 accumulation
-//   error). To keep fp32-like accuracy every value is split exactly into
-//   v = v_hi + v_lo with v_hi = v truncated to tf32, and the three significant
-//   cross terms go side by side along the GEMM's K dimension (K = 32):
+//   kind::f16 (fp16 operands, fp32 accumulation; twice the tf32 rate). All values
+//   are first scaled by one power of two beta per call (the codebook's largest
+//   norm lands in [32, 64), so every operand sits well inside the fp16 range);
+//   that scales g by beta^2 and leaves its sign alone, and every quantity below is
+//   in scaled units. To keep fp32-like accuracy each value is split into
+//   v = v_hi + v_lo + d, v_hi = v truncated to fp16, v_lo = (v - v_hi) truncated
+//   to fp16, and the three significant cross terms go side by side along the
+//   GEMM's K dimension (K = 32):
 //     A[i] = ( x_hi,  1,     x_hi,  1,     x_lo,  -T'0, -R, -T'1 )
 //     B[k] = ( c_hi, -h_hi,  c_lo, -h_lo,  c_hi,  s0,    1,  s1  )   (9 + 1 + 9 + 1 + 9 + 3)
 //   where (s0, s1) = (1, 0) for the first 128 codewords of a tile and (0, 1) for
 //   the other 128, so each half of a tile row sees its own T' (each half is tested
-//   by its own thread, with its own running best). R (tf32, fixed per row, about
-//   |x|^2 / 2) and T' (tf32) are exact; the other half's T' meets an exact 0.
-//   Dropping x_lo.c_lo, truncating the lo parts to tf32 and accumulating 31 terms
-//   in fp32 give
-//     |g - (e - R - T')| <= E = 2^-16 (|x| Cmax + Hmax + |R| + |T'|) + 2^-120 (Cmax + |x| + 1)
+//   by its own thread, with its own running best). R (fixed per row, about
+//   |x|^2 / 2) and T' are normal fp16 values or 0, so they are exact operands
+//   even for a tensor core that flushes fp16 subnormals; the other half's T'
+//   meets an exact 0. |d| <= 2^-20 |v| + 2^-13 (relative while v_lo is a normal
+//   fp16 value, absolute below that, flushed subnormals included); products of
+//   fp16 values are exact in fp32, so dropping x_lo.c_lo and accumulating 31
+//   products in fp32 give
+//     |g - (e - R - T')| <= E = 2^-16 (|x| Cmax + Hmax + |R| + |T'|) + 2^-11 (|x| + Cmax + 1)
 //   (3 * 2^-20 + 31 * 2^-23 (1 + 2^-8) < 2^-16 on the first group, 31 * 2^-23 on R
-//   and T'; the absolute part covers subnormal inputs the tensor core may flush).
+//   and T'; 3 * 2^-13 (|x| + Cmax) + 2^-13 from the absolute parts of d, with
+//   sum_j |v_j| <= 3 |v|, on the second). A row whose scaled norm exceeds 256 (R and
+//   the products would leave the fp16 / exact-product range) enters the GEMM with
+//   x = 0 and is tested exactly against every codeword.
 //   The kernel keeps R + T' + E < thr0, where e < thr0 proves D_dir > best (the
 //   test of kq_assign.cu without its arithmetic slack), so a negative g (sign bit
 //   set, -0 included since E > 0) rules the codeword out. The TMEM load reduces as
@@ -29,14 +38,15 @@
 //   its sign bit set is ruled out with no further work (NaN test values, which the
 //   maximum skips, only arise in rows whose thread tests every codeword anyway: see
 //   T' = -2^100 below). Only a chunk with a non-negative maximum sends the row to
-//   the exact fp32 direct form on the CUDA cores, which reads c = c_hi + c_lo
-//   (exact) from the shared tile. When a row's best improves, its thread rewrites
-//   its T' (one 4-byte shared store). MMAs already issued, or issued before the
+//   the exact fp32 direct form on the CUDA cores, which reads c in fp32 from the
+//   same shared stage (every streamed tile carries its codewords in fp32 after the
+//   fp16 operands). When a row's best improves, its thread rewrites its T' (one
+//   2-byte shared store). MMAs already issued, or issued before the
 //   store is seen, use the older T', which satisfied the inequality for the older,
 //   larger best, and so for the current one: the test stays sound at every moment.
-//   A half row without a usable T' (no running best yet, non-finite inputs) holds
-//   T' = -2^100: its g is then huge and positive (and no infinity meets the other
-//   half's 0), and its thread tests every codeword exactly anyway.
+//   A half row without a usable T' (no running best yet, non-finite or out-of-range
+//   inputs) holds -T' = 2^15, finite so that the other half's 0 meets no
+//   infinity, and its thread tests every codeword exactly.
 //
 // Warm starts (a hint per kernel): a row's own hinted codeword always passes the
 // test (its distance is the best, which the test cannot rule out), so every row
@@ -47,12 +57,13 @@
 // row perm[s]; results do not depend on the order.
 //
 // Warp roles in a CTA of 352 threads that owns 256 kernels (two 128-row tiles):
-//   warp 0      producer: streams packed codeword tiles (256 codewords x 128 B,
-//               already in the tensor-core layout) into a 4-stage shared ring with
-//               one bulk asynchronous copy per tile (TMA engine), mbarrier tx counts;
+//   warp 0      producer: streams packed codeword tiles (256 codewords x 100 B:
+//               64 B of fp16 operands in the tensor-core layout, then 36 B of fp32
+//               codeword) into a 6-stage shared ring with one bulk asynchronous
+//               copy per tile (TMA engine), mbarrier tx counts;
 //   warps 1-2   MMA issuers, one per row tile (warp 1 also owns TMEM: 512 columns,
-//               one 256-column accumulator per row tile): from one thread, the 4
-//               MMAs (M = 128, N = 256, K = 8 each) of its row tile for a codeword
+//               one 256-column accumulator per row tile): from one thread, the 2
+//               MMAs (M = 128, N = 256, K = 16 each) of its row tile for a codeword
 //               tile, then tcgen05.commit. The epilogue drains one accumulator
 //               while the tensor core fills the other. Two issuers, because the
 //               first shared-memory access (a barrier wait) of a thread after its
@@ -72,6 +83,8 @@
 // N = 128 ones lose ~20%.)
 // Every wait is bounded; a wait that runs out sets KQ_FLAG_TIMEOUT and an abort
 // word, every role then drains out, and warp 1 frees TMEM before the CTA exits.
+#include <cuda_fp16.h>
+
 #include "kq_internal.cuh"
 
 namespace kq {
@@ -81,25 +94,30 @@ constexpr int TC_RT = 2;                   // row tiles per CTA
 constexpr int TC_ROWS = TC_M * TC_RT;      // kernels per CTA
 constexpr int TC_N = 256;                  // codewords per tile (N of every MMA)
 constexpr int TC_HALF = TC_N / 2;          // codewords of a tile one epilogue thread tests
-constexpr int TC_KD = 32;                  // K of the GEMM (hi/lo split, see top of file)
-constexpr int TC_STAGES = 4;
-constexpr int TC_TILE_BYTES = TC_N * TC_KD * 4;  // 32 KiB per codeword tile
-constexpr int TC_A_BYTES = TC_M * TC_KD * 4;     // 16 KiB per row tile
+constexpr int TC_KD = 32;                  // K of the GEMM in fp16 elements (hi/lo split, see top of file)
+constexpr int TC_STAGES = 6;
+constexpr int TC_TILE_H = TC_N * TC_KD * 2;      // 16 KiB of fp16 operands per codeword tile
+constexpr int TC_TILE_BYTES = TC_TILE_H + TC_N * D * 4;  // + the tile's codewords in fp32: 25 KiB streamed
+constexpr int TC_A_BYTES = TC_M * TC_KD * 2;     // 8 KiB per row tile
 constexpr int TC_THREADS = 352;
 constexpr int TC_EPI_WARP0 = 3;            // first epilogue warp (0: producer, 1-2: MMA issuers)
 constexpr int TC_EPI_WARPS = 8;
 constexpr uint32_t TC_COLS = 512;          // TMEM columns allocated (2 row tiles x 256)
 constexpr uint32_t TC_LBO = 128;           // K-adjacent core matrices (8 rows x 16 B each)
-constexpr uint32_t TC_SBO = TC_KD / 4 * 128; // next 8-row group (8 core matrices along K)
+constexpr uint32_t TC_SBO = TC_KD / 8 * 128; // next 8-row group (4 core matrices along K)
 constexpr long long TC_WAIT_LIMIT = 4000000;
 constexpr float TWO_G_TC = 3.0517578125e-5f;  // 2 x 2^-16 (see top of file)
+constexpr float TWO_ABS_TC = 9.765625e-4f;     // 2 x 2^-11: twice the absolute part of E, per unit of |x| + Cmax + 1
 constexpr float INV_ONE_M_G11_TC = 1.0000008344650269f;  // 1 + 7 * 2^-23 >= 1 / (1 - gamma_11) (direct-form bound)
 constexpr int TC_SLOT_T0 = 29, TC_SLOT_R = 30, TC_SLOT_T1 = 31;  // K slots of -T'0, -R, -T'1
-constexpr float TC_T_EVERY = 1.2676506002282294e30f;  // 2^100: -T' of a half row tested exactly
+constexpr float TC_T_EVERY = 32768.f;      // -T' of a half row tested exactly (finite in fp16)
+constexpr float TC_T_LIMIT = 16384.f;      // |T'| bound that keeps -T' an fp16 operand
+constexpr float TC_X_LIMIT = 256.f;        // scaled |x| above which a row is tested exactly
+constexpr float F16_MIN_NORMAL = 6.103515625e-05f;  // 2^-14
 
-// Byte offset of element (row, k) in a K-major, no-swizzle core-matrix tile.
+// Byte offset of fp16 element (row, k) in a K-major, no-swizzle core-matrix tile.
 __host__ __device__ __forceinline__ uint32_t tc_offset(int row, int k) {
-    return (uint32_t)(row / 8) * TC_SBO + (uint32_t)(k / 4) * TC_LBO + (uint32_t)(row % 8) * 16 + (uint32_t)(k % 4) * 4;
+    return (uint32_t)(row / 8) * TC_SBO + (uint32_t)(k / 8) * TC_LBO + (uint32_t)(row % 8) * 16 + (uint32_t)(k % 8) * 2;
 }
 
 __device__ __forceinline__ uint64_t tc_smem_desc(uint32_t saddr) {
@@ -110,9 +128,9 @@ __device__ __forceinline__ uint64_t tc_smem_desc(uint32_t saddr) {
     return d;
 }
 
-// kind::tf32 instruction descriptor: D f32, A and B tf32, both K-major, M x N.
+// kind::f16 instruction descriptor: D f32, A and B f16, both K-major, M x N.
 __host__ __device__ constexpr uint32_t tc_idesc(int m, int n) {
-    return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+    return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 
 __device__ __forceinline__ void mbar_init(uint32_t a, uint32_t count) {
@@ -177,91 +195,187 @@ __device__ __forceinline__ uint32_t sign_mask32(const uint32_t (&r)[32]) {
     return s[0];
 }
 
-// v = hi + lo exactly, hi = v truncated to tf32 (10 explicit mantissa bits).
-__device__ __forceinline__ float tf32_hi(float v) { return __uint_as_float(__float_as_uint(v) & 0xFFFFE000u); }
+// v truncated to fp16 (toward zero), back in fp32.
+__device__ __forceinline__ float f16_rz(float v) { return __half2float(__float2half_rz(v)); }
 
-// v rounded toward -inf to tf32 (finite v).
-__device__ __forceinline__ float tf32_rd(float v) {
-    const uint32_t u = __float_as_uint(v);
-    if ((u & 0x1FFFu) == 0u) return v;
-    return __uint_as_float(v > 0.f ? (u & 0xFFFFE000u) : (u & 0xFFFFE000u) + 0x2000u);
+// fp16 bits of a value that fp16 represents exactly.
+__device__ __forceinline__ uint32_t f16_bits(float v) { return (uint32_t)__half_as_ushort(__float2half_rn(v)); }
+
+// v (finite, |v| < 2^14) rounded toward -inf to a normal fp16 value or 0: a
+// subnormal result becomes 0 (v > 0) or -2^-14 (v < 0), still <= v, so a tensor
+// core that flushes subnormal inputs sees the same operand.
+__device__ __forceinline__ float f16_rd_normal(float v) {
+    float r = __half2float(__float2half_rd(v));
+    if (r != 0.f && fabsf(r) < F16_MIN_NORMAL) r = r > 0.f ? 0.f : -F16_MIN_NORMAL;
+    return r;
 }
 
-// The first 29 slots of the K = 32 row layout for one operand (see top of file).
-// `a_side` selects the A pattern (x_hi, 1, x_hi, 1, x_lo) or the B pattern (c_hi,
-// -h_hi, c_lo, -h_lo, c_hi); v holds the 9 values, extra the 10th (1 for A, -h for
-// B). The caller fills slots 29-31.
+// The scale beta = 2^(6 - e) of the fp16 operands for a codebook whose largest
+// norm is f 2^e (f in [0.5, 1)): the scaled norm lands in [32, 64). 1 when that
+// norm is zero or not finite; the exponent stays within +-60 so that beta^2 is a
+// normal fp32 number.
+__device__ __forceinline__ float tc_scale(float craw) {
+    if (!(craw > 0.f) || !(craw <= 3.402823466e38f)) return 1.f;
+    int e;
+    frexpf(craw, &e);
+    return ldexpf(1.f, min(60, max(-60, 6 - e)));
+}
+
+// The first 29 slots of the K = 32 row layout for one operand (see top of file), as
+// fp16-representable values. `a_side` selects the A pattern (x_hi, 1, x_hi, 1,
+// x_lo) or the B pattern (c_hi, -h_hi, c_lo, -h_lo, c_hi); v holds the 9 scaled
+// values, extra the 10th (1 for A, -h for B). The caller fills slots 29-31.
 __device__ __forceinline__ void tc_row(const float (&v)[D], float extra, bool a_side, float (&out)[TC_KD]) {
 #pragma unroll
     for (int j = 0; j < D; ++j) {
-        const float hi = tf32_hi(v[j]), lo = v[j] - hi;
+        const float hi = f16_rz(v[j]), lo = f16_rz(v[j] - hi);
         out[j] = hi;
         out[10 + j] = a_side ? hi : lo;
         out[20 + j] = a_side ? lo : hi;
     }
-    const float ehi = tf32_hi(extra);
+    const float ehi = f16_rz(extra);
     out[D] = a_side ? 1.f : ehi;
-    out[19] = a_side ? 1.f : extra - ehi;
+    out[19] = a_side ? 1.f : f16_rz(extra - ehi);
 }
 
-// Packs C into tensor-core tiles (Kpad codewords, Kpad a multiple of TC_N) and
-// reduces the same codebook bounds as pack_codebook_kernel into hdr->cb_*.
-// Padding codewords get c = 0 and -h = -inf, so their g is -inf.
-__global__ void __launch_bounds__(256) pack_codebook_tc_kernel(const float *__restrict__ C, int32_t K, int32_t Kpad,
-                                                               float *__restrict__ Cpk, Header *hdr) {
-    const int k = blockIdx.x * blockDim.x + threadIdx.x;
-    float cmax = 0.f, hmax = 0.f, qmax = 0.f;
-    if (k < Kpad) {
-        float c[D];
-        float mh = __int_as_float(0xff800000);  // -h; -inf for padding codewords
+// Row `row` of an fp16 operand tile: the 32 slot values, four 16-byte stores.
+__device__ __forceinline__ void tc_store_row(unsigned char *tile, int row, const float (&v)[TC_KD]) {
 #pragma unroll
-        for (int j = 0; j < D; ++j) c[j] = 0.f;
-        if (k < K) {
-            bool ok = true;
-            float s = 0.f, c2lo = 0.f, c2hi = 0.f;
+    for (int q = 0; q < TC_KD / 8; ++q) {
+        uint32_t w[4];
 #pragma unroll
-            for (int j = 0; j < D; ++j) {
-                c[j] = C[(int64_t)k * D + j];
-                ok &= isfinite(c[j]);
-                s = fmaf(c[j], c[j], s);
-                c2lo = __fadd_rd(c2lo, __fmul_rd(c[j], c[j]));
-                c2hi = __fadd_ru(c2hi, __fmul_ru(c[j], c[j]));
-            }
-            const float h = 0.5f * s;
-            const float h2 = h + h;
-            mh = -h;
-            cmax = __fsqrt_ru(c2hi);
-            hmax = fabsf(h);
-            qmax = fmaxf(fabsf(__fsub_ru(c2hi, h2)), fabsf(__fsub_rd(c2lo, h2)));
-            if (!ok) {
-                set_flag(&hdr->status, KQ_FLAG_NONFINITE);
-                cmax = hmax = qmax = __int_as_float(0x7fc00000);  // NaN: disables the test
-            }
+        for (int p = 0; p < 4; ++p) w[p] = f16_bits(v[8 * q + 2 * p]) | (f16_bits(v[8 * q + 2 * p + 1]) << 16);
+        *reinterpret_cast<uint4 *>(tile + tc_offset(row, 8 * q)) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+// Norm of codeword k rounded up, NaN when a value is not finite.
+__device__ __forceinline__ float codeword_norm_ru(const float *__restrict__ C, int64_t k) {
+    bool ok = true;
+    float c2hi = 0.f;
+#pragma unroll
+    for (int j = 0; j < D; ++j) {
+        const float c = C[k * D + j];
+        ok &= isfinite(c);
+        c2hi = __fadd_ru(c2hi, __fmul_ru(c, c));
+    }
+    return ok ? __fsqrt_ru(c2hi) : __int_as_float(0x7fc00000);
+}
+
+// Maximum of non-negative floats and NaN through their bits (NaN orders above all).
+__device__ __forceinline__ float max_bits(float a, float b) {
+    return __uint_as_float(max(__float_as_uint(a), __float_as_uint(b)));
+}
+__device__ __forceinline__ float warp_max_bits(float m) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = __uint_as_float(max(__float_as_uint(m), __shfl_xor_sync(0xffffffffu, __float_as_uint(m), o)));
+    return m;
+}
+
+// Codeword k of the padded codebook (k < Kpad) into its tile: the fp16 operands of
+// beta c, then c in fp32 for the exact path; returns the scaled bounds of
+// pack_codebook_kernel (cmax, hmax, qmax; NaN for a non-finite codeword, 0 for
+// padding). Padding codewords get c = 0 and -h = -inf, so their g is -inf.
+__device__ __forceinline__ void pack_codeword_tc(const float *__restrict__ C, int32_t K, int32_t k, float beta,
+                                                 float *__restrict__ Cpk, Header *hdr, float &cmax, float &hmax,
+                                                 float &qmax) {
+    float c[D], c32[D];
+    float mh = __int_as_float(0xff800000);  // -h; -inf for padding codewords
+#pragma unroll
+    for (int j = 0; j < D; ++j) c[j] = c32[j] = 0.f;
+    cmax = hmax = qmax = 0.f;
+    if (k < K) {
+        bool ok = true;
+        float s = 0.f, c2lo = 0.f, c2hi = 0.f;
+#pragma unroll
+        for (int j = 0; j < D; ++j) {
+            c32[j] = C[(int64_t)k * D + j];
+            c[j] = beta * c32[j];  // exact: a power of two, inside the normal range
+            ok &= isfinite(c[j]);
+            s = fmaf(c[j], c[j], s);
+            c2lo = __fadd_rd(c2lo, __fmul_rd(c[j], c[j]));
+            c2hi = __fadd_ru(c2hi, __fmul_ru(c[j], c[j]));
         }
-        const int kl = k % TC_N;
-        float v[TC_KD];
-        tc_row(c, mh, false, v);
-        if (!(mh >= -3.402823466e38f)) v[19] = 0.f;  // padding: -inf already sits in the hi slot
-        v[TC_SLOT_T0] = kl < TC_HALF ? 1.f : 0.f;
-        v[TC_SLOT_R] = 1.f;
-        v[TC_SLOT_T1] = kl < TC_HALF ? 0.f : 1.f;
-        unsigned char *tile = reinterpret_cast<unsigned char *>(Cpk) + (int64_t)(k / TC_N) * TC_TILE_BYTES;
-#pragma unroll
-        for (int q = 0; q < TC_KD / 4; ++q)
-            *reinterpret_cast<float4 *>(tile + tc_offset(kl, 4 * q)) =
-                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        const float h = 0.5f * s;
+        const float h2 = h + h;
+        mh = -h;
+        cmax = __fsqrt_ru(c2hi);
+        hmax = fabsf(h);
+        qmax = fmaxf(fabsf(__fsub_ru(c2hi, h2)), fabsf(__fsub_rd(c2lo, h2)));
+        if (!ok) {
+            set_flag(&hdr->status, KQ_FLAG_NONFINITE);
+            cmax = hmax = qmax = __int_as_float(0x7fc00000);  // NaN: disables the test
+        }
     }
+    const int kl = k % TC_N;
+    float v[TC_KD];
+    tc_row(c, mh, false, v);
+    if (!(mh >= -3.402823466e38f)) v[19] = 0.f;  // padding: -inf already sits in the hi slot
+    v[TC_SLOT_T0] = kl < TC_HALF ? 1.f : 0.f;
+    v[TC_SLOT_R] = 1.f;
+    v[TC_SLOT_T1] = kl < TC_HALF ? 0.f : 1.f;
+    unsigned char *tile = reinterpret_cast<unsigned char *>(Cpk) + (int64_t)(k / TC_N) * TC_TILE_BYTES;
+    tc_store_row(tile, kl, v);
+    float *cw = reinterpret_cast<float *>(tile + TC_TILE_H) + kl * D;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        cmax = __uint_as_float(max(__float_as_uint(cmax), __shfl_xor_sync(0xffffffffu, __float_as_uint(cmax), o)));
-        hmax = __uint_as_float(max(__float_as_uint(hmax), __shfl_xor_sync(0xffffffffu, __float_as_uint(hmax), o)));
-        qmax = __uint_as_float(max(__float_as_uint(qmax), __shfl_xor_sync(0xffffffffu, __float_as_uint(qmax), o)));
-    }
+    for (int j = 0; j < D; ++j) cw[j] = c32[j];
+}
+
+__device__ __forceinline__ void publish_bounds_tc(float cmax, float hmax, float qmax, Header *hdr) {
+    cmax = warp_max_bits(cmax);
+    hmax = warp_max_bits(hmax);
+    qmax = warp_max_bits(qmax);
     if ((threadIdx.x & 31) == 0) {
         atomicMax(&hdr->cb_cmax, __float_as_uint(cmax));
         atomicMax(&hdr->cb_hmax, __float_as_uint(hmax));
         atomicMax(&hdr->cb_qmax, __float_as_uint(qmax));
     }
+}
+
+// hdr->cb_craw = the codebook's largest norm (rounded up; NaN when a value is not
+// finite), from which the operand scale beta is taken.
+__global__ void __launch_bounds__(256) codebook_norm_tc_kernel(const float *__restrict__ C, int32_t K, Header *hdr) {
+    const int k = blockIdx.x * blockDim.x + threadIdx.x;
+    const float m = warp_max_bits(k < K ? codeword_norm_ru(C, k) : 0.f);
+    if ((threadIdx.x & 31) == 0) atomicMax(&hdr->cb_craw, __float_as_uint(m));
+}
+
+// Packs beta C into tensor-core tiles (Kpad codewords, Kpad a multiple of TC_N) and
+// reduces the scaled codebook bounds into hdr->cb_*; beta from hdr->cb_craw.
+__global__ void __launch_bounds__(256) pack_codebook_tc_kernel(const float *__restrict__ C, int32_t K, int32_t Kpad,
+                                                               float *__restrict__ Cpk, Header *hdr) {
+    const int k = blockIdx.x * blockDim.x + threadIdx.x;
+    const float beta = tc_scale(__uint_as_float(__ldcg(&hdr->cb_craw)));
+    float cmax = 0.f, hmax = 0.f, qmax = 0.f;
+    if (k < Kpad) pack_codeword_tc(C, K, k, beta, Cpk, hdr, cmax, hmax, qmax);
+    publish_bounds_tc(cmax, hmax, qmax, hdr);
+}
+
+// Both steps in one CTA, for small codebooks (one launch instead of two).
+constexpr int32_t TC_PACK_ONE_CTA = 2048;
+__global__ void __launch_bounds__(256) pack_codebook_tc_small_kernel(const float *__restrict__ C, int32_t K,
+                                                                     int32_t Kpad, float *__restrict__ Cpk,
+                                                                     Header *hdr) {
+    __shared__ float s_m[8];
+    float m = 0.f;
+    for (int k = threadIdx.x; k < K; k += 256) m = max_bits(m, codeword_norm_ru(C, k));
+    m = warp_max_bits(m);
+    if ((threadIdx.x & 31) == 0) s_m[threadIdx.x >> 5] = m;
+    __syncthreads();
+    m = s_m[0];
+#pragma unroll
+    for (int w = 1; w < 8; ++w) m = max_bits(m, s_m[w]);
+    if (threadIdx.x == 0) hdr->cb_craw = __float_as_uint(m);
+    const float beta = tc_scale(m);
+    float cmax = 0.f, hmax = 0.f, qmax = 0.f;
+    for (int k = threadIdx.x; k < Kpad; k += 256) {
+        float a, b, c;
+        pack_codeword_tc(C, K, k, beta, Cpk, hdr, a, b, c);
+        cmax = max_bits(cmax, a);
+        hmax = max_bits(hmax, b);
+        qmax = max_bits(qmax, c);
+    }
+    publish_bounds_tc(cmax, hmax, qmax, hdr);
 }
 
 // Per-row constants of the test: k0 = X2lo - Qmax (rounded down), k1 = |x| Cmax +
@@ -270,18 +384,20 @@ struct RowConst {
     float k0, k1, k2, R;
 };
 
-// T' for a running best b: with thr0 = (k0 - b / (1 - gamma_11)) / 2 (rounded down)
-// and dT = thr0 - R (rounded down), T' = dT - 2^-15 (k1 + |dT|) - k2 rounded down
-// to tf32. Then E(T') < thr0 - R - T' (|T'| <= (1 + 2^-9)(|dT| + margin) and
-// 2^-16 (k1 + that) stays below the margin), so R + T' + E < thr0. Returns false
-// (test every codeword) when any of it is not finite or |T'| would reach 2^100.
-__device__ __forceinline__ bool tc_shift(const RowConst &rc, float b, float &tp) {
-    const float thr0 = __fmul_rd(__fsub_rd(rc.k0, __fmul_ru(b, INV_ONE_M_G11_TC)), 0.5f);
+// T' for a running best b (unscaled; beta2 = beta^2): with thr0 = (k0 - beta2 b /
+// (1 - gamma_11)) / 2 (rounded down) and dT = thr0 - R (rounded down), T' = dT -
+// 2^-15 (k1 + |dT|) - k2 rounded down to a normal fp16 value or 0. Then E(T') <
+// thr0 - R - T' (|T'| <= (1 + 2^-10)(|dT| + margin) + 2^-14, and 2^-16 (k1 +
+// that) + k2 / 2 stays below the margin since k2 >= 2^-10), so R + T' + E < thr0.
+// Returns false (test every codeword) when any of it is not finite or |T'| would
+// reach 2^14.
+__device__ __forceinline__ bool tc_shift(const RowConst &rc, float b, float beta2, float &tp) {
+    const float thr0 = __fmul_rd(__fsub_rd(rc.k0, __fmul_ru(__fmul_ru(b, beta2), INV_ONE_M_G11_TC)), 0.5f);
     const float dT = __fsub_rd(thr0, rc.R);
     const float margin = __fadd_ru(__fmul_ru(TWO_G_TC, __fadd_ru(rc.k1, fabsf(dT))), rc.k2);
     const float pre = __fsub_rd(dT, margin);
-    if (!(fabsf(pre) < 1.0e30f)) return false;
-    tp = tf32_rd(pre);
+    if (!(fabsf(pre) < TC_T_LIMIT)) return false;
+    tp = f16_rd_normal(pre);
     return true;
 }
 
@@ -317,6 +433,8 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     volatile uint32_t *abort_flag = &S.abort_flag;
     uint32_t *status = &hdr->status;
+    const float beta = tc_scale(__uint_as_float(__ldcg(&hdr->cb_craw)));  // as pack_codebook_tc_kernel
+    const float beta2 = beta * beta;
 
     // ---- epilogue threads: one kernel in each row tile, one half of every tile
     const bool epi = warp >= TC_EPI_WARP0;
@@ -339,29 +457,33 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
             // slot -> kernel row (rows in the order of a permutation, when given)
             const int64_t slot = (int64_t)blockIdx.x * TC_ROWS + rloc;
             const int64_t row = slot < n ? (perm ? (int64_t)__ldg(perm + slot) : slot) : n;
-            float x[D];
+            float x[D], xs[D];  // the kernel, and beta times it (exact unless out of range)
 #pragma unroll
-            for (int j = 0; j < D; ++j) x[j] = row < n ? W[row * D + j] : 0.f;
+            for (int j = 0; j < D; ++j) {
+                x[j] = row < n ? W[row * D + j] : 0.f;
+                xs[j] = beta * x[j];
+            }
             bool ok = true;
 #pragma unroll
             for (int j = 0; j < D; ++j) ok &= isfinite(x[j]);
             if (row < n && !ok && hsel == 0) set_flag(status, KQ_FLAG_NONFINITE);
-            const float cmax = __uint_as_float(__ldcg(&hdr->cb_cmax));
+            const float cmax = __uint_as_float(__ldcg(&hdr->cb_cmax));  // scaled bounds
             const float hmax = __uint_as_float(__ldcg(&hdr->cb_hmax));
             const float qmax = __uint_as_float(__ldcg(&hdr->cb_qmax));
             float x2lo = 0.f, x2hi = 0.f;
 #pragma unroll
             for (int j = 0; j < D; ++j) {
-                x2lo = __fadd_rd(x2lo, __fmul_rd(x[j], x[j]));
-                x2hi = __fadd_ru(x2hi, __fmul_ru(x[j], x[j]));
+                x2lo = __fadd_rd(x2lo, __fmul_rd(xs[j], xs[j]));
+                x2hi = __fadd_ru(x2hi, __fmul_ru(xs[j], xs[j]));
             }
             const float xn = __fsqrt_ru(x2hi);
+            const bool inrange = xn <= TC_X_LIMIT;  // false for non-finite rows too
             RowConst rc;
-            rc.R = tf32_hi(0.5f * x2lo);
-            if (!(fabsf(rc.R) <= 3.402823466e38f)) rc.R = 0.f;  // any tf32 value is valid
-            rc.k0 = __fsub_rd(x2lo, qmax);
+            rc.R = inrange ? f16_rz(0.5f * x2lo) : 0.f;
+            if (rc.R < F16_MIN_NORMAL) rc.R = 0.f;  // a normal fp16 operand or 0
+            rc.k0 = inrange ? __fsub_rd(x2lo, qmax) : __int_as_float(0x7fc00000);  // NaN: never shifted
             rc.k1 = __fadd_ru(__fadd_ru(hmax, __fmul_ru(xn, cmax)), fabsf(rc.R));
-            rc.k2 = __fmul_ru(1.504632769052528e-36f /* 2 x 2^-120 */, __fadd_ru(__fadd_ru(cmax, xn), 1.f));
+            rc.k2 = __fmul_ru(TWO_ABS_TC, __fadd_ru(__fadd_ru(cmax, xn), 1.f));
             bool ev = true;
             float tp = 0.f;
             if (hint != nullptr && row < n) {
@@ -371,7 +493,7 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                     if (d < best[t]) {
                         best[t] = d;
                         bi[t] = known[t] = h;
-                        ev = !tc_shift(rc, d, tp);
+                        ev = !tc_shift(rc, d, beta2, tp);
                     }
                 }
             }
@@ -380,14 +502,13 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
 #pragma unroll
                 for (int j = 0; j < D; ++j) S.xs[rloc][j] = x[j];
                 S.rc[rloc] = rc;
-                float a[TC_KD];
-                tc_row(x, 1.f, true, a);
+                float a[TC_KD], xa[D];
+#pragma unroll
+                for (int j = 0; j < D; ++j) xa[j] = inrange ? xs[j] : 0.f;
+                tc_row(xa, 1.f, true, a);
                 a[TC_SLOT_T0] = a[TC_SLOT_T1] = ev ? TC_T_EVERY : -tp;
                 a[TC_SLOT_R] = -rc.R;
-#pragma unroll
-                for (int u = 0; u < TC_KD / 4; ++u)
-                    *reinterpret_cast<float4 *>(&S.a[t][tc_offset(r, 4 * u)]) =
-                        make_float4(a[4 * u], a[4 * u + 1], a[4 * u + 2], a[4 * u + 3]);
+                tc_store_row(S.a[t], r, a);
             }
         }
     }
@@ -457,12 +578,12 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t b0 = (uint32_t)__cvta_generic_to_shared(S.b[s]);
 #pragma unroll
-                for (int kb = 0; kb < TC_KD / 8; ++kb) {
+                for (int kb = 0; kb < TC_KD / 16; ++kb) {
                     const uint64_t ad = tc_smem_desc(a0 + kb * 2 * TC_LBO);
-                    const uint64_t bd = tc_smem_desc(b0 + kb * 2 * TC_LBO);  // 8 tf32 of K per MMA
+                    const uint64_t bd = tc_smem_desc(b0 + kb * 2 * TC_LBO);  // 16 fp16 of K per MMA
                     asm volatile(
                         "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-                        " tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}" ::"r"(dcol),
+                        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(dcol),
                         "l"(ad), "l"(bd), "r"(idesc), "r"((uint32_t)kb)
                         : "memory");
                 }
@@ -547,11 +668,11 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                             const int32_t k = i * TC_N + kl;
                             if (k >= K) break;
                             float xr[D], cw[D];
+                            const float *c32 = reinterpret_cast<const float *>(tile + TC_TILE_H) + kl * D;
 #pragma unroll
                             for (int u = 0; u < D; ++u) {
                                 xr[u] = S.xs[rloc][u];
-                                cw[u] = *reinterpret_cast<const float *>(tile + tc_offset(kl, u)) +
-                                        *reinterpret_cast<const float *>(tile + tc_offset(kl, 10 + u));  // c_hi + c_lo = c
+                                cw[u] = c32[u];
                             }
                             const float d = direct_distance(xr, cw);
                             if (d < best[t] || (d == best[t] && k < bi[t])) {
@@ -563,10 +684,10 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                     }
                     if (moved) {
                         float tp = 0.f;
-                        const bool e2 = !tc_shift(S.rc[rloc], best[t], tp);
+                        const bool e2 = !tc_shift(S.rc[rloc], best[t], beta2, tp);
                         every = (every & ~(1u << t)) | ((e2 ? 1u : 0u) << t);
-                        *reinterpret_cast<float *>(&S.a[t][tc_offset(r, hsel ? TC_SLOT_T1 : TC_SLOT_T0)]) =
-                            e2 ? TC_T_EVERY : -tp;
+                        *reinterpret_cast<uint16_t *>(&S.a[t][tc_offset(r, hsel ? TC_SLOT_T1 : TC_SLOT_T0)]) =
+                            (uint16_t)f16_bits(e2 ? TC_T_EVERY : -tp);
                         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // for later MMAs
                     }
                 }
@@ -640,9 +761,17 @@ bool tc_eligible(int64_t n, int32_t K, int num_sms) {
 }
 
 cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Header *hdr, cudaStream_t s) {
-    cudaError_t e = cudaMemsetAsync(&hdr->cb_cmax, 0, 3 * sizeof(uint32_t), s);
+    cudaError_t e = cudaMemsetAsync(&hdr->cb_cmax, 0, 4 * sizeof(uint32_t), s);  // cb_cmax .. cb_craw
     if (e != cudaSuccess) return e;
     const int32_t Kpad = tc_kpad(K);
+    if (Kpad <= TC_PACK_ONE_CTA) {
+        pack_codebook_tc_small_kernel<<<1, 256, 0, s>>>(C, K, Kpad, Cpk, hdr);
+        count_launch();
+        return cudaGetLastError();
+    }
+    codebook_norm_tc_kernel<<<(K + 255) / 256, 256, 0, s>>>(C, K, hdr);
+    count_launch();
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
     pack_codebook_tc_kernel<<<(Kpad + 255) / 256, 256, 0, s>>>(C, K, Kpad, Cpk, hdr);
     count_launch();
     return cudaGetLastError();

@@ -29,7 +29,8 @@ struct Header {
     uint32_t hi_w, hi_a;    // level fit: ordered-int maxima over weighted / all scalars (init 0)
     uint32_t maxv_w;        // level fit: max |v| over weighted scalars (fp32 bits)
     uint32_t pad1;
-    uint32_t cb_cmax, cb_hmax, cb_qmax, pad2;  // assign filter: codebook bounds (fp32 bits, see kq_assign.cu)
+    uint32_t cb_cmax, cb_hmax, cb_qmax;  // assign filter: codebook bounds (fp32 bits, see kq_assign.cu)
+    uint32_t cb_craw;       // tensor-core assign: largest codeword norm before scaling (fp32 bits)
     uint32_t upd_bound;     // update: bound B on |W| the fixed-point scale was chosen for (fp32 bits)
     uint32_t upd_violation; // update: a |w| > B was seen (the exact fallback must run)
     int32_t upd_scale;      // update: the scale exponent S the accumulators hold
