@@ -79,8 +79,11 @@
 // the CTA barrier that opens the teardown: a lone lane waits on a completed
 // mbarrier phase in ~20 cycles, a whole warp (or a lane whose partners wait at a
 // warp-level sync) in ~100-300, all of it idle time for the tensor core when it is
-// the MMA issuer's. (N = 256 MMAs keep the tensor core fully busy from one thread;
-// N = 128 ones lose ~20%.)
+// the MMA issuer's. (Back to back, one thread's MMAs run at the full rate with N = 256
+// or 128; here N = 128 jobs on two accumulators per row tile were slower. What
+// bounds the kernel is the per-job hand-back: issue, execution, commit, TMEM loads,
+// arrive and the next issue take ~880 cycles per row tile, of which only the other
+// row tile's 256 cycles of MMA overlap.)
 // Every wait is bounded; a wait that runs out sets KQ_FLAG_TIMEOUT and an abort
 // word, every role then drains out, and warp 1 frees TMEM before the CTA exits.
 #include <cuda_fp16.h>
