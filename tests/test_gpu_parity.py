@@ -123,10 +123,14 @@ def test_assign_filter_extreme_scales(case):
 TC_MIN_N = 256 * 152  # one row block per SM (from about 256 kernels on the tensor cores run)
 
 
-@pytest.mark.parametrize("case", ["plain", "offset", "mixed", "large", "near_dup", "ragged"])
+@pytest.mark.parametrize("case", ["plain", "offset", "mixed", "large", "near_dup", "ragged", "outlier_codeword",
+                                  "outlier_rows"])
 def test_assign_tensor_core_path(case):
     # n large enough for the tensor-core path; K = 1000 is not a multiple of the
-    # 128-codeword tile, so padding codewords are exercised too.
+    # 128-codeword tile, so padding codewords are exercised too. The fp16 operands
+    # are scaled by one power of two per call: an outlier codeword sets that scale
+    # (every other value then sits low in the fp16 range), and rows far outside the
+    # codebook leave the range (they are tested exactly against every codeword).
     n, K = TC_MIN_N + 1000, 1000
     if case == "ragged":
         n = TC_MIN_N + 77
@@ -142,10 +146,16 @@ def test_assign_tensor_core_path(case):
     elif case == "near_dup":
         C[1::2] = np.nextafter(C[0::2], np.float32(np.inf))[: C[1::2].shape[0]]
         W[:K] = C
+    elif case == "outlier_codeword":
+        C[5] *= 3e4
+    elif case == "outlier_rows":
+        W[::97] *= 1e4
     W, C = W.astype(np.float32), C.astype(np.float32)
     idx, dist, st, _ = gpu_assign(W, C)
     assert st == 0
     rows = np.sort(synth.below(synth.stream_key(203, 9), 6000, n))
+    if case == "outlier_rows":
+        rows = np.unique(np.concatenate([rows, np.arange(0, n, 97)[:500]]))
     rows[-1] = n - 1
     idx_ref, dist_ref = oracle.assign(W[rows], C, threads=THREADS)
     assert check_indices(W, C, idx[rows], idx_ref, rows) == 0
