@@ -299,27 +299,59 @@ def run_kq(args, rank, world, local_rank):
             "codes": torch.empty(K, 9, dtype=torch.uint8).pin_memory(),
             "Wr": torch.empty(n, 9, dtype=torch.float32).pin_memory(),
             "objective": torch.empty(T + 1, dtype=torch.float64).pin_memory()}
-    obj = torch.empty(T + 1, dtype=torch.float64, device=dev)
-    Wd = torch.empty_like(W)
-    seld = torch.empty_like(sel)
+    # Steps are pipelined over two buffer sets: step s computes on the default stream
+    # while a copy stream brings in step s + 1's inputs and reads out step s - 1's
+    # outputs (events order each copy against the compute that produces or consumes
+    # its buffers). Every step's inputs still cross from pinned host memory and all
+    # its outputs come back inside the timed region.
+    main = torch.cuda.current_stream(dev)
+    cs = torch.cuda.Stream(dev)
+    bufs = [{"W": torch.empty_like(W), "sel": torch.empty_like(sel),
+             "C0": torch.empty(K, 9, dtype=torch.float32, device=dev),
+             "C": torch.empty(K, 9, dtype=torch.float32, device=dev),
+             "idx": torch.empty(n, dtype=torch.int32, device=dev),
+             "counts": torch.empty(K, dtype=torch.int32, device=dev),
+             "levels": torch.empty(64, dtype=torch.float32, device=dev),
+             "codes": torch.empty(K, 9, dtype=torch.uint8, device=dev),
+             "Wr": torch.empty_like(W),
+             "objective": torch.empty(T + 1, dtype=torch.float64, device=dev)} for _ in range(2)]
+    ev = {k: [torch.cuda.Event() for _ in range(2)] for k in ("in", "used", "out")}
 
-    def e2e_step():
-        Wd.copy_(W_pin, non_blocking=True)
-        seld.copy_(sel_pin, non_blocking=True)
-        kq.kq_init_codebook(Wd, seld, Ca, ws)
-        kq.kq_fit_codebook(Wd, Ca, T, Cb, idx, counts, obj, ws)
-        kq.kq_quantize_codebook_6bit(Cb, counts, 100, levels, codes, None, ws)
-        kq.kq_reconstruct(idx, None, codes, levels, Wr, ws, K=K)
-        for name, src in (("C", Cb), ("idx", idx), ("counts", counts), ("levels", levels), ("codes", codes),
-                          ("Wr", Wr), ("objective", obj)):
-            outs[name].copy_(src, non_blocking=True)
+    def e2e_run(steps):
+        def fetch(s):
+            b = bufs[s % 2]
+            with torch.cuda.stream(cs):
+                if s >= 2:
+                    cs.wait_event(ev["used"][s % 2])  # step s - 2 is done with these inputs
+                b["W"].copy_(W_pin, non_blocking=True)
+                b["sel"].copy_(sel_pin, non_blocking=True)
+                ev["in"][s % 2].record(cs)
 
-    e2e_steps = max(1, min(args.steps, args.e2e_steps))
-    e2e_step()
+        fetch(0)
+        for s in range(steps):
+            b = bufs[s % 2]
+            if s + 1 < steps:
+                fetch(s + 1)
+            main.wait_event(ev["in"][s % 2])
+            if s >= 2:
+                main.wait_event(ev["out"][s % 2])  # step s - 2's outputs have been read out
+            kq.kq_init_codebook(b["W"], b["sel"], b["C0"], ws)
+            kq.kq_fit_codebook(b["W"], b["C0"], T, b["C"], b["idx"], b["counts"], b["objective"], ws)
+            kq.kq_quantize_codebook_6bit(b["C"], b["counts"], 100, b["levels"], b["codes"], None, ws)
+            kq.kq_reconstruct(b["idx"], None, b["codes"], b["levels"], b["Wr"], ws, K=K)
+            ev["used"][s % 2].record(main)
+            with torch.cuda.stream(cs):
+                cs.wait_event(ev["used"][s % 2])
+                for name in outs:
+                    outs[name].copy_(b[name], non_blocking=True)
+                ev["out"][s % 2].record(cs)
+
+    e2e_steps = max(1, args.e2e_steps)
+    e2e_run(1)
+    torch.cuda.synchronize()
     barrier()
     t0 = time.perf_counter()
-    for _ in range(e2e_steps):
-        e2e_step()
+    e2e_run(e2e_steps)
     torch.cuda.synchronize()
     e2e_s = time.perf_counter() - t0
     e2e_value, _ = replica_throughput(1e3 * e2e_s, pairs_per_step, e2e_steps, world, dev)
@@ -394,7 +426,9 @@ def run_kq(args, rank, world, local_rank):
         "gpu_launches": int(launches),
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                 "steps": e2e_steps, "api": "kq_init_codebook + kq_fit_codebook + kq_quantize_codebook_6bit + "
-                                           "kq_reconstruct, pinned host buffers, all outputs copied back"},
+                                           "kq_reconstruct, pinned host buffers, all outputs copied back; "
+                                           "copies on a second stream, overlapped with the neighbouring "
+                                           "steps' compute (two buffer sets)"},
     }
     if clk:
         out["clocks"] = clk
@@ -583,7 +617,7 @@ def main():
     ap.add_argument("--steps", type=int, default=3)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["kq", "reference"], default="kq")
-    ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--e2e-steps", type=int, default=4)
     ap.add_argument("--ref-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--only", choices=["assign", "update", "quantize", "reconstruct", "gradstep", "levelgrad",
