@@ -19,6 +19,11 @@ namespace {
 
 constexpr int32_t KQ_ABI_VERSION = 3;
 constexpr int32_t HINT_ORDER_MIN_K = 4096;  // warm starts in hint order from 16 codeword tiles on
+// Cold assignments with many codeword tiles start from a pilot pass: rows against the
+// first K / COLD_PILOT_DIV codewords (a random sample when the codebook was drawn from
+// the kernels), whose answers then serve as warm-start hints for the full pass.
+constexpr int32_t COLD_PILOT_MIN_K = 16384;
+constexpr int32_t COLD_PILOT_DIV = 16;
 
 inline bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
@@ -105,6 +110,15 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
                      float *dist, int *nb, const Ws &w, int sms, cudaStream_t s, const int32_t *hint_counts = nullptr) {
     if (tc_eligible(n, K, sms)) {
         KQ_TRY(launch_pack_codebook_tc(C, K, w.cpk, w.hdr, s));
+        // A cold start with many tiles: hints from the pilot pass, written into idx
+        // (each row's hint is read before its own answer is written, by the same CTA).
+        if (!hint && K >= COLD_PILOT_MIN_K) {
+            int nbp = 0;
+            KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K / COLD_PILOT_DIV, nullptr, nullptr, idx, nullptr, nullptr, &nbp,
+                                    w.hdr, s));
+            hint = idx;
+            hint_counts = nullptr;
+        }
         // Warm start with many codeword tiles: rows grouped by hint (see
         // kq_assign_tc.cu); the objective's block sums are then taken over the
         // distances in row order, whatever the grouping. With few tiles the four extra

@@ -184,6 +184,25 @@ def test_assign_paths_agree():
     assert np.array_equal(i_w, i_tc) and bits_equal(d_w, d_tc)
 
 
+def test_assign_cold_pilot_path():
+    # K >= 16384 without a hint: a pilot pass against the first K / 16 codewords
+    # seeds the full pass; the answer is the plain argmin all the same (the CUDA-core
+    # kernel, the oracle on sampled rows, and a run warm-started from the answer).
+    n, K = 2 * TC_MIN_N + 123, 16384 + 77
+    W = synth.random_kernels(n, 9, 261, 0.05)
+    C = W[synth.init_selection(n, K, 262)]
+    i0, d0, st, _ = gpu_assign(W, C)
+    assert st == 0
+    i_cc, d_cc = gpu_assign_cuda_cores(W, C)
+    assert np.array_equal(i0, i_cc) and bits_equal(d0, d_cc)
+    rows = np.sort(synth.below(synth.stream_key(263, 9), 2000, n))
+    idx_ref, dist_ref = oracle.assign(W[rows], C, threads=THREADS)
+    assert check_indices(W, C, i0[rows], idx_ref, rows) == 0
+    assert bits_equal(d0[rows], dist_ref)
+    i1, d1, st, _ = gpu_assign(W, C, hint=i0)
+    assert st == 0 and np.array_equal(i1, i0) and bits_equal(d1, d0)
+
+
 def test_assign_hint_order_path():
     # K >= 4096 on the tensor-core path: warm-started rows are processed grouped by
     # hint; the result must be the cold result, whatever the hints (exact, random,
