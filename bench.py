@@ -603,10 +603,19 @@ def run_configs(args):
         ms = e0.elapsed_time(e1) / args.reps
         statuses = [kq.kq_device_status(L["ws"]) for L in layers]
         evals = sum((T + 1) * L["n"] * L["K"] for L in layers)
+        rate = evals / (ms / 1e3)
+        sms = torch.cuda.get_device_properties(dev).multi_processor_count
+        peaks = _peaks()
+        bf16 = float(peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops", 1700.0)))
+        max_mhz = float(peaks.get("sm_max_mhz", 2070.0))
         print(json.dumps({
             "config": wl.name, "layers": len(layers), "kernels": sum(L["n"] for L in layers),
             "codewords": sum(L["K"] for L in layers), "iters": T, "evals": evals, "ms_per_run": ms,
-            "evals_per_s": evals / (ms / 1e3),
+            "evals_per_s": rate,
+            # whole-run figures (init, fit, 6-bit quantisation and recovery all in the time),
+            # so lower bounds for the assignment kernels alone
+            "frac_of_tensor_peak": rate * TC_FLOPS_PER_PAIR / 1e12 / bf16,
+            "direct_form_frac_of_fp32_peak": rate * DIRECT_OPS_PER_PAIR / (sms * FP32_LANES_PER_SM * max_mhz * 1e6),
             "gpu_launches_per_run": (kq.kq_kernel_launches() - launches0) // args.reps,
             "status": max(st for st, _ in statuses), "reps": args.reps}), flush=True)
 

@@ -356,22 +356,25 @@ __global__ void __launch_bounds__(256) pack_codebook_tc_kernel(const float *__re
 
 // Both steps in one CTA, for small codebooks (one launch instead of two).
 constexpr int32_t TC_PACK_ONE_CTA = 2048;
-__global__ void __launch_bounds__(256) pack_codebook_tc_small_kernel(const float *__restrict__ C, int32_t K,
-                                                                     int32_t Kpad, float *__restrict__ Cpk,
-                                                                     Header *hdr) {
-    __shared__ float s_m[8];
+constexpr int TC_PACK_SMALL_THREADS = 1024;
+__global__ void __launch_bounds__(TC_PACK_SMALL_THREADS) pack_codebook_tc_small_kernel(const float *__restrict__ C,
+                                                                                       int32_t K, int32_t Kpad,
+                                                                                       float *__restrict__ Cpk,
+                                                                                       Header *hdr) {
+    constexpr int WARPS = TC_PACK_SMALL_THREADS / 32;
+    __shared__ float s_m[WARPS];
     float m = 0.f;
-    for (int k = threadIdx.x; k < K; k += 256) m = max_bits(m, codeword_norm_ru(C, k));
+    for (int k = threadIdx.x; k < K; k += TC_PACK_SMALL_THREADS) m = max_bits(m, codeword_norm_ru(C, k));
     m = warp_max_bits(m);
     if ((threadIdx.x & 31) == 0) s_m[threadIdx.x >> 5] = m;
     __syncthreads();
     m = s_m[0];
 #pragma unroll
-    for (int w = 1; w < 8; ++w) m = max_bits(m, s_m[w]);
+    for (int w = 1; w < WARPS; ++w) m = max_bits(m, s_m[w]);
     if (threadIdx.x == 0) hdr->cb_craw = __float_as_uint(m);
     const float beta = tc_scale(m);
     float cmax = 0.f, hmax = 0.f, qmax = 0.f;
-    for (int k = threadIdx.x; k < Kpad; k += 256) {
+    for (int k = threadIdx.x; k < Kpad; k += TC_PACK_SMALL_THREADS) {
         float a, b, c;
         pack_codeword_tc(C, K, k, beta, Cpk, hdr, a, b, c);
         cmax = max_bits(cmax, a);
@@ -438,6 +441,36 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
     uint32_t *status = &hdr->status;
     const float beta = tc_scale(__uint_as_float(__ldcg(&hdr->cb_craw)));  // as pack_codebook_tc_kernel
     const float beta2 = beta * beta;
+
+    // ---- barriers first: the producer starts streaming the first codeword tiles
+    // while the epilogue threads set up their rows (the other roles wait for the
+    // barriers only after the CTA barrier below)
+    const int pre = ntiles < TC_STAGES ? ntiles : TC_STAGES;
+    if (tid == 0) {
+        for (int s = 0; s < TC_STAGES; ++s) {
+            mbar_init((uint32_t)__cvta_generic_to_shared(&S.full[s]), 1);
+            mbar_init((uint32_t)__cvta_generic_to_shared(&S.empty[s]), TC_EPI_WARPS);
+        }
+        for (int t = 0; t < TC_RT; ++t) {
+            mbar_init((uint32_t)__cvta_generic_to_shared(&S.tfull[t]), 1);
+            mbar_init((uint32_t)__cvta_generic_to_shared(&S.tempty[t]), TC_EPI_WARPS);
+        }
+        mbar_init((uint32_t)__cvta_generic_to_shared(&S.done), TC_RT);
+        S.abort_flag = 0u;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // initialised barriers -> bulk copies
+        for (int i = 0; i < pre; ++i) {
+            const uint32_t fb = (uint32_t)__cvta_generic_to_shared(&S.full[i]);
+            asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb), "r"(TC_TILE_BYTES)
+                         : "memory");
+            asm volatile(
+                "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                    (uint32_t)__cvta_generic_to_shared(S.b[i])),
+                "l"(reinterpret_cast<const unsigned char *>(Cpk) + (int64_t)i * TC_TILE_BYTES), "r"(TC_TILE_BYTES),
+                "r"(fb)
+                : "memory");
+        }
+    }
 
     // ---- epilogue threads: one kernel in each row tile, one half of every tile
     const bool epi = warp >= TC_EPI_WARP0;
@@ -516,20 +549,7 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
         }
     }
 
-    // ---- barriers and TMEM
-    if (tid == 0) {
-        for (int s = 0; s < TC_STAGES; ++s) {
-            mbar_init((uint32_t)__cvta_generic_to_shared(&S.full[s]), 1);
-            mbar_init((uint32_t)__cvta_generic_to_shared(&S.empty[s]), TC_EPI_WARPS);
-        }
-        for (int t = 0; t < TC_RT; ++t) {
-            mbar_init((uint32_t)__cvta_generic_to_shared(&S.tfull[t]), 1);
-            mbar_init((uint32_t)__cvta_generic_to_shared(&S.tempty[t]), TC_EPI_WARPS);
-        }
-        mbar_init((uint32_t)__cvta_generic_to_shared(&S.done), TC_RT);
-        S.abort_flag = 0u;
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
+    // ---- TMEM
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          (uint32_t)__cvta_generic_to_shared(&S.tmem_base)),
@@ -546,10 +566,9 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
     if (warp == 0) {
         // ---- producer (lane 0)
         if (lane == 0) {
-            for (int i = 0; i < ntiles; ++i) {
+            for (int i = pre; i < ntiles; ++i) {  // tiles 0 .. pre - 1 are on their way
                 const int s = i % TC_STAGES;
-                if (i >= TC_STAGES &&
-                    !mbar_wait((uint32_t)__cvta_generic_to_shared(&S.empty[s]), ((i / TC_STAGES) - 1) & 1, abort_flag,
+                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.empty[s]), ((i / TC_STAGES) - 1) & 1, abort_flag,
                                status))
                     break;
                 const uint32_t fb = (uint32_t)__cvta_generic_to_shared(&S.full[s]);
@@ -768,7 +787,7 @@ cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Heade
     if (e != cudaSuccess) return e;
     const int32_t Kpad = tc_kpad(K);
     if (Kpad <= TC_PACK_ONE_CTA) {
-        pack_codebook_tc_small_kernel<<<1, 256, 0, s>>>(C, K, Kpad, Cpk, hdr);
+        pack_codebook_tc_small_kernel<<<1, TC_PACK_SMALL_THREADS, 0, s>>>(C, K, Kpad, Cpk, hdr);
         count_launch();
         return cudaGetLastError();
     }
