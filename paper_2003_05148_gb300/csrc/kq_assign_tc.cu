@@ -487,22 +487,43 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
         known[t] = -1;
     }
     if (epi) {
+        // Both rows' loads are issued before any of them is used (two dependent
+        // rounds to global memory per thread instead of four): the kernels and their
+        // hints, then the hinted codewords.
+        int64_t row[TC_RT];
+        float xw[TC_RT][D], ch[TC_RT][D];
+        int32_t hv[TC_RT];
+#pragma unroll
+        for (int t = 0; t < TC_RT; ++t) {
+            // slot -> kernel row (rows in the order of a permutation, when given)
+            const int64_t slot = (int64_t)blockIdx.x * TC_ROWS + t * TC_M + r;
+            row[t] = slot < n ? (perm ? (int64_t)__ldg(perm + slot) : slot) : n;
+        }
+#pragma unroll
+        for (int t = 0; t < TC_RT; ++t) {
+#pragma unroll
+            for (int j = 0; j < D; ++j) xw[t][j] = row[t] < n ? W[row[t] * D + j] : 0.f;
+            hv[t] = (hint != nullptr && row[t] < n) ? hint[row[t]] : -1;
+        }
+#pragma unroll
+        for (int t = 0; t < TC_RT; ++t) {
+            const bool hok = (uint32_t)hv[t] < (uint32_t)K;
+#pragma unroll
+            for (int j = 0; j < D; ++j) ch[t][j] = hok ? C[(int64_t)hv[t] * D + j] : 0.f;
+        }
 #pragma unroll
         for (int t = 0; t < TC_RT; ++t) {
             const int rloc = t * TC_M + r;
-            // slot -> kernel row (rows in the order of a permutation, when given)
-            const int64_t slot = (int64_t)blockIdx.x * TC_ROWS + rloc;
-            const int64_t row = slot < n ? (perm ? (int64_t)__ldg(perm + slot) : slot) : n;
             float x[D], xs[D];  // the kernel, and beta times it (exact unless out of range)
 #pragma unroll
             for (int j = 0; j < D; ++j) {
-                x[j] = row < n ? W[row * D + j] : 0.f;
+                x[j] = xw[t][j];
                 xs[j] = beta * x[j];
             }
             bool ok = true;
 #pragma unroll
             for (int j = 0; j < D; ++j) ok &= isfinite(x[j]);
-            if (row < n && !ok && hsel == 0) set_flag(status, KQ_FLAG_NONFINITE);
+            if (row[t] < n && !ok && hsel == 0) set_flag(status, KQ_FLAG_NONFINITE);
             const float cmax = __uint_as_float(__ldcg(&hdr->cb_cmax));  // scaled bounds
             const float hmax = __uint_as_float(__ldcg(&hdr->cb_hmax));
             const float qmax = __uint_as_float(__ldcg(&hdr->cb_qmax));
@@ -522,15 +543,12 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
             rc.k2 = __fmul_ru(TWO_ABS_TC, __fadd_ru(__fadd_ru(cmax, xn), 1.f));
             bool ev = true;
             float tp = 0.f;
-            if (hint != nullptr && row < n) {
-                const int32_t h = hint[row];
-                if ((uint32_t)h < (uint32_t)K) {
-                    const float d = direct_distance(x, C + (int64_t)h * D);
-                    if (d < best[t]) {
-                        best[t] = d;
-                        bi[t] = known[t] = h;
-                        ev = !tc_shift(rc, d, beta2, tp);
-                    }
+            if ((uint32_t)hv[t] < (uint32_t)K) {
+                const float d = direct_distance(x, ch[t]);
+                if (d < best[t]) {
+                    best[t] = d;
+                    bi[t] = known[t] = hv[t];
+                    ev = !tc_shift(rc, d, beta2, tp);
                 }
             }
             every |= (ev ? 1u : 0u) << t;
