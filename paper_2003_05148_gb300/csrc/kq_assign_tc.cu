@@ -427,6 +427,7 @@ struct TcShared {
     RowConst rc[TC_ROWS];    // rare exact path only (registers go to the tile values)
     float pbest[TC_ROWS];    // second half's result per row, merged at the end
     int32_t pidx[TC_ROWS];
+    int32_t prow[TC_ROWS];   // kernel row of each slot (n for a slot without one)
     double wsum[TC_EPI_WARPS / 2][TC_RT];
 };
 
@@ -553,6 +554,7 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
             }
             every |= (ev ? 1u : 0u) << t;
             if (hsel == 0) {  // both halves start from the same state; one writes it
+                S.prow[rloc] = (int32_t)row[t];
 #pragma unroll
                 for (int j = 0; j < D; ++j) S.xs[rloc][j] = x[j];
                 S.rc[rloc] = rc;
@@ -754,8 +756,7 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
 #pragma unroll
         for (int t = 0; t < TC_RT; ++t) {
             const int rloc = t * TC_M + r;
-            const int64_t slot = (int64_t)blockIdx.x * TC_ROWS + rloc;
-            const int64_t row = slot < n ? (perm ? (int64_t)__ldg(perm + slot) : slot) : n;
+            const int64_t row = S.prow[rloc];
             const float ob = S.pbest[rloc];
             const int32_t oi = S.pidx[rloc];
             if (ob < best[t] || (ob == best[t] && oi < bi[t])) {
