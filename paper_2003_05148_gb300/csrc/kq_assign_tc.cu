@@ -95,6 +95,13 @@ namespace kq {
 constexpr int TC_M = 128;                  // rows per MMA (row tile)
 constexpr int TC_RT = 2;                   // row tiles per CTA
 constexpr int TC_ROWS = TC_M * TC_RT;      // kernels per CTA
+// Warm starts with 1024 to 4096 codewords (no global hint order) group a CTA's rows by
+// the 32-codeword chunk of their hint: at most 128 chunks, plus rows without a hint.
+// (With fewer codeword tiles the sort costs more than it saves: 86 vs 91 us at K = 512,
+// n = 262,144; 148 vs 142 us at K = 2048.)
+constexpr int32_t TC_LGROUP_MINK = 1024;
+constexpr int32_t TC_LGROUP_MAXK = 4096;
+constexpr int TC_LBINS = TC_LGROUP_MAXK / 32 + 1;
 constexpr int TC_N = 256;                  // codewords per tile (N of every MMA)
 constexpr int TC_HALF = TC_N / 2;          // codewords of a tile one epilogue thread tests
 constexpr int TC_KD = 32;                  // K of the GEMM in fp16 elements (hi/lo split, see top of file)
@@ -428,8 +435,15 @@ struct TcShared {
     float pbest[TC_ROWS];    // second half's result per row, merged at the end
     int32_t pidx[TC_ROWS];
     int32_t prow[TC_ROWS];   // kernel row of each slot (n for a slot without one)
+    int32_t lslot[TC_ROWS];  // CTA-local grouping: the CTA row (0..255) slot s works on
+    int32_t lhint[TC_ROWS];  // CTA-local grouping: the hint of each CTA row
+    uint32_t lcnt[TC_LBINS];
+    float rowbest[TC_ROWS];  // each CTA row's distance, for the objective's partial sum in row order
     double wsum[TC_EPI_WARPS / 2][TC_RT];
 };
+
+// Named barrier among the 256 epilogue threads (warps 3-10).
+__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
 
 __global__ void __launch_bounds__(TC_THREADS, 1)
 assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict__ C, const float *__restrict__ Cpk,
@@ -487,7 +501,65 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
         bi[t] = 0;
         known[t] = -1;
     }
+    const bool lgroup = hint != nullptr && perm == nullptr && K >= TC_LGROUP_MINK && K <= TC_LGROUP_MAXK;
     if (epi) {
+        const int64_t row0 = (int64_t)blockIdx.x * TC_ROWS;
+        if (lgroup) {
+            // CTA-local grouping (counting sort of the CTA's rows by hint chunk; the
+            // order within a chunk is free): a warp's rows then share a few chunks,
+            // so the exact path for the hints' own columns is entered a few times
+            // per warp instead of in nearly every chunk.
+            if (hsel == 1)
+                for (int b = r; b < TC_LBINS; b += TC_M) S.lcnt[b] = 0u;
+            int32_t hh[TC_RT];
+            if (hsel == 0) {
+#pragma unroll
+                for (int t = 0; t < TC_RT; ++t) {
+                    const int64_t rw = row0 + t * TC_M + r;
+                    hh[t] = rw < n ? hint[rw] : -1;
+                    S.lhint[t * TC_M + r] = hh[t];
+                }
+            }
+            epi_sync();
+            uint32_t pos[TC_RT];
+            int bin[TC_RT];
+            if (hsel == 0) {
+#pragma unroll
+                for (int t = 0; t < TC_RT; ++t) {
+                    bin[t] = (uint32_t)hh[t] < (uint32_t)K ? hh[t] >> 5 : TC_LBINS - 1;
+                    pos[t] = atomicAdd(&S.lcnt[bin[t]], 1u);
+                }
+            }
+            epi_sync();
+            if (warp == TC_EPI_WARP0) {  // exclusive scan of the bin counts, 5 bins per lane
+                uint32_t c[5], tot = 0;
+#pragma unroll
+                for (int u = 0; u < 5; ++u) {
+                    const int b = lane * 5 + u;
+                    c[u] = b < TC_LBINS ? S.lcnt[b] : 0u;
+                    tot += c[u];
+                }
+                uint32_t inc = tot;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const uint32_t y = __shfl_up_sync(0xffffffffu, inc, o);
+                    if (lane >= o) inc += y;
+                }
+                uint32_t base = inc - tot;
+#pragma unroll
+                for (int u = 0; u < 5; ++u) {
+                    const int b = lane * 5 + u;
+                    if (b < TC_LBINS) S.lcnt[b] = base;
+                    base += c[u];
+                }
+            }
+            epi_sync();
+            if (hsel == 0) {
+#pragma unroll
+                for (int t = 0; t < TC_RT; ++t) S.lslot[S.lcnt[bin[t]] + pos[t]] = t * TC_M + r;
+            }
+            epi_sync();
+        }
         // Both rows' loads are issued before any of them is used (two dependent
         // rounds to global memory per thread instead of four): the kernels and their
         // hints, then the hinted codewords.
@@ -496,15 +568,16 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
         int32_t hv[TC_RT];
 #pragma unroll
         for (int t = 0; t < TC_RT; ++t) {
-            // slot -> kernel row (rows in the order of a permutation, when given)
-            const int64_t slot = (int64_t)blockIdx.x * TC_ROWS + t * TC_M + r;
+            // slot -> kernel row (rows in the order of a global or CTA-local grouping, when given)
+            const int loc = lgroup ? S.lslot[t * TC_M + r] : t * TC_M + r;
+            const int64_t slot = row0 + loc;
             row[t] = slot < n ? (perm ? (int64_t)__ldg(perm + slot) : slot) : n;
         }
 #pragma unroll
         for (int t = 0; t < TC_RT; ++t) {
 #pragma unroll
             for (int j = 0; j < D; ++j) xw[t][j] = row[t] < n ? W[row[t] * D + j] : 0.f;
-            hv[t] = (hint != nullptr && row[t] < n) ? hint[row[t]] : -1;
+            hv[t] = (hint != nullptr && row[t] < n) ? (lgroup ? S.lhint[row[t] - row0] : hint[row[t]]) : -1;
         }
 #pragma unroll
         for (int t = 0; t < TC_RT; ++t) {
@@ -763,12 +836,17 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                 best[t] = ob;
                 bi[t] = oi;
             }
-            double sum = 0.0;
             if (row < n) {
                 idx[row] = bi[t];
                 if (dist) dist[row] = best[t];
-                sum = (double)best[t];
             }
+            // the partial sum runs over the CTA's rows in row order whatever the grouping
+            S.rowbest[lgroup ? S.lslot[rloc] : rloc] = row < n ? best[t] : 0.f;
+        }
+        asm volatile("bar.sync 2, 128;" ::: "memory");  // the 128 threads of the first half
+#pragma unroll
+        for (int t = 0; t < TC_RT; ++t) {
+            double sum = (double)S.rowbest[t * TC_M + r];
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
             if (lane == 0) S.wsum[warp - TC_EPI_WARP0][t] = sum;

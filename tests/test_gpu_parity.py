@@ -224,8 +224,10 @@ def test_assign_hint_order_path():
         assert st == 0 and np.array_equal(i1, i0) and bits_equal(d1, d0)
 
 
-def test_fit_hint_order_deterministic_and_chained():
-    n, K = TC_MIN_N + 21000, 4500
+@pytest.mark.parametrize("K", [2000, 4500])
+def test_fit_hint_order_deterministic_and_chained(K):
+    # K = 4500: warm starts grouped by hint across the grid; K = 2000: within each CTA
+    n = TC_MIN_N + 21000
     W = synth.random_kernels(n, 9, 231, 0.05)
     C0 = W[synth.init_selection(n, K, 232)]
     a = _gpu_fit(W, C0, 3)
