@@ -868,13 +868,14 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
 int32_t tc_kpad(int32_t K) { return (K + TC_N - 1) / TC_N * TC_N; }
 
 // Which assignment kernel is faster, from measured costs on GB300: this kernel runs
-// ceil(n / 256) CTAs, one per SM at a time, each ~12K cycles of setup plus ~1024
-// cycles per 256-codeword tile; the split-K CUDA-core kernel takes at least ~50 us
-// at these sizes (e.g. 56 us for n = 4096, K = 1024) and ~1.4e12 pairs/s beyond.
+// ceil(n / 256) CTAs, one per SM at a time, each ~12K cycles of setup and teardown
+// plus ~1000 cycles per 256-codeword tile; the split-K CUDA-core kernel takes at
+// least ~50 us at these sizes (e.g. 56 us for n = 4096, K = 1024) and ~1.4e12
+// pairs/s beyond.
 bool tc_eligible(int64_t n, int32_t K, int num_sms) {
     const double blocks = (double)((n + TC_ROWS - 1) / TC_ROWS);
-    const double waves = (blocks + num_sms - 1) / num_sms;
-    const double tc_us = (12000.0 + 1024.0 * ((K + TC_N - 1) / TC_N) * (double)(int64_t)waves) / 2070.0;
+    const double waves = (double)(int64_t)((blocks + num_sms - 1) / num_sms);
+    const double tc_us = waves * (12000.0 + 1000.0 * ((K + TC_N - 1) / TC_N)) / 2070.0;
     const double cc_us = fmax(50.0, (double)n * K / 1.4e6);
     return n >= (int64_t)TC_ROWS * num_sms || tc_us < cc_us;
 }
