@@ -72,7 +72,7 @@ struct Ws {
     unsigned long long *cq;
     float *cpk;
     float *dist;
-    int32_t *perm, *pcnt;
+    int32_t *perm, *pcnt, *prev;
 };
 
 Ws carve(void *ws, int64_t n, int32_t K) {
@@ -92,16 +92,8 @@ Ws carve(void *ws, int64_t n, int32_t K) {
     w.dist = reinterpret_cast<float *>(b + L.dist);
     w.perm = reinterpret_cast<int32_t *>(b + L.perm);
     w.pcnt = reinterpret_cast<int32_t *>(b + L.pcnt);
+    w.prev = reinterpret_cast<int32_t *>(b + L.prev);
     return w;
-}
-
-// Update step with the scale chosen once per fit from max|W| (exact mode); the
-// finalise leaves the accumulators zeroed again.
-kq_status run_update_exact(const float *W, int64_t n, const int32_t *idx, int32_t K, const float *C_prev,
-                           float *C_next, int32_t *counts, const Ws &w, int sms, cudaStream_t s) {
-    KQ_TRY(launch_accumulate(W, n, idx, K, w.hdr, w.acc, false, sms, s));
-    KQ_TRY(launch_finalize(w.acc, K, w.hdr, C_prev, C_next, counts, s));
-    return KQ_OK;
 }
 
 // One assignment, on the kernel tc_eligible picks. hint_counts: rows per hinted
@@ -151,19 +143,28 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
     KQ_TRY(cudaMemcpyAsync(w.cbuf0, C_init, cbytes, cudaMemcpyDeviceToDevice, s));
     float *cur = w.cbuf0, *nxt = w.cbuf1;
     int nb = 0;
-    // iteration t > 0 starts every row from its previous assignment (warm start)
+    // Assignment t goes to idx when iters - t is even, else to the workspace's other
+    // index buffer, so the final one lands in idx. Iteration t > 0 starts every row
+    // from assignment t - 1 (warm start; the update wrote its cluster sizes), and its
+    // update moves only the rows whose codeword changed (the sums stay in place).
+    auto buf = [&](int32_t t) -> int32_t * { return ((iters - t) & 1) ? w.prev : idx; };
     for (int32_t t = 0; t < iters; ++t) {
-        // from t > 0 the hint is the last assignment, whose counts the update wrote
-        if ((st = run_assign(W, n, cur, K, t > 0 ? idx : nullptr, idx, nullptr, &nb, w, sms, s,
-                             t > 0 ? counts : nullptr)) != KQ_OK)
+        int32_t *out = buf(t);
+        const int32_t *hint = t > 0 ? buf(t - 1) : nullptr;
+        if ((st = run_assign(W, n, cur, K, hint, out, nullptr, &nb, w, sms, s, t > 0 ? counts : nullptr)) !=
+            KQ_OK)
             return st;
         if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
-        if ((st = run_update_exact(W, n, idx, K, cur, nxt, counts, w, sms, s)) != KQ_OK) return st;
+        if (t == 0)
+            KQ_TRY(launch_accumulate(W, n, out, K, w.hdr, w.acc, false, sms, s));
+        else
+            KQ_TRY(launch_accumulate_delta(W, n, hint, out, K, w.hdr, w.acc, sms, s));
+        KQ_TRY(launch_finalize(w.acc, K, w.hdr, cur, nxt, counts, s, true));
         float *tmp = cur;
         cur = nxt;
         nxt = tmp;
     }
-    if ((st = run_assign(W, n, cur, K, iters > 0 ? idx : nullptr, idx, nullptr, &nb, w, sms, s,
+    if ((st = run_assign(W, n, cur, K, iters > 0 ? buf(iters - 1) : nullptr, idx, nullptr, &nb, w, sms, s,
                          iters > 0 ? counts : nullptr)) != KQ_OK)
         return st;
     if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + iters, s));

@@ -42,7 +42,7 @@ struct Header {
 static_assert(sizeof(Header) <= 4096, "header too large");
 
 struct WsLayout {
-    size_t cd, acc, part, blocksum, cbuf0, cbuf1, cp, cq, cpk, dist, perm, pcnt, total;
+    size_t cd, acc, part, blocksum, cbuf0, cbuf1, cp, cq, cpk, dist, perm, pcnt, prev, total;
 };
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -63,6 +63,7 @@ inline WsLayout ws_layout(int64_t n, int32_t K) {
     L.dist = off;     off = align_up(off + (size_t)n * 4, 256);          // distances when the caller keeps none
     L.perm = off;     off = align_up(off + (size_t)n * 4, 256);          // rows in hint order
     L.pcnt = off;     off = align_up(off + (size_t)(K + 1) * 4, 256);    // per-hint counts / cursors
+    L.prev = off;     off = align_up(off + (size_t)n * 4, 256);          // the fit's other assignment buffer
     L.total = off;
     return L;
 }
@@ -288,7 +289,11 @@ cudaError_t launch_update_fallback(const float *W, int64_t n, const int32_t *idx
 cudaError_t launch_histogram(const int32_t *idx, int64_t n, int32_t K, int32_t *counts, uint32_t *status,
                              int num_sms, cudaStream_t s);
 cudaError_t launch_finalize(unsigned long long *acc, int32_t K, const Header *hdr, const float *C_prev,
-                            float *C_next, int32_t *counts, cudaStream_t s);
+                            float *C_next, int32_t *counts, cudaStream_t s, bool keep_sums = false);
+// The fit's update after its first iteration: the exact fixed-point sums of idx_old
+// (held in acc) become those of idx_new by moving only the rows whose codeword changed.
+cudaError_t launch_accumulate_delta(const float *W, int64_t n, const int32_t *idx_old, const int32_t *idx_new,
+                                    int32_t K, Header *hdr, unsigned long long *acc, int num_sms, cudaStream_t s);
 
 // The whole k-means fit in one cooperative launch, for small codebooks (K <= 512).
 bool small_fit_eligible(int64_t n, int32_t K);

@@ -204,12 +204,13 @@ update_fallback_kernel(const float *__restrict__ W, int64_t n, const int32_t *__
 }
 
 // c_k = (sum * 2^-S) / z_k in fp32 (keep C_prev when z_k = 0); clears the
-// accumulator row for the next call. fp32 arithmetic (GB300's fp64 rate is low):
-// sum -> fp32, exact power-of-two scaling, one IEEE division; within ~1.5 ulp of
-// the exact mean.
+// accumulator row for the next call unless the sums are kept (the fit's next update
+// only moves the rows whose codeword changed). fp32 arithmetic (GB300's fp64 rate is
+// low): sum -> fp32, exact power-of-two scaling, one IEEE division; within ~1.5 ulp
+// of the exact mean.
 __global__ void __launch_bounds__(256)
 finalize_kernel(unsigned long long *__restrict__ acc, int32_t K, const Header *hdr, const float *C_prev,
-                float *C_next, int32_t *__restrict__ counts) {
+                float *C_next, int32_t *__restrict__ counts, bool keep) {
     const int k = blockIdx.x * blockDim.x + threadIdx.x;
     if (k >= K) return;
     const int S = __ldcg(&hdr->upd_scale);
@@ -225,9 +226,52 @@ finalize_kernel(unsigned long long *__restrict__ acc, int32_t K, const Header *h
 #pragma unroll
     for (int j = 0; j < D; ++j) C_next[(int64_t)k * D + j] = c[j];
     counts[k] = (int32_t)z;
+    if (keep) return;
     ulonglong2 *a2 = reinterpret_cast<ulonglong2 *>(a);
 #pragma unroll
     for (int w = 0; w < ACC_WORDS / 2; ++w) a2[w] = make_ulonglong2(0ull, 0ull);
+}
+
+// The sums of idx_old (in acc, at the scale in hdr->upd_scale) become those of
+// idx_new: a row whose codeword changed is subtracted from the old codeword's sums
+// and added to the new one's (the same fixed-point values the full accumulation
+// adds, so the result is the full accumulation's, bit for bit; integer arithmetic
+// is exact whatever the order). Rows that kept their codeword cost two index loads.
+__global__ void __launch_bounds__(256)
+accumulate_delta_kernel(const float *__restrict__ W, int64_t n, const int32_t *__restrict__ idx_old,
+                        const int32_t *__restrict__ idx_new, int32_t K, Header *hdr,
+                        unsigned long long *__restrict__ acc) {
+    const int S = __ldcg(&hdr->upd_scale);
+    bool bad = false;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        const int32_t a = __ldcs(idx_old + i), b = __ldcs(idx_new + i);
+        if (a == b) continue;
+        if ((uint32_t)a >= (uint32_t)K || (uint32_t)b >= (uint32_t)K) {
+            bad = true;
+            continue;
+        }
+        unsigned long long *ra = acc + (int64_t)a * ACC_WORDS, *rb = acc + (int64_t)b * ACC_WORDS;
+#pragma unroll
+        for (int j = 0; j < D; ++j) {
+            const unsigned long long q = (unsigned long long)fixed_rn(W[i * D + j], S);
+            atomicAdd(rb + j, q);
+            atomicAdd(ra + j, 0ull - q);
+        }
+        atomicAdd(rb + D, 1ull);
+        atomicAdd(ra + D, ~0ull);  // - 1
+    }
+    if (bad) set_flag(&hdr->status, KQ_FLAG_INDEX_RANGE);
+}
+
+cudaError_t launch_accumulate_delta(const float *W, int64_t n, const int32_t *idx_old, const int32_t *idx_new,
+                                    int32_t K, Header *hdr, unsigned long long *acc, int num_sms, cudaStream_t s) {
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
+    if (blocks < 1) blocks = 1;
+    accumulate_delta_kernel<<<(unsigned)blocks, 256, 0, s>>>(W, n, idx_old, idx_new, K, hdr, acc);
+    count_launch();
+    return cudaGetLastError();
 }
 
 // counts[k] = #{i : idx[i] == k} with integer atomics (order-independent).
@@ -312,8 +356,8 @@ cudaError_t launch_update_fallback(const float *W, int64_t n, const int32_t *idx
 }
 
 cudaError_t launch_finalize(unsigned long long *acc, int32_t K, const Header *hdr, const float *C_prev,
-                            float *C_next, int32_t *counts, cudaStream_t s) {
-    finalize_kernel<<<(K + 255) / 256, 256, 0, s>>>(acc, K, hdr, C_prev, C_next, counts);
+                            float *C_next, int32_t *counts, cudaStream_t s, bool keep_sums) {
+    finalize_kernel<<<(K + 255) / 256, 256, 0, s>>>(acc, K, hdr, C_prev, C_next, counts, keep_sums);
     count_launch();
     return cudaGetLastError();
 }
