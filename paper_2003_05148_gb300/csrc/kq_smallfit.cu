@@ -19,7 +19,8 @@
 namespace kq {
 
 constexpr int SF_THREADS = 256;
-constexpr int SF_ROWS = 4;             // kernels per thread per pass (codebook loads shared)
+constexpr int SF_ROWS = 4;             // kernels per group (codebook loads shared)
+constexpr int SF_SPLIT = 8;            // lanes that share a group's codebook scan
 constexpr int32_t SF_MAX_K = 512;      // codebook pairs in shared memory: 9 x 256 x 8 B = 18 KB
 
 struct SmallFitArgs {
@@ -40,13 +41,19 @@ struct SmallFitArgs {
 
 // One pass of the assignment against the codebook pairs in shared memory; adds the
 // kernels to the sums (accumulate) or only to the counts (final pass), and returns
-// this thread's share of the objective (its distances in row order, fp64).
+// this thread's share of the objective. A group of SF_ROWS kernels is searched by
+// SF_SPLIT consecutive lanes: lane s of the group takes the codeword pairs p with
+// p % SF_SPLIT == s (consecutive lanes read consecutive pairs: no bank conflicts), and
+// the lanes' (distance, index) minima merge lexicographically, so the lowest index
+// wins ties as in one sequential scan. Lane s < SF_ROWS then records kernel s.
 __device__ __forceinline__ double small_fit_assign(const SmallFitArgs &a, const unsigned long long (*cp)[SF_MAX_K / 2],
                                                    int32_t npairs, int S, bool accumulate, bool &nonfinite) {
-    const int64_t nthr = (int64_t)gridDim.x * SF_THREADS;
+    const int lane = threadIdx.x & 31, slice = lane % SF_SPLIT;
+    const unsigned gmask = 0xffu << (lane & ~(SF_SPLIT - 1));  // the group's lanes
+    const int64_t gstride = (int64_t)gridDim.x * (SF_THREADS / SF_SPLIT);
     double part = 0.0;
     // groups of SF_ROWS kernels dealt round-robin over the CTAs, so every CTA has work
-    for (int64_t g = (int64_t)threadIdx.x * gridDim.x + blockIdx.x; g * SF_ROWS < a.n; g += nthr) {
+    for (int64_t g = (int64_t)(threadIdx.x / SF_SPLIT) * gridDim.x + blockIdx.x; g * SF_ROWS < a.n; g += gstride) {
         const int64_t r0 = g * SF_ROWS;
         unsigned long long x2[SF_ROWS][D];
 #pragma unroll
@@ -63,7 +70,7 @@ __device__ __forceinline__ double small_fit_assign(const SmallFitArgs &a, const 
             best[r] = __int_as_float(0x7f800000);
             bi[r] = 0;
         }
-        for (int32_t p = 0; p < npairs; ++p) {
+        for (int32_t p = slice; p < npairs; p += SF_SPLIT) {
             unsigned long long c2[D];
 #pragma unroll
             for (int j = 0; j < D; ++j) c2[j] = cp[j][p];
@@ -89,20 +96,39 @@ __device__ __forceinline__ double small_fit_assign(const SmallFitArgs &a, const 
             }
         }
 #pragma unroll
-        for (int r = 0; r < SF_ROWS; ++r) {
-            if (r0 + r >= a.n) break;
-            a.idx[r0 + r] = bi[r];
-            part += (double)best[r];
-            unsigned long long *row = a.acc + (int64_t)bi[r] * ACC_WORDS;
+        for (int r = 0; r < SF_ROWS; ++r)
+#pragma unroll
+            for (int o = SF_SPLIT / 2; o > 0; o >>= 1) {
+                const float od = __shfl_xor_sync(gmask, best[r], o);
+                const int32_t oi = __shfl_xor_sync(gmask, bi[r], o);
+                if (od < best[r] || (od == best[r] && oi < bi[r])) {
+                    best[r] = od;
+                    bi[r] = oi;
+                }
+            }
+        // lane s < SF_ROWS of the group records kernel r0 + s (static indexing: a select chain)
+        float mb = best[0];
+        int32_t mi = bi[0];
+#pragma unroll
+        for (int r = 1; r < SF_ROWS; ++r)
+            if (slice == r) {
+                mb = best[r];
+                mi = bi[r];
+            }
+        const int64_t row = r0 + slice;
+        if (slice < SF_ROWS && row < a.n) {
+            a.idx[row] = mi;
+            part += (double)mb;
+            unsigned long long *acc = a.acc + (int64_t)mi * ACC_WORDS;
             if (accumulate) {
 #pragma unroll
                 for (int j = 0; j < D; ++j) {
-                    const float v = a.W[(r0 + r) * D + j];  // the row again (L1)
+                    const float v = a.W[row * D + j];  // the row again (L1)
                     nonfinite |= !isfinite(v);
-                    atomicAdd(row + j, (unsigned long long)fixed_rn(v, S));
+                    atomicAdd(acc + j, (unsigned long long)fixed_rn(v, S));
                 }
             }
-            atomicAdd(row + D, 1ull);
+            atomicAdd(acc + D, 1ull);
         }
     }
     return part;
@@ -187,10 +213,9 @@ __global__ void __launch_bounds__(SF_THREADS) small_fit_kernel(SmallFitArgs a) {
     if (__any_sync(0xffffffffu, nonfinite) && (threadIdx.x & 31) == 0) set_flag(&h->status, KQ_FLAG_NONFINITE);
 }
 
-// Up to 2^22 kernel x codeword pairs per iteration: beyond that the brute-force pass
-// has too few rows per thread to fill the SMs and the multi-launch kernels (split-K
-// CUDA-core assign, tensor cores) are faster (VGG-16 conv3_2, 16.8M pairs: 1.80 vs
-// 1.23 ms per 20-iteration fit; conv 64x64, 65,536 pairs: 0.29 vs 0.50 ms).
+// Up to 2^22 kernel x codeword pairs per iteration: beyond that the multi-launch
+// kernels (tensor cores, split-K CUDA-core assign) are faster (VGG-16 conv3_2, 16.8M
+// pairs: 1.57 vs 1.10 ms per 20-iteration fit; conv 64x64, 65,536 pairs: 0.27 vs 0.50 ms).
 bool small_fit_eligible(int64_t n, int32_t K) { return K <= SF_MAX_K && (int64_t)n * K <= (1LL << 22); }
 
 cudaError_t launch_small_fit(const float *W, int64_t n, const float *C0, int32_t K, int32_t iters, float *C_out,
