@@ -479,6 +479,17 @@ def test_quantize_edge_cases(case):
     assert st == 0 and bits_equal(lv_g, lv_r) and np.array_equal(cd_g, cd_r) and it_g == it_r
 
 
+def test_quantize_negative_count_flagged():
+    # a negative count is flagged and treated as 0
+    C = synth.random_kernels(1000, 9, 23, 0.05)
+    counts = synth.random_counts(1000, 24, 40)
+    counts[5] = -3
+    lv_g, cd_g, it_g, st, flags = gpu_quantize(C, counts)
+    lv_r, cd_r, it_r = oracle.level_fit(C, np.maximum(counts, 0))
+    assert st == 5 and flags & kq.FLAG_INDEX_RANGE
+    assert bits_equal(lv_g, lv_r) and np.array_equal(cd_g, cd_r) and it_g == it_r
+
+
 # --------------------------------------------------------------------------- reconstruction
 
 @pytest.mark.parametrize("n,K", [(1, 1), (31, 5), (4096, 16), (100001, 256), (4194304, 65536)])
