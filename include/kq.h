@@ -66,6 +66,9 @@ typedef enum {
 #define KQ_FLAG_CODE_RANGE 0x4u
 #define KQ_FLAG_TIMEOUT 0x8u
 
+/* kq_fit_codebook flags. */
+#define KQ_STOP_ON_STABLE 0x1
+
 /* Human-readable name of a status. Never NULL. */
 const char *kq_status_string(kq_status s);
 
@@ -157,16 +160,25 @@ kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int
  *   W          n x 9 fp32 (device, 16-byte aligned)
  *   C_init     K x 9 fp32 (device); C_out K x 9 fp32 output (device; may equal C_init)
  *   iters      >= 0
- *   flags      must be 0 (reserved)
+ *   flags      0 or KQ_STOP_ON_STABLE: stop iterating once an assignment equals
+ *              the previous one. That is a fixed point of the iteration (the
+ *              update rebuilds the same codebook from the same clusters, bit for
+ *              bit, and every later assignment repeats this one), so the outputs
+ *              are exactly those of all `iters` iterations; the objective entries
+ *              of the skipped steps repeat the last one computed. The call then
+ *              synchronises `stream` once per iteration to read the test.
  *   idx        n int32 output: the final assignment (device)
  *   counts     K int32 output: cluster sizes of the final assignment (device)
  *   objective  iters + 1 fp64 outputs (device) or NULL: Eq. 1 objective per step,
  *              summed in a fixed order (bitwise reproducible)
+ *   iters_run  1 int32 output (host) or NULL: codebook updates performed (iters,
+ *              or fewer when KQ_STOP_ON_STABLE stopped at a fixed point)
  * Every assignment after the first is warm-started from the previous one (see
- * kq_assign's hint). Runs entirely on `stream`; no host synchronisation. */
+ * kq_assign's hint). Without KQ_STOP_ON_STABLE it runs entirely on `stream` with
+ * no host synchronisation. */
 kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_init, int32_t iters, int32_t flags,
-                          float *C_out, int32_t *idx, int32_t *counts, double *objective, void *ws, size_t ws_bytes,
-                          kq_stream_t stream);
+                          float *C_out, int32_t *idx, int32_t *counts, double *objective, int32_t *iters_run,
+                          void *ws, size_t ws_bytes, kq_stream_t stream);
 
 /* Adaptive codebook size, Algorithm 1 with Eq. 3 (Sec. 3.1): a binary search for
  * the smallest codebook that keeps a layer's quality above a target. The paper's

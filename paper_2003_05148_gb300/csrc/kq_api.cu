@@ -17,7 +17,7 @@ void count_launch(int kernels) { g_launches.fetch_add((unsigned long long)kernel
 
 namespace {
 
-constexpr int32_t KQ_ABI_VERSION = 3;
+constexpr int32_t KQ_ABI_VERSION = 4;
 constexpr int32_t HINT_ORDER_MIN_K = 4096;  // warm starts in hint order from 16 codeword tiles on
 // Cold assignments with many codeword tiles start from a pilot pass: rows against the
 // first K / COLD_PILOT_DIV codewords (a random sample when the codebook was drawn from
@@ -133,9 +133,14 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
 // The k-means fit of kq_fit_codebook on carved workspace regions (sized for at
 // least K codewords). objective: iters + 1 device doubles or null; final_obj: one
 // device double receiving the objective of the final assignment, or null.
+// stop_on_stable: after every incremental update, read on the host whether any row
+// changed codeword; if none did, the fit is at a fixed point (the next update would
+// rebuild the same codebook from the same sets, bit for bit, and every later
+// assignment would repeat this one), so the outputs of the remaining iterations are
+// written directly. iters_run (host, nullable): the codebook updates performed.
 kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int32_t iters, float *C_out,
                   int32_t *idx, int32_t *counts, double *objective, double *final_obj, const Ws &w, int sms,
-                  cudaStream_t s) {
+                  cudaStream_t s, bool stop_on_stable = false, int32_t *iters_run = nullptr) {
     const size_t cbytes = (size_t)K * D * sizeof(float);
     kq_status st;
     KQ_TRY(launch_update_prepare(nullptr, K, w.acc, w.hdr, false, s));
@@ -155,10 +160,26 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
             KQ_OK)
             return st;
         if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
-        if (t == 0)
+        if (t == 0) {
             KQ_TRY(launch_accumulate(W, n, out, K, w.hdr, w.acc, false, sms, s));
-        else
+        } else if (!stop_on_stable) {
             KQ_TRY(launch_accumulate_delta(W, n, hint, out, K, w.hdr, w.acc, sms, s));
+        } else {
+            KQ_TRY(cudaMemsetAsync(&w.hdr->fit_moved, 0, sizeof(uint32_t), s));
+            KQ_TRY(launch_accumulate_delta(W, n, hint, out, K, w.hdr, w.acc, sms, s, &w.hdr->fit_moved));
+            uint32_t moved = 1;
+            KQ_TRY(cudaMemcpyAsync(&moved, &w.hdr->fit_moved, sizeof(moved), cudaMemcpyDeviceToHost, s));
+            KQ_TRY(cudaStreamSynchronize(s));
+            if (!moved) {  // assignment t repeats assignment t - 1: C_t is the fixed point
+                if (out != idx) KQ_TRY(cudaMemcpyAsync(idx, out, (size_t)n * sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
+                if (objective) KQ_TRY(launch_fill_objective(objective, t, iters, s));
+                if (final_obj) KQ_TRY(launch_sum_blocks(w.blocksum, nb, final_obj, s));
+                KQ_TRY(launch_histogram(idx, n, K, counts, &w.hdr->status, sms, s));
+                KQ_TRY(cudaMemcpyAsync(C_out, cur, cbytes, cudaMemcpyDeviceToDevice, s));
+                if (iters_run) *iters_run = t;
+                return KQ_OK;
+            }
+        }
         KQ_TRY(launch_finalize(w.acc, K, w.hdr, cur, nxt, counts, s, true));
         float *tmp = cur;
         cur = nxt;
@@ -171,6 +192,7 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
     if (final_obj) KQ_TRY(launch_sum_blocks(w.blocksum, nb, final_obj, s));
     KQ_TRY(launch_histogram(idx, n, K, counts, &w.hdr->status, sms, s));
     KQ_TRY(cudaMemcpyAsync(C_out, cur, cbytes, cudaMemcpyDeviceToDevice, s));
+    if (iters_run) *iters_run = iters;
     return KQ_OK;
 }
 
@@ -269,10 +291,10 @@ kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int
 }
 
 kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_init, int32_t iters, int32_t flags,
-                          float *C_out, int32_t *idx, int32_t *counts, double *objective, void *ws, size_t ws_bytes,
-                          kq_stream_t stream) {
+                          float *C_out, int32_t *idx, int32_t *counts, double *objective, int32_t *iters_run,
+                          void *ws, size_t ws_bytes, kq_stream_t stream) {
     if (!sizes_ok(n, K) || !W || !C_init || !C_out || !idx || !counts) return KQ_ERR_INVALID_ARG;
-    if (iters < 0 || flags != 0) return KQ_ERR_INVALID_ARG;
+    if (iters < 0 || (flags & ~KQ_STOP_ON_STABLE) != 0) return KQ_ERR_INVALID_ARG;
     if (!aligned(W, 16) || !aligned(C_init, 4) || !aligned(C_out, 4) || !aligned(idx, 4) || !aligned(counts, 4) ||
         !aligned(objective, 8))
         return KQ_ERR_ALIGNMENT;
@@ -282,12 +304,22 @@ kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_i
     if ((st = num_sms(&sms)) != KQ_OK) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     const Ws w = carve(ws, n, K);
+    const bool stop = (flags & KQ_STOP_ON_STABLE) != 0;
     if (small_fit_eligible(n, K)) {  // the whole fit in one cooperative launch
         const int nblk = (int)((n + 255) / 256) + MAX_PART_BLOCKS;
-        return cuda_status(launch_small_fit(W, n, C_init, K, iters, C_out, idx, counts, objective, w.acc, w.cbuf0,
-                                            w.cbuf1, w.blocksum, nblk, w.hdr, sms, s));
+        KQ_TRY(launch_small_fit(W, n, C_init, K, iters, C_out, idx, counts, objective, w.acc, w.cbuf0, w.cbuf1,
+                                w.blocksum, nblk, w.hdr, sms, s, stop));
+        if (iters_run && stop) {  // the iteration count is on the device
+            int32_t run = iters;
+            KQ_TRY(cudaMemcpyAsync(&run, &w.hdr->fit_iters, sizeof(run), cudaMemcpyDeviceToHost, s));
+            KQ_TRY(cudaStreamSynchronize(s));
+            *iters_run = run;
+        } else if (iters_run) {
+            *iters_run = iters;
+        }
+        return KQ_OK;
     }
-    return run_fit(W, n, K, C_init, iters, C_out, idx, counts, objective, nullptr, w, sms, s);
+    return run_fit(W, n, K, C_init, iters, C_out, idx, counts, objective, nullptr, w, sms, s, stop, iters_run);
 }
 
 kq_status kq_search_codebook_size(const float *W, int64_t n, const int64_t *sel, int32_t sel_len, double alpha,

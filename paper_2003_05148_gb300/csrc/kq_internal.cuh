@@ -24,17 +24,17 @@ struct Header {
     uint32_t barrier;       // grid-barrier arrival counter (level fit)
     uint32_t abort;         // set when a bounded wait gives up
     uint32_t changed[3];    // level fit: "some code changed" per iteration (triple buffered)
-    uint32_t pad0;
+    uint32_t fit_moved;     // fit (stop on stable): some row changed codeword in the last update
     uint32_t lo_w, lo_a;    // level fit: ordered-int minima over weighted / all scalars (init 0xff..)
     uint32_t hi_w, hi_a;    // level fit: ordered-int maxima over weighted / all scalars (init 0)
     uint32_t maxv_w;        // level fit: max |v| over weighted scalars (fp32 bits)
-    uint32_t pad1;
+    uint32_t fit_moved1;    // one-launch fit (stop on stable): the same for odd iterations
     uint32_t cb_cmax, cb_hmax, cb_qmax;  // assign filter: codebook bounds (fp32 bits, see kq_assign.cu)
     uint32_t cb_craw;       // tensor-core assign: largest codeword norm before scaling (fp32 bits)
     uint32_t upd_bound;     // update: bound B on |W| the fixed-point scale was chosen for (fp32 bits)
     uint32_t upd_violation; // update: a |w| > B was seen (the exact fallback must run)
     int32_t upd_scale;      // update: the scale exponent S the accumulators hold
-    uint32_t pad3;
+    int32_t fit_iters;      // one-launch fit: codebook updates performed
     unsigned long long wtotal;          // level fit: sum of weights
     unsigned long long lacc[3][LEVELS][2];  // level fit: (weight sum, fixed-point sum) per level
     double obj;                         // codebook-size search: objective of the last fit
@@ -292,15 +292,21 @@ cudaError_t launch_finalize(unsigned long long *acc, int32_t K, const Header *hd
                             float *C_next, int32_t *counts, cudaStream_t s, bool keep_sums = false);
 // The fit's update after its first iteration: the exact fixed-point sums of idx_old
 // (held in acc) become those of idx_new by moving only the rows whose codeword changed.
+// moved (nullable): set to 1 when some row's codeword changed.
 cudaError_t launch_accumulate_delta(const float *W, int64_t n, const int32_t *idx_old, const int32_t *idx_new,
-                                    int32_t K, Header *hdr, unsigned long long *acc, int num_sms, cudaStream_t s);
+                                    int32_t K, Header *hdr, unsigned long long *acc, int num_sms, cudaStream_t s,
+                                    uint32_t *moved = nullptr);
+// obj[j] = obj[from] for from < j <= to (the objective of a fit stopped at a fixed point).
+cudaError_t launch_fill_objective(double *obj, int32_t from, int32_t to, cudaStream_t s);
 
 // The whole k-means fit in one cooperative launch, for small codebooks (K <= 512).
 bool small_fit_eligible(int64_t n, int32_t K);
+// stop_on_stable: end at the first assignment equal to the previous one (the
+// outputs are then those of all iters; hdr->fit_iters receives the updates made).
 cudaError_t launch_small_fit(const float *W, int64_t n, const float *C0, int32_t K, int32_t iters, float *C_out,
                              int32_t *idx, int32_t *counts, double *objective, unsigned long long *acc, float *cbuf0,
                              float *cbuf1, double *blocksum, int max_blocksum, Header *hdr, int num_sms,
-                             cudaStream_t s);
+                             cudaStream_t s, bool stop_on_stable = false);
 
 cudaError_t launch_level_fit(const float *C, int64_t N, const int32_t *counts, int32_t max_iters, float *levels,
                              uint8_t *codes, int32_t *iters_run, Header *hdr, int num_sms, cudaStream_t s);

@@ -10,6 +10,9 @@
 //                its codeword; barrier; C_{t+1} = sums / counts (empty keeps C_t),
 //                objective J_t = sum of the distances; barrier;
 //   final        assign against C_T, cluster sizes of that assignment, J_T.
+// With stop_on_stable an assignment equal to the previous one ends the fit early: it
+// is a fixed point (C_{t+1} would be C_t bit for bit), so it is the final assignment,
+// C_t the final codebook and J_t every later objective entry.
 // The distances are the definition's (t_j = fl(x_j - c_j), acc = fma(t_j, t_j, acc),
 // j = 0..8), two codewords at a time with packed fp32x2 arithmetic (each half is the
 // scalar sequence); the sums use the integer conversion and scale of the update
@@ -37,6 +40,7 @@ struct SmallFitArgs {
     float *cbuf0, *cbuf1;     // C_t alternates between the two
     double *blocksum;         // one partial objective per CTA
     Header *hdr;
+    int stop_on_stable;
 };
 
 // One pass of the assignment against the codebook pairs in shared memory; adds the
@@ -47,7 +51,8 @@ struct SmallFitArgs {
 // the lanes' (distance, index) minima merge lexicographically, so the lowest index
 // wins ties as in one sequential scan. Lane s < SF_ROWS then records kernel s.
 __device__ __forceinline__ double small_fit_assign(const SmallFitArgs &a, const unsigned long long (*cp)[SF_MAX_K / 2],
-                                                   int32_t npairs, int S, bool accumulate, bool &nonfinite) {
+                                                   int32_t npairs, int S, bool accumulate, bool &nonfinite,
+                                                   bool compare, bool &moved) {
     const int lane = threadIdx.x & 31, slice = lane % SF_SPLIT;
     const unsigned gmask = 0xffu << (lane & ~(SF_SPLIT - 1));  // the group's lanes
     const int64_t gstride = (int64_t)gridDim.x * (SF_THREADS / SF_SPLIT);
@@ -117,6 +122,7 @@ __device__ __forceinline__ double small_fit_assign(const SmallFitArgs &a, const 
             }
         const int64_t row = r0 + slice;
         if (slice < SF_ROWS && row < a.n) {
+            if (compare) moved |= a.idx[row] != mi;  // the previous assignment, written by this lane
             a.idx[row] = mi;
             part += (double)mb;
             unsigned long long *acc = a.acc + (int64_t)mi * ACC_WORDS;
@@ -152,6 +158,7 @@ __global__ void __launch_bounds__(SF_THREADS) small_fit_kernel(SmallFitArgs a) {
         for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
         if ((threadIdx.x & 31) == 0) atomicMax(&h->maxabs_bits, __float_as_uint(m));
         for (int64_t e = gtid; e < (int64_t)a.K * D; e += nthr) a.cbuf0[e] = a.C0[e];
+        if (gtid == 0) h->fit_moved = h->fit_moved1 = 0u;  // first set after the barrier below
     }
     if (!grid_barrier(h, gridDim.x, epoch)) return;
     const int S = fit_sum_scale(__uint_as_float(__ldcg(&h->maxabs_bits)), a.n);
@@ -170,7 +177,10 @@ __global__ void __launch_bounds__(SF_THREADS) small_fit_kernel(SmallFitArgs a) {
             cp[j][p] = pack2(c0, c1);
         }
         __syncthreads();
-        double part = small_fit_assign(a, cp, npairs, S, !last, nonfinite);
+        bool moved = false;
+        double part = small_fit_assign(a, cp, npairs, S, !last, nonfinite, a.stop_on_stable && t > 0, moved);
+        uint32_t *moved_word = (t & 1) ? &h->fit_moved1 : &h->fit_moved;
+        if (__any_sync(0xffffffffu, moved) && (threadIdx.x & 31) == 0) atomicOr(moved_word, 1u);
         // per-CTA partial of the objective, fixed order
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
@@ -182,13 +192,18 @@ __global__ void __launch_bounds__(SF_THREADS) small_fit_kernel(SmallFitArgs a) {
             a.blocksum[blockIdx.x] = s;
         }
         if (!grid_barrier(h, gridDim.x, epoch)) return;
+        // a fixed point: this assignment is the final one (the same word in every CTA;
+        // the other parity's word was last read before the previous barrier)
+        const bool stable = a.stop_on_stable && t > 0 && !last && __ldcg(moved_word) == 0u;
+        if (gtid == 0) *((t & 1) ? &h->fit_moved : &h->fit_moved1) = 0u;
+        const bool fin = last || stable;
         // C_{t+1} = mean of each set (the update's arithmetic), or the cluster sizes of
         // the final assignment; the accumulators are cleared for the next pass
         float *Cn = (t & 1) ? a.cbuf0 : a.cbuf1;
         for (int64_t k = gtid; k < a.K; k += nthr) {
             unsigned long long *row = a.acc + k * ACC_WORDS;
             const long long z = (long long)__ldcg(row + D);
-            if (!last) {
+            if (!fin) {
                 const float zf = (float)z;
 #pragma unroll
                 for (int j = 0; j < D; ++j) {
@@ -206,9 +221,11 @@ __global__ void __launch_bounds__(SF_THREADS) small_fit_kernel(SmallFitArgs a) {
         if (a.objective && gtid == 0) {
             double s = 0.0;
             for (unsigned b = 0; b < gridDim.x; ++b) s += __ldcg(a.blocksum + b);
-            a.objective[t] = s;
+            for (int32_t u = t; u <= (stable ? a.iters : t); ++u) a.objective[u] = s;
         }
-        if (!last && !grid_barrier(h, gridDim.x, epoch)) return;
+        if (gtid == 0 && fin) h->fit_iters = t;
+        if (fin) break;
+        if (!grid_barrier(h, gridDim.x, epoch)) return;
     }
     if (__any_sync(0xffffffffu, nonfinite) && (threadIdx.x & 31) == 0) set_flag(&h->status, KQ_FLAG_NONFINITE);
 }
@@ -221,7 +238,7 @@ bool small_fit_eligible(int64_t n, int32_t K) { return K <= SF_MAX_K && (int64_t
 cudaError_t launch_small_fit(const float *W, int64_t n, const float *C0, int32_t K, int32_t iters, float *C_out,
                              int32_t *idx, int32_t *counts, double *objective, unsigned long long *acc, float *cbuf0,
                              float *cbuf1, double *blocksum, int max_blocksum, Header *hdr, int num_sms,
-                             cudaStream_t s) {
+                             cudaStream_t s, bool stop_on_stable) {
     cudaError_t e = cudaMemsetAsync(acc, 0, (size_t)K * ACC_WORDS * sizeof(unsigned long long), s);
     if (e != cudaSuccess) return e;
     e = cudaMemsetAsync(&hdr->maxabs_bits, 0, 3 * sizeof(uint32_t), s);  // max|W|, barrier counter, abort word
@@ -235,7 +252,8 @@ cudaError_t launch_small_fit(const float *W, int64_t n, const float *C0, int32_t
     if (blocks > (int64_t)per_sm * num_sms) blocks = (int64_t)per_sm * num_sms;  // co-resident by construction
     if (blocks > max_blocksum) blocks = max_blocksum;
     if (blocks < 1) blocks = 1;
-    SmallFitArgs a{W, n, C0, K, iters, C_out, idx, counts, objective, acc, cbuf0, cbuf1, blocksum, hdr};
+    SmallFitArgs a{W, n, C0, K, iters, C_out, idx, counts, objective, acc, cbuf0, cbuf1, blocksum, hdr,
+                   stop_on_stable ? 1 : 0};
     void *params[] = {&a};
     e = cudaLaunchCooperativeKernel((const void *)small_fit_kernel, dim3((unsigned)blocks), dim3(SF_THREADS), params, 0,
                                     s);

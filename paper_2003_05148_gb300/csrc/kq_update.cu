@@ -240,13 +240,14 @@ finalize_kernel(unsigned long long *__restrict__ acc, int32_t K, const Header *h
 __global__ void __launch_bounds__(256)
 accumulate_delta_kernel(const float *__restrict__ W, int64_t n, const int32_t *__restrict__ idx_old,
                         const int32_t *__restrict__ idx_new, int32_t K, Header *hdr,
-                        unsigned long long *__restrict__ acc) {
+                        unsigned long long *__restrict__ acc, uint32_t *moved) {
     const int S = __ldcg(&hdr->upd_scale);
-    bool bad = false;
+    bool bad = false, any = false;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
         const int32_t a = __ldcs(idx_old + i), b = __ldcs(idx_new + i);
         if (a == b) continue;
+        any = true;
         if ((uint32_t)a >= (uint32_t)K || (uint32_t)b >= (uint32_t)K) {
             bad = true;
             continue;
@@ -262,14 +263,32 @@ accumulate_delta_kernel(const float *__restrict__ W, int64_t n, const int32_t *_
         atomicAdd(ra + D, ~0ull);  // - 1
     }
     if (bad) set_flag(&hdr->status, KQ_FLAG_INDEX_RANGE);
+    if (moved && __any_sync(0xffffffffu, any) && (threadIdx.x & 31) == 0) atomicOr(moved, 1u);
 }
 
 cudaError_t launch_accumulate_delta(const float *W, int64_t n, const int32_t *idx_old, const int32_t *idx_new,
-                                    int32_t K, Header *hdr, unsigned long long *acc, int num_sms, cudaStream_t s) {
+                                    int32_t K, Header *hdr, unsigned long long *acc, int num_sms, cudaStream_t s,
+                                    uint32_t *moved) {
     int64_t blocks = (n + 255) / 256;
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
     if (blocks < 1) blocks = 1;
-    accumulate_delta_kernel<<<(unsigned)blocks, 256, 0, s>>>(W, n, idx_old, idx_new, K, hdr, acc);
+    accumulate_delta_kernel<<<(unsigned)blocks, 256, 0, s>>>(W, n, idx_old, idx_new, K, hdr, acc, moved);
+    count_launch();
+    return cudaGetLastError();
+}
+
+__global__ void __launch_bounds__(256) fill_objective_kernel(double *obj, int32_t from, int32_t to) {
+    const double v = obj[from];
+    for (int64_t j = (int64_t)from + 1 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j <= to;
+         j += (int64_t)gridDim.x * blockDim.x)
+        obj[j] = v;
+}
+
+cudaError_t launch_fill_objective(double *obj, int32_t from, int32_t to, cudaStream_t s) {
+    if (to <= from) return cudaSuccess;
+    int64_t blocks = ((int64_t)to - from + 255) / 256;
+    if (blocks > 1024) blocks = 1024;
+    fill_objective_kernel<<<(unsigned)blocks, 256, 0, s>>>(obj, from, to);
     count_launch();
     return cudaGetLastError();
 }

@@ -20,6 +20,7 @@ KQ_OK = 0
 STATUS_NAMES = {0: "KQ_OK", 1: "KQ_ERR_INVALID_ARG", 2: "KQ_ERR_ALIGNMENT", 3: "KQ_ERR_NONFINITE",
                 4: "KQ_ERR_CUDA", 5: "KQ_ERR_DEVICE_CHECK", 6: "KQ_ERR_WORKSPACE", 7: "KQ_ERR_TIMEOUT"}
 FLAG_NONFINITE, FLAG_INDEX_RANGE, FLAG_CODE_RANGE, FLAG_TIMEOUT = 0x1, 0x2, 0x4, 0x8
+STOP_ON_STABLE = 0x1  # kq_fit_codebook flag
 
 EXPORTS = ["kq_status_string", "kq_abi_version", "kq_kernel_launches", "kq_workspace_bytes", "kq_device_status", "kq_init_codebook",
            "kq_assign", "kq_update_centroids", "kq_fit_codebook", "kq_quantize_codebook_6bit", "kq_reconstruct",
@@ -58,7 +59,7 @@ def lib() -> ctypes.CDLL:
             "kq_init_codebook": ([P, i64, P, i32, P, P, sz, P], ctypes.c_int),
             "kq_assign": ([P, i64, P, i32, P, P, P, P, sz, P], ctypes.c_int),
             "kq_update_centroids": ([P, i64, P, i32, P, P, P, P, sz, P], ctypes.c_int),
-            "kq_fit_codebook": ([P, i64, i32, P, i32, i32, P, P, P, P, P, sz, P], ctypes.c_int),
+            "kq_fit_codebook": ([P, i64, i32, P, i32, i32, P, P, P, P, P, P, sz, P], ctypes.c_int),
             "kq_quantize_codebook_6bit": ([P, i32, P, i32, P, P, P, P, sz, P], ctypes.c_int),
             "kq_reconstruct": ([P, i64, P, i32, P, P, P, P, sz, P], ctypes.c_int),
             "kq_compression_report": ([i64, i32, i32, i32, ctypes.POINTER(Report)], ctypes.c_int),
@@ -158,11 +159,15 @@ def kq_update_centroids(W, idx, C_prev, C_next, counts, ws, stream=None) -> None
         _dev(counts, "counts", torch.int32), _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
 
 
-def kq_fit_codebook(W, C_init, iters, C_out, idx, counts, objective, ws, stream=None, flags: int = 0) -> None:
+def kq_fit_codebook(W, C_init, iters, C_out, idx, counts, objective, ws, stream=None, flags: int = 0) -> int:
+    """Returns the number of codebook updates performed (iters unless STOP_ON_STABLE stopped early)."""
+    run = ctypes.c_int32(0)
     _check("kq_fit_codebook", lib().kq_fit_codebook(
         _dev(W, "W", torch.float32), _rows(W), _rows(C_init), _dev(C_init, "C_init", torch.float32), iters, flags,
         _dev(C_out, "C_out", torch.float32), _dev(idx, "idx", torch.int32), _dev(counts, "counts", torch.int32),
-        _dev(objective, "objective", torch.float64), _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+        _dev(objective, "objective", torch.float64), ctypes.byref(run), _dev(ws, "ws", torch.uint8), ws.numel(),
+        _stream(stream)))
+    return run.value
 
 
 def kq_quantize_codebook_6bit(C, counts, max_iters, levels, codes, iters_run, ws, stream=None) -> None:

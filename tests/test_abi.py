@@ -35,7 +35,7 @@ def test_exports_every_declared_symbol(lib):
 
 
 def test_status_strings_and_version(lib):
-    assert kq.kq_abi_version() == 3
+    assert kq.kq_abi_version() == 4
     for code, name in kq.STATUS_NAMES.items():
         assert kq.kq_status_string(code) == name
     assert kq.kq_status_string(99) == "KQ_ERR_UNKNOWN"
@@ -65,8 +65,9 @@ def test_host_validation_before_any_device_work(lib):
     assert L.kq_assign(good, 1024, good, 16, None, good, None, good, ws_bytes - 1, None) == 6  # too small
     assert L.kq_assign(good, 1024, good, 16, None, good, None, odd, ws_bytes, None) == 2  # ws alignment
     assert L.kq_update_centroids(good, 1024, good, 16, None, good, good, good, ws_bytes, None) == 1
-    assert L.kq_fit_codebook(good, 1024, 16, good, -1, 0, good, good, good, None, good, ws_bytes, None) == 1
-    assert L.kq_fit_codebook(good, 1024, 16, good, 3, 7, good, good, good, None, good, ws_bytes, None) == 1
+    assert L.kq_fit_codebook(good, 1024, 16, good, -1, 0, good, good, good, None, None, good, ws_bytes, None) == 1
+    assert L.kq_fit_codebook(good, 1024, 16, good, 3, 7, good, good, good, None, None, good, ws_bytes, None) == 1
+    assert L.kq_fit_codebook(good, 1024, 16, good, 3, 2, good, good, good, None, None, good, ws_bytes, None) == 1
     assert L.kq_quantize_codebook_6bit(good, 16, good, -1, good, good, None, good, ws_bytes, None) == 1
     assert L.kq_quantize_codebook_6bit(good, 16, good, 10, good, good, None, good, 100, None) == 6
     assert L.kq_reconstruct(good, 1024, None, 16, None, None, good, good, ws_bytes, None) == 1  # nothing to decode
@@ -156,7 +157,7 @@ def test_cuda_failure_returns_status_without_device(lib):
     ws_bytes = kq.kq_workspace_bytes(1024, 16)
     assert L.kq_assign(good, 1024, good, 16, None, good, None, good, ws_bytes, None) == 4
     assert L.kq_update_centroids(good, 1024, good, 16, good, good, good, good, ws_bytes, None) == 4
-    assert L.kq_fit_codebook(good, 1024, 16, good, 3, 0, good, good, good, None, good, ws_bytes, None) == 4
+    assert L.kq_fit_codebook(good, 1024, 16, good, 3, 0, good, good, good, None, None, good, ws_bytes, None) == 4
     assert L.kq_quantize_codebook_6bit(good, 16, good, 10, good, good, None, good, ws_bytes, None) == 4
     assert L.kq_reconstruct(good, 1024, good, 16, None, None, good, good, ws_bytes, None) == 4
     assert L.kq_quantize_reconstruct(good, 1024, good, 16, good, None, good, good, ws_bytes, None) == 4

@@ -407,6 +407,57 @@ def test_fit_stepwise(cfg, li):
     assert np.all(obj_T[1:] <= obj_T[:-1] * (1 + 1e-6))
 
 
+def _gpu_fit_run(W, C0, iters, flags):
+    n, K = W.shape[0], C0.shape[0]
+    C = torch.empty(K, 9, dtype=torch.float32, device=dev())
+    idx = torch.empty(n, dtype=torch.int32, device=dev())
+    counts = torch.empty(K, dtype=torch.int32, device=dev())
+    obj = torch.empty(iters + 1, dtype=torch.float64, device=dev())
+    ws = kq.workspace(n, K, dev())
+    run = kq.kq_fit_codebook(to_dev(W), to_dev(C0), iters, C, idx, counts, obj, ws, flags=flags)
+    st, _ = kq.kq_device_status(ws)
+    assert st == 0
+    return (C.cpu().numpy(), idx.cpu().numpy(), counts.cpu().numpy(), obj.cpu().numpy()), run
+
+
+def _separated(n, P, seed):
+    # n kernels around P well-separated prototypes (noise 1e-3 of their spread): no
+    # near-ties, and Lloyd reaches a fixed point within a few iterations
+    protos = synth.random_kernels(P, 9, seed, 1.0)
+    which = synth.below(synth.stream_key(seed, 5), n, P)
+    return (protos[which] + synth.random_kernels(n, 9, seed + 1, 1e-3)).astype(np.float32)
+
+
+@pytest.mark.parametrize("case", ["one_launch", "tensor_cores", "layer"])
+def test_fit_stop_on_stable(case):
+    if case == "layer":
+        lay, W, C0 = _layer(4, 0)  # ResNet-18 conv 64x64, K = 1024: multi-launch path
+        iters = 30
+    else:
+        n, K = (6000, 64) if case == "one_launch" else (40000, 4096)
+        W = _separated(n, 2 * K, 31 if case == "one_launch" else 32)
+        C0 = W[:K].copy()
+        iters = 40
+    full, run_full = _gpu_fit_run(W, C0, iters, 0)
+    stop, run = _gpu_fit_run(W, C0, iters, kq.STOP_ON_STABLE)
+    # a fixed point repeats itself: every output is that of all iterations, bit for bit
+    assert run_full == iters and 0 <= run <= iters
+    for a, b in zip(full, stop):
+        assert bits_equal(a, b)
+    if case == "layer":
+        return
+    # the oracle's own fixed point: the first assignment equal to the previous one
+    C, prev, t_ref = C0, None, iters
+    for t in range(iters):
+        idx, _ = oracle.assign(W, C, threads=THREADS)
+        if prev is not None and np.array_equal(idx, prev):
+            t_ref = t
+            break
+        C, _ = oracle.update(W, idx, C)
+        prev = idx
+    assert run == t_ref < iters
+
+
 def test_fit_end_to_end_against_oracle():
     lay, W, C0 = _layer(1)
     C_g, idx_g, cnt_g, obj_g = _gpu_fit(W, C0, 10)
