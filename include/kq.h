@@ -328,6 +328,18 @@ typedef struct {
 
 kq_status kq_compression_report(int64_t n, int32_t k, int32_t omega, int32_t b_c, kq_report *out);
 
+/* The seeded draw of K distinct kernel rows that initialises a codebook
+ * (kq_init_codebook's sel; the paper leaves the initialisation open, Sec. 3.1):
+ * a partial Fisher-Yates shuffle of [0, n) whose step j = 0..K-1 swaps position j
+ * with j + (u_j mod (n - j)); out[j] is position j afterwards. u_j is output j of
+ * the SplitMix64 stream (Steele, Lea and Flood, OOPSLA 2014) with key
+ * mix(seed * 0x100000001B3 + 4), output j = mix(key + (j + 1) * 0x9E3779B97F4A7C15),
+ * mix the SplitMix64 finaliser; all arithmetic modulo 2^64.
+ *   n    1 <= n < 2^31;  K  1 <= K <= n
+ *   out  K int64 (host)
+ * Host only (no device work); uses a temporary host map of at most K entries. */
+kq_status kq_seed_indices(int64_t n, int32_t K, uint64_t seed, int64_t *out);
+
 /* Eq. 5 (host only): compression ratio of conventional per-weight quantisation,
  * C_con = n * omega^2 * b_fp / (u * b_1 + n * omega^2 * ceil(log2 u)), with u
  * codebook entries of b_1 bits each and b_fp-bit full-precision weights. */

@@ -5,6 +5,7 @@
 
 #include <atomic>
 #include <cmath>
+#include <unordered_map>
 
 #include "kq_internal.cuh"
 
@@ -194,6 +195,13 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
     KQ_TRY(cudaMemcpyAsync(C_out, cur, cbytes, cudaMemcpyDeviceToDevice, s));
     if (iters_run) *iters_run = iters;
     return KQ_OK;
+}
+
+// SplitMix64 finaliser (Steele, Lea and Flood, OOPSLA 2014).
+uint64_t splitmix_mix(uint64_t z) {
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
 }
 
 int ceil_log2_i64(int64_t k) {
@@ -495,6 +503,32 @@ kq_status kq_quantize_reconstruct(const int32_t *idx, int64_t n, const float *C,
     Ws w = carve(ws, n, K);
     return cuda_status(launch_encode_gather(C, K, levels, codes, w.cq, idx, n, W_out, w.hdr, sms,
                                             reinterpret_cast<cudaStream_t>(stream)));
+}
+
+kq_status kq_seed_indices(int64_t n, int32_t K, uint64_t seed, int64_t *out) {
+    if (!out || n < 1 || n >= (1LL << 31) || K < 1 || (int64_t)K > n) return KQ_ERR_INVALID_ARG;
+    const uint64_t golden = 0x9E3779B97F4A7C15ull;
+    const uint64_t key = splitmix_mix(seed * 0x100000001B3ull + 4u);  // the initial-selection stream
+    // positions below K live in out; the few larger positions a swap touched, in a map
+    std::unordered_map<int64_t, int64_t> far;
+    far.reserve((size_t)K);
+    for (int32_t j = 0; j < K; ++j) out[j] = j;
+    auto get = [&](int64_t p) -> int64_t {
+        if (p < K) return out[p];
+        const auto it = far.find(p);
+        return it == far.end() ? p : it->second;
+    };
+    for (int32_t j = 0; j < K; ++j) {
+        const uint64_t u = splitmix_mix(key + (uint64_t)(j + 1) * golden);
+        const int64_t r = j + (int64_t)(u % (uint64_t)(n - j));
+        const int64_t vj = out[j], vr = get(r);
+        if (r < K)
+            out[r] = vj;
+        else
+            far[r] = vj;
+        out[j] = vr;
+    }
+    return KQ_OK;
 }
 
 kq_status kq_compression_report(int64_t n, int32_t k, int32_t omega, int32_t b_c, kq_report *out) {

@@ -25,7 +25,8 @@ STOP_ON_STABLE = 0x1  # kq_fit_codebook flag
 EXPORTS = ["kq_status_string", "kq_abi_version", "kq_kernel_launches", "kq_workspace_bytes", "kq_device_status", "kq_init_codebook",
            "kq_assign", "kq_update_centroids", "kq_fit_codebook", "kq_quantize_codebook_6bit", "kq_reconstruct",
            "kq_compression_report", "kq_conventional_ratio", "kq_assign_noalloc", "kq_quantize_scalars_6bit",
-           "kq_codebook_grad_step", "kq_levels_grad_step", "kq_search_codebook_size", "kq_quantize_reconstruct"]
+           "kq_codebook_grad_step", "kq_levels_grad_step", "kq_search_codebook_size", "kq_quantize_reconstruct",
+           "kq_seed_indices"]
 
 
 class KQError(RuntimeError):
@@ -63,6 +64,7 @@ def lib() -> ctypes.CDLL:
             "kq_quantize_codebook_6bit": ([P, i32, P, i32, P, P, P, P, sz, P], ctypes.c_int),
             "kq_reconstruct": ([P, i64, P, i32, P, P, P, P, sz, P], ctypes.c_int),
             "kq_compression_report": ([i64, i32, i32, i32, ctypes.POINTER(Report)], ctypes.c_int),
+            "kq_seed_indices": ([i64, i32, ctypes.c_uint64, P], ctypes.c_int),
             "kq_conventional_ratio": ([i64, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
             "kq_assign_noalloc": ([P, i64, P, i32, P, P, P], ctypes.c_int),
             "kq_quantize_scalars_6bit": ([P, i64, i32, P, P, P, P, sz, P], ctypes.c_int),
@@ -234,6 +236,13 @@ def kq_compression_report(n: int, k: int, omega: int = 3, b_c: int = 32) -> dict
     r = Report()
     _check("kq_compression_report", lib().kq_compression_report(n, k, omega, b_c, ctypes.byref(r)))
     return {f: getattr(r, f) for f, _ in Report._fields_}
+
+
+def kq_seed_indices(n: int, K: int, seed: int) -> torch.Tensor:
+    """K distinct row numbers in [0, n) (int64, host): the seeded draw that initialises a codebook."""
+    out = torch.empty(K, dtype=torch.int64)
+    _check("kq_seed_indices", lib().kq_seed_indices(n, K, seed & 0xFFFFFFFFFFFFFFFF, out.data_ptr()))
+    return out
 
 
 def kq_conventional_ratio(n: int, omega: int, u: int, b_1: int, b_fp: int = 32) -> float:

@@ -6,9 +6,11 @@ import os
 import re
 from fractions import Fraction
 
+import numpy as np
 import pytest
 
 import oracle
+import synth
 from paper_2003_05148_gb300 import build, kq
 
 HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "kq.h")
@@ -49,6 +51,25 @@ def test_workspace_bytes_rules(lib):
     a = kq.kq_workspace_bytes(4096, 16)
     b = kq.kq_workspace_bytes(4194304, 65536)
     assert 4096 < a < b and a % 256 == 0 and b % 256 == 0
+
+
+@pytest.mark.parametrize("n,K,seed", [(1, 1, 0), (50, 50, 9), (4096, 16, 1001), (65536, 256, 1202),
+                                     (4194304, 65536, 1502), (2 ** 31 - 1, 300, 2 ** 64 - 1), (10, 3, 12345)])
+def test_seed_indices_match_the_input_generator(lib, n, K, seed):
+    # the library's draw and the seeded input module's are written separately from
+    # the same definition (SplitMix64 stream 4, partial Fisher-Yates)
+    got = kq.kq_seed_indices(n, K, seed).numpy()
+    assert np.array_equal(got, synth.init_selection(n, K, seed))
+    assert len(np.unique(got)) == K and got.min() >= 0 and got.max() < n
+
+
+def test_seed_indices_rejects_bad_sizes(lib):
+    out = (ctypes.c_int64 * 4)()
+    assert lib.kq_seed_indices(0, 1, 1, out) == 1
+    assert lib.kq_seed_indices(3, 4, 1, out) == 1
+    assert lib.kq_seed_indices(2 ** 31, 1, 1, out) == 1
+    assert lib.kq_seed_indices(10, 0, 1, out) == 1
+    assert lib.kq_seed_indices(10, 2, 1, None) == 1
 
 
 def test_host_validation_before_any_device_work(lib):
