@@ -458,6 +458,43 @@ def test_fit_stop_on_stable(case):
     assert run == t_ref < iters
 
 
+def test_layers_on_concurrent_streams_match_sequential():
+    # A network's layers are independent problems: fitted, quantised and recovered on
+    # their own streams with their own workspaces, concurrently, they give the
+    # sequential results bit for bit (one-launch fits, tensor-core and CUDA-core
+    # assigns, cooperative level fits sharing the GPU).
+    picks = [_layer(3, 0), _layer(3, 2), _layer(3, 5), _layer(4, 0)]
+    T = 5
+
+    def run(lay, W, C0, stream):
+        n, K = W.shape[0], C0.shape[0]
+        with torch.cuda.stream(stream):
+            Wd, Cd = to_dev(W), to_dev(C0)
+            o = {"C": torch.empty(K, 9, device=dev()), "idx": torch.empty(n, dtype=torch.int32, device=dev()),
+                 "counts": torch.empty(K, dtype=torch.int32, device=dev()),
+                 "obj": torch.empty(T + 1, dtype=torch.float64, device=dev()),
+                 "levels": torch.empty(64, device=dev()), "codes": torch.empty(K, 9, dtype=torch.uint8, device=dev()),
+                 "Wr": torch.empty(n, 9, device=dev())}
+            ws = kq.workspace(n, K, dev())
+            kq.kq_fit_codebook(Wd, Cd, T, o["C"], o["idx"], o["counts"], o["obj"], ws)
+            kq.kq_quantize_codebook_6bit(o["C"], o["counts"], 100, o["levels"], o["codes"], None, ws)
+            kq.kq_reconstruct(o["idx"], None, o["codes"], o["levels"], o["Wr"], ws, K=K)
+        return o, ws
+
+    seq = []
+    for lay, W, C0 in picks:
+        o, ws = run(lay, W, C0, torch.cuda.current_stream())
+        assert kq.kq_device_status(ws)[0] == 0
+        seq.append({k: v.cpu().numpy() for k, v in o.items()})
+    streams = [torch.cuda.Stream(device=dev()) for _ in picks]
+    conc = [run(lay, W, C0, s) for (lay, W, C0), s in zip(picks, streams)]
+    torch.cuda.synchronize()
+    for (o, ws), ref in zip(conc, seq):
+        assert kq.kq_device_status(ws)[0] == 0
+        for k, v in o.items():
+            assert bits_equal(v.cpu().numpy(), ref[k]), k
+
+
 def test_fit_end_to_end_against_oracle():
     lay, W, C0 = _layer(1)
     C_g, idx_g, cnt_g, obj_g = _gpu_fit(W, C0, 10)
