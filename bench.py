@@ -438,9 +438,12 @@ def run_kq(args, rank, world, local_rank):
         threads = oracle.default_threads()
         C0 = oracle.gather_rows(W_h, sel_h)
         rows, dt = _cpu_sample(W_h, C0, args.ref_seconds, threads)
+        rows1, dt1 = _cpu_sample(W_h, C0, min(args.ref_seconds, 3.0), 1)  # and on one core
         out["cpu_baseline"] = {"value": rows * K / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
                                "sample": f"oracle assign of {rows} seeded rows against all K={K} codewords "
-                                         f"({rows * K:.3g} evals, {dt:.1f} s)"}
+                                         f"({rows * K:.3g} evals, {dt:.1f} s)",
+                               "value_1core": rows1 * K / dt1,
+                               "sample_1core": f"{rows1} rows on one thread ({dt1:.1f} s)"}
     print(json.dumps(out), flush=True)
 
 
