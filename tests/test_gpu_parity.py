@@ -458,6 +458,20 @@ def test_fit_stop_on_stable(case):
     assert run == t_ref < iters
 
 
+@pytest.mark.parametrize("iters", [0, 1, 2])
+@pytest.mark.parametrize("shape", ["one_launch", "multi_launch"])
+def test_fit_stop_on_stable_short_fits(shape, iters):
+    # no assignment can repeat before the second one: the flag changes nothing
+    W = _separated(6000, 128, 33) if shape == "one_launch" else _separated(20000, 1024, 34)
+    K = 64 if shape == "one_launch" else 1024
+    C0 = W[:K].copy()
+    full, run_full = _gpu_fit_run(W, C0, iters, 0)
+    stop, run = _gpu_fit_run(W, C0, iters, kq.STOP_ON_STABLE)
+    assert run_full == iters and run == iters
+    for a, b in zip(full, stop):
+        assert bits_equal(a, b)
+
+
 def test_layers_on_concurrent_streams_match_sequential():
     # A network's layers are independent problems: fitted, quantised and recovered on
     # their own streams with their own workspaces, concurrently, they give the
