@@ -511,7 +511,7 @@ kq_status kq_seed_indices(int64_t n, int32_t K, uint64_t seed, int64_t *out) {
     const uint64_t key = splitmix_mix(seed * 0x100000001B3ull + 4u);  // the initial-selection stream
     // positions below K live in out; the few larger positions a swap touched, in a map
     std::unordered_map<int64_t, int64_t> far;
-    far.reserve((size_t)K);
+    far.reserve((size_t)(n - K < K ? n - K : K));  // at most one entry per step, none past n
     for (int32_t j = 0; j < K; ++j) out[j] = j;
     auto get = [&](int64_t p) -> int64_t {
         if (p < K) return out[p];
