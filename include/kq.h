@@ -17,13 +17,16 @@
  *   K rows of 9 floats. Indices are int32, counts int32, codes uint8 (one 6-bit
  *   code per byte, values 0..63), levels 64 floats.
  * - Memory. Every pointer except those documented as host pointers is device
- *   memory owned by the caller. The library allocates nothing and frees nothing.
+ *   memory owned by the caller. The library allocates no device memory (the
+ *   host-only kq_seed_indices uses a temporary host map).
  *   Scratch lives in a caller-allocated workspace of kq_workspace_bytes(n, K)
  *   bytes (256-byte aligned), which must be zero-filled once before its first
  *   use (e.g. torch.zeros); the library keeps it consistent afterwards. One
  *   workspace must not be used by two calls that can run at the same time.
  * - Streams. Work is enqueued on the given stream and the call returns without
- *   waiting for it (except kq_device_status, which synchronises the stream).
+ *   waiting for it, except where a call documents otherwise: kq_device_status,
+ *   kq_search_codebook_size (host decisions between trial fits) and
+ *   kq_fit_codebook with KQ_STOP_ON_STABLE synchronise the stream.
  * - Errors. Arguments are validated on the host before anything is enqueued; a
  *   bad argument returns a status and enqueues nothing. Problems that only the
  *   device can see (a non-finite input, an index or code out of range, a bounded
