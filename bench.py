@@ -1,17 +1,19 @@
 """Benchmark of the KQ hot path on GB300: kernel x codeword distance evals/s.
 
 One step = one pass of the whole hot path over the 2048x2048 stress layer
-(n = 4,194,304 kernels, K = 65,536 codewords, 10 Lloyd iterations):
-codebook init from seeded kernels, 10 x (assign + centroid update), final assign,
-cluster sizes, 6-bit codebook quantisation, K+C reconstruction of the weights.
-The metric counts (iters + 1) * n * K distance evaluations per step.
+(n = 4,194,304 kernels, K = 65,536 codewords, 10 Lloyd iterations) through the
+entry points a user calls: kq_init_codebook (codebook from seeded kernels),
+kq_fit_codebook (10 x (assignment + centroid update), the final assignment and
+its cluster sizes), kq_quantize_codebook_6bit, kq_reconstruct (K+C). The metric
+counts (iters + 1) * n * K distance evaluations per step.
 
 Default (impl "kq"): the CUDA path through the C ABI, inputs resident in HBM
 (the 151 MB weight matrix is larger than the 129 MB L2, so no flush is needed),
-timed with CUDA events on the launching stream. "e2e" re-times the step through
-kq_fit_codebook with the weights coming from pinned host memory and every output
-copied back. --impl reference times the CPU oracle on a bounded row sample of
-the same workload on the host cores.
+timed with CUDA events on the launching stream; a kernel trace (kq_trace_*)
+times every kernel of the timed steps on its stream, from which the rooflines
+come. "e2e" re-times the same calls with the weights coming from pinned host
+memory and every output copied back. --impl reference times the CPU oracle on a
+bounded row sample of the same workload on the host cores.
 
 Multi-GPU (torchrun): the path does not shard here, so every rank runs an
 independent replica; value = all ranks' evals / max-over-ranks time.
@@ -38,12 +40,10 @@ METRIC = "kernel x codeword distance evals/s per Lloyd iteration"
 UNIT = "evals/s"
 SM_COUNT_NOMINAL = 152
 FP32_LANES_PER_SM = 128
-OPS_PER_PAIR = 9  # FP32-pipe lane ops per pair executed by the assign kernel: the 9 FFMA of its certified test
 DIRECT_OPS_PER_PAIR = 18  # the fp32 direct form: 9 FSUB + 9 FFMA
-# Tensor-core assign: the certified test is an (n x 32) . (32 x K) split-fp16 GEMM, 2 * 32 flops per pair.
-TC_FLOPS_PER_PAIR = 64
-TC_ROWS_PER_CTA = 256  # the library takes the tensor-core kernel when n >= 256 * SMs
-F16_FLOPS_PER_CLK_SM = 8192  # dense fp16 / bf16 tensor rate per SM per clock
+METHOD_FLOPS_PER_PAIR = 18  # the contraction of Eq. 1's distance: the 9-term dot product x . c
+# What the tensor-core assign executes per pair: an (n x 32) . (32 x K) split-fp16 GEMM, 2 * 32 flops.
+GEMM_FLOPS_PER_PAIR = 64
 WORKLOAD_CFG = 5
 
 
@@ -202,6 +202,21 @@ def run_reference(args, rank, world):
     print(json.dumps(out), flush=True)
 
 
+def _trace_summary(trace, steps):
+    """Per kernel: launches, total device ms and share of the traced time."""
+    tot = sum(ms for _, ms in trace) or 1.0
+    out = {}
+    for name, ms in trace:
+        d = out.setdefault(name, {"launches": 0, "ms_total": 0.0})
+        d["launches"] += 1
+        d["ms_total"] += ms
+    for d in out.values():
+        d["share"] = round(d["ms_total"] / tot, 5)
+        d["ms_per_step"] = round(d["ms_total"] / steps, 4)
+        d["ms_total"] = round(d["ms_total"], 4)
+    return dict(sorted(out.items(), key=lambda kv: -kv[1]["ms_total"]))
+
+
 def run_kq(args, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -220,45 +235,35 @@ def run_kq(args, rank, world, local_rank):
     W = torch.from_numpy(W_h).to(dev)
     sel = torch.from_numpy(sel_h).to(dev)
     ws = kq.workspace(n, K, dev)
-    Ca = torch.empty(K, 9, dtype=torch.float32, device=dev)
-    Cb = torch.empty_like(Ca)
+    C0 = torch.empty(K, 9, dtype=torch.float32, device=dev)
+    C = torch.empty_like(C0)
     idx = torch.empty(n, dtype=torch.int32, device=dev)
     counts = torch.empty(K, dtype=torch.int32, device=dev)
+    obj = torch.empty(T + 1, dtype=torch.float64, device=dev)
     levels = torch.empty(64, dtype=torch.float32, device=dev)
     codes = torch.empty(K, 9, dtype=torch.uint8, device=dev)
     Wr = torch.empty_like(W)
-    n_assign = T + 1
 
     def pair():
         return (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
 
-    def new_events():
-        return {"assign": [pair() for _ in range(n_assign)], "update": [pair() for _ in range(n_assign)],
-                "reconstruct": [pair()]}
+    def step(rec=None):
+        """One pass of the hot path through the entry points a user calls: codebook
+        init, the k-means fit (T updates and the final assignment), 6-bit codebook
+        quantisation, K+C recovery. `rec` brackets the recovery call."""
+        kq.kq_init_codebook(W, sel, C0, ws)
+        kq.kq_fit_codebook(W, C0, T, C, idx, counts, obj, ws)
+        kq.kq_quantize_codebook_6bit(C, counts, 100, levels, codes, None, ws)
+        if rec:
+            rec[0].record(stream)
+        kq.kq_reconstruct(idx, None, codes, levels, Wr, ws, K=K)
+        if rec:
+            rec[1].record(stream)
 
-    def timed(ev, name, i, fn):
-        if ev:
-            ev[name][i][0].record(stream)
-        fn()
-        if ev:
-            ev[name][i][1].record(stream)
-
-    def step(ev=None):
-        """One pass of the hot path through the public entry points; `ev` brackets the calls."""
-        kq.kq_init_codebook(W, sel, Ca, ws)
-        cur, nxt = Ca, Cb
-        for t in range(T + 1):
-            # iterations after the first start from the previous assignment (as kq_fit_codebook does)
-            timed(ev, "assign", t, lambda: kq.kq_assign(W, cur, idx, None, ws, hint=idx if t > 0 else None))
-            # after the last assignment the update gives the cluster sizes the quantiser weighs by
-            timed(ev, "update", t, lambda: kq.kq_update_centroids(W, idx, cur, nxt, counts, ws))
-            if t < T:
-                cur, nxt = nxt, cur
-        kq.kq_quantize_codebook_6bit(cur, counts, 100, levels, codes, None, ws)
-        timed(ev, "reconstruct", 0, lambda: kq.kq_reconstruct(idx, None, codes, levels, Wr, ws, K=K))
-
+    l0 = kq.kq_kernel_launches()
     for _ in range(args.warmup):
         step()
+    per_step_launches = (kq.kq_kernel_launches() - l0) // max(1, args.warmup)
     st, flags = kq.kq_device_status(ws)
     if st != 0:
         raise RuntimeError(f"device status {st} flags {flags:#x} after warm-up")
@@ -268,28 +273,43 @@ def run_kq(args, rank, world, local_rank):
             dist.barrier()
         torch.cuda.synchronize()
 
-    evs = [new_events() for _ in range(args.steps)]
+    recs = [pair() for _ in range(args.steps)]
+    # every kernel of the timed steps gets a pair of events on its launch stream
+    kq.kq_trace_start(per_step_launches * args.steps + 64)
     launches0 = kq.kq_kernel_launches()
     barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(_smi_id(dev)) as clocks:
         e0.record(stream)
         for s in range(args.steps):
-            step(evs[s])
+            step(recs[s])
         e1.record(stream)
         barrier()
+    kq.kq_trace_stop()
     launches = kq.kq_kernel_launches() - launches0
     ms_total = e0.elapsed_time(e1)
-    call_ms = {name: [a.elapsed_time(b) for ev in evs for a, b in ev[name]] for name in evs[0]}
-    assign_ms = call_ms["assign"]
-    pairs_per_step = n_assign * n * K
+    trace = kq.kq_trace_read()
+    rec_ms = [a.elapsed_time(b) for a, b in recs]
+    pairs_per_step = (T + 1) * n * K
     value, ms_max = replica_throughput(ms_total, pairs_per_step, args.steps, world, dev)
 
     st, flags = kq.kq_device_status(ws)
     if st != 0:
         raise RuntimeError(f"device status {st} flags {flags:#x} after the timed steps")
 
-    # ---- end to end through kq_fit_codebook: pinned host in, every output back ----
+    # the standalone update call (every row accumulated: the step of Eq. 1 as defined),
+    # on the fit's final assignment, for its HBM roofline
+    Cn = torch.empty_like(C)
+    cnt2 = torch.empty_like(counts)
+    upd = [pair() for _ in range(args.update_reps)]
+    for a, b in upd:
+        a.record(stream)
+        kq.kq_update_centroids(W, idx, C, Cn, cnt2, ws)
+        b.record(stream)
+    torch.cuda.synchronize()
+    upd_ms = [a.elapsed_time(b) for a, b in upd]
+
+    # ---- end to end through the same calls: pinned host in, every output back ----
     W_pin = torch.from_numpy(W_h).pin_memory()
     sel_pin = torch.from_numpy(sel_h).pin_memory()
     outs = {"C": torch.empty(K, 9, dtype=torch.float32).pin_memory(),
@@ -346,7 +366,7 @@ def run_kq(args, rank, world, local_rank):
                     outs[name].copy_(b[name], non_blocking=True)
                 ev["out"][s % 2].record(cs)
 
-    e2e_steps = max(1, args.e2e_steps)
+    e2e_steps = args.e2e_steps if args.e2e_steps > 0 else args.steps
     e2e_run(1)
     torch.cuda.synchronize()
     barrier()
@@ -357,6 +377,9 @@ def run_kq(args, rank, world, local_rank):
     e2e_value, _ = replica_throughput(1e3 * e2e_s, pairs_per_step, e2e_steps, world, dev)
     h2d = W_pin.numel() * 4 + sel_pin.numel() * 8
     d2h = sum(t.numel() * t.element_size() for t in outs.values())
+    # the e2e fit must give what the device-timed one gave (same inputs, deterministic)
+    if not (torch.equal(outs["idx"], idx.cpu()) and torch.equal(outs["Wr"], Wr.cpu())):
+        raise RuntimeError("end-to-end outputs differ from the device-timed step's")
 
     if rank != 0:
         return
@@ -364,39 +387,52 @@ def run_kq(args, rank, world, local_rank):
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     clk = clocks.summary()
     max_mhz = float(peaks.get("sm_max_mhz", 2070.0))
-    peak_tops = sms * FP32_LANES_PER_SM * max_mhz * 1e6 / 1e12
-    t_assign = statistics.mean(assign_ms) / 1e3
+    fp32_peak = sms * FP32_LANES_PER_SM * max_mhz * 1e6 / 1e12
     traffic = _ncu_traffic()
-    if n >= TC_ROWS_PER_CTA * sms:
+    kernels = _trace_summary(trace, args.steps)
+    tc_ms = [ms for name, ms in trace if name == "assign_tc_kernel"]
+    cc_ms = [ms for name, ms in trace if name == "assign_kernel"]
+    if tc_ms:
         # kernel timed inside a long step: the sustained bf16 figure (fp16 runs at the bf16 rate)
         bf16 = float(peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops", 1700.0)))
-        peak = bf16
-        achieved = TC_FLOPS_PER_PAIR * n * K / t_assign / 1e12
-        roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
-                    "traffic": traffic.get("assign_tc_kernel"), "kernel": "assign_tc_kernel",
-                    "peak_basis": f"measured cuBLAS bf16 sustained {bf16:.1f} TFLOP/s (dense fp16 and bf16 share "
-                                  f"one rate); flops = {TC_FLOPS_PER_PAIR} per pair (the split-fp16 GEMM of the "
-                                  f"certified test, K = 32 fp16 per row, fp32 accumulation); the exact fp32 "
-                                  f"re-evaluations of the few candidate pairs run on the CUDA cores and are not counted",
-                    "frac_of_burst": achieved / float(peaks.get("bf16_tflops", bf16)),
-                    "peak_at_max_clock": sms * F16_FLOPS_PER_CLK_SM * max_mhz * 1e6 / 1e12,
-                    "assign_ms_mean": 1e3 * t_assign, "assign_launches": len(assign_ms)}
-        roofline["frac_of_peak_at_max_clock"] = achieved / roofline["peak_at_max_clock"]
+        per_step = len(tc_ms) // args.steps
+        pilots = per_step - (T + 1)  # the cold first assignment's pilot pass (K / 16 codewords)
+        full = [ms for i, ms in enumerate(tc_ms) if i % per_step >= pilots]
+        t_step = sum(tc_ms) / args.steps / 1e3  # s of tensor-core assign per step, pilot included
+        achieved = METHOD_FLOPS_PER_PAIR * pairs_per_step / t_step / 1e12
+        gemm_pairs = n * (K * (T + 1) + pilots * (K // 16))
+        gemm = GEMM_FLOPS_PER_PAIR * gemm_pairs / t_step / 1e12
+        roofline = {
+            "bound": "tensor", "achieved": achieved, "peak": bf16, "unit": "TFLOP/s", "frac": achieved / bf16,
+            "traffic": traffic.get("assign_tc_kernel"), "kernel": "assign_tc_kernel",
+            "work": f"{METHOD_FLOPS_PER_PAIR} flops per kernel x codeword pair (the 9-term dot product x . c of "
+                    f"Eq. 1's distance), (T + 1) n K = {pairs_per_step:.4g} pairs per step, over the device time "
+                    f"of every assign_tc_kernel launch of the step (the cold pass's pilot included)",
+            "peak_basis": f"measured cuBLAS bf16 sustained {bf16:.1f} TFLOP/s (of measured; dense fp16 and bf16 "
+                          f"share one rate); the kernel is timed inside the long step",
+            "launches": len(tc_ms), "ms_mean": statistics.mean(tc_ms),
+            "ms_mean_full_pass": statistics.mean(full), "ms_mean_pilot": statistics.mean(
+                [ms for i, ms in enumerate(tc_ms) if i % per_step < pilots]) if pilots > 0 else None,
+            "frac_of_burst": achieved / float(peaks.get("bf16_tflops", bf16)),
+            "gemm": {"flops_per_pair": GEMM_FLOPS_PER_PAIR, "achieved": gemm, "frac_of_peak": gemm / bf16,
+                     "overhead_vs_method": GEMM_FLOPS_PER_PAIR / METHOD_FLOPS_PER_PAIR,
+                     "note": "what the tensor core executes: the split-fp16 test GEMM, K = 32 fp16 per row "
+                             "(three cross terms of the hi/lo split plus the threshold slots; 27 of 32 used), "
+                             "pilot pairs included; the exact fp32 re-evaluations of candidate pairs run on the "
+                             "CUDA cores and are not counted"},
+        }
     else:
-        achieved = OPS_PER_PAIR * n * K / t_assign / 1e12
-        roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tops, "unit": "Tops/s",
-                    "frac": achieved / peak_tops, "traffic": traffic.get("assign_kernel"), "kernel": "assign_kernel",
-                    "peak_basis": f"{sms} SMs x {FP32_LANES_PER_SM} FP32 lanes x {max_mhz:.0f} MHz (max SM clock); "
-                                  f"op = one FP32-pipe lane op; {OPS_PER_PAIR} per pair (the FFMA of the certified "
-                                  f"expanded-form test every pair gets; the exact re-evaluations of the few "
-                                  f"candidate pairs are not counted)",
-                    "assign_ms_mean": 1e3 * t_assign, "assign_launches": len(assign_ms)}
-        if clk:
-            roofline["frac_at_sampled_clock"] = achieved / (sms * FP32_LANES_PER_SM * clk["sm_mhz"] * 1e6 / 1e12)
-    roofline["direct_form_equivalent"] = {"achieved_tops": DIRECT_OPS_PER_PAIR * n * K / t_assign / 1e12,
-                                          "frac_of_fp32_peak": DIRECT_OPS_PER_PAIR * n * K / t_assign / 1e12 / peak_tops,
-                                          "note": "18 FP32 ops/pair: the rate a direct-form CUDA-core kernel "
-                                                  "would need for the same time"}
+        t_step = sum(cc_ms) / args.steps / 1e3
+        achieved = DIRECT_OPS_PER_PAIR * pairs_per_step / t_step / 1e12
+        roofline = {"bound": "alu", "achieved": achieved, "peak": fp32_peak, "unit": "Tops/s",
+                    "frac": achieved / fp32_peak, "traffic": traffic.get("assign_kernel"), "kernel": "assign_kernel",
+                    "peak_basis": f"{sms} SMs x {FP32_LANES_PER_SM} FP32 lanes x {max_mhz:.0f} MHz",
+                    "launches": len(cc_ms)}
+    roofline["direct_form_equivalent"] = {
+        "achieved_tops": DIRECT_OPS_PER_PAIR * pairs_per_step / t_step / 1e12,
+        "frac_of_fp32_peak": DIRECT_OPS_PER_PAIR * pairs_per_step / t_step / 1e12 / fp32_peak,
+        "note": "18 FP32 lane ops per pair (9 FSUB + 9 FFMA): the rate a direct-form CUDA-core kernel would "
+                f"need for the same time, against {sms} x {FP32_LANES_PER_SM} lanes x {max_mhz:.0f} MHz"}
     hbm = float(peaks.get("hbm_gbs", 6776.3))
 
     def hbm_roofline(kernel, bytes_per_call, ms_list, note):
@@ -408,27 +444,31 @@ def run_kq(args, rank, world, local_rank):
 
     upd_bytes = n * (36 + 4) + K * (36 + 36 + 4)
     rec_bytes = n * (4 + 36) + 9 * K + 256
-    roofline_update = hbm_roofline("accumulate_kernel", upd_bytes, call_ms["update"],
-                                   "whole kq_update_centroids call (prepare + accumulate + fallback check + finalize)")
-    roofline_reconstruct = hbm_roofline("gather_codes_kernel", rec_bytes, call_ms["reconstruct"],
-                                        "whole kq_reconstruct call, K+C (decode codes + gather)")
+    roofline_update = hbm_roofline("accumulate_kernel", upd_bytes, upd_ms,
+                                   "standalone kq_update_centroids calls (prepare + accumulate + fallback check + "
+                                   "finalize) on the fit's final assignment, after the timed steps; inside the fit "
+                                   "the update moves only the rows whose codeword changed (see kernels)")
+    roofline_reconstruct = hbm_roofline("gather_codes_kernel", rec_bytes, rec_ms,
+                                        "whole kq_reconstruct call of every timed step, K+C (decode codes + gather)")
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms_max / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "f32", "data": "synthetic",
         "config": {"workload": "stress_2048x2048_K65536_T10", "n": n, "K": K, "iters": T,
-                   "step": "init + 10x(assign+update) + assign + counts + 6-bit quantize + K+C reconstruct",
+                   "step": "kq_init_codebook + kq_fit_codebook (10 updates, final assignment, counts) + "
+                           "kq_quantize_codebook_6bit + kq_reconstruct (K+C)",
                    "l2": "inputs larger than L2 (W is 151 MB, L2 129 MB): no flush",
                    "parallelism": f"replicas x{world}"},
         "roofline": roofline,
         "roofline_update": roofline_update,
         "roofline_reconstruct": roofline_reconstruct,
+        "kernels": kernels,
         "gpu_launches": int(launches),
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                 "steps": e2e_steps, "api": "kq_init_codebook + kq_fit_codebook + kq_quantize_codebook_6bit + "
                                            "kq_reconstruct, pinned host buffers, all outputs copied back; "
                                            "copies on a second stream, overlapped with the neighbouring "
-                                           "steps' compute (two buffer sets)"},
+                                           "steps' compute (two buffer sets); host clock"},
     }
     if clk:
         out["clocks"] = clk
@@ -436,12 +476,12 @@ def run_kq(args, rank, world, local_rank):
         import oracle
 
         threads = oracle.default_threads()
-        C0 = oracle.gather_rows(W_h, sel_h)
-        rows, dt = _cpu_sample(W_h, C0, args.ref_seconds, threads)
-        rows1, dt1 = _cpu_sample(W_h, C0, min(args.ref_seconds, 3.0), 1)  # and on one core
+        C0_h = oracle.gather_rows(W_h, sel_h)
+        rows, dt = _cpu_sample(W_h, C0_h, args.ref_seconds, threads)
+        rows1, dt1 = _cpu_sample(W_h, C0_h, min(args.ref_seconds, 3.0), 1)  # and on one core
         out["cpu_baseline"] = {"value": rows * K / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
-                               "sample": f"oracle assign of {rows} seeded rows against all K={K} codewords "
-                                         f"({rows * K:.3g} evals, {dt:.1f} s)",
+                               "sample": f"oracle assign (the step holding ~all of the work) of {rows} seeded rows "
+                                         f"against all K={K} codewords ({rows * K:.3g} evals, {dt:.1f} s)",
                                "value_1core": rows1 * K / dt1,
                                "sample_1core": f"{rows1} rows on one thread ({dt1:.1f} s)"}
     print(json.dumps(out), flush=True)
@@ -627,7 +667,7 @@ def run_configs(args):
             "evals_per_s": rate,
             # whole-run figures (init, fit, 6-bit quantisation and recovery all in the time),
             # so lower bounds for the assignment kernels alone
-            "frac_of_tensor_peak": rate * TC_FLOPS_PER_PAIR / 1e12 / bf16,
+            "frac_of_tensor_peak": rate * METHOD_FLOPS_PER_PAIR / 1e12 / bf16,
             "direct_form_frac_of_fp32_peak": rate * DIRECT_OPS_PER_PAIR / (sms * FP32_LANES_PER_SM * max_mhz * 1e6),
             "gpu_launches_per_run": (kq.kq_kernel_launches() - launches0) // args.reps,
             "status": max(st for st, _ in statuses), "reps": args.reps, "streams": len(side)}), flush=True)
@@ -639,7 +679,8 @@ def main():
     ap.add_argument("--steps", type=int, default=3)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["kq", "reference"], default="kq")
-    ap.add_argument("--e2e-steps", type=int, default=4)
+    ap.add_argument("--e2e-steps", type=int, default=0, help="end-to-end steps (default: --steps)")
+    ap.add_argument("--update-reps", type=int, default=10, help="standalone update calls for its roofline")
     ap.add_argument("--ref-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--only", choices=["assign", "update", "quantize", "reconstruct", "gradstep", "levelgrad",

@@ -82,6 +82,25 @@ int32_t kq_abi_version(void);
  * devices, all threads). A diagnostic for tracing and launch accounting. */
 uint64_t kq_kernel_launches(void);
 
+/* Kernel trace, a diagnostic for per-kernel device time. kq_trace_start makes
+ * `capacity` (1 .. 2^20) pairs of CUDA events on the current device (host-side
+ * objects: no device memory) and starts a trace: from then on each kernel libkq
+ * launches, up to `capacity` of them, gets one event recorded on its launch
+ * stream just before it and one just after it. kq_trace_stop stops recording (the
+ * recorded pairs stay readable); kq_trace_count returns the launches recorded;
+ * kq_trace_get waits for launch i's second event and returns the kernel's name (a
+ * static string) and the time between the two events in ms. A new
+ * kq_trace_start discards the previous trace. One trace per process: trace calls
+ * from one host thread on one device at a time. While a trace runs, each launch
+ * costs two more stream commands, and a kernel that would otherwise start while
+ * its predecessor finishes (a programmatic dependent launch) starts after it.
+ * Errors: KQ_ERR_INVALID_ARG for a capacity or index out of range or a NULL
+ * output, KQ_ERR_CUDA when an event cannot be made or read. */
+kq_status kq_trace_start(int32_t capacity);
+kq_status kq_trace_stop(void);
+int32_t kq_trace_count(void);
+kq_status kq_trace_get(int32_t i, const char **name, float *ms);
+
 /* Bytes of workspace needed by any entry point for n kernels and K codewords.
  * Returns 0 when (n, K) is outside the supported range. */
 size_t kq_workspace_bytes(int64_t n, int32_t K);
@@ -132,9 +151,15 @@ kq_status kq_assign(const float *W, int64_t n, const float *C, int32_t K, const 
  * Same inputs, outputs and rules as kq_assign, without the workspace: the
  * scratch is a fixed array of about 10 MB built into libkq, which every GPU that
  * loads the library holds until the process exits. Limits: n <= 16,777,216 and
- * K <= 65,536; larger sizes return KQ_ERR_WORKSPACE. The first call on a device
- * looks up the array's device address (once per device, so make that first call
- * before any stream capture). Every call on a device shares the array, so calls
+ * K <= 65,536; larger sizes return KQ_ERR_WORKSPACE. It always runs the
+ * CUDA-core assignment kernel (the tensor-core one needs packed codeword tiles
+ * that the fixed array has no room for), so it returns the same indices and
+ * distances as kq_assign, bit for bit, at lower throughput. The first call on a
+ * device looks up the array's device address and keeps it (once per device, so
+ * make that first call before any stream capture); a cudaDeviceReset of that
+ * device invalidates the kept address, so do not call this entry point again in
+ * a process after resetting a device it has used. The pointers passed must
+ * belong to the current device. Every call on a device shares the array, so calls
  * whose work can overlap on the GPU race: issue them in order on one stream.
  * Device-side flags (e.g. a non-finite input) are not reported by this variant.
  * It never allocates or frees memory. */
@@ -156,8 +181,8 @@ kq_status kq_assign_noalloc(const float *W, int64_t n, const float *C, int32_t K
 kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int32_t K, const float *C_prev,
                               float *C_next, int32_t *counts, void *ws, size_t ws_bytes, kq_stream_t stream);
 
-/* k-means fit of the kernel codebook, Sec. 3.1 Eq. 1 (the "Quantize kernel ...
- * with k-means" step of Algorithm 1): from C_init, `iters` times
+/* k-means fit of the kernel codebook, Sec. 3.1 Eq. 1 (the k-means quantisation
+ * step of Algorithm 1): from C_init, `iters` times
  * { assign against C_t; objective[t] = sum_i dist_i; C_{t+1} = update },
  * then a final assign against C_iters, objective[iters] = its sum.
  *   W          n x 9 fp32 (device, 16-byte aligned)
@@ -215,7 +240,7 @@ kq_status kq_search_codebook_size(const float *W, int64_t n, const int64_t *sel,
 
 /* 6-bit kernel-codebook quantisation, Sec. 3.2: k-means with 64 levels over all
  * K*9 codebook scalars v_kj, each weighted by its entry's appearance count
- * z_k ("entry appearance time"), then the code of every scalar.
+ * z_k (how often the entry occurs in W), then the code of every scalar.
  *   - levels start at linspace(min, max, 64) over the scalars with z_k > 0 (all
  *     scalars if no count is positive), computed in fp64 and rounded to fp32;
  *   - a scalar's code is its nearest level by fp32 |v - level|, lower index on ties;
@@ -266,8 +291,8 @@ kq_status kq_quantize_scalars_6bit(const float *v, int64_t m, int32_t max_iters,
 kq_status kq_codebook_grad_step(const float *G, int64_t n, const int32_t *idx, int32_t K, float lr, const float *C,
                                 float *C_next, int32_t *counts, void *ws, size_t ws_bytes, kq_stream_t stream);
 
-/* Retraining step of the quantised codebook, Sec. 3.2 ("Retraining of codebook
- * quantization follows the same scheme"): a network weight is
+/* Retraining step of the quantised codebook, Sec. 3.2 (retrained the same way
+ * as the kernel codebook, with averaged gradients): a network weight is
  * W'_ij = levels[codes[idx_i * 9 + j]], so level l moves against the average
  * gradient of every weight whose value it is:
  *   counts[l]      = #{ (i, j) : codes[idx_i * 9 + j] == l },
@@ -319,6 +344,10 @@ kq_status kq_quantize_reconstruct(const int32_t *idx, int64_t n, const float *C,
  *           the 64-entry level table of the 6-bit codebook is not counted)
  *   Eq. 7  beta = B / (n * omega^2)             bits per parameter
  *   Eq. 6  ratio_kq = n * omega^2 * 32 / B      compression ratio C_KQ
+ *   Eq. 5  ratio_con_1bit = n * omega^2 * 32 / (2 * 32 + n * omega^2)
+ *          the same layer under conventional per-weight quantisation at its
+ *          limit (a codebook of u = 2 fp32 entries, one index bit per weight;
+ *          Sec. 3.3 puts that limit at 32), for comparison with ratio_kq
  * b_c = 32 for kernel-level quantisation only, 6 after codebook quantisation.
  * Requires n >= 1, 1 <= k, omega >= 1, b_c >= 1, out != NULL (host pointer). */
 typedef struct {
@@ -327,6 +356,7 @@ typedef struct {
     int64_t total_bits;
     double beta;
     double ratio_kq;
+    double ratio_con_1bit;
 } kq_report;
 
 kq_status kq_compression_report(int64_t n, int32_t k, int32_t omega, int32_t b_c, kq_report *out);

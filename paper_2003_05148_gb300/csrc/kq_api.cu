@@ -5,7 +5,9 @@
 
 #include <atomic>
 #include <cmath>
+#include <mutex>
 #include <unordered_map>
+#include <vector>
 
 #include "kq_internal.cuh"
 
@@ -13,12 +15,38 @@ using namespace kq;
 
 namespace kq {
 static std::atomic<unsigned long long> g_launches{0};
-void count_launch(int kernels) { g_launches.fetch_add((unsigned long long)kernels, std::memory_order_relaxed); }
+
+// Kernel trace (kq_trace_*): event pairs created up front, filled in launch order.
+struct TraceRec {
+    const char *name;
+    cudaEvent_t begin, end;
+};
+static std::mutex g_trace_mu;
+static std::vector<TraceRec> g_trace;
+static size_t g_trace_used = 0;
+static std::atomic<bool> g_trace_on{false};
+
+void launch_begin(cudaStream_t s) {
+    if (!g_trace_on.load(std::memory_order_relaxed)) return;
+    std::lock_guard<std::mutex> lock(g_trace_mu);
+    if (g_trace_on && g_trace_used < g_trace.size()) cudaEventRecord(g_trace[g_trace_used].begin, s);
+}
+
+void launch_end(cudaStream_t s, const char *name) {
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    if (!g_trace_on.load(std::memory_order_relaxed)) return;
+    std::lock_guard<std::mutex> lock(g_trace_mu);
+    if (g_trace_on && g_trace_used < g_trace.size()) {
+        cudaEventRecord(g_trace[g_trace_used].end, s);
+        g_trace[g_trace_used].name = name;
+        ++g_trace_used;
+    }
+}
 }  // namespace kq
 
 namespace {
 
-constexpr int32_t KQ_ABI_VERSION = 4;
+constexpr int32_t KQ_ABI_VERSION = 5;
 constexpr int32_t HINT_ORDER_MIN_K = 4096;  // warm starts in hint order from 16 codeword tiles on
 // Cold assignments with many codeword tiles start from a pilot pass: rows against the
 // first K / COLD_PILOT_DIV codewords (a random sample when the codebook was drawn from
@@ -231,6 +259,52 @@ const char *kq_status_string(kq_status s) {
 int32_t kq_abi_version(void) { return KQ_ABI_VERSION; }
 
 uint64_t kq_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
+
+kq_status kq_trace_start(int32_t capacity) {
+    if (capacity < 1 || capacity > (1 << 20)) return KQ_ERR_INVALID_ARG;
+    std::lock_guard<std::mutex> lock(g_trace_mu);
+    g_trace_on = false;
+    // events belong to the device current when they were made: remake them all
+    for (TraceRec &r : g_trace) {
+        cudaEventDestroy(r.begin);
+        cudaEventDestroy(r.end);
+    }
+    g_trace.clear();
+    g_trace_used = 0;
+    g_trace.reserve((size_t)capacity);
+    for (int32_t i = 0; i < capacity; ++i) {
+        TraceRec r{nullptr, nullptr, nullptr};
+        if (cudaEventCreate(&r.begin) != cudaSuccess) return KQ_ERR_CUDA;
+        if (cudaEventCreate(&r.end) != cudaSuccess) {
+            cudaEventDestroy(r.begin);
+            return KQ_ERR_CUDA;
+        }
+        g_trace.push_back(r);
+    }
+    g_trace_on = true;
+    return KQ_OK;
+}
+
+kq_status kq_trace_stop(void) {
+    std::lock_guard<std::mutex> lock(g_trace_mu);
+    g_trace_on = false;
+    return KQ_OK;
+}
+
+int32_t kq_trace_count(void) {
+    std::lock_guard<std::mutex> lock(g_trace_mu);
+    return (int32_t)g_trace_used;
+}
+
+kq_status kq_trace_get(int32_t i, const char **name, float *ms) {
+    std::lock_guard<std::mutex> lock(g_trace_mu);
+    if (i < 0 || (size_t)i >= g_trace_used || !name || !ms) return KQ_ERR_INVALID_ARG;
+    const TraceRec &r = g_trace[(size_t)i];
+    if (cudaEventSynchronize(r.end) != cudaSuccess) return KQ_ERR_CUDA;
+    if (cudaEventElapsedTime(ms, r.begin, r.end) != cudaSuccess) return KQ_ERR_CUDA;
+    *name = r.name;
+    return KQ_OK;
+}
 
 size_t kq_workspace_bytes(int64_t n, int32_t K) {
     if (!sizes_ok(n, K)) return 0;
@@ -540,6 +614,7 @@ kq_status kq_compression_report(int64_t n, int32_t k, int32_t omega, int32_t b_c
     out->total_bits = out->index_bits + out->codebook_bits;
     out->beta = (double)out->total_bits / (double)(n * w2);
     out->ratio_kq = (double)(n * w2 * 32) / (double)out->total_bits;
+    out->ratio_con_1bit = (double)(n * w2 * 32) / (double)(2 * 32 + n * w2);  // Eq. 5, u = 2, b_1 = 32
     return KQ_OK;
 }
 

@@ -288,8 +288,9 @@ __global__ void __launch_bounds__(256) sum_blocks_kernel(const double *__restric
 cudaError_t launch_pack_codebook(const float *C, int32_t K, float *Cd, Header *hdr, cudaStream_t s) {
     cudaError_t e = cudaMemsetAsync(&hdr->cb_cmax, 0, 3 * sizeof(uint32_t), s);
     if (e != cudaSuccess) return e;
+    launch_begin(s);
     pack_codebook_kernel<<<(K + 255) / 256, 256, 0, s>>>(C, K, Cd, hdr);
-    count_launch();
+    launch_end(s, "pack_codebook_kernel");
     return cudaGetLastError();
 }
 
@@ -315,14 +316,16 @@ cudaError_t launch_assign(const float *W, int64_t n, const float *Cd, const floa
     G = (K + kps - 1) / kps;
     const int64_t part_stride = row_blocks * ROW_BLOCK;
     dim3 grid((unsigned)row_blocks, (unsigned)G);
+    launch_begin(s);
     assign_kernel<<<grid, A_THREADS, 0, s>>>(W, n, Cd, C, K, kps, hint, idx, dist, blocksum, part, part_stride, hdr);
-    count_launch();
+    launch_end(s, "assign_kernel");
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     if (G > 1) {
         const int64_t cb = (n + 255) / 256;
+        launch_begin(s);
         combine_kernel<<<(unsigned)cb, 256, 0, s>>>(part, part_stride, (int)G, n, idx, dist, blocksum);
-        count_launch();
+        launch_end(s, "combine_kernel");
         *nblocksum = (int)cb;
     } else {
         *nblocksum = (int)row_blocks;
@@ -331,8 +334,9 @@ cudaError_t launch_assign(const float *W, int64_t n, const float *Cd, const floa
 }
 
 cudaError_t launch_sum_blocks(const double *blocksum, int nblocks, double *out, cudaStream_t s) {
+    launch_begin(s);
     sum_blocks_kernel<<<1, 256, 0, s>>>(blocksum, nblocks, out);
-    count_launch();
+    launch_end(s, "sum_blocks_kernel");
     return cudaGetLastError();
 }
 

@@ -37,7 +37,7 @@
 //   it reads (tcgen05.ld.red.max, sm_103a): a 32-codeword chunk whose maximum g has
 //   its sign bit set is ruled out with no further work (NaN test values, which the
 //   maximum skips, only arise in rows whose thread tests every codeword anyway: see
-//   T' = -2^100 below). Only a chunk with a non-negative maximum sends the row to
+//   -T' = 2^15 below). Only a chunk with a non-negative maximum sends the row to
 //   the exact fp32 direct form on the CUDA cores, which reads c in fp32 from the
 //   same shared stage (every streamed tile carries its codewords in fp32 after the
 //   fp16 operands). When a row's best improves, its thread rewrites its T' (one
@@ -885,15 +885,18 @@ cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Heade
     if (e != cudaSuccess) return e;
     const int32_t Kpad = tc_kpad(K);
     if (Kpad <= TC_PACK_ONE_CTA) {
+        launch_begin(s);
         pack_codebook_tc_small_kernel<<<1, TC_PACK_SMALL_THREADS, 0, s>>>(C, K, Kpad, Cpk, hdr);
-        count_launch();
+        launch_end(s, "pack_codebook_tc_small_kernel");
         return cudaGetLastError();
     }
+    launch_begin(s);
     codebook_norm_tc_kernel<<<(K + 255) / 256, 256, 0, s>>>(C, K, hdr);
-    count_launch();
+    launch_end(s, "codebook_norm_tc_kernel");
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    launch_begin(s);
     pack_codebook_tc_kernel<<<(Kpad + 255) / 256, 256, 0, s>>>(C, K, Kpad, Cpk, hdr);
-    count_launch();
+    launch_end(s, "pack_codebook_tc_kernel");
     return cudaGetLastError();
 }
 
@@ -1010,26 +1013,31 @@ cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, c
     if (hint_counts) {
         // the rows per hinted codeword are known (all hints valid): start offsets
         // straight from them, K + 1 entries with the last count 0
+        launch_begin(s);
         scan_counts_kernel<<<1, SCAN_THREADS, 0, s>>>(hint_counts, K, K + 1, cnt);
-        count_launch();
+        launch_end(s, "scan_counts_kernel");
     } else {
         cudaError_t e = cudaMemsetAsync(cnt, 0, (size_t)(K + 1) * sizeof(int32_t), s);
         if (e != cudaSuccess) return e;
+        launch_begin(s);
         hint_histogram_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cnt);
-        count_launch();
+        launch_end(s, "hint_histogram_kernel");
         // the scan turns cnt into start offsets in place
+        launch_begin(s);
         scan_counts_kernel<<<1, SCAN_THREADS, 0, s>>>(cnt, K + 1, K + 1, cnt);
-        count_launch();
+        launch_end(s, "scan_counts_kernel");
     }
+    launch_begin(s);
     hint_scatter_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cnt, perm);
-    count_launch();
+    launch_end(s, "hint_scatter_kernel");
     return cudaGetLastError();
 }
 
 cudaError_t launch_dist_block_sums(const float *dist, int64_t n, double *blocksum, int *nblocksum, cudaStream_t s) {
     const int64_t blocks = (n + 255) / 256;
+    launch_begin(s);
     dist_block_sums_kernel<<<(unsigned)blocks, 256, 0, s>>>(dist, n, blocksum);
-    count_launch();
+    launch_end(s, "dist_block_sums_kernel");
     *nblocksum = (int)blocks;
     return cudaGetLastError();
 }
@@ -1045,9 +1053,10 @@ cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const fl
     if (e != cudaSuccess) return e;
     const int64_t blocks = (n + TC_ROWS - 1) / TC_ROWS;
     const int32_t ntiles = tc_kpad(K) / TC_N;
+    launch_begin(s);
     assign_tc_kernel<<<(unsigned)blocks, TC_THREADS, smem, s>>>(W, n, C, Cpk, K, ntiles, hint, perm, idx, dist,
                                                                 blocksum, hdr);
-    count_launch();
+    launch_end(s, "assign_tc_kernel");
     *nblocksum = (int)blocks;
     return cudaGetLastError();
 }

@@ -249,8 +249,12 @@ __device__ __forceinline__ bool grid_barrier(Header *h, unsigned nblocks, unsign
     return s_ok != 0;
 }
 
-// Process-wide count of kernels libkq has launched (kq_kernel_launches()).
-void count_launch(int kernels = 1);
+// Every kernel launch is bracketed by launch_begin(s) before it and launch_end(s,
+// name) after it (s: the launch stream, name: the kernel's, a string literal).
+// launch_end counts the launch (kq_kernel_launches()); while a trace is on
+// (kq_trace_start), the pair also records CUDA events around the kernel on s.
+void launch_begin(cudaStream_t s);
+void launch_end(cudaStream_t s, const char *name);
 
 // ---- launchers (defined in the .cu files; all return cudaGetLastError()) ----
 // Packs C for the assign kernel and computes the filter's codebook bounds into

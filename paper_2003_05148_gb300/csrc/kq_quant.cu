@@ -320,10 +320,11 @@ cudaError_t launch_level_fit_t(const LevelArgs &args, int num_sms, cudaStream_t 
     LevelArgs a = args;
     a.use_table = args.N / (blocks * T) >= 64;  // the table pays for itself from ~64 scalars per thread
     void *params[] = {&a};
+    launch_begin(s);
     e = cudaLaunchCooperativeKernel((const void *)level_fit_kernel<UNIT>, dim3((unsigned)blocks), dim3(T), params,
                                     smem, s);
     if (e != cudaSuccess) return e;
-    count_launch();
+    launch_end(s, "level_fit_kernel");
     return cudaGetLastError();
 }
 

@@ -276,8 +276,9 @@ init_codebook_kernel(const float *__restrict__ W, int64_t n, const int64_t *__re
 
 cudaError_t launch_decode_codebook(const float *C, int32_t K, const uint8_t *codes, float *Cp,
                                    unsigned long long *Cq, uint32_t *status, cudaStream_t s) {
+    launch_begin(s);
     decode_codebook_kernel<<<(K + 255) / 256, 256, 0, s>>>(C, K, codes, Cp, Cq, status);
-    count_launch();
+    launch_end(s, "decode_codebook_kernel");
     return cudaGetLastError();
 }
 
@@ -297,16 +298,18 @@ cudaError_t launch_gather_rows(const int32_t *idx, int64_t n, const float *Cp, c
         attr[0].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
+        launch_begin(s);
         const cudaError_t e = cudaLaunchKernelEx(&cfg, gather_codes_kernel, idx, n, Cq, levels, K, W_out, status);
-        count_launch();
+        launch_end(s, "gather_codes_kernel");
         return e != cudaSuccess ? e : cudaGetLastError();
     }
     const int64_t groups = n / G_ROWS;
     int64_t blocks = (groups + R_WARPS - 1) / R_WARPS;
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
     if (blocks < 1) blocks = 1;
+    launch_begin(s);
     gather_rows_kernel<<<(unsigned)blocks, R_THREADS, 0, s>>>(idx, n, Cp, K, W_out, status);
-    count_launch();
+    launch_end(s, "gather_rows_kernel");
     return cudaGetLastError();
 }
 
@@ -326,18 +329,20 @@ cudaError_t launch_encode_gather(const float *C, int32_t K, const float *levels,
     if (blocks < 1) blocks = 1;
     void *params[] = {(void *)&C, (void *)&K, (void *)&levels, (void *)&codes, (void *)&Cq,
                       (void *)&idx, (void *)&n, (void *)&W_out, (void *)&hdr};
+    launch_begin(s);
     e = cudaLaunchCooperativeKernel((const void *)encode_gather_kernel, dim3((unsigned)blocks), dim3(R_THREADS),
                                     params, 0, s);
     if (e != cudaSuccess) return e;
-    count_launch();
+    launch_end(s, "encode_gather_kernel");
     return cudaGetLastError();
 }
 
 cudaError_t launch_init_codebook(const float *W, int64_t n, const int64_t *sel, int32_t K, float *C0,
                                  uint32_t *status, cudaStream_t s) {
     const int64_t total = (int64_t)K * D;
+    launch_begin(s);
     init_codebook_kernel<<<(unsigned)((total + 255) / 256), 256, 0, s>>>(W, n, sel, K, C0, status);
-    count_launch();
+    launch_end(s, "init_codebook_kernel");
     return cudaGetLastError();
 }
 

@@ -171,8 +171,9 @@ __global__ void level_grad_finalize_kernel(const Header *hdr, float lr, const fl
 
 cudaError_t launch_grad_finalize(unsigned long long *acc, int32_t K, const Header *hdr, float lr, const float *C,
                                  float *C_next, int32_t *counts, cudaStream_t s) {
+    launch_begin(s);
     grad_finalize_kernel<<<(K + 255) / 256, 256, 0, s>>>(acc, K, hdr, lr, C, C_next, counts);
-    count_launch();
+    launch_end(s, "grad_finalize_kernel");
     return cudaGetLastError();
 }
 
@@ -188,11 +189,13 @@ cudaError_t launch_level_grad(const float *G, int64_t n, const int32_t *idx, int
     int64_t blocks = (chunks + LG_WARPS * LG_UNROLL - 1) / (LG_WARPS * LG_UNROLL);
     if (blocks > 2LL * num_sms) blocks = 2LL * num_sms;  // two CTAs per SM fit in shared memory
     if (blocks < 1) blocks = 1;
+    launch_begin(s);
     level_grad_kernel<<<(unsigned)blocks, LG_THREADS, smem, s>>>(G, n, idx, K, codes, hdr);
-    count_launch();
+    launch_end(s, "level_grad_kernel");
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    launch_begin(s);
     level_grad_finalize_kernel<<<1, LEVELS, 0, s>>>(hdr, lr, levels, levels_next, counts);
-    count_launch();
+    launch_end(s, "level_grad_finalize_kernel");
     return cudaGetLastError();
 }
 

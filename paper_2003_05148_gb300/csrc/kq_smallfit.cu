@@ -255,10 +255,11 @@ cudaError_t launch_small_fit(const float *W, int64_t n, const float *C0, int32_t
     SmallFitArgs a{W, n, C0, K, iters, C_out, idx, counts, objective, acc, cbuf0, cbuf1, blocksum, hdr,
                    stop_on_stable ? 1 : 0};
     void *params[] = {&a};
+    launch_begin(s);
     e = cudaLaunchCooperativeKernel((const void *)small_fit_kernel, dim3((unsigned)blocks), dim3(SF_THREADS), params, 0,
                                     s);
     if (e != cudaSuccess) return e;
-    count_launch();
+    launch_end(s, "small_fit_kernel");
     return cudaGetLastError();
 }
 

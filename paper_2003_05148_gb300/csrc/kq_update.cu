@@ -272,8 +272,9 @@ cudaError_t launch_accumulate_delta(const float *W, int64_t n, const int32_t *id
     int64_t blocks = (n + 255) / 256;
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
     if (blocks < 1) blocks = 1;
+    launch_begin(s);
     accumulate_delta_kernel<<<(unsigned)blocks, 256, 0, s>>>(W, n, idx_old, idx_new, K, hdr, acc, moved);
-    count_launch();
+    launch_end(s, "accumulate_delta_kernel");
     return cudaGetLastError();
 }
 
@@ -288,8 +289,9 @@ cudaError_t launch_fill_objective(double *obj, int32_t from, int32_t to, cudaStr
     if (to <= from) return cudaSuccess;
     int64_t blocks = ((int64_t)to - from + 255) / 256;
     if (blocks > 1024) blocks = 1024;
+    launch_begin(s);
     fill_objective_kernel<<<(unsigned)blocks, 256, 0, s>>>(obj, from, to);
-    count_launch();
+    launch_end(s, "fill_objective_kernel");
     return cudaGetLastError();
 }
 
@@ -313,8 +315,9 @@ cudaError_t launch_histogram(const int32_t *idx, int64_t n, int32_t K, int32_t *
     int64_t blocks = (n + 255) / 256;
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
     if (blocks < 1) blocks = 1;
+    launch_begin(s);
     histogram_kernel<<<(unsigned)blocks, 256, 0, s>>>(idx, n, K, counts, status);
-    count_launch();
+    launch_end(s, "histogram_kernel");
     return cudaGetLastError();
 }
 
@@ -325,8 +328,9 @@ cudaError_t launch_maxabs(const float *W, int64_t count, uint32_t *maxabs_bits, 
     int64_t blocks = (count / 4 + 255) / 256;
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
     if (blocks < 1) blocks = 1;
+    launch_begin(s);
     maxabs_kernel<<<(unsigned)blocks, 256, 0, s>>>(W, count, maxabs_bits, status);
-    count_launch();
+    launch_end(s, "maxabs_kernel");
     return cudaGetLastError();
 }
 
@@ -344,8 +348,9 @@ cudaError_t launch_update_prepare(const float *C_prev, int32_t K, unsigned long 
     int64_t blocks = ((int64_t)K * ACC_WORDS / 2 + 255) / 256;
     if (blocks > 4 * 152) blocks = 4 * 152;
     if (blocks < 1) blocks = 1;
+    launch_begin(s);
     update_prepare_kernel<<<(unsigned)blocks, 256, 0, s>>>(C_prev, K, acc, hdr, guess_from_codebook);
-    count_launch();
+    launch_end(s, "update_prepare_kernel");
     return cudaGetLastError();
 }
 
@@ -355,8 +360,9 @@ cudaError_t launch_accumulate(const float *W, int64_t n, const int32_t *idx, int
     int64_t blocks = (chunks + U_THREADS / 32 - 1) / (U_THREADS / 32);
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
     if (blocks < 1) blocks = 1;
+    launch_begin(s);
     accumulate_kernel<<<(unsigned)blocks, U_THREADS, 0, s>>>(W, n, idx, K, hdr, acc, guess);
-    count_launch();
+    launch_end(s, "accumulate_kernel");
     return cudaGetLastError();
 }
 
@@ -368,16 +374,18 @@ cudaError_t launch_update_fallback(const float *W, int64_t n, const int32_t *idx
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
     const unsigned blocks = (unsigned)num_sms;  // one CTA per SM: co-resident by construction
     void *params[] = {(void *)&W, (void *)&n, (void *)&idx, (void *)&K, (void *)&hdr, (void *)&acc};
+    launch_begin(s);
     e = cudaLaunchCooperativeKernel((const void *)update_fallback_kernel, dim3(blocks), dim3(U_THREADS), params, 0, s);
     if (e != cudaSuccess) return e;
-    count_launch();
+    launch_end(s, "update_fallback_kernel");
     return cudaGetLastError();
 }
 
 cudaError_t launch_finalize(unsigned long long *acc, int32_t K, const Header *hdr, const float *C_prev,
                             float *C_next, int32_t *counts, cudaStream_t s, bool keep_sums) {
+    launch_begin(s);
     finalize_kernel<<<(K + 255) / 256, 256, 0, s>>>(acc, K, hdr, C_prev, C_next, counts, keep_sums);
-    count_launch();
+    launch_end(s, "finalize_kernel");
     return cudaGetLastError();
 }
 

@@ -26,7 +26,7 @@ EXPORTS = ["kq_status_string", "kq_abi_version", "kq_kernel_launches", "kq_works
            "kq_assign", "kq_update_centroids", "kq_fit_codebook", "kq_quantize_codebook_6bit", "kq_reconstruct",
            "kq_compression_report", "kq_conventional_ratio", "kq_assign_noalloc", "kq_quantize_scalars_6bit",
            "kq_codebook_grad_step", "kq_levels_grad_step", "kq_search_codebook_size", "kq_quantize_reconstruct",
-           "kq_seed_indices"]
+           "kq_seed_indices", "kq_trace_start", "kq_trace_stop", "kq_trace_count", "kq_trace_get"]
 
 
 class KQError(RuntimeError):
@@ -37,7 +37,7 @@ class KQError(RuntimeError):
 
 class Report(ctypes.Structure):
     _fields_ = [("index_bits", ctypes.c_int64), ("codebook_bits", ctypes.c_int64), ("total_bits", ctypes.c_int64),
-                ("beta", ctypes.c_double), ("ratio_kq", ctypes.c_double)]
+                ("beta", ctypes.c_double), ("ratio_kq", ctypes.c_double), ("ratio_con_1bit", ctypes.c_double)]
 
 
 _lib = None
@@ -55,6 +55,10 @@ def lib() -> ctypes.CDLL:
             "kq_status_string": ([ctypes.c_int], ctypes.c_char_p),
             "kq_abi_version": ([], i32),
             "kq_kernel_launches": ([], ctypes.c_uint64),
+            "kq_trace_start": ([i32], ctypes.c_int),
+            "kq_trace_stop": ([], ctypes.c_int),
+            "kq_trace_count": ([], i32),
+            "kq_trace_get": ([i32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(ctypes.c_float)], ctypes.c_int),
             "kq_workspace_bytes": ([i64, i32], sz),
             "kq_device_status": ([P, sz, P, P], ctypes.c_int),
             "kq_init_codebook": ([P, i64, P, i32, P, P, sz, P], ctypes.c_int),
@@ -99,9 +103,36 @@ def _dev(t: Optional[torch.Tensor], name: str, dtype: torch.dtype):
     return ctypes.c_void_p(t.data_ptr())
 
 
-def _stream(stream) -> ctypes.c_void_p:
-    s = torch.cuda.current_stream() if stream is None else stream
-    return ctypes.c_void_p(s.cuda_stream)
+class _Call:
+    """Marshalling for one call of an entry point that takes device memory: every
+    tensor must live on one CUDA device; the call runs with that device current
+    (the library reads the current device for its SM count and launches there) and
+    on that device's current stream unless a stream of the same device is given."""
+
+    def __init__(self, fn: str):
+        self.fn = fn
+        self.device = None
+
+    def ptr(self, t: Optional[torch.Tensor], name: str, dtype: torch.dtype):
+        p = _dev(t, name, dtype)
+        if t is not None:
+            if self.device is None:
+                self.device = t.device
+            elif t.device != self.device:
+                raise ValueError(f"{self.fn}: {name} is on {t.device}, other arguments on {self.device}")
+        return p
+
+    def stream(self, stream) -> ctypes.c_void_p:
+        if self.device is None:
+            raise ValueError(f"{self.fn}: no device tensor given")
+        s = torch.cuda.current_stream(self.device) if stream is None else stream
+        if s.device != self.device:
+            raise ValueError(f"{self.fn}: the stream is on {s.device}, the tensors on {self.device}")
+        return ctypes.c_void_p(s.cuda_stream)
+
+    def __call__(self, *args) -> None:
+        with torch.cuda.device(self.device):
+            _check(self.fn, getattr(lib(), self.fn)(*args))
 
 
 def _rows(W: torch.Tensor) -> int:
@@ -122,6 +153,26 @@ def kq_kernel_launches() -> int:
     return int(lib().kq_kernel_launches())
 
 
+def kq_trace_start(capacity: int) -> None:
+    """Start a kernel trace of up to `capacity` launches (events on the current device)."""
+    _check("kq_trace_start", lib().kq_trace_start(capacity))
+
+
+def kq_trace_stop() -> None:
+    _check("kq_trace_stop", lib().kq_trace_stop())
+
+
+def kq_trace_read() -> list:
+    """[(kernel name, device ms)] of every launch the current trace recorded, in launch order."""
+    out = []
+    name = ctypes.c_char_p()
+    ms = ctypes.c_float()
+    for i in range(lib().kq_trace_count()):
+        _check("kq_trace_get", lib().kq_trace_get(i, ctypes.byref(name), ctypes.byref(ms)))
+        out.append((name.value.decode(), ms.value))
+    return out
+
+
 def kq_workspace_bytes(n: int, K: int) -> int:
     return int(lib().kq_workspace_bytes(n, K))
 
@@ -137,68 +188,79 @@ def workspace(n: int, K: int, device=None) -> torch.Tensor:
 def kq_device_status(ws: torch.Tensor, stream=None):
     """(status, flags): read and clear the sticky device status word (synchronises the stream)."""
     flags = ctypes.c_uint32(0)
-    st = lib().kq_device_status(_dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream), ctypes.byref(flags))
+    c = _Call("kq_device_status")
+    ptr = c.ptr(ws, "ws", torch.uint8)
+    with torch.cuda.device(c.device):
+        st = lib().kq_device_status(ptr, ws.numel(), c.stream(stream), ctypes.byref(flags))
     return st, flags.value
 
 
 def kq_init_codebook(W, sel, C0, ws, stream=None) -> None:
-    _check("kq_init_codebook", lib().kq_init_codebook(
-        _dev(W, "W", torch.float32), _rows(W), _dev(sel, "sel", torch.int64), sel.numel(),
-        _dev(C0, "C0", torch.float32), _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+    c = _Call("kq_init_codebook")
+    c(
+        c.ptr(W, "W", torch.float32), _rows(W), c.ptr(sel, "sel", torch.int64), sel.numel(),
+        c.ptr(C0, "C0", torch.float32), c.ptr(ws, "ws", torch.uint8), ws.numel(), c.stream(stream))
 
 
 def kq_assign(W, C, idx, dist, ws, hint=None, stream=None) -> None:
-    _check("kq_assign", lib().kq_assign(
-        _dev(W, "W", torch.float32), _rows(W), _dev(C, "C", torch.float32), _rows(C),
-        _dev(hint, "hint", torch.int32), _dev(idx, "idx", torch.int32), _dev(dist, "dist", torch.float32),
-        _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+    c = _Call("kq_assign")
+    c(
+        c.ptr(W, "W", torch.float32), _rows(W), c.ptr(C, "C", torch.float32), _rows(C),
+        c.ptr(hint, "hint", torch.int32), c.ptr(idx, "idx", torch.int32), c.ptr(dist, "dist", torch.float32),
+        c.ptr(ws, "ws", torch.uint8), ws.numel(), c.stream(stream))
 
 
 def kq_update_centroids(W, idx, C_prev, C_next, counts, ws, stream=None) -> None:
-    _check("kq_update_centroids", lib().kq_update_centroids(
-        _dev(W, "W", torch.float32), _rows(W), _dev(idx, "idx", torch.int32), _rows(C_prev),
-        _dev(C_prev, "C_prev", torch.float32), _dev(C_next, "C_next", torch.float32),
-        _dev(counts, "counts", torch.int32), _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+    c = _Call("kq_update_centroids")
+    c(
+        c.ptr(W, "W", torch.float32), _rows(W), c.ptr(idx, "idx", torch.int32), _rows(C_prev),
+        c.ptr(C_prev, "C_prev", torch.float32), c.ptr(C_next, "C_next", torch.float32),
+        c.ptr(counts, "counts", torch.int32), c.ptr(ws, "ws", torch.uint8), ws.numel(), c.stream(stream))
 
 
 def kq_fit_codebook(W, C_init, iters, C_out, idx, counts, objective, ws, stream=None, flags: int = 0) -> int:
     """Returns the number of codebook updates performed (iters unless STOP_ON_STABLE stopped early)."""
     run = ctypes.c_int32(0)
-    _check("kq_fit_codebook", lib().kq_fit_codebook(
-        _dev(W, "W", torch.float32), _rows(W), _rows(C_init), _dev(C_init, "C_init", torch.float32), iters, flags,
-        _dev(C_out, "C_out", torch.float32), _dev(idx, "idx", torch.int32), _dev(counts, "counts", torch.int32),
-        _dev(objective, "objective", torch.float64), ctypes.byref(run), _dev(ws, "ws", torch.uint8), ws.numel(),
-        _stream(stream)))
+    c = _Call("kq_fit_codebook")
+    c(
+        c.ptr(W, "W", torch.float32), _rows(W), _rows(C_init), c.ptr(C_init, "C_init", torch.float32), iters, flags,
+        c.ptr(C_out, "C_out", torch.float32), c.ptr(idx, "idx", torch.int32), c.ptr(counts, "counts", torch.int32),
+        c.ptr(objective, "objective", torch.float64), ctypes.byref(run), c.ptr(ws, "ws", torch.uint8), ws.numel(),
+        c.stream(stream))
     return run.value
 
 
 def kq_quantize_codebook_6bit(C, counts, max_iters, levels, codes, iters_run, ws, stream=None) -> None:
-    _check("kq_quantize_codebook_6bit", lib().kq_quantize_codebook_6bit(
-        _dev(C, "C", torch.float32), _rows(C), _dev(counts, "counts", torch.int32), max_iters,
-        _dev(levels, "levels", torch.float32), _dev(codes, "codes", torch.uint8),
-        _dev(iters_run, "iters_run", torch.int32), _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+    c = _Call("kq_quantize_codebook_6bit")
+    c(
+        c.ptr(C, "C", torch.float32), _rows(C), c.ptr(counts, "counts", torch.int32), max_iters,
+        c.ptr(levels, "levels", torch.float32), c.ptr(codes, "codes", torch.uint8),
+        c.ptr(iters_run, "iters_run", torch.int32), c.ptr(ws, "ws", torch.uint8), ws.numel(), c.stream(stream))
 
 
 def kq_quantize_scalars_6bit(v, max_iters, levels, codes, iters_run, ws, stream=None) -> None:
-    _check("kq_quantize_scalars_6bit", lib().kq_quantize_scalars_6bit(
-        _dev(v, "v", torch.float32), v.numel(), max_iters, _dev(levels, "levels", torch.float32),
-        _dev(codes, "codes", torch.uint8), _dev(iters_run, "iters_run", torch.int32), _dev(ws, "ws", torch.uint8),
-        ws.numel(), _stream(stream)))
+    c = _Call("kq_quantize_scalars_6bit")
+    c(
+        c.ptr(v, "v", torch.float32), v.numel(), max_iters, c.ptr(levels, "levels", torch.float32),
+        c.ptr(codes, "codes", torch.uint8), c.ptr(iters_run, "iters_run", torch.int32), c.ptr(ws, "ws", torch.uint8),
+        ws.numel(), c.stream(stream))
 
 
 def kq_codebook_grad_step(G, idx, lr: float, C, C_next, counts, ws, stream=None) -> None:
-    _check("kq_codebook_grad_step", lib().kq_codebook_grad_step(
-        _dev(G, "G", torch.float32), _rows(G), _dev(idx, "idx", torch.int32), _rows(C), float(lr),
-        _dev(C, "C", torch.float32), _dev(C_next, "C_next", torch.float32), _dev(counts, "counts", torch.int32),
-        _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+    c = _Call("kq_codebook_grad_step")
+    c(
+        c.ptr(G, "G", torch.float32), _rows(G), c.ptr(idx, "idx", torch.int32), _rows(C), float(lr),
+        c.ptr(C, "C", torch.float32), c.ptr(C_next, "C_next", torch.float32), c.ptr(counts, "counts", torch.int32),
+        c.ptr(ws, "ws", torch.uint8), ws.numel(), c.stream(stream))
 
 
 def kq_levels_grad_step(G, idx, codes, lr: float, levels, levels_next, counts, ws, stream=None) -> None:
-    _check("kq_levels_grad_step", lib().kq_levels_grad_step(
-        _dev(G, "G", torch.float32), _rows(G), _dev(idx, "idx", torch.int32), codes.numel() // 9,
-        _dev(codes, "codes", torch.uint8), float(lr), _dev(levels, "levels", torch.float32),
-        _dev(levels_next, "levels_next", torch.float32), _dev(counts, "counts", torch.int64),
-        _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+    c = _Call("kq_levels_grad_step")
+    c(
+        c.ptr(G, "G", torch.float32), _rows(G), c.ptr(idx, "idx", torch.int32), codes.numel() // 9,
+        c.ptr(codes, "codes", torch.uint8), float(lr), c.ptr(levels, "levels", torch.float32),
+        c.ptr(levels_next, "levels_next", torch.float32), c.ptr(counts, "counts", torch.int64),
+        c.ptr(ws, "ws", torch.uint8), ws.numel(), c.stream(stream))
 
 
 def kq_search_codebook_size(W, sel, alpha: float, r: float, max_steps: int, lloyd_iters: int, C_out, idx, counts,
@@ -209,27 +271,30 @@ def kq_search_codebook_size(W, sel, alpha: float, r: float, max_steps: int, lloy
     steps = ctypes.c_int32(0)
     tK = (ctypes.c_int32 * (max_steps + 1))()
     tE = (ctypes.c_double * (max_steps + 1))()
-    _check("kq_search_codebook_size", lib().kq_search_codebook_size(
-        _dev(W, "W", torch.float32), _rows(W), _dev(sel, "sel", torch.int64), sel.numel(), float(alpha), float(r),
-        max_steps, lloyd_iters, _dev(C_out, "C_out", torch.float32), _dev(idx, "idx", torch.int32),
-        _dev(counts, "counts", torch.int32), ctypes.byref(k), ctypes.byref(err), tK, tE, ctypes.byref(steps),
-        _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+    c = _Call("kq_search_codebook_size")
+    c(
+        c.ptr(W, "W", torch.float32), _rows(W), c.ptr(sel, "sel", torch.int64), sel.numel(), float(alpha), float(r),
+        max_steps, lloyd_iters, c.ptr(C_out, "C_out", torch.float32), c.ptr(idx, "idx", torch.int32),
+        c.ptr(counts, "counts", torch.int32), ctypes.byref(k), ctypes.byref(err), tK, tE, ctypes.byref(steps),
+        c.ptr(ws, "ws", torch.uint8), ws.numel(), c.stream(stream))
     return k.value, err.value, [(tK[i], tE[i]) for i in range(steps.value + 1)]
 
 
 def kq_quantize_reconstruct(idx, C, levels, codes, W_out, ws, stream=None) -> None:
-    _check("kq_quantize_reconstruct", lib().kq_quantize_reconstruct(
-        _dev(idx, "idx", torch.int32), idx.numel(), _dev(C, "C", torch.float32), _rows(C),
-        _dev(levels, "levels", torch.float32), _dev(codes, "codes", torch.uint8), _dev(W_out, "W_out", torch.float32),
-        _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+    c = _Call("kq_quantize_reconstruct")
+    c(
+        c.ptr(idx, "idx", torch.int32), idx.numel(), c.ptr(C, "C", torch.float32), _rows(C),
+        c.ptr(levels, "levels", torch.float32), c.ptr(codes, "codes", torch.uint8), c.ptr(W_out, "W_out", torch.float32),
+        c.ptr(ws, "ws", torch.uint8), ws.numel(), c.stream(stream))
 
 
 def kq_reconstruct(idx, C, codes, levels, W_out, ws, K: Optional[int] = None, stream=None) -> None:
     K = _rows(C) if C is not None else codes.numel() // 9 if K is None else K
-    _check("kq_reconstruct", lib().kq_reconstruct(
-        _dev(idx, "idx", torch.int32), idx.numel(), _dev(C, "C", torch.float32), K,
-        _dev(codes, "codes", torch.uint8), _dev(levels, "levels", torch.float32),
-        _dev(W_out, "W_out", torch.float32), _dev(ws, "ws", torch.uint8), ws.numel(), _stream(stream)))
+    c = _Call("kq_reconstruct")
+    c(
+        c.ptr(idx, "idx", torch.int32), idx.numel(), c.ptr(C, "C", torch.float32), K,
+        c.ptr(codes, "codes", torch.uint8), c.ptr(levels, "levels", torch.float32),
+        c.ptr(W_out, "W_out", torch.float32), c.ptr(ws, "ws", torch.uint8), ws.numel(), c.stream(stream))
 
 
 def kq_compression_report(n: int, k: int, omega: int = 3, b_c: int = 32) -> dict:
@@ -253,6 +318,7 @@ def kq_conventional_ratio(n: int, omega: int, u: int, b_1: int, b_fp: int = 32) 
 
 def kq_assign_noalloc(W, C, idx, dist, stream=None) -> None:
     """kq_assign without a workspace, for callers that cannot allocate device memory."""
-    _check("kq_assign_noalloc", lib().kq_assign_noalloc(
-        _dev(W, "W", torch.float32), _rows(W), _dev(C, "C", torch.float32), _rows(C),
-        _dev(idx, "idx", torch.int32), _dev(dist, "dist", torch.float32), _stream(stream)))
+    c = _Call("kq_assign_noalloc")
+    c(
+        c.ptr(W, "W", torch.float32), _rows(W), c.ptr(C, "C", torch.float32), _rows(C),
+        c.ptr(idx, "idx", torch.int32), c.ptr(dist, "dist", torch.float32), c.stream(stream))

@@ -37,7 +37,7 @@ def test_exports_every_declared_symbol(lib):
 
 
 def test_status_strings_and_version(lib):
-    assert kq.kq_abi_version() == 4
+    assert kq.kq_abi_version() == 5
     for code, name in kq.STATUS_NAMES.items():
         assert kq.kq_status_string(code) == name
     assert kq.kq_status_string(99) == "KQ_ERR_UNKNOWN"
@@ -154,6 +154,8 @@ def test_report_matches_oracle(lib, n, k, b_c):
     assert got["total_bits"] == ref.total_bits
     assert Fraction(got["beta"]) == pytest.approx(ref.beta, rel=1e-15)
     assert Fraction(got["ratio_kq"]) == pytest.approx(ref.ratio_kq, rel=1e-15)
+    # Eq. 5 at its limit (u = 2 fp32 entries, one bit per weight) for the same layer
+    assert Fraction(got["ratio_con_1bit"]) == pytest.approx(oracle.ratio_conventional(n, 3, 2, 32), rel=1e-15)
 
 
 def test_conventional_ratio_matches_oracle(lib):
@@ -164,6 +166,15 @@ def test_conventional_ratio_matches_oracle(lib):
         kq.kq_conventional_ratio(10, 3, 1, 32)
     with pytest.raises(kq.KQError):
         kq.kq_compression_report(0, 4)
+
+
+def test_trace_arguments_checked_on_host(lib):
+    assert lib.kq_trace_start(0) == 1
+    assert lib.kq_trace_start((1 << 20) + 1) == 1
+    name, ms = ctypes.c_char_p(), ctypes.c_float()
+    assert lib.kq_trace_get(-1, ctypes.byref(name), ctypes.byref(ms)) == 1
+    assert lib.kq_trace_get(lib.kq_trace_count(), ctypes.byref(name), ctypes.byref(ms)) == 1
+    assert lib.kq_trace_stop() == 0
 
 
 def test_cuda_failure_returns_status_without_device(lib):
@@ -183,3 +194,4 @@ def test_cuda_failure_returns_status_without_device(lib):
     assert L.kq_reconstruct(good, 1024, good, 16, None, None, good, good, ws_bytes, None) == 4
     assert L.kq_quantize_reconstruct(good, 1024, good, 16, good, None, good, good, ws_bytes, None) == 4
     assert L.kq_device_status(good, ws_bytes, None, None) == 4
+    assert L.kq_trace_start(4) == 4  # no device to make events on

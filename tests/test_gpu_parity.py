@@ -670,3 +670,35 @@ def test_init_codebook():
     kq.kq_init_codebook(to_dev(W), to_dev(sel), C0, ws)
     assert kq.kq_device_status(ws)[0] == 0
     assert bits_equal(C0.cpu().numpy(), oracle.gather_rows(W, sel))
+
+
+# --------------------------------------------------------------------------- kernel trace
+
+def test_trace_times_every_launch_of_a_fit():
+    # a fit on the tensor-core path, traced: one record per launch, in launch order,
+    # each with a kernel name and a positive device time (ResNet-18 conv5: n = 8192,
+    # K = 2048, multi-launch fit on the tensor-core path, no pilot pass)
+    lay, W, C0 = _layer(4, 4)
+    n, K = W.shape[0], C0.shape[0]
+    Wd, Cd = to_dev(W), to_dev(C0)
+    C = torch.empty_like(Cd)
+    idx = torch.empty(n, dtype=torch.int32, device=dev())
+    counts = torch.empty(K, dtype=torch.int32, device=dev())
+    ws = kq.workspace(n, K, dev())
+    kq.kq_fit_codebook(Wd, Cd, 2, C, idx, counts, None, ws)  # warm-up
+    torch.cuda.synchronize()
+    kq.kq_trace_start(256)
+    l0 = kq.kq_kernel_launches()
+    kq.kq_fit_codebook(Wd, Cd, 2, C, idx, counts, None, ws)
+    launched = kq.kq_kernel_launches() - l0
+    kq.kq_trace_stop()
+    kq.kq_fit_codebook(Wd, Cd, 1, C, idx, counts, None, ws)  # not recorded
+    trace = kq.kq_trace_read()
+    assert kq.kq_device_status(ws)[0] == 0
+    assert len(trace) == launched > 0
+    names = [name for name, _ in trace]
+    assert names.count("assign_tc_kernel") == 3  # two updates, then the final assignment
+    assert all(ms > 0 for _, ms in trace)
+    assert names[-1] == "histogram_kernel"  # the final assignment's cluster sizes
+    with pytest.raises(kq.KQError):
+        kq.kq_trace_start(0)
