@@ -71,6 +71,7 @@ typedef enum {
 
 /* kq_fit_codebook flags. */
 #define KQ_STOP_ON_STABLE 0x1
+#define KQ_FIT_PLAIN 0x2
 
 /* Human-readable name of a status. Never NULL. */
 const char *kq_status_string(kq_status s);
@@ -188,13 +189,24 @@ kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int
  *   W          n x 9 fp32 (device, 16-byte aligned)
  *   C_init     K x 9 fp32 (device); C_out K x 9 fp32 output (device; may equal C_init)
  *   iters      >= 0
- *   flags      0 or KQ_STOP_ON_STABLE: stop iterating once an assignment equals
- *              the previous one. That is a fixed point of the iteration (the
- *              update rebuilds the same codebook from the same clusters, bit for
- *              bit, and every later assignment repeats this one), so the outputs
- *              are exactly those of all `iters` iterations; the objective entries
- *              of the skipped steps repeat the last one computed. The call then
+ *   flags      0 or a combination of
+ *              KQ_STOP_ON_STABLE: stop iterating once an assignment equals the
+ *              previous one. That is a fixed point of the iteration (the update
+ *              rebuilds the same codebook from the same clusters, bit for bit, and
+ *              every later assignment repeats this one), so the outputs are
+ *              exactly those of all `iters` iterations; the objective entries of
+ *              the skipped steps repeat the last one computed. The call then
  *              synchronises `stream` once per iteration to read the test.
+ *              KQ_FIT_PLAIN: test every kernel against every codeword in every
+ *              assignment. Without it, fits of 4096 to 65536 codewords on the
+ *              tensor-core path prune, as Yinyang k-means does (Sec. 4.1): the
+ *              codebook is ordered by a k-d tree so that each 256-codeword tile
+ *              holds nearby codewords, every kernel keeps a lower bound on its
+ *              distance to each tile (lowered by the tile's codeword drift after
+ *              every update), and a tile that cannot hold a codeword as close as
+ *              the kernel's previous one is skipped for a whole block of kernels.
+ *              The first assignment then starts from each kernel's nearest
+ *              codeword in its k-d leaf. The outputs are identical either way.
  *   idx        n int32 output: the final assignment (device)
  *   counts     K int32 output: cluster sizes of the final assignment (device)
  *   objective  iters + 1 fp64 outputs (device) or NULL: Eq. 1 objective per step,

@@ -102,6 +102,13 @@ struct Ws {
     float *cpk;
     float *dist;
     int32_t *perm, *pcnt, *prev;
+    // pruned fit (yy_cap: the largest codebook the regions hold, 0 when absent)
+    int32_t yy_cap;
+    int32_t *cperm, *cpos, *kdtmp, *leaf;
+    unsigned long long *kdkey;
+    KdNode *nodes;
+    float *tdrift, *ydist;
+    unsigned char *yrec;
 };
 
 Ws carve(void *ws, int64_t n, int32_t K) {
@@ -122,6 +129,16 @@ Ws carve(void *ws, int64_t n, int32_t K) {
     w.perm = reinterpret_cast<int32_t *>(b + L.perm);
     w.pcnt = reinterpret_cast<int32_t *>(b + L.pcnt);
     w.prev = reinterpret_cast<int32_t *>(b + L.prev);
+    w.yy_cap = yy_sizes(K) ? K : 0;
+    w.cperm = reinterpret_cast<int32_t *>(b + L.cperm);
+    w.cpos = reinterpret_cast<int32_t *>(b + L.cpos);
+    w.kdtmp = reinterpret_cast<int32_t *>(b + L.kdtmp);
+    w.kdkey = reinterpret_cast<unsigned long long *>(b + L.kdkey);
+    w.nodes = reinterpret_cast<KdNode *>(b + L.kdnode);
+    w.tdrift = reinterpret_cast<float *>(b + L.tdrift);
+    w.yrec = reinterpret_cast<unsigned char *>(b + L.yrec);
+    w.ydist = reinterpret_cast<float *>(b + L.ydist);
+    w.leaf = reinterpret_cast<int32_t *>(b + L.leaf);
     return w;
 }
 
@@ -145,7 +162,7 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
         // distances in row order, whatever the grouping. With few tiles the four extra
         // launches cost more than they save, and rows stay in order.
         if (hint && K >= HINT_ORDER_MIN_K) {
-            KQ_TRY(launch_hint_permutation(hint, n, K, hint_counts, w.pcnt, w.perm, sms, s));
+            KQ_TRY(launch_hint_permutation(hint, n, K, nullptr, nullptr, hint_counts, w.pcnt, w.perm, sms, s));
             float *d = dist ? dist : w.dist;
             KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K, hint, w.perm, idx, d, nullptr, nb, w.hdr, s));
             KQ_TRY(launch_dist_block_sums(d, n, w.blocksum, nb, s));
@@ -159,6 +176,29 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
     return KQ_OK;
 }
 
+// One assignment of a pruned fit (kq_assign_tc.cu, kq_order.cu): the codebook
+// packed in k-d order, rows grouped by the codebook position of their hint, tiles
+// ruled out by the rows' bound records. read: the records are those of the
+// previous pass, whose codebook is Cprev (tile drifts from it); otherwise every
+// tile is processed and the records are written fresh. Without a hint (the fit's
+// first pass) the hints come from the k-d leaves, written into idx.
+kq_status run_assign_pruned(const float *W, int64_t n, const float *C, int32_t K, const int32_t *hint, int32_t *idx,
+                            int *nb, const Ws &w, int sms, cudaStream_t s, const int32_t *hint_counts,
+                            const float *Cprev, bool read) {
+    const TcYy st{w.cperm, w.cpos, w.tdrift, w.yrec, w.ydist, yy_stride(w.yy_cap), read ? 1 : 0};
+    KQ_TRY(launch_pack_codebook_tc(C, K, w.cpk, w.hdr, s, w.cperm, read ? Cprev : nullptr,
+                                   read ? w.tdrift : nullptr));
+    if (!hint) {
+        KQ_TRY(launch_kd_hints(W, n, w.nodes, K, w.cpk, w.cperm, w.leaf, w.pcnt, w.perm, idx, sms, s));
+        hint = idx;
+        hint_counts = nullptr;
+    }
+    KQ_TRY(launch_hint_permutation(hint, n, K, w.cpos, w.cperm, hint_counts, w.pcnt, w.perm, sms, s));
+    KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K, hint, w.perm, idx, w.dist, nullptr, nb, w.hdr, s, &st));
+    KQ_TRY(launch_dist_block_sums(w.dist, n, w.blocksum, nb, s));
+    return KQ_OK;
+}
+
 // The k-means fit of kq_fit_codebook on carved workspace regions (sized for at
 // least K codewords). objective: iters + 1 device doubles or null; final_obj: one
 // device double receiving the objective of the final assignment, or null.
@@ -169,7 +209,7 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
 // written directly. iters_run (host, nullable): the codebook updates performed.
 kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int32_t iters, float *C_out,
                   int32_t *idx, int32_t *counts, double *objective, double *final_obj, const Ws &w, int sms,
-                  cudaStream_t s, bool stop_on_stable = false, int32_t *iters_run = nullptr) {
+                  cudaStream_t s, bool stop_on_stable = false, int32_t *iters_run = nullptr, bool plain = false) {
     const size_t cbytes = (size_t)K * D * sizeof(float);
     kq_status st;
     KQ_TRY(launch_update_prepare(nullptr, K, w.acc, w.hdr, false, s));
@@ -177,6 +217,13 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
     KQ_TRY(cudaMemcpyAsync(w.cbuf0, C_init, cbytes, cudaMemcpyDeviceToDevice, s));
     float *cur = w.cbuf0, *nxt = w.cbuf1;
     int nb = 0;
+    // pruned assignments: the codebook's k-d order is taken once, from C_init
+    const bool pruned = !plain && K <= w.yy_cap && yy_sizes(K) && tc_eligible(n, K, sms);
+    if (pruned) KQ_TRY(launch_codebook_order(cur, K, w.cperm, w.cpos, w.kdtmp, w.kdkey, w.nodes, w.hdr, s));
+    auto assign = [&](int32_t t, const int32_t *hint, int32_t *out, const int32_t *hint_counts) -> kq_status {
+        if (pruned) return run_assign_pruned(W, n, cur, K, hint, out, &nb, w, sms, s, hint_counts, nxt, t > 0);
+        return run_assign(W, n, cur, K, hint, out, nullptr, &nb, w, sms, s, hint_counts);
+    };
     // Assignment t goes to idx when iters - t is even, else to the workspace's other
     // index buffer, so the final one lands in idx. Iteration t > 0 starts every row
     // from assignment t - 1 (warm start; the update wrote its cluster sizes), and its
@@ -185,9 +232,7 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
     for (int32_t t = 0; t < iters; ++t) {
         int32_t *out = buf(t);
         const int32_t *hint = t > 0 ? buf(t - 1) : nullptr;
-        if ((st = run_assign(W, n, cur, K, hint, out, nullptr, &nb, w, sms, s, t > 0 ? counts : nullptr)) !=
-            KQ_OK)
-            return st;
+        if ((st = assign(t, hint, out, t > 0 ? counts : nullptr)) != KQ_OK) return st;
         if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
         if (t == 0) {
             KQ_TRY(launch_accumulate(W, n, out, K, w.hdr, w.acc, false, sms, s));
@@ -214,8 +259,7 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
         cur = nxt;
         nxt = tmp;
     }
-    if ((st = run_assign(W, n, cur, K, iters > 0 ? buf(iters - 1) : nullptr, idx, nullptr, &nb, w, sms, s,
-                         iters > 0 ? counts : nullptr)) != KQ_OK)
+    if ((st = assign(iters, iters > 0 ? buf(iters - 1) : nullptr, idx, iters > 0 ? counts : nullptr)) != KQ_OK)
         return st;
     if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + iters, s));
     if (final_obj) KQ_TRY(launch_sum_blocks(w.blocksum, nb, final_obj, s));
@@ -376,7 +420,7 @@ kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_i
                           float *C_out, int32_t *idx, int32_t *counts, double *objective, int32_t *iters_run,
                           void *ws, size_t ws_bytes, kq_stream_t stream) {
     if (!sizes_ok(n, K) || !W || !C_init || !C_out || !idx || !counts) return KQ_ERR_INVALID_ARG;
-    if (iters < 0 || (flags & ~KQ_STOP_ON_STABLE) != 0) return KQ_ERR_INVALID_ARG;
+    if (iters < 0 || (flags & ~(KQ_STOP_ON_STABLE | KQ_FIT_PLAIN)) != 0) return KQ_ERR_INVALID_ARG;
     if (!aligned(W, 16) || !aligned(C_init, 4) || !aligned(C_out, 4) || !aligned(idx, 4) || !aligned(counts, 4) ||
         !aligned(objective, 8))
         return KQ_ERR_ALIGNMENT;
@@ -401,7 +445,8 @@ kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_i
         }
         return KQ_OK;
     }
-    return run_fit(W, n, K, C_init, iters, C_out, idx, counts, objective, nullptr, w, sms, s, stop, iters_run);
+    return run_fit(W, n, K, C_init, iters, C_out, idx, counts, objective, nullptr, w, sms, s, stop, iters_run,
+                   (flags & KQ_FIT_PLAIN) != 0);
 }
 
 kq_status kq_search_codebook_size(const float *W, int64_t n, const int64_t *sel, int32_t sel_len, double alpha,

@@ -102,12 +102,12 @@ constexpr int TC_ROWS = TC_M * TC_RT;      // kernels per CTA
 constexpr int32_t TC_LGROUP_MINK = 1024;
 constexpr int32_t TC_LGROUP_MAXK = 4096;
 constexpr int TC_LBINS = TC_LGROUP_MAXK / 32 + 1;
-constexpr int TC_N = 256;                  // codewords per tile (N of every MMA)
+// TC_N codewords per tile (N of every MMA), TC_KD = K of the GEMM in fp16 elements
+// (hi/lo split, see top of file); a tile is TC_TILE_H bytes of fp16 operands and
+// the tile's codewords in fp32, TC_TILE_BYTES = 25 KiB streamed (kq_internal.cuh).
 constexpr int TC_HALF = TC_N / 2;          // codewords of a tile one epilogue thread tests
-constexpr int TC_KD = 32;                  // K of the GEMM in fp16 elements (hi/lo split, see top of file)
-constexpr int TC_STAGES = 6;
-constexpr int TC_TILE_H = TC_N * TC_KD * 2;      // 16 KiB of fp16 operands per codeword tile
-constexpr int TC_TILE_BYTES = TC_TILE_H + TC_N * D * 4;  // + the tile's codewords in fp32: 25 KiB streamed
+constexpr int TC_STAGES = 6;               // tile ring of the plain kernel
+constexpr int TC_STAGES_YY = 4;            // and of the pruned one (its records take the rest; as fast)
 constexpr int TC_A_BYTES = TC_M * TC_KD * 2;     // 8 KiB per row tile
 constexpr int TC_THREADS = 352;
 constexpr int TC_EPI_WARP0 = 3;            // first epilogue warp (0: producer, 1-2: MMA issuers)
@@ -282,19 +282,20 @@ __device__ __forceinline__ float warp_max_bits(float m) {
     return m;
 }
 
-// Codeword k of the padded codebook (k < Kpad) into its tile: the fp16 operands of
-// beta c, then c in fp32 for the exact path; returns the scaled bounds of
-// pack_codebook_kernel (cmax, hmax, qmax; NaN for a non-finite codeword, 0 for
-// padding). Padding codewords get c = 0 and -h = -inf, so their g is -inf.
-__device__ __forceinline__ void pack_codeword_tc(const float *__restrict__ C, int32_t K, int32_t k, float beta,
-                                                 float *__restrict__ Cpk, Header *hdr, float &cmax, float &hmax,
-                                                 float &qmax) {
+// Codeword k into position p of the padded codebook (p < Kpad; p >= K: padding):
+// the fp16 operands of beta c, then c in fp32 for the exact path; returns the
+// scaled bounds of pack_codebook_kernel (cmax, hmax, qmax; NaN for a non-finite
+// codeword, 0 for padding). Padding codewords get c = 0 and -h = -inf, so their g
+// is -inf.
+__device__ __forceinline__ void pack_codeword_tc(const float *__restrict__ C, int32_t K, int32_t k, int32_t p,
+                                                 float beta, float *__restrict__ Cpk, Header *hdr, float &cmax,
+                                                 float &hmax, float &qmax) {
     float c[D], c32[D];
     float mh = __int_as_float(0xff800000);  // -h; -inf for padding codewords
 #pragma unroll
     for (int j = 0; j < D; ++j) c[j] = c32[j] = 0.f;
     cmax = hmax = qmax = 0.f;
-    if (k < K) {
+    if (p < K) {
         bool ok = true;
         float s = 0.f, c2lo = 0.f, c2hi = 0.f;
 #pragma unroll
@@ -317,14 +318,14 @@ __device__ __forceinline__ void pack_codeword_tc(const float *__restrict__ C, in
             cmax = hmax = qmax = __int_as_float(0x7fc00000);  // NaN: disables the test
         }
     }
-    const int kl = k % TC_N;
+    const int kl = p % TC_N;
     float v[TC_KD];
     tc_row(c, mh, false, v);
     if (!(mh >= -3.402823466e38f)) v[19] = 0.f;  // padding: -inf already sits in the hi slot
     v[TC_SLOT_T0] = kl < TC_HALF ? 1.f : 0.f;
     v[TC_SLOT_R] = 1.f;
     v[TC_SLOT_T1] = kl < TC_HALF ? 0.f : 1.f;
-    unsigned char *tile = reinterpret_cast<unsigned char *>(Cpk) + (int64_t)(k / TC_N) * TC_TILE_BYTES;
+    unsigned char *tile = reinterpret_cast<unsigned char *>(Cpk) + (int64_t)(p / TC_N) * TC_TILE_BYTES;
     tc_store_row(tile, kl, v);
     float *cw = reinterpret_cast<float *>(tile + TC_TILE_H) + kl * D;
 #pragma unroll
@@ -352,13 +353,44 @@ __global__ void __launch_bounds__(256) codebook_norm_tc_kernel(const float *__re
 
 // Packs beta C into tensor-core tiles (Kpad codewords, Kpad a multiple of TC_N) and
 // reduces the scaled codebook bounds into hdr->cb_*; beta from hdr->cb_craw.
+// cperm (nullable): position p holds codeword cperm[p]. Cprev, tdrift (nullable):
+// tdrift[tile] = the largest |C[k] - Cprev[k]| (rounded up; NaN if not finite) over
+// the tile's codewords (one CTA of 256 threads per tile).
 __global__ void __launch_bounds__(256) pack_codebook_tc_kernel(const float *__restrict__ C, int32_t K, int32_t Kpad,
-                                                               float *__restrict__ Cpk, Header *hdr) {
-    const int k = blockIdx.x * blockDim.x + threadIdx.x;
+                                                               float *__restrict__ Cpk, Header *hdr,
+                                                               const int32_t *__restrict__ cperm,
+                                                               const float *__restrict__ Cprev,
+                                                               float *__restrict__ tdrift) {
+    const int p = blockIdx.x * blockDim.x + threadIdx.x;
     const float beta = tc_scale(__uint_as_float(__ldcg(&hdr->cb_craw)));
     float cmax = 0.f, hmax = 0.f, qmax = 0.f;
-    if (k < Kpad) pack_codeword_tc(C, K, k, beta, Cpk, hdr, cmax, hmax, qmax);
+    const int32_t k = (cperm != nullptr && p < K) ? cperm[p] : p;
+    if (p < Kpad) pack_codeword_tc(C, K, k, p, beta, Cpk, hdr, cmax, hmax, qmax);
     publish_bounds_tc(cmax, hmax, qmax, hdr);
+    if (tdrift) {
+        __shared__ float s_dr[8];
+        float dr = 0.f;
+        if (p < K) {
+            float s2 = 0.f;
+            bool ok = true;
+#pragma unroll
+            for (int u = 0; u < D; ++u) {
+                const float dlt = C[(int64_t)k * D + u] - Cprev[(int64_t)k * D + u];
+                ok &= isfinite(dlt);
+                s2 = __fadd_ru(s2, __fmul_ru(dlt, dlt));
+            }
+            // |fl(a - b)| may be below |a - b| by half an ulp: one more ulp per coordinate
+            dr = ok ? __fmul_ru(__fsqrt_ru(s2), 1.0000002384185791f) : __int_as_float(0x7fc00000);
+        }
+        dr = warp_max_bits(dr);
+        if ((threadIdx.x & 31) == 0) s_dr[threadIdx.x >> 5] = dr;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float m = 0.f;
+            for (int w = 0; w < 8; ++w) m = max_bits(m, s_dr[w]);
+            tdrift[blockIdx.x] = m;
+        }
+    }
 }
 
 // Both steps in one CTA, for small codebooks (one launch instead of two).
@@ -383,7 +415,7 @@ __global__ void __launch_bounds__(TC_PACK_SMALL_THREADS) pack_codebook_tc_small_
     float cmax = 0.f, hmax = 0.f, qmax = 0.f;
     for (int k = threadIdx.x; k < Kpad; k += TC_PACK_SMALL_THREADS) {
         float a, b, c;
-        pack_codeword_tc(C, K, k, beta, Cpk, hdr, a, b, c);
+        pack_codeword_tc(C, K, k, k, beta, Cpk, hdr, a, b, c);
         cmax = max_bits(cmax, a);
         hmax = max_bits(hmax, b);
         qmax = max_bits(qmax, c);
@@ -424,10 +456,11 @@ __device__ __forceinline__ float direct_distance(const float (&x)[D], const floa
     return acc;
 }
 
-struct TcShared {
+template <int NST>
+struct __align__(16) TcShared {
     unsigned char a[TC_RT][TC_A_BYTES];             // row tiles (tensor-core layout)
-    unsigned char b[TC_STAGES][TC_TILE_BYTES];      // codeword tiles
-    unsigned long long full[TC_STAGES], empty[TC_STAGES], tfull[TC_RT], tempty[TC_RT], done;
+    unsigned char b[NST][TC_TILE_BYTES];            // codeword tiles
+    unsigned long long full[NST], empty[NST], tfull[TC_RT], tempty[TC_RT], done;
     uint32_t tmem_base;
     uint32_t abort_flag;
     float xs[TC_ROWS][D];    // the CTA's kernels and test constants, read on the
@@ -442,27 +475,94 @@ struct TcShared {
     double wsum[TC_EPI_WARPS / 2][TC_RT];
 };
 
+// Pruned kernel only (after TcShared; then the records, TC_ROWS x stride bytes).
+struct __align__(16) TcYyShared {
+    unsigned long long xfull[4][2], xempty[4][2];  // hand-over of the second half's bound, per lane quarter
+    uint32_t mask[YY_MAX_TILES / 32];              // tiles this CTA processes
+    int32_t nt;                                    // their number
+    int32_t pad_;
+    uint16_t tl[YY_MAX_TILES];                     // the tiles, in processing order
+    float tmax[2][TC_ROWS];                        // per half row: largest T' an MMA may have read
+    float tabs[2][TC_ROWS];                        // and largest |T'|
+    float xch[2][TC_RT][TC_M];                     // the second half's bound, for the first half's thread
+    float drift[YY_MAX_TILES];                     // per tile: largest codeword move since the last pass
+    float dprev[TC_ROWS];                          // each slot's record distance (when read)
+    float fin[TC_ROWS];                            // each slot's final best distance
+};
+
+constexpr int YY_DELTA_SHIFT = 10;  // bound step: 2^(e - 10) for an initial codebook whose largest norm is f 2^e
+constexpr float YY_ONE_M_G11 = 0.99999904632568359375f;  // 1 - 8 * 2^-23 <= 1 - gamma_11 <= 1 / (1 + gamma_11)
+constexpr float TWO_M16 = 1.52587890625e-05f;            // 2^-16
+
+// Record byte of a slack x (a lower bound of distance minus a distance reference,
+// in units of the bound step: inv = 1 / step): floor(x / step) clamped to [0, 255],
+// 0 for a negative or NaN x.
+__device__ __forceinline__ uint32_t yy_encode(float x, float inv) {
+    const float v = __fmul_rd(x, inv);
+    if (!(v >= 1.f)) return 0u;
+    return v >= 255.f ? 255u : (uint32_t)v;
+}
+
 // Named barrier among the 256 epilogue threads (warps 3-10).
 __device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
 
+// The tile holding the hinted codeword of slot row0's row (the pruned kernel reading
+// records streams it before the tile list is known); 0 without a usable hint.
+__device__ __forceinline__ int yy_first_tile(const int32_t *hint, const int32_t *perm, int64_t row0, int64_t n,
+                                             int32_t K, const int32_t *cpos) {
+    const int64_t r0 = perm ? (int64_t)__ldg(perm + row0) : row0;
+    const int32_t h = (hint != nullptr && (uint64_t)r0 < (uint64_t)n) ? hint[r0] : -1;
+    return (uint32_t)h < (uint32_t)K ? __ldg(cpos + h) / TC_N : 0;
+}
+
+// YY: the pruned kernel of the fit (yy: its state). The codebook is packed in the
+// order yy.cperm (tile g = positions [256 g, 256 g + 256)); indices and the tie rule
+// stay those of the original numbering. Every row keeps a record of one byte per
+// tile: q with q * step + dprev <= the distance from the row to every codeword of
+// the tile (dprev <= its distance to every codeword), written at the end of each
+// pass and, in the next pass, lowered by the tile's drift (triangle inequality). A
+// tile whose bound proves every codeword farther than the row's hinted codeword for
+// all 256 rows of the CTA is not streamed, multiplied or tested at all; the answer
+// is the same, since no skipped codeword could improve or tie the row's best.
+template <bool YY>
 __global__ void __launch_bounds__(TC_THREADS, 1)
 assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict__ C, const float *__restrict__ Cpk,
                  int32_t K, int32_t ntiles, const int32_t *hint, const int32_t *__restrict__ perm, int32_t *idx,
-                 float *__restrict__ dist, double *__restrict__ blocksum, Header *hdr) {
+                 float *__restrict__ dist, double *__restrict__ blocksum, Header *hdr, TcYy yy) {
+    constexpr int NST = YY ? TC_STAGES_YY : TC_STAGES;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
-    TcShared &S = *reinterpret_cast<TcShared *>(smem_raw);
+    TcShared<NST> &S = *reinterpret_cast<TcShared<NST> *>(smem_raw);
+    TcYyShared &Y = *reinterpret_cast<TcYyShared *>(smem_raw + sizeof(TcShared<NST>));  // YY only
+    unsigned char *yrec = smem_raw + sizeof(TcShared<NST>) + sizeof(TcYyShared);      // YY only
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     volatile uint32_t *abort_flag = &S.abort_flag;
     uint32_t *status = &hdr->status;
     const float beta = tc_scale(__uint_as_float(__ldcg(&hdr->cb_craw)));  // as pack_codebook_tc_kernel
     const float beta2 = beta * beta;
+    const float inv_beta = 1.f / beta;  // exact: a power of two
+    const int64_t row0 = (int64_t)blockIdx.x * TC_ROWS;
+    // pruned kernel: bound step (fixed for the fit) and whether the records are valid
+    float ystep = 0.f, yinv = 0.f;
+    bool yread = false;
+    if (YY) {
+        const float cn = __uint_as_float(__ldcg(&hdr->yy_cnorm));
+        if (cn > 0.f && cn <= 3.402823466e38f) {
+            int e;
+            frexpf(cn, &e);
+            const int ex = max(-100, min(100, e - YY_DELTA_SHIFT));
+            ystep = ldexpf(1.f, ex);
+            yinv = ldexpf(1.f, -ex);
+        }
+        yread = yy.read != 0 && ystep > 0.f;
+    }
 
     // ---- barriers first: the producer starts streaming the first codeword tiles
     // while the epilogue threads set up their rows (the other roles wait for the
-    // barriers only after the CTA barrier below)
-    const int pre = ntiles < TC_STAGES ? ntiles : TC_STAGES;
+    // barriers only after the CTA barrier below). The pruned kernel reading records
+    // streams one tile early: the one holding the first slot's hinted codeword.
+    const int pre = (YY && yread) ? 1 : (ntiles < NST ? ntiles : NST);
     if (tid == 0) {
-        for (int s = 0; s < TC_STAGES; ++s) {
+        for (int s = 0; s < NST; ++s) {
             mbar_init((uint32_t)__cvta_generic_to_shared(&S.full[s]), 1);
             mbar_init((uint32_t)__cvta_generic_to_shared(&S.empty[s]), TC_EPI_WARPS);
         }
@@ -471,17 +571,26 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
             mbar_init((uint32_t)__cvta_generic_to_shared(&S.tempty[t]), TC_EPI_WARPS);
         }
         mbar_init((uint32_t)__cvta_generic_to_shared(&S.done), TC_RT);
+        if (YY) {
+            for (int qq = 0; qq < 4; ++qq)
+                for (int b = 0; b < 2; ++b) {
+                    mbar_init((uint32_t)__cvta_generic_to_shared(&Y.xfull[qq][b]), 1);
+                    mbar_init((uint32_t)__cvta_generic_to_shared(&Y.xempty[qq][b]), 1);
+                }
+        }
         S.abort_flag = 0u;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // initialised barriers -> bulk copies
+        const int g0 = (YY && yread) ? yy_first_tile(hint, perm, row0, n, K, yy.cpos) : 0;
         for (int i = 0; i < pre; ++i) {
+            const int g = (YY && yread) ? g0 : i;
             const uint32_t fb = (uint32_t)__cvta_generic_to_shared(&S.full[i]);
             asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb), "r"(TC_TILE_BYTES)
                          : "memory");
             asm volatile(
                 "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
                     (uint32_t)__cvta_generic_to_shared(S.b[i])),
-                "l"(reinterpret_cast<const unsigned char *>(Cpk) + (int64_t)i * TC_TILE_BYTES), "r"(TC_TILE_BYTES),
+                "l"(reinterpret_cast<const unsigned char *>(Cpk) + (int64_t)g * TC_TILE_BYTES), "r"(TC_TILE_BYTES),
                 "r"(fb)
                 : "memory");
         }
@@ -501,9 +610,13 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
         bi[t] = 0;
         known[t] = -1;
     }
-    const bool lgroup = hint != nullptr && perm == nullptr && K >= TC_LGROUP_MINK && K <= TC_LGROUP_MAXK;
+    const bool lgroup = !YY && hint != nullptr && perm == nullptr && K >= TC_LGROUP_MINK && K <= TC_LGROUP_MAXK;
     if (epi) {
-        const int64_t row0 = (int64_t)blockIdx.x * TC_ROWS;
+        if (YY) {  // cleared before the epilogue barrier that precedes their first use
+            const int et = tid - TC_EPI_WARP0 * 32;
+            if (et < YY_MAX_TILES / 32) Y.mask[et] = 0u;
+            for (int g = et; g < ntiles; g += TC_EPI_WARPS * 32) Y.drift[g] = yread ? __ldg(yy.tdrift + g) : 0.f;
+        }
         if (lgroup) {
             // CTA-local grouping (counting sort of the CTA's rows by hint chunk; the
             // order within a chunk is free): a warp's rows then share a few chunks,
@@ -621,11 +734,16 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                 const float d = direct_distance(x, ch[t]);
                 if (d < best[t]) {
                     best[t] = d;
-                    bi[t] = known[t] = hv[t];
+                    bi[t] = hv[t];
+                    known[t] = YY ? __ldg(yy.cpos + hv[t]) : hv[t];  // known: the codebook position
                     ev = !tc_shift(rc, d, beta2, tp);
                 }
             }
             every |= (ev ? 1u : 0u) << t;
+            if (YY) {
+                Y.tmax[hsel][rloc] = ev ? -TC_T_EVERY : tp;
+                Y.tabs[hsel][rloc] = ev ? TC_T_EVERY : fabsf(tp);
+            }
             if (hsel == 0) {  // both halves start from the same state; one writes it
                 S.prow[rloc] = (int32_t)row[t];
 #pragma unroll
@@ -638,6 +756,75 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                 a[TC_SLOT_T0] = a[TC_SLOT_T1] = ev ? TC_T_EVERY : -tp;
                 a[TC_SLOT_R] = -rc.R;
                 tc_store_row(S.a[t], r, a);
+            }
+        }
+        if (YY) {
+            // The tiles this CTA needs: thread (hsel, r) reads the record of the row in
+            // row tile hsel (its best so far is the hinted codeword's exact distance B);
+            // tile g can be skipped for that row when the record's bound, lowered by
+            // the tile's drift, proves every codeword of g farther than B.
+            epi_sync();  // mask cleared, drifts staged
+            const int sl = hsel * TC_M + r;
+            const int64_t rw = row[hsel];
+            const float B = best[hsel];
+            const bool all = !yread || !(B <= 3.402823466e38f);  // no valid record or no finite hint distance
+            const float dp = (yread && rw < n) ? yy.dprev[rw] : 0.f;
+            if (yread) Y.dprev[sl] = dp;
+            const uint4 *src = reinterpret_cast<const uint4 *>(yy.rec + (rw < n ? rw : 0) * (int64_t)yy.stride);
+            uint4 *dst = reinterpret_cast<uint4 *>(yrec + sl * yy.stride);
+            for (int w = 0; w < (ntiles + 31) / 32; ++w) {
+                uint32_t need = 0u;
+                if (rw < n) {
+                    if (all) {
+                        need = 0xffffffffu;
+                    } else {
+#pragma unroll
+                        for (int h2 = 0; h2 < 2; ++h2) {
+                            const int c = 2 * w + h2;
+                            if (c * 16 >= yy.stride) continue;  // a stride of 16 (mod 32) bytes
+                            const uint4 v = src[c];
+                            dst[c] = v;
+#pragma unroll
+                            for (int u = 0; u < 16; ++u) {
+                                const uint32_t wsel = (u >> 2) == 0 ? v.x : (u >> 2) == 1 ? v.y : (u >> 2) == 2 ? v.z : v.w;
+                                const float qv = (float)((wsel >> (8 * (u & 3))) & 255u);
+                                const float lb = __fsub_rd(__fadd_rd(__fmul_rd(qv, ystep), dp), Y.drift[c * 16 + u < ntiles ? c * 16 + u : 0]);
+                                const bool skip = lb > 0.f && __fmul_rd(__fmul_rd(lb, lb), YY_ONE_M_G11) > B;
+                                need |= (skip ? 0u : 1u) << (16 * h2 + u);
+                            }
+                        }
+                    }
+                    const int left = ntiles - 32 * w;
+                    if (left < 32) need &= (1u << left) - 1u;
+                }
+                need = __reduce_or_sync(0xffffffffu, need);
+                if (lane == 0 && need) atomicOr(&Y.mask[w], need);
+            }
+            epi_sync();
+            if (warp == TC_EPI_WARP0) {
+                // the list: the early tile first (read mode), then the others in order;
+                // lane l takes tiles 8 l .. 8 l + 7
+                const int g0 = yread ? yy_first_tile(hint, perm, row0, n, K, yy.cpos) : -1;  // as streamed
+                uint32_t bits = (Y.mask[lane >> 2] >> ((lane & 3) * 8)) & 0xffu;
+                if (g0 >= 0 && (g0 >> 3) == lane) bits &= ~(1u << (g0 & 7));
+                const int cnt = __popc(bits);
+                int incl = cnt;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const int y2 = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += y2;
+                }
+                int pos = (g0 >= 0 ? 1 : 0) + incl - cnt;
+                while (bits) {
+                    const int b = __ffs(bits) - 1;
+                    bits &= bits - 1u;
+                    Y.tl[pos++] = (uint16_t)(lane * 8 + b);
+                }
+                if (lane == 31) Y.nt = (g0 >= 0 ? 1 : 0) + incl;
+                if (lane == 0 && g0 >= 0) {
+                    Y.tl[0] = (uint16_t)g0;
+                    atomicOr(&Y.mask[g0 >> 5], 1u << (g0 & 31));  // the mask now marks every processed tile
+                }
             }
         }
     }
@@ -655,13 +842,15 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = S.tmem_base;
+    const int nt = YY ? Y.nt : ntiles;  // tiles this CTA processes (the list's length)
 
     if (warp == 0) {
         // ---- producer (lane 0)
         if (lane == 0) {
-            for (int i = pre; i < ntiles; ++i) {  // tiles 0 .. pre - 1 are on their way
-                const int s = i % TC_STAGES;
-                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.empty[s]), ((i / TC_STAGES) - 1) & 1, abort_flag,
+            for (int i = pre; i < nt; ++i) {  // list entries 0 .. pre - 1 are on their way
+                const int s = i % NST;
+                const int g = YY ? (int)Y.tl[i] : i;
+                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.empty[s]), ((i / NST) - 1) & 1, abort_flag,
                                status))
                     break;
                 const uint32_t fb = (uint32_t)__cvta_generic_to_shared(&S.full[s]);
@@ -670,7 +859,7 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                 asm volatile(
                     "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
                         (uint32_t)__cvta_generic_to_shared(S.b[s])),
-                    "l"(reinterpret_cast<const unsigned char *>(Cpk) + (int64_t)i * TC_TILE_BYTES), "r"(TC_TILE_BYTES),
+                    "l"(reinterpret_cast<const unsigned char *>(Cpk) + (int64_t)g * TC_TILE_BYTES), "r"(TC_TILE_BYTES),
                     "r"(fb)
                     : "memory");
             }
@@ -682,9 +871,9 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
             constexpr uint32_t idesc = tc_idesc(TC_M, TC_N);
             const uint32_t a0 = (uint32_t)__cvta_generic_to_shared(S.a[t]);
             const uint32_t dcol = tmem + (uint32_t)(t * TC_N);
-            for (int i = 0; i < ntiles; ++i) {
-                const int s = i % TC_STAGES;
-                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.full[s]), (i / TC_STAGES) & 1, abort_flag, status))
+            for (int i = 0; i < nt; ++i) {
+                const int s = i % NST;
+                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.full[s]), (i / NST) & 1, abort_flag, status))
                     break;
                 // the accumulator is free once the epilogue read tile i - 1
                 if (i >= 1 &&
@@ -734,8 +923,17 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
         // or tie the running best.
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         bool go = true;
-        for (int i = 0; i < ntiles && go; ++i) {
-            const int st = i % TC_STAGES;
+        for (int i = 0; i < nt && go; ++i) {
+            const int st = i % NST;
+            const int gb = (YY ? (int)Y.tl[i] : i) * TC_N;  // codebook position of the tile's first codeword
+            float own[TC_RT];                                // pruned: this half's bound per row tile
+            // pruned, second half: its exchange slot must have been read (tile i - 2)
+            if (YY && hsel == 1 && i >= 2 &&
+                !mbar_wait((uint32_t)__cvta_generic_to_shared(&Y.xempty[q][i & 1]), ((i >> 1) - 1) & 1, abort_flag,
+                           status)) {
+                go = false;
+                break;
+            }
 #pragma unroll
             for (int t = 0; t < TC_RT; ++t) {
                 if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.tfull[t]), i & 1, abort_flag, status)) {
@@ -774,14 +972,14 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                         // the running best itself needs no decision (in a warm start it
                         // is almost always the only codeword that passes)
                         uint32_t mask = !need ? 0u : (ev ? 0xffffffffu : ~sign_mask32(v[c]));
-                        const int kloc = known[t] - (i * TC_N + hsel * TC_HALF + 32 * c);
+                        const int kloc = known[t] - (gb + hsel * TC_HALF + 32 * c);
                         if ((uint32_t)kloc < 32u) mask &= ~(1u << kloc);
                         while (mask) {
                             const int j = __ffs(mask) - 1;
                             mask &= mask - 1u;
                             const int kl = hsel * TC_HALF + 32 * c + j;
-                            const int32_t k = i * TC_N + kl;
-                            if (k >= K) break;
+                            const int32_t p = gb + kl;  // codebook position (the index unless pruned)
+                            if (p >= K) break;
                             float xr[D], cw[D];
                             const float *c32 = reinterpret_cast<const float *>(tile + TC_TILE_H) + kl * D;
 #pragma unroll
@@ -790,10 +988,15 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                                 cw[u] = c32[u];
                             }
                             const float d = direct_distance(xr, cw);
-                            if (d < best[t] || (d == best[t] && k < bi[t])) {
-                                best[t] = d;
-                                bi[t] = known[t] = k;
-                                moved = true;
+                            if (d <= best[t]) {
+                                // the lowest original index wins a tie, whatever the packing order
+                                const int32_t k = YY ? __ldg(yy.cperm + p) : p;
+                                if (d < best[t] || k < bi[t]) {
+                                    best[t] = d;
+                                    bi[t] = k;
+                                    known[t] = p;
+                                    moved = true;
+                                }
                             }
                         }
                     }
@@ -804,7 +1007,53 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                         *reinterpret_cast<uint16_t *>(&S.a[t][tc_offset(r, hsel ? TC_SLOT_T1 : TC_SLOT_T0)]) =
                             (uint16_t)f16_bits(e2 ? TC_T_EVERY : -tp);
                         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // for later MMAs
+                        if (YY) {
+                            const float tn = e2 ? -TC_T_EVERY : tp;
+                            Y.tmax[hsel][rloc] = fmaxf(Y.tmax[hsel][rloc], tn);
+                            Y.tabs[hsel][rloc] = fmaxf(Y.tabs[hsel][rloc], fabsf(tn));
+                        }
                     }
+                }
+                if (YY) {
+                    // a lower bound on the distance from the row to every codeword of this
+                    // half tile: D >= X2lo - Qmax - 2 e and e <= g + R + T' + E for each of
+                    // them (scaled units), with g at most the half's maximum m and T' at most
+                    // the largest value an MMA may have read
+                    const int rloc = t * TC_M + r;
+                    const RowConst rq = S.rc[rloc];
+                    const float E = __fadd_ru(__fmul_ru(TWO_M16, __fadd_ru(rq.k1, Y.tabs[hsel][rloc])),
+                                              __fmul_ru(0.5f, rq.k2));
+                    const float up = __fadd_ru(__fadd_ru(__fadd_ru(m, rq.R), Y.tmax[hsel][rloc]), E);
+                    const float lbD = __fsub_rd(rq.k0, __fmul_ru(2.f, up));  // NaN for rows tested exactly
+                    own[t] = __fmul_rd(__fsqrt_rd(fmaxf(lbD, 0.f)), inv_beta);
+                    if (hsel == 1) Y.xch[i & 1][t][r] = own[t];
+                }
+            }
+            if (YY && go) {
+                // the row's bound for the tile is the smaller of its two halves': the
+                // second half hands its value over, the first half records the byte
+                // (as slack over its current best, which is at least the final one)
+                if (hsel == 1) {
+                    __syncwarp();
+                    if (lane == 0)
+                        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(
+                                         (uint32_t)__cvta_generic_to_shared(&Y.xfull[q][i & 1]))
+                                     : "memory");
+                } else if (mbar_wait((uint32_t)__cvta_generic_to_shared(&Y.xfull[q][i & 1]), (i >> 1) & 1,
+                                     abort_flag, status)) {
+#pragma unroll
+                    for (int t = 0; t < TC_RT; ++t) {
+                        const float lb = fminf(own[t], Y.xch[i & 1][t][r]);
+                        const float dref = __fsqrt_ru(__fmul_ru(best[t], INV_ONE_M_G11_TC));
+                        yrec[(t * TC_M + r) * yy.stride + gb / TC_N] = (unsigned char)yy_encode(__fsub_rd(lb, dref), yinv);
+                    }
+                    __syncwarp();
+                    if (lane == 0)
+                        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(
+                                         (uint32_t)__cvta_generic_to_shared(&Y.xempty[q][i & 1]))
+                                     : "memory");
+                } else {
+                    go = false;
                 }
             }
             __syncwarp();
@@ -842,6 +1091,7 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
             }
             // the partial sum runs over the CTA's rows in row order whatever the grouping
             S.rowbest[lgroup ? S.lslot[rloc] : rloc] = row < n ? best[t] : 0.f;
+            if (YY) Y.fin[rloc] = best[t];
         }
         asm volatile("bar.sync 2, 128;" ::: "memory");  // the 128 threads of the first half
 #pragma unroll
@@ -863,6 +1113,41 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TC_COLS) : "memory");
     }
+    if (YY && epi) {
+        // Records for the next pass, relative to this pass's final best: processed
+        // tiles keep the byte of this pass (its slack over a best at least the final
+        // one); the others take last pass's bound lowered by the tile's drift.
+        const int sl = hsel * TC_M + r;
+        const int64_t rw = S.prow[sl];
+        const bool valid = *abort_flag == 0u;  // after a wait gave up, records start over (no bound)
+        if (rw < n) {
+            const float Df = Y.fin[sl];
+            const bool fin = valid && Df <= 3.402823466e38f;
+            const float dpn = fin ? __fsqrt_rd(__fmul_rd(Df, YY_ONE_M_G11)) : 0.f;  // <= the distance to any codeword
+            const float dref = fin ? __fsqrt_ru(__fmul_ru(Df, INV_ONE_M_G11_TC)) : __int_as_float(0x7f800000);
+            const float dpo = yread ? Y.dprev[sl] : 0.f;
+            const unsigned char *rs = yrec + sl * yy.stride;
+            uint4 *dst = reinterpret_cast<uint4 *>(yy.rec + rw * (int64_t)yy.stride);
+            for (int c = 0; c < yy.stride / 16; ++c) {
+                uint32_t wv[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+                for (int u = 0; u < 16; ++u) {
+                    const int g = c * 16 + u;
+                    uint32_t b = 0u;
+                    if (g < ntiles && fin) {
+                        b = rs[g];
+                        if (!((Y.mask[g >> 5] >> (g & 31)) & 1u)) {
+                            const float lb = __fsub_rd(__fadd_rd(__fmul_rd((float)b, ystep), dpo), Y.drift[g]);
+                            b = yy_encode(__fsub_rd(lb, dref), yinv);
+                        }
+                    }
+                    wv[u >> 2] |= b << (8 * (u & 3));
+                }
+                dst[c] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+            }
+            yy.dprev[rw] = dpn;
+        }
+    }
 }
 
 int32_t tc_kpad(int32_t K) { return (K + TC_N - 1) / TC_N * TC_N; }
@@ -880,11 +1165,12 @@ bool tc_eligible(int64_t n, int32_t K, int num_sms) {
     return n >= (int64_t)TC_ROWS * num_sms || tc_us < cc_us;
 }
 
-cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Header *hdr, cudaStream_t s) {
+cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Header *hdr, cudaStream_t s,
+                                    const int32_t *cperm, const float *Cprev, float *tdrift) {
     cudaError_t e = cudaMemsetAsync(&hdr->cb_cmax, 0, 4 * sizeof(uint32_t), s);  // cb_cmax .. cb_craw
     if (e != cudaSuccess) return e;
     const int32_t Kpad = tc_kpad(K);
-    if (Kpad <= TC_PACK_ONE_CTA) {
+    if (Kpad <= TC_PACK_ONE_CTA && !cperm && !tdrift) {
         launch_begin(s);
         pack_codebook_tc_small_kernel<<<1, TC_PACK_SMALL_THREADS, 0, s>>>(C, K, Kpad, Cpk, hdr);
         launch_end(s, "pack_codebook_tc_small_kernel");
@@ -895,7 +1181,8 @@ cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Heade
     launch_end(s, "codebook_norm_tc_kernel");
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     launch_begin(s);
-    pack_codebook_tc_kernel<<<(Kpad + 255) / 256, 256, 0, s>>>(C, K, Kpad, Cpk, hdr);
+    pack_codebook_tc_kernel<<<(Kpad + 255) / 256, 256, 0, s>>>(C, K, Kpad, Cpk, hdr, cperm, tdrift ? Cprev : nullptr,
+                                                                Cprev ? tdrift : nullptr);
     launch_end(s, "pack_codebook_tc_kernel");
     return cudaGetLastError();
 }
@@ -905,14 +1192,18 @@ cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Heade
 // own running best, whose column the test cannot rule out) is entered once per warp
 // instead of once per distinct hint. Results do not depend on the order.
 
-// cnt[h] = rows hinted to codeword h; cnt[K] = rows without a usable hint.
+// The group of hint h: cpos[h] (the codebook position) or h; K without a usable hint.
+__device__ __forceinline__ int32_t hint_key(int32_t h, int32_t K, const int32_t *__restrict__ cpos) {
+    if ((uint32_t)h >= (uint32_t)K) return K;
+    return cpos ? __ldg(cpos + h) : h;
+}
+
+// cnt[key] = rows whose hint has that group key (see hint_key).
 __global__ void __launch_bounds__(256) hint_histogram_kernel(const int32_t *__restrict__ hint, int64_t n, int32_t K,
-                                                             int32_t *cnt) {
+                                                             const int32_t *__restrict__ cpos, int32_t *cnt) {
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
-        const int32_t h = __ldcs(hint + i);
-        atomicAdd(cnt + ((uint32_t)h < (uint32_t)K ? h : K), 1);
-    }
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride)
+        atomicAdd(cnt + hint_key(__ldcs(hint + i), K, cpos), 1);
 }
 
 // cursor[0..m) = exclusive prefix sum of cnt[0..m) (one CTA), where entries past
@@ -921,8 +1212,10 @@ __global__ void __launch_bounds__(256) hint_histogram_kernel(const int32_t *__re
 // round's total carried into the next. cursor may be cnt itself: each round reads
 // all its entries before any are written.
 constexpr int SCAN_THREADS = 1024;
+// map (nullable): entry k reads cnt[map[k]] (counts per codeword scanned in
+// codebook-position order).
 __global__ void __launch_bounds__(SCAN_THREADS) scan_counts_kernel(const int32_t *cnt, int32_t mc, int32_t m,
-                                                                   int32_t *cursor) {
+                                                                   int32_t *cursor, const int32_t *__restrict__ map) {
     __shared__ int32_t wsum[SCAN_THREADS / 32];
     __shared__ int32_t s_carry;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -931,12 +1224,12 @@ __global__ void __launch_bounds__(SCAN_THREADS) scan_counts_kernel(const int32_t
     for (int32_t base = 0; base < m; base += 4 * SCAN_THREADS) {
         const int32_t k0 = base + 4 * tid;
         int32_t c[4];
-        if (k0 + 3 < mc && ((reinterpret_cast<uintptr_t>(cnt + k0) & 15) == 0)) {
+        if (!map && k0 + 3 < mc && ((reinterpret_cast<uintptr_t>(cnt + k0) & 15) == 0)) {
             const int4 v = *reinterpret_cast<const int4 *>(cnt + k0);
             c[0] = v.x; c[1] = v.y; c[2] = v.z; c[3] = v.w;
         } else {
 #pragma unroll
-            for (int u = 0; u < 4; ++u) c[u] = k0 + u < mc ? cnt[k0 + u] : 0;
+            for (int u = 0; u < 4; ++u) c[u] = k0 + u < mc ? cnt[map ? map[k0 + u] : k0 + u] : 0;
         }
         const int32_t local = c[0] + c[1] + c[2] + c[3];
         int32_t incl = local;
@@ -978,13 +1271,13 @@ __global__ void __launch_bounds__(SCAN_THREADS) scan_counts_kernel(const int32_t
     }
 }
 
-// perm = the rows grouped by hint (any order within a group).
+// perm = the rows grouped by hint key (any order within a group).
 __global__ void __launch_bounds__(256) hint_scatter_kernel(const int32_t *__restrict__ hint, int64_t n, int32_t K,
-                                                           int32_t *cursor, int32_t *__restrict__ perm) {
+                                                           const int32_t *__restrict__ cpos, int32_t *cursor,
+                                                           int32_t *__restrict__ perm) {
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
-        const int32_t h = __ldcs(hint + i);
-        const int32_t pos = atomicAdd(cursor + ((uint32_t)h < (uint32_t)K ? h : K), 1);
+        const int32_t pos = atomicAdd(cursor + hint_key(__ldcs(hint + i), K, cpos), 1);
         if ((uint32_t)pos < (uint32_t)n) perm[pos] = (int32_t)i;  // counts that do not match the hints: no stray write
     }
 }
@@ -1006,29 +1299,30 @@ __global__ void __launch_bounds__(256) dist_block_sums_kernel(const float *__res
     }
 }
 
-cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, const int32_t *hint_counts,
-                                    int32_t *cnt, int32_t *perm, int num_sms, cudaStream_t s) {
+cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, const int32_t *cpos,
+                                    const int32_t *cperm, const int32_t *hint_counts, int32_t *cnt, int32_t *perm,
+                                    int num_sms, cudaStream_t s) {
     int64_t blocks = (n + 255) / 256;
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
     if (hint_counts) {
         // the rows per hinted codeword are known (all hints valid): start offsets
         // straight from them, K + 1 entries with the last count 0
         launch_begin(s);
-        scan_counts_kernel<<<1, SCAN_THREADS, 0, s>>>(hint_counts, K, K + 1, cnt);
+        scan_counts_kernel<<<1, SCAN_THREADS, 0, s>>>(hint_counts, K, K + 1, cnt, cpos ? cperm : nullptr);
         launch_end(s, "scan_counts_kernel");
     } else {
         cudaError_t e = cudaMemsetAsync(cnt, 0, (size_t)(K + 1) * sizeof(int32_t), s);
         if (e != cudaSuccess) return e;
         launch_begin(s);
-        hint_histogram_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cnt);
+        hint_histogram_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cpos, cnt);
         launch_end(s, "hint_histogram_kernel");
         // the scan turns cnt into start offsets in place
         launch_begin(s);
-        scan_counts_kernel<<<1, SCAN_THREADS, 0, s>>>(cnt, K + 1, K + 1, cnt);
+        scan_counts_kernel<<<1, SCAN_THREADS, 0, s>>>(cnt, K + 1, K + 1, cnt, nullptr);
         launch_end(s, "scan_counts_kernel");
     }
     launch_begin(s);
-    hint_scatter_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cnt, perm);
+    hint_scatter_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cpos, cnt, perm);
     launch_end(s, "hint_scatter_kernel");
     return cudaGetLastError();
 }
@@ -1044,19 +1338,35 @@ cudaError_t launch_dist_block_sums(const float *dist, int64_t n, double *blocksu
 
 cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const float *Cpk, int32_t K,
                              const int32_t *hint, const int32_t *perm, int32_t *idx, float *dist, double *blocksum,
-                             int *nblocksum, Header *hdr, cudaStream_t s) {
+                             int *nblocksum, Header *hdr, cudaStream_t s, const TcYy *yy) {
     // One CTA per SM (it owns all of TMEM); the shared layout alone rules out a second.
-    const int smem = (int)sizeof(TcShared) + 1024;  // + alignment slack of the dynamic base
-    static_assert(sizeof(TcShared) + 1024 <= 227 * 1024, "shared layout too large");
-    static_assert(sizeof(TcShared) + 1024 > 114 * 1024, "two CTAs per SM would share TMEM");
-    cudaError_t e = cudaFuncSetAttribute(assign_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
+    // (+ 1024: alignment slack of the dynamic base)
+    constexpr size_t plain = sizeof(TcShared<TC_STAGES>) + 1024;
+    constexpr size_t pruned_max = sizeof(TcShared<TC_STAGES_YY>) + sizeof(TcYyShared) + (size_t)TC_ROWS * YY_MAX_TILES + 1024;
+    static_assert(plain <= 227 * 1024 && pruned_max <= 227 * 1024, "shared layout too large");
+    static_assert(plain > 114 * 1024 && sizeof(TcShared<TC_STAGES_YY>) + 1024 > 114 * 1024,
+                  "two CTAs per SM would share TMEM");
+    static_assert(sizeof(TcShared<TC_STAGES_YY>) % 16 == 0 && sizeof(TcYyShared) % 16 == 0, "record alignment");
     const int64_t blocks = (n + TC_ROWS - 1) / TC_ROWS;
     const int32_t ntiles = tc_kpad(K) / TC_N;
-    launch_begin(s);
-    assign_tc_kernel<<<(unsigned)blocks, TC_THREADS, smem, s>>>(W, n, C, Cpk, K, ntiles, hint, perm, idx, dist,
-                                                                blocksum, hdr);
-    launch_end(s, "assign_tc_kernel");
+    cudaError_t e;
+    if (yy) {
+        if (ntiles > YY_MAX_TILES || yy->stride < ntiles || yy->stride % 16 != 0) return cudaErrorInvalidValue;
+        const int smem = (int)(sizeof(TcShared<TC_STAGES_YY>) + sizeof(TcYyShared) + (size_t)TC_ROWS * yy->stride) + 1024;
+        e = cudaFuncSetAttribute(assign_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess) return e;
+        launch_begin(s);
+        assign_tc_kernel<true><<<(unsigned)blocks, TC_THREADS, smem, s>>>(W, n, C, Cpk, K, ntiles, hint, perm, idx,
+                                                                        dist, blocksum, hdr, *yy);
+        launch_end(s, "assign_tc_kernel");
+    } else {
+        e = cudaFuncSetAttribute(assign_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plain);
+        if (e != cudaSuccess) return e;
+        launch_begin(s);
+        assign_tc_kernel<false><<<(unsigned)blocks, TC_THREADS, (int)plain, s>>>(W, n, C, Cpk, K, ntiles, hint, perm,
+                                                                               idx, dist, blocksum, hdr, TcYy{});
+        launch_end(s, "assign_tc_kernel");
+    }
     *nblocksum = (int)blocks;
     return cudaGetLastError();
 }

@@ -16,6 +16,38 @@ constexpr int CP_FLOATS = 12;    // padded codeword row for the reconstruct gath
 constexpr int ACC_WORDS = 16;    // int64 accumulator row per codeword: 9 sums, count, pad (128 B)
 constexpr int ROW_BLOCK = 1024;  // kernels per assign CTA (128 threads x 8 rows)
 constexpr int MAX_PART_BLOCKS = 512;  // bound on (row blocks x codeword splits) with split-K
+// Tensor-core assign: a codeword tile is 256 codewords, streamed as 16 KiB of fp16
+// operands (K = 32 per codeword) followed by the 256 codewords in fp32.
+constexpr int TC_N = 256;
+constexpr int TC_KD = 32;
+constexpr int TC_TILE_H = TC_N * TC_KD * 2;
+constexpr int TC_TILE_BYTES = TC_TILE_H + TC_N * D * 4;
+// Pruned assignment in the fit (Yinyang-style tile bounds, kq_order.cu and
+// kq_assign_tc.cu): codebooks of YY_MIN_K .. YY_MAX_K codewords (16 .. 256 tiles).
+constexpr int32_t YY_MIN_K = 4096;
+constexpr int32_t YY_MAX_K = 65536;
+constexpr int YY_MAX_TILES = YY_MAX_K / TC_N;
+inline bool yy_sizes(int32_t K) { return K >= YY_MIN_K && K <= YY_MAX_K; }
+inline int32_t yy_stride(int32_t K) { return ((K + TC_N - 1) / TC_N + 15) / 16 * 16; }  // record bytes per kernel
+
+// Split plane of an inner node of the codebook's k-d tree (kq_order.cu).
+struct KdNode {
+    float mean[D];
+    float axis[D];
+    float pivot;  // projections below go left
+};
+
+// Pruned assignment state (kq_assign_tc.cu): the codebook is packed in the order
+// cperm (position -> codeword), and every kernel carries a record of one byte per
+// tile, a lower bound on its distance to the tile's codewords (see kq_assign_tc.cu).
+struct TcYy {
+    const int32_t *cperm, *cpos;
+    const float *tdrift;   // per tile: largest move of its codewords since the last pass
+    unsigned char *rec;    // n x stride bytes
+    float *dprev;          // n: lower bound on the kernel's distance to every codeword
+    int32_t stride;
+    int32_t read;          // 0: the records are not valid yet (every tile is processed)
+};
 
 // Fixed part of the workspace (first 4 KiB).
 struct Header {
@@ -38,11 +70,15 @@ struct Header {
     unsigned long long wtotal;          // level fit: sum of weights
     unsigned long long lacc[3][LEVELS][2];  // level fit: (weight sum, fixed-point sum) per level
     double obj;                         // codebook-size search: objective of the last fit
+    uint32_t yy_cnorm;                  // pruned fit: largest norm of the initial codebook (fp32 bits)
 };
 static_assert(sizeof(Header) <= 4096, "header too large");
 
 struct WsLayout {
-    size_t cd, acc, part, blocksum, cbuf0, cbuf1, cp, cq, cpk, dist, perm, pcnt, prev, total;
+    size_t cd, acc, part, blocksum, cbuf0, cbuf1, cp, cq, cpk, dist, perm, pcnt, prev;
+    // pruned fit (only when yy_sizes(K)): codebook order and its inverse, k-d tree
+    // nodes and scratch, per-tile drift, per-kernel bound records and distances
+    size_t cperm, cpos, kdtmp, kdkey, kdnode, tdrift, yrec, ydist, leaf, total;
 };
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -64,6 +100,16 @@ inline WsLayout ws_layout(int64_t n, int32_t K) {
     L.perm = off;     off = align_up(off + (size_t)n * 4, 256);          // rows in hint order
     L.pcnt = off;     off = align_up(off + (size_t)(K + 1) * 4, 256);    // per-hint counts / cursors
     L.prev = off;     off = align_up(off + (size_t)n * 4, 256);          // the fit's other assignment buffer
+    const bool yy = yy_sizes(K);
+    L.cperm = off;    off = align_up(off + (yy ? (size_t)K * 4 : 0), 256);
+    L.cpos = off;     off = align_up(off + (yy ? (size_t)K * 4 : 0), 256);
+    L.kdtmp = off;    off = align_up(off + (yy ? (size_t)K * 4 : 0), 256);
+    L.kdkey = off;    off = align_up(off + (yy ? (size_t)K * 8 : 0), 256);
+    L.kdnode = off;   off = align_up(off + (yy ? (size_t)2 * YY_MAX_TILES * sizeof(KdNode) : 0), 256);
+    L.tdrift = off;   off = align_up(off + (yy ? (size_t)YY_MAX_TILES * 4 : 0), 256);
+    L.yrec = off;     off = align_up(off + (yy ? (size_t)n * yy_stride(K) : 0), 256);
+    L.ydist = off;    off = align_up(off + (yy ? (size_t)n * 4 : 0), 256);
+    L.leaf = off;     off = align_up(off + (yy ? (size_t)n * 4 : 0), 256);
     L.total = off;
     return L;
 }
@@ -266,15 +312,32 @@ cudaError_t launch_assign(const float *W, int64_t n, const float *Cd, const floa
                           Header *hdr, int num_sms, cudaStream_t s);
 // Tensor-core assignment (kq_assign_tc.cu): used where tc_eligible's cost estimate favours it.
 bool tc_eligible(int64_t n, int32_t K, int num_sms);
-cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Header *hdr, cudaStream_t s);
+// cperm (nullable): pack the codebook in that order; Cprev, tdrift (nullable): the
+// largest codeword move per tile since Cprev.
+cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Header *hdr, cudaStream_t s,
+                                    const int32_t *cperm = nullptr, const float *Cprev = nullptr,
+                                    float *tdrift = nullptr);
+// yy (nullable): the pruned assignment over a codebook packed in yy->cperm order.
 cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const float *Cpk, int32_t K,
                              const int32_t *hint, const int32_t *perm, int32_t *idx, float *dist, double *blocksum,
-                             int *nblocksum, Header *hdr, cudaStream_t s);
+                             int *nblocksum, Header *hdr, cudaStream_t s, const TcYy *yy = nullptr);
 // Rows grouped by their hinted codeword (cnt: K + 1 ints of scratch, perm: n ints).
-// hint_counts: the number of rows per hinted codeword when the caller knows it (every
-// hint then valid), else null (counted here).
-cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, const int32_t *hint_counts,
-                                    int32_t *cnt, int32_t *perm, int num_sms, cudaStream_t s);
+// cpos (nullable): groups ordered by cpos[hint] instead of the hint (the codebook's
+// tile order); cperm is its inverse (needed with hint_counts). hint_counts: the
+// number of rows per hinted codeword when the caller knows it (every hint then
+// valid), else null (counted here).
+cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, const int32_t *cpos,
+                                    const int32_t *cperm, const int32_t *hint_counts, int32_t *cnt, int32_t *perm,
+                                    int num_sms, cudaStream_t s);
+// The k-d order of the codebook (kq_order.cu): cperm / cpos, tree nodes, and the
+// initial codebook's largest norm in hdr->yy_cnorm.
+cudaError_t launch_codebook_order(const float *C, int32_t K, int32_t *cperm, int32_t *cpos, int32_t *tmp,
+                                  unsigned long long *keys, KdNode *nodes, Header *hdr, cudaStream_t s);
+// First-pass hints: each kernel's nearest codeword within its k-d leaf tile
+// (Cpk: the codebook packed in cperm order). leaf, cnt, perm: scratch.
+cudaError_t launch_kd_hints(const float *W, int64_t n, const KdNode *nodes, int32_t K, const float *Cpk,
+                            const int32_t *cperm, int32_t *leaf, int32_t *cnt, int32_t *perm, int32_t *hint,
+                            int num_sms, cudaStream_t s);
 // blocksum[b] = fp64 sum of dist over rows [256 b, 256 b + 256), in row order.
 cudaError_t launch_dist_block_sums(const float *dist, int64_t n, double *blocksum, int *nblocksum, cudaStream_t s);
 cudaError_t launch_sum_blocks(const double *blocksum, int nblocks, double *out, cudaStream_t s);

@@ -20,7 +20,7 @@ KQ_OK = 0
 STATUS_NAMES = {0: "KQ_OK", 1: "KQ_ERR_INVALID_ARG", 2: "KQ_ERR_ALIGNMENT", 3: "KQ_ERR_NONFINITE",
                 4: "KQ_ERR_CUDA", 5: "KQ_ERR_DEVICE_CHECK", 6: "KQ_ERR_WORKSPACE", 7: "KQ_ERR_TIMEOUT"}
 FLAG_NONFINITE, FLAG_INDEX_RANGE, FLAG_CODE_RANGE, FLAG_TIMEOUT = 0x1, 0x2, 0x4, 0x8
-STOP_ON_STABLE = 0x1  # kq_fit_codebook flag
+STOP_ON_STABLE, FIT_PLAIN = 0x1, 0x2  # kq_fit_codebook flags
 
 EXPORTS = ["kq_status_string", "kq_abi_version", "kq_kernel_launches", "kq_workspace_bytes", "kq_device_status", "kq_init_codebook",
            "kq_assign", "kq_update_centroids", "kq_fit_codebook", "kq_quantize_codebook_6bit", "kq_reconstruct",

@@ -88,7 +88,7 @@ def test_host_validation_before_any_device_work(lib):
     assert L.kq_update_centroids(good, 1024, good, 16, None, good, good, good, ws_bytes, None) == 1
     assert L.kq_fit_codebook(good, 1024, 16, good, -1, 0, good, good, good, None, None, good, ws_bytes, None) == 1
     assert L.kq_fit_codebook(good, 1024, 16, good, 3, 7, good, good, good, None, None, good, ws_bytes, None) == 1
-    assert L.kq_fit_codebook(good, 1024, 16, good, 3, 2, good, good, good, None, None, good, ws_bytes, None) == 1
+    assert L.kq_fit_codebook(good, 1024, 16, good, 3, 4, good, good, good, None, None, good, ws_bytes, None) == 1
     assert L.kq_quantize_codebook_6bit(good, 16, good, -1, good, good, None, good, ws_bytes, None) == 1
     assert L.kq_quantize_codebook_6bit(good, 16, good, 10, good, good, None, good, 100, None) == 6
     assert L.kq_reconstruct(good, 1024, None, 16, None, None, good, good, ws_bytes, None) == 1  # nothing to decode

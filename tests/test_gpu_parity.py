@@ -702,3 +702,72 @@ def test_trace_times_every_launch_of_a_fit():
     assert names[-1] == "histogram_kernel"  # the final assignment's cluster sizes
     with pytest.raises(kq.KQError):
         kq.kq_trace_start(0)
+
+
+# --------------------------------------------------------------------------- pruned fit
+
+def _fit_both(W, C0, iters):
+    pruned, run_p = _gpu_fit_run(W, C0, iters, 0)
+    plain, run_q = _gpu_fit_run(W, C0, iters, kq.FIT_PLAIN)
+    return pruned, plain
+
+
+@pytest.mark.parametrize("case", ["k4096", "k4097_ragged_tile", "k12345", "dup_codewords", "resnet_k16384",
+                                  "iters0", "iters1"])
+def test_fit_pruned_matches_plain(case):
+    # Tile pruning (k-d codebook order, per-tile bound records, skipped tiles) only
+    # changes speed: every output equals the plain fit's, bit for bit.
+    iters = 4
+    if case == "resnet_k16384":
+        lay, W, C0 = _layer(4, 9)  # 256 -> 256, n = 65536, K = 16384
+    else:
+        n = {"k4096": 40000, "k4097_ragged_tile": 41000, "k12345": 60000, "dup_codewords": 40000,
+             "iters0": 40000, "iters1": 40000}[case]
+        K = {"k4097_ragged_tile": 4097, "k12345": 12345}.get(case, 4096)
+        lay = synth.Layer("t", 64, n // 64, K, 4 * K, 70 + len(case))
+        W = synth.conv_weights(lay)[:n]
+        C0 = oracle.gather_rows(W, synth.init_selection(n, K, 71 + len(case)))
+        if case == "dup_codewords":
+            # exact ties between codewords far apart in the original numbering
+            C0[[5, 700, 2900, 4000]] = C0[[3000, 4095, 12, 64]]
+        iters = {"iters0": 0, "iters1": 1}.get(case, iters)
+    pruned, plain = _fit_both(W, C0, iters)
+    for a, b in zip(pruned, plain):
+        assert bits_equal(a, b)
+
+
+def test_fit_pruned_stepwise_against_oracle():
+    # ResNet-18 128 -> 256 layer (n = 32768, K = 8192): the pruned fit's every step
+    # against the oracle from the same codebook, and a 3-iteration fit equal to the
+    # chained one-iteration fits
+    lay, W, C0 = _layer(4, 8)
+    C = C0
+    for t in range(3):
+        (C_next, idx_next, cnt_next, obj), _ = _gpu_fit_run(W, C, 1, 0)
+        idx_ref, dist_ref = oracle.assign(W, C, threads=THREADS)
+        C_ref, _ = oracle.update(W, idx_ref, C)
+        check_centroids(C_next, C_ref)
+        assert obj[0] == pytest.approx(oracle.objective(dist_ref), rel=1e-12)
+        i2, d2 = oracle.assign(W, C_next, threads=THREADS)
+        assert check_indices(W, C_next, idx_next, i2) == 0
+        assert np.array_equal(cnt_next, np.bincount(idx_next, minlength=lay.K))
+        C = C_next
+    (C_T, idx_T, _, obj_T), _ = _gpu_fit_run(W, C0, 3, 0)
+    assert bits_equal(C_T, C)
+    i3, _ = oracle.assign(W, C_T, threads=THREADS)
+    assert check_indices(W, C_T, idx_T, i3) == 0
+    assert np.all(obj_T[1:] <= obj_T[:-1] * (1 + 1e-6))
+
+
+def test_fit_pruned_full_size_stress():
+    # the stress layer (n = 4,194,304, K = 65,536: 256 tiles, the largest pruned
+    # codebook), 3 iterations, pruned and plain bit for bit; sampled rows of the
+    # final assignment against the oracle
+    lay, W, C0 = _layer(5)
+    pruned, plain = _fit_both(W, C0, 3)
+    for a, b in zip(pruned, plain):
+        assert bits_equal(a, b)
+    C_T, idx_T = pruned[0], pruned[1]
+    rows = np.sort(synth.below(synth.stream_key(lay.seed, 11), 2048, lay.n))
+    idx_ref, _ = oracle.assign(W[rows], C_T, threads=THREADS)
+    assert check_indices(W, C_T, idx_T[rows], idx_ref, rows) == 0
