@@ -170,6 +170,37 @@ def _cpu_sample(W, C, seconds: float, threads: int):
     return rows, dt
 
 
+def _cpu_lloyd_iteration(wl, seconds: float):
+    """The oracle's ms per Lloyd iteration of a whole workload on the host cores: per
+    layer, its assignment timed on a seeded row sample (rows are independent) and
+    scaled to every row, plus its update over every row."""
+    import oracle
+
+    threads = oracle.default_threads()
+    per_layer = max(0.05, seconds / len(wl.layers))
+    total_ms, sampled, rows_all = 0.0, 0, 0
+    for lay in wl.layers:
+        W, sel = synth.layer_inputs(lay)
+        C0 = oracle.gather_rows(W, sel)
+        n = W.shape[0]
+        rows, dt = _cpu_sample(W, C0, per_layer, threads) if n * lay.K > 2e8 else (n, None)
+        if dt is None:
+            t0 = time.perf_counter()
+            idx, _ = oracle.assign(W, C0, threads=threads)
+            dt = time.perf_counter() - t0
+        else:
+            idx = synth.below(synth.stream_key(lay.seed, 17), n, lay.K).astype(np.int32)
+        t0 = time.perf_counter()
+        oracle.update(W, idx, C0)
+        du = time.perf_counter() - t0
+        total_ms += 1e3 * (dt * n / rows + du)
+        sampled += rows
+        rows_all += n
+    return {"ms_per_lloyd_iter": total_ms, "cores": threads, "kind": "oracle",
+            "sample": f"assignment timed on {sampled} of {rows_all} rows and scaled to all; update over every row "
+                      f"(indices: the oracle's own where every row was assigned, else seeded)"}
+
+
 def run_reference(args, rank, world):
     """CPU oracle on the host cores (rank 0 only)."""
     if rank != 0:
@@ -661,16 +692,21 @@ def run_configs(args):
         peaks = _peaks()
         bf16 = float(peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops", 1700.0)))
         max_mhz = float(peaks.get("sm_max_mhz", 2070.0))
-        print(json.dumps({
+        line = {
             "config": wl.name, "layers": len(layers), "kernels": sum(L["n"] for L in layers),
             "codewords": sum(L["K"] for L in layers), "iters": T, "evals": evals, "ms_per_run": ms,
-            "evals_per_s": rate,
+            "ms_per_lloyd_iter": ms / (T + 1), "evals_per_s": rate,
             # whole-run figures (init, fit, 6-bit quantisation and recovery all in the time),
-            # so lower bounds for the assignment kernels alone
+            # so lower bounds for the assignment kernels alone; method work = 18 flops per pair
             "frac_of_tensor_peak": rate * METHOD_FLOPS_PER_PAIR / 1e12 / bf16,
             "direct_form_frac_of_fp32_peak": rate * DIRECT_OPS_PER_PAIR / (sms * FP32_LANES_PER_SM * max_mhz * 1e6),
             "gpu_launches_per_run": (kq.kq_kernel_launches() - launches0) // args.reps,
-            "status": max(st for st, _ in statuses), "reps": args.reps, "streams": len(side)}), flush=True)
+            "status": max(st for st, _ in statuses), "reps": args.reps, "streams": len(side)}
+        if not args.no_cpu_baseline:
+            line["cpu_baseline"] = _cpu_lloyd_iteration(wl, args.ref_seconds)
+            line["cpu_baseline"]["speedup_per_lloyd_iter"] = line["cpu_baseline"]["ms_per_lloyd_iter"] / line[
+                "ms_per_lloyd_iter"]
+        print(json.dumps(line), flush=True)
 
 
 def main():

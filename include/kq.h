@@ -71,7 +71,7 @@ typedef enum {
 
 /* kq_fit_codebook flags. */
 #define KQ_STOP_ON_STABLE 0x1
-#define KQ_FIT_PLAIN 0x2
+#define KQ_FIT_PRUNE 0x2
 
 /* Human-readable name of a status. Never NULL. */
 const char *kq_status_string(kq_status s);
@@ -101,6 +101,27 @@ kq_status kq_trace_start(int32_t capacity);
 kq_status kq_trace_stop(void);
 int32_t kq_trace_count(void);
 kq_status kq_trace_get(int32_t i, const char **name, float *ms);
+
+/* Failure-detection test hook (no paper counterpart): makes the bounded device-side
+ * waits of later calls on this workspace run out, so that tests can check that a
+ * wait that gives up is reported (KQ_FLAG_TIMEOUT / KQ_ERR_TIMEOUT from
+ * kq_device_status) and that the call still returns, without any GPU fault.
+ *   faults      KQ_TEST_SKIP_ARRIVAL: in the grid barriers of the cooperative
+ *               kernels (6-bit quantisation, one-launch small fits, fused recovery,
+ *               update fallback) CTA 0 never arrives, so the others wait until the
+ *               limit; KQ_TEST_STOP_TILE_STREAM: the tensor-core assignment streams
+ *               no codeword tile beyond those it starts before its setup, so its
+ *               MMA issuers wait until the limit. 0 clears both.
+ *   wait_limit  polls before a bounded wait gives up (0: the normal limits, about
+ *               2 s for grid barriers and 4M mbarrier polls).
+ * Enqueued on `stream` (a one-thread kernel writes the workspace header); stays in
+ * effect for this workspace until cleared. The outputs of a call whose wait gave
+ * up are unspecified; the workspace's grid-barrier state is left inconsistent, so
+ * zero-fill it (or use another) before its next use. ws_bytes >= 4096. */
+#define KQ_TEST_SKIP_ARRIVAL 0x1u
+#define KQ_TEST_STOP_TILE_STREAM 0x2u
+kq_status kq_test_inject_wait_fault(void *ws, size_t ws_bytes, uint32_t faults, uint32_t wait_limit,
+                                    kq_stream_t stream);
 
 /* Bytes of workspace needed by any entry point for n kernels and K codewords.
  * Returns 0 when (n, K) is outside the supported range. */
@@ -197,16 +218,17 @@ kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int
  *              exactly those of all `iters` iterations; the objective entries of
  *              the skipped steps repeat the last one computed. The call then
  *              synchronises `stream` once per iteration to read the test.
- *              KQ_FIT_PLAIN: test every kernel against every codeword in every
- *              assignment. Without it, fits of 4096 to 65536 codewords on the
- *              tensor-core path prune, as Yinyang k-means does (Sec. 4.1): the
+ *              KQ_FIT_PRUNE: for fits of 4096 to 65536 codewords on the
+ *              tensor-core path, prune as Yinyang k-means does (Sec. 4.1): the
  *              codebook is ordered by a k-d tree so that each 256-codeword tile
  *              holds nearby codewords, every kernel keeps a lower bound on its
  *              distance to each tile (lowered by the tile's codeword drift after
  *              every update), and a tile that cannot hold a codeword as close as
  *              the kernel's previous one is skipped for a whole block of kernels.
- *              The first assignment then starts from each kernel's nearest
- *              codeword in its k-d leaf. The outputs are identical either way.
+ *              The outputs are identical either way; the workspace holds the
+ *              bounds. (On the 2048 x 2048 stress layer it skips 16-46% of the
+ *              tiles per update but each processed tile costs more, so it is not
+ *              the default.)
  *   idx        n int32 output: the final assignment (device)
  *   counts     K int32 output: cluster sizes of the final assignment (device)
  *   objective  iters + 1 fp64 outputs (device) or NULL: Eq. 1 objective per step,

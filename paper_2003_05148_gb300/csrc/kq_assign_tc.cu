@@ -147,10 +147,11 @@ __device__ __forceinline__ void mbar_init(uint32_t a, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(count) : "memory");
 }
 
-// Bounded wait for the phase with the given parity; false if it ran out or the CTA aborted.
+// Bounded wait for the phase with the given parity; false if it ran out (after
+// `limit` polls) or the CTA aborted.
 __device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, volatile uint32_t *abort_flag,
-                                          uint32_t *status) {
-    for (long long it = 0; it < TC_WAIT_LIMIT; ++it) {
+                                          uint32_t *status, long long limit) {
+    for (long long it = 0; it < limit; ++it) {
         uint32_t done;
         asm volatile(
             "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
@@ -456,11 +457,10 @@ __device__ __forceinline__ float direct_distance(const float (&x)[D], const floa
     return acc;
 }
 
-template <int NST>
-struct __align__(16) TcShared {
+struct TcShared {
     unsigned char a[TC_RT][TC_A_BYTES];             // row tiles (tensor-core layout)
-    unsigned char b[NST][TC_TILE_BYTES];            // codeword tiles
-    unsigned long long full[NST], empty[NST], tfull[TC_RT], tempty[TC_RT], done;
+    unsigned char b[TC_STAGES][TC_TILE_BYTES];      // codeword tiles
+    unsigned long long full[TC_STAGES], empty[TC_STAGES], tfull[TC_RT], tempty[TC_RT], done;
     uint32_t tmem_base;
     uint32_t abort_flag;
     float xs[TC_ROWS][D];    // the CTA's kernels and test constants, read on the
@@ -475,20 +475,35 @@ struct __align__(16) TcShared {
     double wsum[TC_EPI_WARPS / 2][TC_RT];
 };
 
-// Pruned kernel only (after TcShared; then the records, TC_ROWS x stride bytes).
-struct __align__(16) TcYyShared {
-    unsigned long long xfull[4][2], xempty[4][2];  // hand-over of the second half's bound, per lane quarter
-    uint32_t mask[YY_MAX_TILES / 32];              // tiles this CTA processes
-    int32_t nt;                                    // their number
+// Shared layout of the pruned kernel (assign_tc_pruned_kernel); the per-row bound
+// records follow it, TC_ROWS rows of stride + 4 bytes (the 4 put consecutive rows one
+// bank apart).
+struct __align__(16) TcPrunedShared {
+    unsigned char a[TC_RT][TC_A_BYTES];
+    unsigned char b[TC_STAGES_YY][TC_TILE_BYTES];
+    unsigned long long full[TC_STAGES_YY], empty[TC_STAGES_YY], tfull[TC_RT], tempty[TC_RT], done;
+    uint32_t tmem_base;
+    uint32_t abort_flag;
+    float xs[TC_ROWS][D];
+    RowConst rc[TC_ROWS];
+    int32_t prow[TC_ROWS];
+    uint32_t mask[YY_MAX_TILES / 32];  // tiles this CTA processes
+    int32_t nt;                        // their number
     int32_t pad_;
-    uint16_t tl[YY_MAX_TILES];                     // the tiles, in processing order
-    float tmax[2][TC_ROWS];                        // per half row: largest T' an MMA may have read
-    float tabs[2][TC_ROWS];                        // and largest |T'|
-    float xch[2][TC_RT][TC_M];                     // the second half's bound, for the first half's thread
-    float drift[YY_MAX_TILES];                     // per tile: largest codeword move since the last pass
-    float dprev[TC_ROWS];                          // each slot's record distance (when read)
-    float fin[TC_ROWS];                            // each slot's final best distance
+    uint16_t tl[YY_MAX_TILES];         // the tiles, in processing order
+    uint32_t dq[YY_MAX_TILES / 4];     // per tile, a byte: its drift since the last pass in bound steps (rounded up)
+    uint32_t msk[TC_ROWS][8];          // candidate masks of a row's chunks (rare: only those with candidates)
 };
+
+// Byte b of the result: bit b of bits (4 bits -> 4 bytes of 0 or 1).
+__device__ __forceinline__ uint32_t bits_to_bytes01(uint32_t bits) { return (bits * 0x00204081u) & 0x01010101u; }
+// Bit b of the result: byte b of v, which is 0 or 1 (4 bytes -> 4 bits).
+__device__ __forceinline__ uint32_t bytes01_to_bits(uint32_t v) { return (v * 0x01020408u) >> 24; }
+// min(255, ceil(x)) for x >= 0 as an integer; 255 for NaN or +inf, 0 for x <= 0.
+__device__ __forceinline__ uint32_t ceil_byte(float x) {
+    if (!(x < 255.f)) return 255u;
+    return x > 0.f ? (uint32_t)ceilf(x) : 0u;
+}
 
 constexpr int YY_DELTA_SHIFT = 10;  // bound step: 2^(e - 10) for an initial codebook whose largest norm is f 2^e
 constexpr float YY_ONE_M_G11 = 0.99999904632568359375f;  // 1 - 8 * 2^-23 <= 1 - gamma_11 <= 1 / (1 + gamma_11)
@@ -503,6 +518,36 @@ __device__ __forceinline__ uint32_t yy_encode(float x, float inv) {
     return v >= 255.f ? 255u : (uint32_t)v;
 }
 
+// Bounds of sqrt(x) from rsqrtf (at most 2 ulp off) with a 2^-16 relative margin:
+// below <= sqrt(x) <= above, for any x (0 / +inf outside [2^-100, 2^100]; NaN: 0 / +inf).
+__device__ __forceinline__ float sqrt_below(float x) {
+    if (!(x >= 7.888609052e-31f)) return 0.f;
+    if (!(x <= 1.267650600e30f)) return 1.125899906842624e15f;  // 2^50
+    return __fmul_rd(__fmul_rd(x, rsqrtf(x)), 0.9999847412109375f);
+}
+__device__ __forceinline__ float sqrt_above(float x) {
+    if (!(x <= 1.267650600e30f)) return __int_as_float(0x7f800000);
+    if (!(x >= 7.888609052e-31f)) return 8.881784197e-16f;  // 2^-50
+    return __fmul_ru(__fmul_ru(x, rsqrtf(x)), 1.0000152587890625f);
+}
+
+// The part of a half row's lower bound that does not depend on the tile (scaled
+// units): X2lo - Qmax - 2 (R + T'max + E), E = 2^-16 (k1 + |T'|max) + k2 / 2; the
+// tile's bound is this minus twice the half's largest g (see the epilogue).
+// The largest g for which a tile's byte saturates (slack >= 255 steps): with
+// X = beta^2 (dref + 255 step)^2 rounded up, g <= (base - X) / 2 rounded down means
+// base - 2 g >= X. -inf when any of it is not finite.
+__device__ __forceinline__ float yy_saturation(float base, float dref, float step, float beta2) {
+    const float dd = __fadd_ru(dref, __fmul_ru(255.f, step));
+    const float r = __fmul_rd(__fsub_rd(base, __fmul_ru(beta2, __fmul_ru(dd, dd))), 0.5f);
+    return r == r && r <= 3.402823466e38f ? r : __int_as_float(0xff800000);
+}
+
+__device__ __forceinline__ float yy_base(const RowConst &rq, float tmax, float tabs) {
+    const float E = __fadd_ru(__fmul_ru(TWO_M16, __fadd_ru(rq.k1, tabs)), __fmul_ru(0.5f, rq.k2));
+    return __fsub_rd(rq.k0, __fmul_ru(2.f, __fadd_ru(__fadd_ru(rq.R, tmax), E)));  // NaN for rows tested exactly
+}
+
 // Named barrier among the 256 epilogue threads (warps 3-10).
 __device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
 
@@ -515,54 +560,31 @@ __device__ __forceinline__ int yy_first_tile(const int32_t *hint, const int32_t 
     return (uint32_t)h < (uint32_t)K ? __ldg(cpos + h) / TC_N : 0;
 }
 
-// YY: the pruned kernel of the fit (yy: its state). The codebook is packed in the
-// order yy.cperm (tile g = positions [256 g, 256 g + 256)); indices and the tie rule
-// stay those of the original numbering. Every row keeps a record of one byte per
-// tile: q with q * step + dprev <= the distance from the row to every codeword of
-// the tile (dprev <= its distance to every codeword), written at the end of each
-// pass and, in the next pass, lowered by the tile's drift (triangle inequality). A
-// tile whose bound proves every codeword farther than the row's hinted codeword for
-// all 256 rows of the CTA is not streamed, multiplied or tested at all; the answer
-// is the same, since no skipped codeword could improve or tie the row's best.
-template <bool YY>
+// TH: the instantiation with the failure-detection test hooks (kq_test_inject_wait_fault);
+// the other keeps its wait limits compile-time constants, which its hot loops need.
+template <bool TH>
 __global__ void __launch_bounds__(TC_THREADS, 1)
 assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict__ C, const float *__restrict__ Cpk,
                  int32_t K, int32_t ntiles, const int32_t *hint, const int32_t *__restrict__ perm, int32_t *idx,
-                 float *__restrict__ dist, double *__restrict__ blocksum, Header *hdr, TcYy yy) {
-    constexpr int NST = YY ? TC_STAGES_YY : TC_STAGES;
+                 float *__restrict__ dist, double *__restrict__ blocksum, Header *hdr) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
-    TcShared<NST> &S = *reinterpret_cast<TcShared<NST> *>(smem_raw);
-    TcYyShared &Y = *reinterpret_cast<TcYyShared *>(smem_raw + sizeof(TcShared<NST>));  // YY only
-    unsigned char *yrec = smem_raw + sizeof(TcShared<NST>) + sizeof(TcYyShared);      // YY only
+    TcShared &S = *reinterpret_cast<TcShared *>(smem_raw);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     volatile uint32_t *abort_flag = &S.abort_flag;
     uint32_t *status = &hdr->status;
     const float beta = tc_scale(__uint_as_float(__ldcg(&hdr->cb_craw)));  // as pack_codebook_tc_kernel
     const float beta2 = beta * beta;
-    const float inv_beta = 1.f / beta;  // exact: a power of two
-    const int64_t row0 = (int64_t)blockIdx.x * TC_ROWS;
-    // pruned kernel: bound step (fixed for the fit) and whether the records are valid
-    float ystep = 0.f, yinv = 0.f;
-    bool yread = false;
-    if (YY) {
-        const float cn = __uint_as_float(__ldcg(&hdr->yy_cnorm));
-        if (cn > 0.f && cn <= 3.402823466e38f) {
-            int e;
-            frexpf(cn, &e);
-            const int ex = max(-100, min(100, e - YY_DELTA_SHIFT));
-            ystep = ldexpf(1.f, ex);
-            yinv = ldexpf(1.f, -ex);
-        }
-        yread = yy.read != 0 && ystep > 0.f;
-    }
+    // failure-detection tests (kq_test_inject_wait_fault): shorter waits, tile stream cut
+    const uint32_t tfault = TH ? __ldcg(&hdr->test_faults) : 0u;
+    const uint32_t tlim = TH ? __ldcg(&hdr->test_wait_limit) : 0u;
+    const long long wlim = (TH && tlim) ? (long long)tlim : TC_WAIT_LIMIT;
 
     // ---- barriers first: the producer starts streaming the first codeword tiles
     // while the epilogue threads set up their rows (the other roles wait for the
-    // barriers only after the CTA barrier below). The pruned kernel reading records
-    // streams one tile early: the one holding the first slot's hinted codeword.
-    const int pre = (YY && yread) ? 1 : (ntiles < NST ? ntiles : NST);
+    // barriers only after the CTA barrier below)
+    const int pre = ntiles < TC_STAGES ? ntiles : TC_STAGES;
     if (tid == 0) {
-        for (int s = 0; s < NST; ++s) {
+        for (int s = 0; s < TC_STAGES; ++s) {
             mbar_init((uint32_t)__cvta_generic_to_shared(&S.full[s]), 1);
             mbar_init((uint32_t)__cvta_generic_to_shared(&S.empty[s]), TC_EPI_WARPS);
         }
@@ -571,26 +593,17 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
             mbar_init((uint32_t)__cvta_generic_to_shared(&S.tempty[t]), TC_EPI_WARPS);
         }
         mbar_init((uint32_t)__cvta_generic_to_shared(&S.done), TC_RT);
-        if (YY) {
-            for (int qq = 0; qq < 4; ++qq)
-                for (int b = 0; b < 2; ++b) {
-                    mbar_init((uint32_t)__cvta_generic_to_shared(&Y.xfull[qq][b]), 1);
-                    mbar_init((uint32_t)__cvta_generic_to_shared(&Y.xempty[qq][b]), 1);
-                }
-        }
         S.abort_flag = 0u;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // initialised barriers -> bulk copies
-        const int g0 = (YY && yread) ? yy_first_tile(hint, perm, row0, n, K, yy.cpos) : 0;
         for (int i = 0; i < pre; ++i) {
-            const int g = (YY && yread) ? g0 : i;
             const uint32_t fb = (uint32_t)__cvta_generic_to_shared(&S.full[i]);
             asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb), "r"(TC_TILE_BYTES)
                          : "memory");
             asm volatile(
                 "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
                     (uint32_t)__cvta_generic_to_shared(S.b[i])),
-                "l"(reinterpret_cast<const unsigned char *>(Cpk) + (int64_t)g * TC_TILE_BYTES), "r"(TC_TILE_BYTES),
+                "l"(reinterpret_cast<const unsigned char *>(Cpk) + (int64_t)i * TC_TILE_BYTES), "r"(TC_TILE_BYTES),
                 "r"(fb)
                 : "memory");
         }
@@ -610,13 +623,9 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
         bi[t] = 0;
         known[t] = -1;
     }
-    const bool lgroup = !YY && hint != nullptr && perm == nullptr && K >= TC_LGROUP_MINK && K <= TC_LGROUP_MAXK;
+    const bool lgroup = hint != nullptr && perm == nullptr && K >= TC_LGROUP_MINK && K <= TC_LGROUP_MAXK;
     if (epi) {
-        if (YY) {  // cleared before the epilogue barrier that precedes their first use
-            const int et = tid - TC_EPI_WARP0 * 32;
-            if (et < YY_MAX_TILES / 32) Y.mask[et] = 0u;
-            for (int g = et; g < ntiles; g += TC_EPI_WARPS * 32) Y.drift[g] = yread ? __ldg(yy.tdrift + g) : 0.f;
-        }
+        const int64_t row0 = (int64_t)blockIdx.x * TC_ROWS;
         if (lgroup) {
             // CTA-local grouping (counting sort of the CTA's rows by hint chunk; the
             // order within a chunk is free): a warp's rows then share a few chunks,
@@ -734,16 +743,11 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                 const float d = direct_distance(x, ch[t]);
                 if (d < best[t]) {
                     best[t] = d;
-                    bi[t] = hv[t];
-                    known[t] = YY ? __ldg(yy.cpos + hv[t]) : hv[t];  // known: the codebook position
+                    bi[t] = known[t] = hv[t];
                     ev = !tc_shift(rc, d, beta2, tp);
                 }
             }
             every |= (ev ? 1u : 0u) << t;
-            if (YY) {
-                Y.tmax[hsel][rloc] = ev ? -TC_T_EVERY : tp;
-                Y.tabs[hsel][rloc] = ev ? TC_T_EVERY : fabsf(tp);
-            }
             if (hsel == 0) {  // both halves start from the same state; one writes it
                 S.prow[rloc] = (int32_t)row[t];
 #pragma unroll
@@ -756,75 +760,6 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                 a[TC_SLOT_T0] = a[TC_SLOT_T1] = ev ? TC_T_EVERY : -tp;
                 a[TC_SLOT_R] = -rc.R;
                 tc_store_row(S.a[t], r, a);
-            }
-        }
-        if (YY) {
-            // The tiles this CTA needs: thread (hsel, r) reads the record of the row in
-            // row tile hsel (its best so far is the hinted codeword's exact distance B);
-            // tile g can be skipped for that row when the record's bound, lowered by
-            // the tile's drift, proves every codeword of g farther than B.
-            epi_sync();  // mask cleared, drifts staged
-            const int sl = hsel * TC_M + r;
-            const int64_t rw = row[hsel];
-            const float B = best[hsel];
-            const bool all = !yread || !(B <= 3.402823466e38f);  // no valid record or no finite hint distance
-            const float dp = (yread && rw < n) ? yy.dprev[rw] : 0.f;
-            if (yread) Y.dprev[sl] = dp;
-            const uint4 *src = reinterpret_cast<const uint4 *>(yy.rec + (rw < n ? rw : 0) * (int64_t)yy.stride);
-            uint4 *dst = reinterpret_cast<uint4 *>(yrec + sl * yy.stride);
-            for (int w = 0; w < (ntiles + 31) / 32; ++w) {
-                uint32_t need = 0u;
-                if (rw < n) {
-                    if (all) {
-                        need = 0xffffffffu;
-                    } else {
-#pragma unroll
-                        for (int h2 = 0; h2 < 2; ++h2) {
-                            const int c = 2 * w + h2;
-                            if (c * 16 >= yy.stride) continue;  // a stride of 16 (mod 32) bytes
-                            const uint4 v = src[c];
-                            dst[c] = v;
-#pragma unroll
-                            for (int u = 0; u < 16; ++u) {
-                                const uint32_t wsel = (u >> 2) == 0 ? v.x : (u >> 2) == 1 ? v.y : (u >> 2) == 2 ? v.z : v.w;
-                                const float qv = (float)((wsel >> (8 * (u & 3))) & 255u);
-                                const float lb = __fsub_rd(__fadd_rd(__fmul_rd(qv, ystep), dp), Y.drift[c * 16 + u < ntiles ? c * 16 + u : 0]);
-                                const bool skip = lb > 0.f && __fmul_rd(__fmul_rd(lb, lb), YY_ONE_M_G11) > B;
-                                need |= (skip ? 0u : 1u) << (16 * h2 + u);
-                            }
-                        }
-                    }
-                    const int left = ntiles - 32 * w;
-                    if (left < 32) need &= (1u << left) - 1u;
-                }
-                need = __reduce_or_sync(0xffffffffu, need);
-                if (lane == 0 && need) atomicOr(&Y.mask[w], need);
-            }
-            epi_sync();
-            if (warp == TC_EPI_WARP0) {
-                // the list: the early tile first (read mode), then the others in order;
-                // lane l takes tiles 8 l .. 8 l + 7
-                const int g0 = yread ? yy_first_tile(hint, perm, row0, n, K, yy.cpos) : -1;  // as streamed
-                uint32_t bits = (Y.mask[lane >> 2] >> ((lane & 3) * 8)) & 0xffu;
-                if (g0 >= 0 && (g0 >> 3) == lane) bits &= ~(1u << (g0 & 7));
-                const int cnt = __popc(bits);
-                int incl = cnt;
-#pragma unroll
-                for (int o = 1; o < 32; o <<= 1) {
-                    const int y2 = __shfl_up_sync(0xffffffffu, incl, o);
-                    if (lane >= o) incl += y2;
-                }
-                int pos = (g0 >= 0 ? 1 : 0) + incl - cnt;
-                while (bits) {
-                    const int b = __ffs(bits) - 1;
-                    bits &= bits - 1u;
-                    Y.tl[pos++] = (uint16_t)(lane * 8 + b);
-                }
-                if (lane == 31) Y.nt = (g0 >= 0 ? 1 : 0) + incl;
-                if (lane == 0 && g0 >= 0) {
-                    Y.tl[0] = (uint16_t)g0;
-                    atomicOr(&Y.mask[g0 >> 5], 1u << (g0 & 31));  // the mask now marks every processed tile
-                }
             }
         }
     }
@@ -842,16 +777,15 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = S.tmem_base;
-    const int nt = YY ? Y.nt : ntiles;  // tiles this CTA processes (the list's length)
 
     if (warp == 0) {
         // ---- producer (lane 0)
         if (lane == 0) {
-            for (int i = pre; i < nt; ++i) {  // list entries 0 .. pre - 1 are on their way
-                const int s = i % NST;
-                const int g = YY ? (int)Y.tl[i] : i;
-                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.empty[s]), ((i / NST) - 1) & 1, abort_flag,
-                               status))
+            const int nlast = (TH && (tfault & KQ_TEST_STOP_TILE_STREAM)) ? pre : ntiles;
+            for (int i = pre; i < nlast; ++i) {  // tiles 0 .. pre - 1 are on their way
+                const int s = i % TC_STAGES;
+                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.empty[s]), ((i / TC_STAGES) - 1) & 1, abort_flag,
+                               status, wlim))
                     break;
                 const uint32_t fb = (uint32_t)__cvta_generic_to_shared(&S.full[s]);
                 asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb), "r"(TC_TILE_BYTES)
@@ -859,7 +793,7 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                 asm volatile(
                     "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
                         (uint32_t)__cvta_generic_to_shared(S.b[s])),
-                    "l"(reinterpret_cast<const unsigned char *>(Cpk) + (int64_t)g * TC_TILE_BYTES), "r"(TC_TILE_BYTES),
+                    "l"(reinterpret_cast<const unsigned char *>(Cpk) + (int64_t)i * TC_TILE_BYTES), "r"(TC_TILE_BYTES),
                     "r"(fb)
                     : "memory");
             }
@@ -871,13 +805,13 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
             constexpr uint32_t idesc = tc_idesc(TC_M, TC_N);
             const uint32_t a0 = (uint32_t)__cvta_generic_to_shared(S.a[t]);
             const uint32_t dcol = tmem + (uint32_t)(t * TC_N);
-            for (int i = 0; i < nt; ++i) {
-                const int s = i % NST;
-                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.full[s]), (i / NST) & 1, abort_flag, status))
+            for (int i = 0; i < ntiles; ++i) {
+                const int s = i % TC_STAGES;
+                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.full[s]), (i / TC_STAGES) & 1, abort_flag, status, wlim))
                     break;
                 // the accumulator is free once the epilogue read tile i - 1
                 if (i >= 1 &&
-                    !mbar_wait((uint32_t)__cvta_generic_to_shared(&S.tempty[t]), (i - 1) & 1, abort_flag, status))
+                    !mbar_wait((uint32_t)__cvta_generic_to_shared(&S.tempty[t]), (i - 1) & 1, abort_flag, status, wlim))
                     break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t b0 = (uint32_t)__cvta_generic_to_shared(S.b[s]);
@@ -904,7 +838,7 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
             asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(db)
                          : "memory");
             if (t == 0) {
-                for (long long it = 0; it < TC_WAIT_LIMIT; ++it) {
+                for (long long it = 0; it < wlim; ++it) {
                     uint32_t ok;
                     asm volatile(
                         "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n selp.u32 %0, 1, 0, p;\n}"
@@ -912,7 +846,7 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                         : "r"(db)
                         : "memory");
                     if (ok) break;
-                    if (it + 1 == TC_WAIT_LIMIT) set_flag(status, KQ_FLAG_TIMEOUT);
+                    if (it + 1 == wlim) set_flag(status, KQ_FLAG_TIMEOUT);
                 }
             }
         }
@@ -923,20 +857,11 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
         // or tie the running best.
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
         bool go = true;
-        for (int i = 0; i < nt && go; ++i) {
-            const int st = i % NST;
-            const int gb = (YY ? (int)Y.tl[i] : i) * TC_N;  // codebook position of the tile's first codeword
-            float own[TC_RT];                                // pruned: this half's bound per row tile
-            // pruned, second half: its exchange slot must have been read (tile i - 2)
-            if (YY && hsel == 1 && i >= 2 &&
-                !mbar_wait((uint32_t)__cvta_generic_to_shared(&Y.xempty[q][i & 1]), ((i >> 1) - 1) & 1, abort_flag,
-                           status)) {
-                go = false;
-                break;
-            }
+        for (int i = 0; i < ntiles && go; ++i) {
+            const int st = i % TC_STAGES;
 #pragma unroll
             for (int t = 0; t < TC_RT; ++t) {
-                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.tfull[t]), i & 1, abort_flag, status)) {
+                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.tfull[t]), i & 1, abort_flag, status, wlim)) {
                     go = false;
                     break;
                 }
@@ -972,14 +897,14 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                         // the running best itself needs no decision (in a warm start it
                         // is almost always the only codeword that passes)
                         uint32_t mask = !need ? 0u : (ev ? 0xffffffffu : ~sign_mask32(v[c]));
-                        const int kloc = known[t] - (gb + hsel * TC_HALF + 32 * c);
+                        const int kloc = known[t] - (i * TC_N + hsel * TC_HALF + 32 * c);
                         if ((uint32_t)kloc < 32u) mask &= ~(1u << kloc);
                         while (mask) {
                             const int j = __ffs(mask) - 1;
                             mask &= mask - 1u;
                             const int kl = hsel * TC_HALF + 32 * c + j;
-                            const int32_t p = gb + kl;  // codebook position (the index unless pruned)
-                            if (p >= K) break;
+                            const int32_t k = i * TC_N + kl;
+                            if (k >= K) break;
                             float xr[D], cw[D];
                             const float *c32 = reinterpret_cast<const float *>(tile + TC_TILE_H) + kl * D;
 #pragma unroll
@@ -988,15 +913,10 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                                 cw[u] = c32[u];
                             }
                             const float d = direct_distance(xr, cw);
-                            if (d <= best[t]) {
-                                // the lowest original index wins a tie, whatever the packing order
-                                const int32_t k = YY ? __ldg(yy.cperm + p) : p;
-                                if (d < best[t] || k < bi[t]) {
-                                    best[t] = d;
-                                    bi[t] = k;
-                                    known[t] = p;
-                                    moved = true;
-                                }
+                            if (d < best[t] || (d == best[t] && k < bi[t])) {
+                                best[t] = d;
+                                bi[t] = known[t] = k;
+                                moved = true;
                             }
                         }
                     }
@@ -1007,53 +927,7 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
                         *reinterpret_cast<uint16_t *>(&S.a[t][tc_offset(r, hsel ? TC_SLOT_T1 : TC_SLOT_T0)]) =
                             (uint16_t)f16_bits(e2 ? TC_T_EVERY : -tp);
                         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // for later MMAs
-                        if (YY) {
-                            const float tn = e2 ? -TC_T_EVERY : tp;
-                            Y.tmax[hsel][rloc] = fmaxf(Y.tmax[hsel][rloc], tn);
-                            Y.tabs[hsel][rloc] = fmaxf(Y.tabs[hsel][rloc], fabsf(tn));
-                        }
                     }
-                }
-                if (YY) {
-                    // a lower bound on the distance from the row to every codeword of this
-                    // half tile: D >= X2lo - Qmax - 2 e and e <= g + R + T' + E for each of
-                    // them (scaled units), with g at most the half's maximum m and T' at most
-                    // the largest value an MMA may have read
-                    const int rloc = t * TC_M + r;
-                    const RowConst rq = S.rc[rloc];
-                    const float E = __fadd_ru(__fmul_ru(TWO_M16, __fadd_ru(rq.k1, Y.tabs[hsel][rloc])),
-                                              __fmul_ru(0.5f, rq.k2));
-                    const float up = __fadd_ru(__fadd_ru(__fadd_ru(m, rq.R), Y.tmax[hsel][rloc]), E);
-                    const float lbD = __fsub_rd(rq.k0, __fmul_ru(2.f, up));  // NaN for rows tested exactly
-                    own[t] = __fmul_rd(__fsqrt_rd(fmaxf(lbD, 0.f)), inv_beta);
-                    if (hsel == 1) Y.xch[i & 1][t][r] = own[t];
-                }
-            }
-            if (YY && go) {
-                // the row's bound for the tile is the smaller of its two halves': the
-                // second half hands its value over, the first half records the byte
-                // (as slack over its current best, which is at least the final one)
-                if (hsel == 1) {
-                    __syncwarp();
-                    if (lane == 0)
-                        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(
-                                         (uint32_t)__cvta_generic_to_shared(&Y.xfull[q][i & 1]))
-                                     : "memory");
-                } else if (mbar_wait((uint32_t)__cvta_generic_to_shared(&Y.xfull[q][i & 1]), (i >> 1) & 1,
-                                     abort_flag, status)) {
-#pragma unroll
-                    for (int t = 0; t < TC_RT; ++t) {
-                        const float lb = fminf(own[t], Y.xch[i & 1][t][r]);
-                        const float dref = __fsqrt_ru(__fmul_ru(best[t], INV_ONE_M_G11_TC));
-                        yrec[(t * TC_M + r) * yy.stride + gb / TC_N] = (unsigned char)yy_encode(__fsub_rd(lb, dref), yinv);
-                    }
-                    __syncwarp();
-                    if (lane == 0)
-                        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(
-                                         (uint32_t)__cvta_generic_to_shared(&Y.xempty[q][i & 1]))
-                                     : "memory");
-                } else {
-                    go = false;
                 }
             }
             __syncwarp();
@@ -1091,7 +965,6 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
             }
             // the partial sum runs over the CTA's rows in row order whatever the grouping
             S.rowbest[lgroup ? S.lslot[rloc] : rloc] = row < n ? best[t] : 0.f;
-            if (YY) Y.fin[rloc] = best[t];
         }
         asm volatile("bar.sync 2, 128;" ::: "memory");  // the 128 threads of the first half
 #pragma unroll
@@ -1113,40 +986,498 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TC_COLS) : "memory");
     }
-    if (YY && epi) {
-        // Records for the next pass, relative to this pass's final best: processed
-        // tiles keep the byte of this pass (its slack over a best at least the final
-        // one); the others take last pass's bound lowered by the tile's drift.
-        const int sl = hsel * TC_M + r;
-        const int64_t rw = S.prow[sl];
-        const bool valid = *abort_flag == 0u;  // after a wait gave up, records start over (no bound)
-        if (rw < n) {
-            const float Df = Y.fin[sl];
-            const bool fin = valid && Df <= 3.402823466e38f;
-            const float dpn = fin ? __fsqrt_rd(__fmul_rd(Df, YY_ONE_M_G11)) : 0.f;  // <= the distance to any codeword
-            const float dref = fin ? __fsqrt_ru(__fmul_ru(Df, INV_ONE_M_G11_TC)) : __int_as_float(0x7f800000);
-            const float dpo = yread ? Y.dprev[sl] : 0.f;
-            const unsigned char *rs = yrec + sl * yy.stride;
-            uint4 *dst = reinterpret_cast<uint4 *>(yy.rec + rw * (int64_t)yy.stride);
-            for (int c = 0; c < yy.stride / 16; ++c) {
-                uint32_t wv[4] = {0u, 0u, 0u, 0u};
+}
+
+// The pruned assignment of the fit (yy: its state). The codebook is packed in the
+// order yy.cperm (tile g = positions [256 g, 256 g + 256)); indices and the tie rule
+// stay those of the original numbering. Every row keeps a record of one byte per
+// tile, q, with q * step + dprev <= its distance to every codeword of the tile, and
+// dprev <= its distance to every codeword: written at the end of each pass and, in
+// the next pass, lowered by the tile's drift (triangle inequality). A tile whose
+// bound proves every codeword farther than the row's hinted codeword, for all 256
+// rows of the CTA, is not streamed, multiplied or tested: the answer is the same,
+// since no skipped codeword could improve or tie the row's best.
+// Roles as in assign_tc_kernel (producer warp 0, MMA issuers warps 1-2, epilogue
+// warps 3-10), except that an epilogue thread owns one whole row: warps 3-6 drain
+// row tile 0 and warps 7-10 row tile 1, each thread reading all 256 columns of its
+// row per tile (two batches of four reducing 32-column loads; the candidate masks
+// are taken before the accumulator goes back). A row's best, threshold and bound
+// over a tile then live in one thread, and the bound costs one fused multiply-add
+// and a byte store per tile.
+template <bool TH>  // as assign_tc_kernel
+__global__ void __launch_bounds__(TC_THREADS, 1)
+assign_tc_pruned_kernel(const float *__restrict__ W, int64_t n, const float *__restrict__ C,
+                        const float *__restrict__ Cpk, int32_t K, int32_t ntiles, const int32_t *hint,
+                        const int32_t *__restrict__ perm, int32_t *idx, float *__restrict__ dist, Header *hdr,
+                        TcYy yy) {
+    constexpr int NST = TC_STAGES_YY;
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    TcPrunedShared &S = *reinterpret_cast<TcPrunedShared *>(smem_raw);
+    unsigned char *yrec = smem_raw + sizeof(TcPrunedShared);
+    const int ys = yy.stride + 4;  // record row pitch in shared memory
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    volatile uint32_t *abort_flag = &S.abort_flag;
+    uint32_t *status = &hdr->status;
+    const float beta = tc_scale(__uint_as_float(__ldcg(&hdr->cb_craw)));  // as pack_codebook_tc_kernel
+    const float beta2 = beta * beta;
+    const float inv_beta = 1.f / beta;  // exact: a power of two
+    const uint32_t tfault = TH ? __ldcg(&hdr->test_faults) : 0u;
+    const uint32_t tlim = TH ? __ldcg(&hdr->test_wait_limit) : 0u;
+    const long long wlim = (TH && tlim) ? (long long)tlim : TC_WAIT_LIMIT;
+    const int64_t row0 = (int64_t)blockIdx.x * TC_ROWS;
+    // bound step (fixed for the fit) and whether the records are valid
+    float ystep = 0.f, yinv = 0.f;
+    {
+        const float cn = __uint_as_float(__ldcg(&hdr->yy_cnorm));
+        if (cn > 0.f && cn <= 3.402823466e38f) {
+            int e;
+            frexpf(cn, &e);
+            const int ex = max(-100, min(100, e - YY_DELTA_SHIFT));
+            ystep = ldexpf(1.f, ex);
+            yinv = ldexpf(1.f, -ex);
+        }
+    }
+    const bool yread = yy.read != 0 && ystep > 0.f;
+
+    // ---- barriers first; the first tiles stream while the rows are set up: a run of
+    // NST consecutive tiles starting at (or just before) the one that holds the first
+    // slot's hinted codeword (the kd order puts neighbouring tiles close together);
+    // they are processed whatever the records say
+    const int pre = ntiles < NST ? ntiles : NST;
+    if (tid == 0) {
+        for (int s = 0; s < NST; ++s) {
+            mbar_init((uint32_t)__cvta_generic_to_shared(&S.full[s]), 1);
+            mbar_init((uint32_t)__cvta_generic_to_shared(&S.empty[s]), TC_EPI_WARPS);
+        }
+        for (int t = 0; t < TC_RT; ++t) {
+            mbar_init((uint32_t)__cvta_generic_to_shared(&S.tfull[t]), 1);
+            mbar_init((uint32_t)__cvta_generic_to_shared(&S.tempty[t]), TC_EPI_WARPS / TC_RT);
+        }
+        mbar_init((uint32_t)__cvta_generic_to_shared(&S.done), TC_RT);
+        S.abort_flag = 0u;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // initialised barriers -> bulk copies
+        const int g0 = yread ? yy_first_tile(hint, perm, row0, n, K, yy.cpos) : 0;
+        const int e0 = min(g0, ntiles - pre);
+        for (int i = 0; i < pre; ++i) {
+            const int g = e0 + i;
+            const uint32_t fb = (uint32_t)__cvta_generic_to_shared(&S.full[i]);
+            asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb), "r"(TC_TILE_BYTES)
+                         : "memory");
+            asm volatile(
+                "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                    (uint32_t)__cvta_generic_to_shared(S.b[i])),
+                "l"(reinterpret_cast<const unsigned char *>(Cpk) + (int64_t)g * TC_TILE_BYTES), "r"(TC_TILE_BYTES),
+                "r"(fb)
+                : "memory");
+        }
+    }
+
+    // ---- epilogue threads: one row each
+    const bool epi = warp >= TC_EPI_WARP0;
+    const int q = warp & 3;                                    // TMEM lane quarter this warp may access
+    const int t = epi ? (warp - TC_EPI_WARP0) >> 2 : 0;       // its row tile
+    const int r = q * 32 + lane;                               // row within the row tile
+    const int sl = t * TC_M + r;                               // the row's CTA slot
+    float best = __int_as_float(0x7f800000);
+    int32_t bi = 0, known = -1;  // known: codebook position of the codeword whose distance is best (-1: none)
+    bool ev = true;              // the row tests every codeword exactly
+    float tmaxv = -TC_T_EVERY, tabsv = TC_T_EVERY;  // largest T' and |T'| any MMA may have read
+    float ybase = __int_as_float(0x7fc00000), ydref = __int_as_float(0x7f800000);
+    float ysat = __int_as_float(0xff800000);  // yy_saturation of the row
+    float dpo = 0.f;  // the record's distance from the last pass
+    int64_t row = n;
+    if (epi) {
+        {
+            const int et = tid - TC_EPI_WARP0 * 32;
+            if (et < YY_MAX_TILES / 32) S.mask[et] = 0u;
+            if (et < YY_MAX_TILES / 4) {  // 4 tiles per word; tiles past the codebook never skip
+                uint32_t wd = 0u;
 #pragma unroll
-                for (int u = 0; u < 16; ++u) {
-                    const int g = c * 16 + u;
-                    uint32_t b = 0u;
-                    if (g < ntiles && fin) {
-                        b = rs[g];
-                        if (!((Y.mask[g >> 5] >> (g & 31)) & 1u)) {
-                            const float lb = __fsub_rd(__fadd_rd(__fmul_rd((float)b, ystep), dpo), Y.drift[g]);
-                            b = yy_encode(__fsub_rd(lb, dref), yinv);
+                for (int u = 0; u < 4; ++u) {
+                    const int g = 4 * et + u;
+                    const uint32_t b = (g < ntiles && yread) ? ceil_byte(__fmul_ru(__ldg(yy.tdrift + g), yinv)) : 255u;
+                    wd |= b << (8 * u);
+                }
+                S.dq[et] = wd;
+            }
+        }
+        const int64_t slot = row0 + sl;
+        row = slot < n ? (int64_t)__ldg(perm + slot) : n;
+        float x[D], ch[D];
+        const int32_t hv = (hint != nullptr && row < n) ? hint[row] : -1;
+        const bool hok = (uint32_t)hv < (uint32_t)K;
+#pragma unroll
+        for (int j = 0; j < D; ++j) x[j] = row < n ? W[row * D + j] : 0.f;
+#pragma unroll
+        for (int j = 0; j < D; ++j) ch[j] = hok ? C[(int64_t)hv * D + j] : 0.f;
+        float xs[D];
+#pragma unroll
+        for (int j = 0; j < D; ++j) xs[j] = beta * x[j];
+        bool ok = true;
+#pragma unroll
+        for (int j = 0; j < D; ++j) ok &= isfinite(x[j]);
+        if (row < n && !ok) set_flag(status, KQ_FLAG_NONFINITE);
+        const float cmax = __uint_as_float(__ldcg(&hdr->cb_cmax));  // scaled bounds
+        const float hmax = __uint_as_float(__ldcg(&hdr->cb_hmax));
+        const float qmax = __uint_as_float(__ldcg(&hdr->cb_qmax));
+        float x2lo = 0.f, x2hi = 0.f;
+#pragma unroll
+        for (int j = 0; j < D; ++j) {
+            x2lo = __fadd_rd(x2lo, __fmul_rd(xs[j], xs[j]));
+            x2hi = __fadd_ru(x2hi, __fmul_ru(xs[j], xs[j]));
+        }
+        const float xn = __fsqrt_ru(x2hi);
+        const bool inrange = xn <= TC_X_LIMIT;  // false for non-finite rows too
+        RowConst rc;
+        rc.R = inrange ? f16_rz(0.5f * x2lo) : 0.f;
+        if (rc.R < F16_MIN_NORMAL) rc.R = 0.f;
+        rc.k0 = inrange ? __fsub_rd(x2lo, qmax) : __int_as_float(0x7fc00000);  // NaN: never shifted
+        rc.k1 = __fadd_ru(__fadd_ru(hmax, __fmul_ru(xn, cmax)), fabsf(rc.R));
+        rc.k2 = __fmul_ru(TWO_ABS_TC, __fadd_ru(__fadd_ru(cmax, xn), 1.f));
+        float tp = 0.f;
+        if (hok) {
+            const float d = direct_distance(x, ch);
+            if (d < best) {
+                best = d;
+                bi = hv;
+                known = __ldg(yy.cpos + hv);
+                ev = !tc_shift(rc, d, beta2, tp);
+            }
+        }
+        S.prow[sl] = (int32_t)row;
+#pragma unroll
+        for (int j = 0; j < D; ++j) S.xs[sl][j] = x[j];
+        S.rc[sl] = rc;
+        {
+            float a[TC_KD], xa[D];
+#pragma unroll
+            for (int j = 0; j < D; ++j) xa[j] = inrange ? xs[j] : 0.f;
+            tc_row(xa, 1.f, true, a);
+            a[TC_SLOT_T0] = a[TC_SLOT_T1] = ev ? TC_T_EVERY : -tp;
+            a[TC_SLOT_R] = -rc.R;
+            tc_store_row(S.a[t], r, a);
+        }
+        tmaxv = ev ? -TC_T_EVERY : tp;
+        tabsv = ev ? TC_T_EVERY : fabsf(tp);
+        ybase = yy_base(rc, tmaxv, tabsv);
+        ydref = sqrt_above(__fmul_ru(best, INV_ONE_M_G11_TC));
+        ysat = yy_saturation(ybase, ydref, ystep, beta2);
+
+        // The tiles this CTA needs: tile g can be skipped for this row when its record's
+        // bound, lowered by the tile's drift, proves every codeword of g farther than
+        // the hinted codeword's distance (the row's best so far).
+        epi_sync();  // mask cleared, drifts staged
+        const bool all = !yread || !(best <= 3.402823466e38f);  // no valid record or no finite hint distance
+        dpo = (yread && row < n) ? yy.dprev[row] : 0.f;
+        const uint4 *src = reinterpret_cast<const uint4 *>(yy.rec + (row < n ? row : 0) * (int64_t)yy.stride);
+        uint32_t *dst = reinterpret_cast<uint32_t *>(yrec + sl * ys);
+        // the whole record in flight at once (one round trip to memory, not eight)
+        uint4 rv[YY_MAX_TILES / 16];
+#pragma unroll
+        for (int c = 0; c < YY_MAX_TILES / 16; ++c)
+            rv[c] = (row < n && !all && c * 16 < yy.stride) ? src[c] : make_uint4(0u, 0u, 0u, 0u);
+        // Tile g is skipped for this row when q_g step + dprev - drift_g > S, S >= the
+        // distance whose square times (1 - gamma_11) is the hint's distance (then every
+        // codeword of g is farther, in the direct form, than the hinted one): in whole
+        // steps, when q_g > base + dq_g (4 tiles per instruction, saturating at 255).
+        const float Sr = sqrt_above(__fmul_ru(best, INV_ONE_M_G11_TC));
+        const uint32_t base4 = ceil_byte(__fmul_ru(__fsub_ru(Sr, dpo), yinv)) * 0x01010101u;
+#pragma unroll
+        for (int w = 0; w < YY_MAX_TILES / 32; ++w) {
+            if (32 * w >= ntiles) break;
+            uint32_t need = 0u;
+            if (row < n) {
+                if (all) {
+                    need = 0xffffffffu;
+                } else {
+#pragma unroll
+                    for (int h2 = 0; h2 < 2; ++h2) {
+                        const int c = 2 * w + h2;
+                        if (c * 16 >= yy.stride) continue;  // a stride of 16 (mod 32) bytes
+                        const uint4 v = rv[c];
+                        dst[4 * c] = v.x;
+                        dst[4 * c + 1] = v.y;
+                        dst[4 * c + 2] = v.z;
+                        dst[4 * c + 3] = v.w;
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const uint32_t qw = k == 0 ? v.x : k == 1 ? v.y : k == 2 ? v.z : v.w;
+                            const uint32_t thr = __vaddus4(base4, S.dq[4 * c + k]);
+                            const uint32_t skip = bytes01_to_bits(__vcmpgtu4(qw, thr) & 0x01010101u);
+                            need |= ((~skip) & 0xfu) << (16 * h2 + 4 * k);
                         }
                     }
-                    wv[u >> 2] |= b << (8 * (u & 3));
                 }
-                dst[c] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+                const int left = ntiles - 32 * w;
+                if (left < 32) need &= (1u << left) - 1u;
             }
-            yy.dprev[rw] = dpn;
+            need = __reduce_or_sync(0xffffffffu, need);
+            if (lane == 0 && need) atomicOr(&S.mask[w], need);
         }
+        epi_sync();
+        if (warp == TC_EPI_WARP0) {
+            // the list: the early tile first (records read), then the others in order;
+            // lane l takes tiles 8 l .. 8 l + 7
+            const int g0 = yread ? yy_first_tile(hint, perm, row0, n, K, yy.cpos) : 0;  // as streamed
+            const int e0 = min(g0, ntiles - pre);
+            uint32_t bits = (S.mask[lane >> 2] >> ((lane & 3) * 8)) & 0xffu;
+#pragma unroll
+            for (int b = 0; b < 8; ++b)  // the early run goes first
+                if ((uint32_t)(lane * 8 + b - e0) < (uint32_t)pre) bits &= ~(1u << b);
+            const int cnt = __popc(bits);
+            int incl = cnt;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y2 = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += y2;
+            }
+            int pos = pre + incl - cnt;
+            while (bits) {
+                const int b = __ffs(bits) - 1;
+                bits &= bits - 1u;
+                S.tl[pos++] = (uint16_t)(lane * 8 + b);
+            }
+            if (lane == 31) S.nt = pre + incl;
+            if (lane < pre) {
+                const int g = e0 + lane;
+                S.tl[lane] = (uint16_t)g;
+                atomicOr(&S.mask[g >> 5], 1u << (g & 31));  // the mask now marks every processed tile
+            }
+        }
+    }
+
+    // ---- TMEM
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         (uint32_t)__cvta_generic_to_shared(&S.tmem_base)),
+                     "r"(TC_COLS)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // A tiles -> tensor core
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = S.tmem_base;
+    const int nt = S.nt;
+
+    if (warp == 0) {
+        // ---- producer (lane 0)
+        if (lane == 0) {
+            const int nlast = (TH && (tfault & KQ_TEST_STOP_TILE_STREAM)) ? pre : nt;
+            for (int i = pre; i < nlast; ++i) {  // list entries 0 .. pre - 1 are on their way
+                const int s = i % NST;
+                const int g = S.tl[i];
+                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.empty[s]), ((i / NST) - 1) & 1, abort_flag,
+                               status, wlim))
+                    break;
+                const uint32_t fb = (uint32_t)__cvta_generic_to_shared(&S.full[s]);
+                asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb), "r"(TC_TILE_BYTES)
+                             : "memory");
+                asm volatile(
+                    "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                        (uint32_t)__cvta_generic_to_shared(S.b[s])),
+                    "l"(reinterpret_cast<const unsigned char *>(Cpk) + (int64_t)g * TC_TILE_BYTES), "r"(TC_TILE_BYTES),
+                    "r"(fb)
+                    : "memory");
+            }
+        }
+    } else if (warp <= TC_RT) {
+        // ---- MMA issuer of row tile warp - 1 (lane 0)
+        const int ti = warp - 1;
+        if (lane == 0) {
+            constexpr uint32_t idesc = tc_idesc(TC_M, TC_N);
+            const uint32_t a0 = (uint32_t)__cvta_generic_to_shared(S.a[ti]);
+            const uint32_t dcol = tmem + (uint32_t)(ti * TC_N);
+            for (int i = 0; i < nt; ++i) {
+                const int s = i % NST;
+                if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.full[s]), (i / NST) & 1, abort_flag, status, wlim))
+                    break;
+                // the accumulator is free once its row tile's epilogue warps read tile i - 1
+                if (i >= 1 &&
+                    !mbar_wait((uint32_t)__cvta_generic_to_shared(&S.tempty[ti]), (i - 1) & 1, abort_flag, status, wlim))
+                    break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t b0 = (uint32_t)__cvta_generic_to_shared(S.b[s]);
+#pragma unroll
+                for (int kb = 0; kb < TC_KD / 16; ++kb) {
+                    const uint64_t ad = tc_smem_desc(a0 + kb * 2 * TC_LBO);
+                    const uint64_t bd = tc_smem_desc(b0 + kb * 2 * TC_LBO);
+                    asm volatile(
+                        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+                        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(dcol),
+                        "l"(ad), "l"(bd), "r"(idesc), "r"((uint32_t)kb)
+                        : "memory");
+                }
+                asm volatile(
+                    "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                        (uint32_t)__cvta_generic_to_shared(&S.tfull[ti]))
+                    : "memory");
+            }
+            const uint32_t db = (uint32_t)__cvta_generic_to_shared(&S.done);
+            asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(db)
+                         : "memory");
+            if (ti == 0) {
+                for (long long it = 0; it < wlim; ++it) {
+                    uint32_t okd;
+                    asm volatile(
+                        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n selp.u32 %0, 1, 0, p;\n}"
+                        : "=r"(okd)
+                        : "r"(db)
+                        : "memory");
+                    if (okd) break;
+                    if (it + 1 == wlim) set_flag(status, KQ_FLAG_TIMEOUT);
+                }
+            }
+        }
+    } else {
+        // ---- epilogue: per tile, load the row's 256 values in two batches with their
+        // chunk maxima, take the candidate masks of the chunks that may hold a codeword
+        // improving or tying the best, hand the accumulator back, then test the
+        // candidates exactly and record the row's bound for the tile
+        const uint32_t taddr0 = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(t * TC_N);
+        bool go = true;
+        for (int i = 0; i < nt && go; ++i) {
+            const int st = i % NST;
+            const int gb = (int)S.tl[i] * TC_N;  // codebook position of the tile's first codeword
+            if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&S.tfull[t]), i & 1, abort_flag, status, wlim)) {
+                go = false;
+                break;
+            }
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            uint32_t v[4][32];
+            float cm[4];
+            float m = __int_as_float(0xff800000);  // the row's largest g over the tile
+            uint32_t anym = 0u;                     // bit c: chunk c has candidates (masks in S.msk)
+#pragma unroll
+            for (int hb = 0; hb < 2; ++hb) {  // columns 128 hb .. 128 hb + 127
+#pragma unroll
+                for (int c = 0; c < 4; ++c) tc_ld32_max(taddr0 + (uint32_t)(128 * hb + 32 * c), v[c], cm[c]);
+                asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+                for (int c = 0; c < 4; ++c) tc_regs_ready(v[c], cm[c]);
+                const float mb = fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3]));
+                m = fmaxf(m, mb);
+                // one warp vote on the way to the hand-back; the masks only in the rare case
+                if (__any_sync(0xffffffffu, !(__float_as_uint(mb) >> 31) || ev)) {
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        const bool need = ev || !(__float_as_uint(cm[c]) >> 31);
+                        if (__any_sync(0xffffffffu, need) && need) {
+                            S.msk[sl][4 * hb + c] = ev ? 0xffffffffu : ~sign_mask32(v[c]);
+                            anym |= 1u << (4 * hb + c);
+                        }
+                    }
+                }
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            __syncwarp();
+            if (lane == 0)
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(
+                                 (uint32_t)__cvta_generic_to_shared(&S.tempty[t]))
+                             : "memory");
+            if (__any_sync(0xffffffffu, anym != 0u)) {  // rare: candidates
+                const unsigned char *tile = S.b[st];
+                bool moved = false;
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    uint32_t mask = ((anym >> c) & 1u) ? S.msk[sl][c] : 0u;
+                    const int kloc = known - (gb + 32 * c);
+                    if ((uint32_t)kloc < 32u) mask &= ~(1u << kloc);  // the best itself needs no test
+                    while (mask) {
+                        const int j = __ffs(mask) - 1;
+                        mask &= mask - 1u;
+                        const int kl = 32 * c + j;
+                        const int32_t p = gb + kl;
+                        if (p >= K) break;
+                        float xr[D], cw[D];
+                        const float *c32 = reinterpret_cast<const float *>(tile + TC_TILE_H) + kl * D;
+#pragma unroll
+                        for (int u = 0; u < D; ++u) {
+                            xr[u] = S.xs[sl][u];
+                            cw[u] = c32[u];
+                        }
+                        const float d = direct_distance(xr, cw);
+                        if (d <= best) {
+                            // the lowest original index wins a tie, whatever the packing order
+                            const int32_t k = __ldg(yy.cperm + p);
+                            if (d < best || k < bi) {
+                                best = d;
+                                bi = k;
+                                known = p;
+                                moved = true;
+                            }
+                        }
+                    }
+                }
+                if (moved) {
+                    float tp = 0.f;
+                    const bool e2 = !tc_shift(S.rc[sl], best, beta2, tp);
+                    ev = e2;
+                    const uint16_t tb = (uint16_t)f16_bits(e2 ? TC_T_EVERY : -tp);
+                    *reinterpret_cast<uint16_t *>(&S.a[t][tc_offset(r, TC_SLOT_T0)]) = tb;
+                    *reinterpret_cast<uint16_t *>(&S.a[t][tc_offset(r, TC_SLOT_T1)]) = tb;
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // for later MMAs
+                    const float tn = e2 ? -TC_T_EVERY : tp;
+                    tmaxv = fmaxf(tmaxv, tn);
+                    tabsv = fmaxf(tabsv, fabsf(tn));
+                    ybase = yy_base(S.rc[sl], tmaxv, tabsv);
+                    ydref = sqrt_above(__fmul_ru(best, INV_ONE_M_G11_TC));
+                    ysat = yy_saturation(ybase, ydref, ystep, beta2);
+                }
+            }
+            // the row's bound for this tile (D >= X2lo - Qmax - 2 e, e <= g + R + T' + E,
+            // g <= m, scaled units), recorded as slack over its current best
+            uint32_t qb = 255u;  // far tiles saturate: no square root
+            if (!(m <= ysat)) {
+                const float lb = __fmul_rd(sqrt_below(__fmaf_rd(-2.f, m, ybase)), inv_beta);
+                qb = yy_encode(__fsub_rd(lb, ydref), yinv);
+            }
+            yrec[sl * ys + gb / TC_N] = (unsigned char)qb;
+            __syncwarp();
+            if (lane == 0)
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"((uint32_t)__cvta_generic_to_shared(&S.empty[st]))
+                             : "memory");
+        }
+    }
+
+    // ---- teardown (a CTA barrier first)
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 1) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TC_COLS) : "memory");
+    }
+    if (epi && row < n) {
+        idx[row] = bi;
+        if (dist) dist[row] = best;
+        // the record for the next pass, relative to this pass's final best: processed
+        // tiles keep this pass's byte (slack over a best at least the final one), the
+        // others last pass's bound lowered by the tile's drift; after a wait gave up,
+        // no bound (zeros)
+        const bool fin = *abort_flag == 0u && best <= 3.402823466e38f;
+        const float dpn = fin ? __fsqrt_rd(__fmul_rd(best, YY_ONE_M_G11)) : 0.f;  // <= the distance to any codeword
+        const float dref = fin ? __fsqrt_ru(__fmul_ru(best, INV_ONE_M_G11_TC)) : __int_as_float(0x7f800000);
+        const uint32_t *rs = reinterpret_cast<const uint32_t *>(yrec + sl * ys);
+        uint4 *dstg = reinterpret_cast<uint4 *>(yy.rec + row * (int64_t)yy.stride);
+        // unprocessed tiles: q - dq_g - cr (saturating), cr = the change of reference in
+        // steps, rounded up: (q - dq - cr) step + dref <= q step + dprev - drift <= the
+        // distance to the tile, and the next pass decodes with dpn <= dref
+        const uint32_t cr4 = (fin ? ceil_byte(__fmul_ru(__fsub_ru(dref, dpo), yinv)) : 255u) * 0x01010101u;
+        for (int c = 0; c < yy.stride / 16; ++c) {
+            uint32_t wv[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int g0 = 16 * c + 4 * k;  // first of the word's 4 tiles
+                const uint32_t qw = rs[4 * c + k];
+                const uint32_t proc = bits_to_bytes01((S.mask[g0 >> 5] >> (g0 & 31)) & 0xfu) * 0xffu;
+                const uint32_t adj = __vsubus4(qw, __vaddus4(S.dq[4 * c + k], cr4));
+                wv[k] = fin ? ((qw & proc) | (adj & ~proc)) : 0u;
+            }
+            dstg[c] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+        }
+        yy.dprev[row] = dpn;
     }
 }
 
@@ -1341,30 +1672,31 @@ cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const fl
                              int *nblocksum, Header *hdr, cudaStream_t s, const TcYy *yy) {
     // One CTA per SM (it owns all of TMEM); the shared layout alone rules out a second.
     // (+ 1024: alignment slack of the dynamic base)
-    constexpr size_t plain = sizeof(TcShared<TC_STAGES>) + 1024;
-    constexpr size_t pruned_max = sizeof(TcShared<TC_STAGES_YY>) + sizeof(TcYyShared) + (size_t)TC_ROWS * YY_MAX_TILES + 1024;
+    constexpr size_t plain = sizeof(TcShared) + 1024;
+    constexpr size_t pruned_max = sizeof(TcPrunedShared) + (size_t)TC_ROWS * (YY_MAX_TILES + 4) + 1024;
     static_assert(plain <= 227 * 1024 && pruned_max <= 227 * 1024, "shared layout too large");
-    static_assert(plain > 114 * 1024 && sizeof(TcShared<TC_STAGES_YY>) + 1024 > 114 * 1024,
-                  "two CTAs per SM would share TMEM");
-    static_assert(sizeof(TcShared<TC_STAGES_YY>) % 16 == 0 && sizeof(TcYyShared) % 16 == 0, "record alignment");
+    static_assert(plain > 114 * 1024 && sizeof(TcPrunedShared) + 1024 > 114 * 1024, "two CTAs per SM would share TMEM");
+    static_assert(sizeof(TcPrunedShared) % 16 == 0, "record alignment");
     const int64_t blocks = (n + TC_ROWS - 1) / TC_ROWS;
     const int32_t ntiles = tc_kpad(K) / TC_N;
     cudaError_t e;
     if (yy) {
-        if (ntiles > YY_MAX_TILES || yy->stride < ntiles || yy->stride % 16 != 0) return cudaErrorInvalidValue;
-        const int smem = (int)(sizeof(TcShared<TC_STAGES_YY>) + sizeof(TcYyShared) + (size_t)TC_ROWS * yy->stride) + 1024;
-        e = cudaFuncSetAttribute(assign_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (ntiles > YY_MAX_TILES || yy->stride < ntiles || yy->stride % 16 != 0 || !perm || !dist)
+            return cudaErrorInvalidValue;
+        const int smem = (int)(sizeof(TcPrunedShared) + (size_t)TC_ROWS * (yy->stride + 4)) + 1024;
+        auto kern = test_hooks(hdr) ? assign_tc_pruned_kernel<true> : assign_tc_pruned_kernel<false>;
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
         launch_begin(s);
-        assign_tc_kernel<true><<<(unsigned)blocks, TC_THREADS, smem, s>>>(W, n, C, Cpk, K, ntiles, hint, perm, idx,
-                                                                        dist, blocksum, hdr, *yy);
-        launch_end(s, "assign_tc_kernel");
+        kern<<<(unsigned)blocks, TC_THREADS, smem, s>>>(W, n, C, Cpk, K, ntiles, hint, perm, idx, dist, hdr, *yy);
+        launch_end(s, "assign_tc_pruned_kernel");
     } else {
-        e = cudaFuncSetAttribute(assign_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plain);
+        auto kern = test_hooks(hdr) ? assign_tc_kernel<true> : assign_tc_kernel<false>;
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plain);
         if (e != cudaSuccess) return e;
         launch_begin(s);
-        assign_tc_kernel<false><<<(unsigned)blocks, TC_THREADS, (int)plain, s>>>(W, n, C, Cpk, K, ntiles, hint, perm,
-                                                                               idx, dist, blocksum, hdr, TcYy{});
+        kern<<<(unsigned)blocks, TC_THREADS, (int)plain, s>>>(W, n, C, Cpk, K, ntiles, hint, perm, idx, dist, blocksum,
+                                                             hdr);
         launch_end(s, "assign_tc_kernel");
     }
     *nblocksum = (int)blocks;

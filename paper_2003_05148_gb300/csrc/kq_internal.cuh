@@ -52,6 +52,9 @@ struct TcYy {
 // Fixed part of the workspace (first 4 KiB).
 struct Header {
     uint32_t status;        // sticky KQ_FLAG_* bits
+    // kq_test_inject_wait_fault (before the fields the entry points clear per call)
+    uint32_t test_faults;       // KQ_TEST_* bits
+    uint32_t test_wait_limit;   // poll limit of bounded waits (0: the normal ones)
     uint32_t maxabs_bits;   // max |W| as fp32 bits (update scale)
     uint32_t barrier;       // grid-barrier arrival counter (level fit)
     uint32_t abort;         // set when a bounded wait gives up
@@ -271,7 +274,9 @@ __device__ __forceinline__ bool grid_barrier(Header *h, unsigned nblocks, unsign
     ++epoch;
     if (threadIdx.x == 0) {
         __threadfence();
-        atomicAdd(&h->barrier, 1u);
+        // (failure-detection tests: CTA 0 may be told not to arrive, and the limit shortened)
+        if (!((h->test_faults & KQ_TEST_SKIP_ARRIVAL) && blockIdx.x == 0)) atomicAdd(&h->barrier, 1u);
+        const long long limit = h->test_wait_limit ? (long long)h->test_wait_limit : BARRIER_SPIN_LIMIT;
         const unsigned target = epoch * nblocks;
         int ok = 1;
         for (long long spin = 0;; ++spin) {
@@ -280,7 +285,7 @@ __device__ __forceinline__ bool grid_barrier(Header *h, unsigned nblocks, unsign
                 ok = 0;
                 break;
             }
-            if (spin > BARRIER_SPIN_LIMIT) {
+            if (spin > limit) {
                 atomicExch(&h->abort, 1u);
                 set_flag(&h->status, KQ_FLAG_TIMEOUT);
                 ok = 0;
@@ -294,6 +299,11 @@ __device__ __forceinline__ bool grid_barrier(Header *h, unsigned nblocks, unsign
     __syncthreads();
     return s_ok != 0;
 }
+
+// Whether kq_test_inject_wait_fault has set test faults or a wait limit on the workspace
+// whose header this is: the tensor-core assign kernels then run their instantiation
+// with the test hooks (the normal one keeps its wait limits compile-time constants).
+bool test_hooks(const Header *hdr);
 
 // Every kernel launch is bracketed by launch_begin(s) before it and launch_end(s,
 // name) after it (s: the launch stream, name: the kernel's, a string literal).

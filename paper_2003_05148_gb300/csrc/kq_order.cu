@@ -22,7 +22,7 @@ namespace kq {
 constexpr int KD_THREADS = 512;
 constexpr int KD_WARPS = KD_THREADS / 32;
 constexpr int KD_COV = D * (D + 1) / 2;  // distinct entries of the 9 x 9 covariance
-constexpr int KD_POWER_ITERS = 64;
+constexpr int KD_POWER_ITERS = 24;
 
 __device__ __forceinline__ int kd_tile_at(int64_t j, int32_t T, int level) { return (int)((j * T) >> level); }
 
@@ -104,30 +104,29 @@ __global__ void __launch_bounds__(KD_THREADS) kd_split_kernel(const float *__res
         s_cov[tid] = s;
     }
     __syncthreads();
-    if (tid == 0) {  // principal axis by power iteration (fp64)
-        double A[D][D];
-        int q = 0;
-        for (int a = 0; a < D; ++a)
-            for (int b = a; b < D; ++b) A[a][b] = A[b][a] = (double)s_cov[q++];
-        double v[D];
-        for (int u = 0; u < D; ++u) v[u] = 1.0 + 0.01 * u;  // not orthogonal to a dominant axis in practice
+    if (warp == 0) {  // principal axis by power iteration: lane a < 9 holds row a and v[a]
+        float Arow[D];
+#pragma unroll
+        for (int b = 0; b < D; ++b) {
+            const int lo = min(lane, b), hi = max(lane, b);  // upper-triangle index of (lo, hi)
+            Arow[b] = lane < D ? s_cov[lo * D - lo * (lo - 1) / 2 + (hi - lo)] : 0.f;
+        }
+        float v = lane < D ? 1.f + 0.01f * lane : 0.f;  // not orthogonal to a dominant axis in practice
         bool ok = true;
-        for (int it = 0; it < KD_POWER_ITERS && ok; ++it) {
-            double w[D], nrm = 0.0;
-            for (int a = 0; a < D; ++a) {
-                double s = 0.0;
-                for (int b = 0; b < D; ++b) s += A[a][b] * v[b];
-                w[a] = s;
-                nrm += s * s;
-            }
-            if (!(nrm > 0.0) || !(nrm < 1e300)) {
-                ok = false;
+        for (int it = 0; it < KD_POWER_ITERS; ++it) {
+            float w = 0.f;
+#pragma unroll
+            for (int b = 0; b < D; ++b) w = fmaf(Arow[b], __shfl_sync(0xffffffffu, v, b), w);
+            float nrm = w * w;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) nrm += __shfl_xor_sync(0xffffffffu, nrm, o);
+            if (!(nrm > 1e-36f) || !(nrm < 1e36f)) {  // degenerate or out of range: keep the last axis
+                ok = it > 0;
                 break;
             }
-            nrm = sqrt(nrm);
-            for (int a = 0; a < D; ++a) v[a] = w[a] / nrm;
+            v = w * rsqrtf(nrm);
         }
-        for (int a = 0; a < D; ++a) s_axis[a] = ok ? (float)v[a] : (a == 0 ? 1.f : 0.f);
+        if (lane < D) s_axis[lane] = ok ? v : (lane == 0 ? 1.f : 0.f);
     }
     __syncthreads();
     float ax[D];
@@ -152,9 +151,16 @@ __global__ void __launch_bounds__(KD_THREADS) kd_split_kernel(const float *__res
         for (int i = tid; i < 256; i += KD_THREADS) hist[i] = 0u;
         __syncthreads();
         const unsigned long long pre = s_prefix, msk = s_mask;
-        for (int64_t e = ea + tid; e < eb; e += KD_THREADS) {
-            const unsigned long long key = keys[e];
-            if ((key & msk) == pre) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+        for (int64_t e0 = ea; e0 < eb; e0 += KD_THREADS) {  // warp-uniform trip count
+            const int64_t e = e0 + tid;
+            unsigned int dg = 256u;  // no bin
+            if (e < eb) {
+                const unsigned long long key = keys[e];
+                if ((key & msk) == pre) dg = (unsigned int)(key >> shift) & 255u;
+            }
+            // lanes with the same digit add once (keys of a node cluster in few bins)
+            const unsigned int peers = __match_any_sync(0xffffffffu, dg);
+            if (dg < 256u && lane == __ffs(peers) - 1) atomicAdd(&hist[dg], (unsigned int)__popc(peers));
         }
         __syncthreads();
         if (tid == 0) {
@@ -176,15 +182,30 @@ __global__ void __launch_bounds__(KD_THREADS) kd_split_kernel(const float *__res
         __syncthreads();
     }
     const unsigned long long pivot = s_prefix;  // exactly r keys are below it
-    for (int64_t e = ea + tid; e < eb; e += KD_THREADS) {
-        const unsigned long long key = keys[e];
-        const int32_t k = (int32_t)(uint32_t)key;
-        if (key < pivot) {
-            const unsigned int s = atomicAdd(&s_left, 1u);
-            if ((int64_t)s < r) nxt[ea + s] = k;
-        } else {
-            const unsigned int s = atomicAdd(&s_right, 1u);
-            if (ea + r + (int64_t)s < eb) nxt[ea + r + s] = k;
+    for (int64_t e0 = ea; e0 < eb; e0 += KD_THREADS) {  // warp-uniform trip count
+        const int64_t e = e0 + tid;
+        const bool in = e < eb;
+        const unsigned long long key = in ? keys[e] : 0ull;
+        const bool left = in && key < pivot;
+        // one atomic per warp and side, lanes placed by their rank within the warp
+        const unsigned int bl = __ballot_sync(0xffffffffu, left), br = __ballot_sync(0xffffffffu, in && !left);
+        unsigned int basel = 0u, baser = 0u;
+        if (lane == 0) {
+            if (bl) basel = atomicAdd(&s_left, (unsigned int)__popc(bl));
+            if (br) baser = atomicAdd(&s_right, (unsigned int)__popc(br));
+        }
+        basel = __shfl_sync(0xffffffffu, basel, 0);
+        baser = __shfl_sync(0xffffffffu, baser, 0);
+        const unsigned int below = (1u << lane) - 1u;
+        if (in) {
+            const int32_t k = (int32_t)(uint32_t)key;
+            if (left) {
+                const unsigned int s = basel + __popc(bl & below);
+                if ((int64_t)s < r) nxt[ea + s] = k;
+            } else {
+                const unsigned int s = baser + __popc(br & below);
+                if (ea + r + (int64_t)s < eb) nxt[ea + r + s] = k;
+            }
         }
     }
     if (tid == 0) {

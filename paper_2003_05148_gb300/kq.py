@@ -20,13 +20,15 @@ KQ_OK = 0
 STATUS_NAMES = {0: "KQ_OK", 1: "KQ_ERR_INVALID_ARG", 2: "KQ_ERR_ALIGNMENT", 3: "KQ_ERR_NONFINITE",
                 4: "KQ_ERR_CUDA", 5: "KQ_ERR_DEVICE_CHECK", 6: "KQ_ERR_WORKSPACE", 7: "KQ_ERR_TIMEOUT"}
 FLAG_NONFINITE, FLAG_INDEX_RANGE, FLAG_CODE_RANGE, FLAG_TIMEOUT = 0x1, 0x2, 0x4, 0x8
-STOP_ON_STABLE, FIT_PLAIN = 0x1, 0x2  # kq_fit_codebook flags
+STOP_ON_STABLE, FIT_PRUNE = 0x1, 0x2  # kq_fit_codebook flags
+TEST_SKIP_ARRIVAL, TEST_STOP_TILE_STREAM = 0x1, 0x2  # kq_test_inject_wait_fault faults
 
 EXPORTS = ["kq_status_string", "kq_abi_version", "kq_kernel_launches", "kq_workspace_bytes", "kq_device_status", "kq_init_codebook",
            "kq_assign", "kq_update_centroids", "kq_fit_codebook", "kq_quantize_codebook_6bit", "kq_reconstruct",
            "kq_compression_report", "kq_conventional_ratio", "kq_assign_noalloc", "kq_quantize_scalars_6bit",
            "kq_codebook_grad_step", "kq_levels_grad_step", "kq_search_codebook_size", "kq_quantize_reconstruct",
-           "kq_seed_indices", "kq_trace_start", "kq_trace_stop", "kq_trace_count", "kq_trace_get"]
+           "kq_seed_indices", "kq_trace_start", "kq_trace_stop", "kq_trace_count", "kq_trace_get",
+           "kq_test_inject_wait_fault"]
 
 
 class KQError(RuntimeError):
@@ -58,6 +60,7 @@ def lib() -> ctypes.CDLL:
             "kq_trace_start": ([i32], ctypes.c_int),
             "kq_trace_stop": ([], ctypes.c_int),
             "kq_trace_count": ([], i32),
+            "kq_test_inject_wait_fault": ([P, sz, ctypes.c_uint32, ctypes.c_uint32, P], ctypes.c_int),
             "kq_trace_get": ([i32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(ctypes.c_float)], ctypes.c_int),
             "kq_workspace_bytes": ([i64, i32], sz),
             "kq_device_status": ([P, sz, P, P], ctypes.c_int),
@@ -193,6 +196,12 @@ def kq_device_status(ws: torch.Tensor, stream=None):
     with torch.cuda.device(c.device):
         st = lib().kq_device_status(ptr, ws.numel(), c.stream(stream), ctypes.byref(flags))
     return st, flags.value
+
+
+def kq_test_inject_wait_fault(ws, faults: int, wait_limit: int, stream=None) -> None:
+    """Failure-detection test hook: later calls on `ws` meet bounded waits that run out."""
+    c = _Call("kq_test_inject_wait_fault")
+    c(c.ptr(ws, "ws", torch.uint8), ws.numel(), faults, wait_limit, c.stream(stream))
 
 
 def kq_init_codebook(W, sel, C0, ws, stream=None) -> None:

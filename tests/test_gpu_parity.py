@@ -184,17 +184,22 @@ def test_assign_paths_agree():
     assert np.array_equal(i_w, i_tc) and bits_equal(d_w, d_tc)
 
 
-def test_assign_cold_pilot_path():
-    # K >= 16384 without a hint: a pilot pass against the first K / 16 codewords
-    # seeds the full pass; the answer is the plain argmin all the same (the CUDA-core
+@pytest.mark.parametrize("case", ["kd_leaf_hints", "pilot", "pilot_above_tree"])
+def test_assign_cold_start_paths(case):
+    # Without a hint on the tensor-core path, the full pass is seeded with hints: on
+    # large problems (n K >= 1e10, up to 65536 codewords) each kernel's nearest codeword
+    # in its k-d leaf tile, otherwise (from 16384 codewords) a pilot pass against the
+    # first K / 16 codewords. The answer is the plain argmin all the same (the CUDA-core
     # kernel, the oracle on sampled rows, and a run warm-started from the answer).
-    n, K = 2 * TC_MIN_N + 123, 16384 + 77
+    n, K = {"kd_leaf_hints": (655360 + 123, 16384 + 77), "pilot": (2 * TC_MIN_N + 123, 16384 + 77),
+            "pilot_above_tree": (2 * TC_MIN_N + 123, 65536 + 1000)}[case]
     W = synth.random_kernels(n, 9, 261, 0.05)
     C = W[synth.init_selection(n, K, 262)]
     i0, d0, st, _ = gpu_assign(W, C)
     assert st == 0
-    i_cc, d_cc = gpu_assign_cuda_cores(W, C)
-    assert np.array_equal(i0, i_cc) and bits_equal(d0, d_cc)
+    if K <= 65536:  # the allocation-free CUDA-core variant holds up to 65536 codewords
+        i_cc, d_cc = gpu_assign_cuda_cores(W, C)
+        assert np.array_equal(i0, i_cc) and bits_equal(d0, d_cc)
     rows = np.sort(synth.below(synth.stream_key(263, 9), 2000, n))
     idx_ref, dist_ref = oracle.assign(W[rows], C, threads=THREADS)
     assert check_indices(W, C, i0[rows], idx_ref, rows) == 0
@@ -707,8 +712,8 @@ def test_trace_times_every_launch_of_a_fit():
 # --------------------------------------------------------------------------- pruned fit
 
 def _fit_both(W, C0, iters):
-    pruned, run_p = _gpu_fit_run(W, C0, iters, 0)
-    plain, run_q = _gpu_fit_run(W, C0, iters, kq.FIT_PLAIN)
+    pruned, run_p = _gpu_fit_run(W, C0, iters, kq.FIT_PRUNE)
+    plain, run_q = _gpu_fit_run(W, C0, iters, 0)
     return pruned, plain
 
 
@@ -743,7 +748,7 @@ def test_fit_pruned_stepwise_against_oracle():
     lay, W, C0 = _layer(4, 8)
     C = C0
     for t in range(3):
-        (C_next, idx_next, cnt_next, obj), _ = _gpu_fit_run(W, C, 1, 0)
+        (C_next, idx_next, cnt_next, obj), _ = _gpu_fit_run(W, C, 1, kq.FIT_PRUNE)
         idx_ref, dist_ref = oracle.assign(W, C, threads=THREADS)
         C_ref, _ = oracle.update(W, idx_ref, C)
         check_centroids(C_next, C_ref)
@@ -752,7 +757,7 @@ def test_fit_pruned_stepwise_against_oracle():
         assert check_indices(W, C_next, idx_next, i2) == 0
         assert np.array_equal(cnt_next, np.bincount(idx_next, minlength=lay.K))
         C = C_next
-    (C_T, idx_T, _, obj_T), _ = _gpu_fit_run(W, C0, 3, 0)
+    (C_T, idx_T, _, obj_T), _ = _gpu_fit_run(W, C0, 3, kq.FIT_PRUNE)
     assert bits_equal(C_T, C)
     i3, _ = oracle.assign(W, C_T, threads=THREADS)
     assert check_indices(W, C_T, idx_T, i3) == 0
