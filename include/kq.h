@@ -371,6 +371,53 @@ kq_status kq_reconstruct(const int32_t *idx, int64_t n, const float *C, int32_t 
 kq_status kq_quantize_reconstruct(const int32_t *idx, int64_t n, const float *C, int32_t K, const float *levels,
                                   uint8_t *codes, float *W_out, void *ws, size_t ws_bytes, kq_stream_t stream);
 
+/* One layer of a network for kq_fit_layers. Every pointer is device memory owned
+ * by the caller, laid out as for the single-layer calls.
+ *   W, n, K    the layer's kernel matrix (n x 9 fp32, 16-byte aligned) and codebook size
+ *   sel        K row numbers (int64) or NULL: when given, the codebook starts as
+ *              C_0 = W[sel] (kq_init_codebook); when NULL, C holds C_0 on entry
+ *   C          K x 9 fp32: C_0 (read) and the fitted codebook (written)
+ *   idx, counts, objective   the fit's outputs (kq_fit_codebook; objective may be NULL)
+ *   levels, codes            64 fp32 / K x 9 uint8 outputs of the 6-bit codebook
+ *              quantisation (kq_quantize_codebook_6bit with `level_iters`), or both NULL
+ *   W_out      n x 9 fp32 output (16-byte aligned) of the K+C recovery
+ *              (kq_reconstruct from idx, codes and levels), or NULL; needs codes
+ *   ws, ws_bytes  this layer's own workspace of kq_workspace_bytes(n, K) bytes */
+typedef struct {
+    const float *W;
+    int64_t n;
+    int32_t K;
+    const int64_t *sel;
+    float *C;
+    int32_t *idx;
+    int32_t *counts;
+    double *objective;
+    float *levels;
+    uint8_t *codes;
+    float *W_out;
+    void *ws;
+    size_t ws_bytes;
+} kq_layer_job;
+
+/* Kernel quantisation of a whole network (Sec. 3.1-3.2 applied layer by layer):
+ * for every job, in one call,
+ *   [kq_init_codebook from sel] -> kq_fit_codebook(iters, flags)
+ *   -> [kq_quantize_codebook_6bit(level_iters)] -> [kq_reconstruct, K+C],
+ * a convenience over those calls with the same results, bit for bit. The layers
+ * are independent problems, so the library spreads them over up to eight internal
+ * streams of the current device (largest (iters + 1) n K first, each to the
+ * least-loaded stream), forked from `stream` and joined back into it: the
+ * latency-bound phases of one layer (small grids, grid barriers, launch gaps)
+ * overlap the work of others. Work enqueued on `stream` after the call starts
+ * after every layer is done; the call itself does not wait for the device.
+ *   jobs       count >= 1 layers (host array); every job needs its own workspace
+ *   iters      >= 0;  level_iters 0 .. 100000 (used when levels/codes are given)
+ *   flags      0 or KQ_FIT_PRUNE (KQ_STOP_ON_STABLE would synchronise per layer)
+ * Argument errors are reported before any work is enqueued; a failure while
+ * enqueueing returns its status after the streams already forked are joined. */
+kq_status kq_fit_layers(const kq_layer_job *jobs, int32_t count, int32_t iters, int32_t level_iters, int32_t flags,
+                        kq_stream_t stream);
+
 /* Storage accounting of one layer (host only, no device work), Sec. 3.2-3.3 and
  * Sec. 4.1:
  *   Eq. 4  total_bits B = k * omega^2 * b_c + n * ceil(log2 k)

@@ -60,7 +60,7 @@ __global__ void test_inject_kernel(Header *h, uint32_t faults, uint32_t limit) {
 
 namespace {
 
-constexpr int32_t KQ_ABI_VERSION = 5;
+constexpr int32_t KQ_ABI_VERSION = 6;
 constexpr int32_t HINT_ORDER_MIN_K = 4096;  // warm starts in hint order from 16 codeword tiles on
 // Cold assignments with many codeword tiles start from a pilot pass: rows against the
 // first K / COLD_PILOT_DIV codewords (a random sample when the codebook was drawn from

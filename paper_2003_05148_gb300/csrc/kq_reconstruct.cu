@@ -111,9 +111,29 @@ gather_rows_kernel(const int32_t *__restrict__ idx, int64_t n, const float *__re
     if (__any_sync(0xffffffffu, bad) && lane == 0) set_flag(status, KQ_FLAG_INDEX_RANGE);
 }
 
-// The loop of gather_codes_kernel over the chunks of CTA `cta` of `ncta` (and the
-// ragged end in CTA 0); lv is the replicated level table, ra/j0/split the lane's
-// float4 slots. Returns whether this thread saw an index outside [0, K).
+// Index loads of chunk pair c2 (two chunks of 32 kernels, the second only when it
+// exists) and the code-word gathers of a loaded pair.
+__device__ __forceinline__ void gc_load_idx(const int32_t *__restrict__ idx, int64_t nch, int64_t c2, int lane,
+                                            int32_t (&k)[2]) {
+    k[0] = __ldcs(idx + 2 * c2 * 32 + lane);
+    k[1] = 2 * c2 + 1 < nch ? __ldcs(idx + (2 * c2 + 1) * 32 + lane) : 0;
+}
+__device__ __forceinline__ void gc_gather(const unsigned long long *__restrict__ Cq, int32_t K, const int32_t (&k)[2],
+                                          bool two, unsigned long long (&q)[2], bool &bad) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const bool ok = (uint32_t)k[h] < (uint32_t)K;
+        bad |= !ok && (h == 0 || two);
+        q[h] = ok ? __ldg(Cq + k[h]) : ALL_CODES_OUT_OF_RANGE;
+    }
+}
+
+// The loop of gather_codes_kernel over the chunk pairs of CTA `cta` of `ncta` (and
+// the ragged end in CTA 0); lv is the replicated level table, ra/j0/split the lane's
+// float4 slots. Software-pipelined by one pair: while pair c2 is decoded and
+// stored, the code words of the warp's next pair and the indices of the one after
+// are already in flight, so a warp waits for neither the index read from DRAM nor
+// the gather from L2. Returns whether this thread saw an index outside [0, K).
 __device__ __forceinline__ bool gather_codes_rows(const int32_t *__restrict__ idx, int64_t n,
                                                   const unsigned long long *__restrict__ Cq, int32_t K,
                                                   float *__restrict__ W_out, const float (*lv)[32], const int *ra,
@@ -121,26 +141,28 @@ __device__ __forceinline__ bool gather_codes_rows(const int32_t *__restrict__ id
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     bool bad = false;
     const int64_t nch = n / 32;
-    // two chunks per warp step: both index loads, then both code gathers are in
-    // flight before any decoding
-    const int64_t nch2 = nch / 2;
-    for (int64_t c2 = cta * R_WARPS + warp; c2 < nch2 + (nch & 1); c2 += ncta * R_WARPS) {
-        const int64_t ch0 = 2 * c2;
-        const bool two = ch0 + 1 < nch;
+    const int64_t npairs = nch / 2 + (nch & 1);
+    const int64_t step = ncta * R_WARPS;
+    int64_t c2 = cta * R_WARPS + warp;
+    int32_t kn[2] = {0, 0};
+    unsigned long long q[2] = {0ull, 0ull};
+    if (c2 < npairs) {
         int32_t k[2];
-        k[0] = __ldcs(idx + ch0 * 32 + lane);
-        k[1] = two ? __ldcs(idx + (ch0 + 1) * 32 + lane) : 0;
-        unsigned long long q[2];
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const bool ok = (uint32_t)k[h] < (uint32_t)K;
-            bad |= !ok && (h == 0 || two);
-            q[h] = ok ? __ldg(Cq + k[h]) : ALL_CODES_OUT_OF_RANGE;
-        }
+        gc_load_idx(idx, nch, c2, lane, k);
+        if (c2 + step < npairs) gc_load_idx(idx, nch, c2 + step, lane, kn);
+        gc_gather(Cq, K, k, 2 * c2 + 1 < nch, q, bad);
+    }
+    for (; c2 < npairs; c2 += step) {
+        const int64_t c2n = c2 + step;
+        unsigned long long qn[2] = {0ull, 0ull};
+        int32_t knn[2] = {0, 0};
+        if (c2n < npairs) gc_gather(Cq, K, kn, 2 * c2n + 1 < nch, qn, bad);
+        if (c2n + step < npairs) gc_load_idx(idx, nch, c2n + step, lane, knn);
+        const bool two = 2 * c2 + 1 < nch;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
             if (h == 1 && !two) break;
-            const int64_t r0 = (ch0 + h) * 32;
+            const int64_t r0 = (2 * c2 + h) * 32;
             const uint32_t qlo = (uint32_t)q[h], qhi = (uint32_t)(q[h] >> 32);
             float4 *d4 = reinterpret_cast<float4 *>(W_out + r0 * D);
 #pragma unroll
@@ -160,6 +182,10 @@ __device__ __forceinline__ bool gather_codes_rows(const int32_t *__restrict__ id
                 if (s < 2 || lane < 32 * D / 4 - 64) __stcs(d4 + lane + 32 * s, make_float4(r[0], r[1], r[2], r[3]));
             }
         }
+        q[0] = qn[0];
+        q[1] = qn[1];
+        kn[0] = knn[0];
+        kn[1] = knn[1];
     }
     // ragged end (< 32 kernels): CTA 0, plain loads and stores
     if (cta == 0) {
@@ -175,25 +201,27 @@ __device__ __forceinline__ bool gather_codes_rows(const int32_t *__restrict__ id
     return bad;
 }
 
-// K+C recovery. A warp owns 32 consecutive kernels (1152 output bytes = 72 float4).
-// Each lane fetches the packed codes of its own kernel (one 8-byte word, instead of
-// a 36-byte row), then produces output float4 number lane, lane + 32 and (lanes
-// 0-7) lane + 64 directly: the at most two kernels a float4 spans send their code
-// words by shuffle, and every code is looked up in a level table replicated across
-// the 32 shared-memory banks (level l for lane L at [l][L]: no bank conflicts). No
-// staging tile; the stores are coalesced streaming float4 stores. Launched as a
-// programmatic dependent of decode_codebook_kernel (the launch and the level table
-// overlap the decode; Cq is read after griddepcontrol.wait): 47.3 -> 44.0 us per
-// call on the stress layer. (Prefetching the next step's indices, and 4 instead
-// of 8 CTAs per SM, measured faster alone but slower inside the fit's step.)
-__global__ void __launch_bounds__(R_THREADS)
+// K+C recovery. A warp owns pairs of 32-kernel chunks (1152 output bytes = 72
+// float4 each). Each lane fetches the packed codes of its own kernel (one 8-byte
+// word, instead of a 36-byte row), then produces output float4 number lane,
+// lane + 32 and (lanes 0-7) lane + 64 of a chunk directly: the at most two
+// kernels a float4 spans send their code words by shuffle, and every code is
+// looked up in a level table replicated across the 32 shared-memory banks (level
+// l for lane L at [l][L]: no bank conflicts). The stores are coalesced streaming
+// float4 stores; one resident wave of CTAs, each warp's loop software-pipelined
+// (gather_codes_rows). Launched as a programmatic dependent of
+// decode_codebook_kernel (the launch and the level table overlap the decode; Cq is
+// read after griddepcontrol.wait). Stress layer (n = 4,194,304), minimum of 30
+// calls: 42.9 us with two waves and no pipelining, 41.5 us as here; decoding
+// each lane's own kernel into a staging tile instead of the shuffles: 42.8 us.
+__global__ void __launch_bounds__(R_THREADS, 4)
 gather_codes_kernel(const int32_t *__restrict__ idx, int64_t n, const unsigned long long *__restrict__ Cq,
                     const float *__restrict__ levels, int32_t K, float *__restrict__ W_out, uint32_t *status) {
     __shared__ float lv[LEVELS + 1][32];  // row LEVELS decodes out-of-range codes to 0
     for (int e = threadIdx.x; e < (LEVELS + 1) * 32; e += R_THREADS)
         lv[e / 32][e % 32] = e / 32 < LEVELS ? levels[e / 32] : 0.f;
     __syncthreads();
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int lane = threadIdx.x & 31;
     // slot s: float4 v = lane + 32 s of the chunk; its first element is coordinate
     // j0 of kernel ra, elements e < split belong to ra, the rest to ra + 1
     int ra[3], j0[3], split[3];
@@ -214,7 +242,7 @@ gather_codes_kernel(const int32_t *__restrict__ idx, int64_t n, const unsigned l
 // kernel indices), one cooperative launch: every CTA encodes a grid-stride share of
 // the codewords into the packed code words of gather_codes_kernel (and the code
 // bytes, when asked for), all CTAs meet at a bounded grid barrier, then gather.
-__global__ void __launch_bounds__(R_THREADS)
+__global__ void __launch_bounds__(R_THREADS, 3)
 encode_gather_kernel(const float *__restrict__ C, int32_t K, const float *__restrict__ levels,
                      uint8_t *__restrict__ codes, unsigned long long *__restrict__ Cq, const int32_t *__restrict__ idx,
                      int64_t n, float *__restrict__ W_out, Header *hdr) {
@@ -286,8 +314,13 @@ cudaError_t launch_gather_rows(const int32_t *idx, int64_t n, const float *Cp, c
                                const float *levels, int32_t K, float *W_out, uint32_t *status, int num_sms,
                                cudaStream_t s) {
     if (Cq) {
+        // one resident wave (the loop is pipelined across a warp's pairs)
+        int per_sm = 0;
+        cudaError_t e0 = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, gather_codes_kernel, R_THREADS, 0);
+        if (e0 != cudaSuccess) return e0;
+        if (per_sm < 1) per_sm = 1;
         int64_t blocks = ((n / 32 + 1) / 2 + R_WARPS - 1) / R_WARPS;
-        if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
+        if (blocks > (int64_t)per_sm * num_sms) blocks = (int64_t)per_sm * num_sms;
         if (blocks < 1) blocks = 1;
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3((unsigned)blocks);

@@ -28,13 +28,21 @@ EXPORTS = ["kq_status_string", "kq_abi_version", "kq_kernel_launches", "kq_works
            "kq_compression_report", "kq_conventional_ratio", "kq_assign_noalloc", "kq_quantize_scalars_6bit",
            "kq_codebook_grad_step", "kq_levels_grad_step", "kq_search_codebook_size", "kq_quantize_reconstruct",
            "kq_seed_indices", "kq_trace_start", "kq_trace_stop", "kq_trace_count", "kq_trace_get",
-           "kq_test_inject_wait_fault"]
+           "kq_test_inject_wait_fault", "kq_fit_layers"]
 
 
 class KQError(RuntimeError):
     def __init__(self, fn: str, status: int):
         self.status = status
         super().__init__(f"{fn} failed: {STATUS_NAMES.get(status, status)}")
+
+
+class LayerJob(ctypes.Structure):
+    """kq_layer_job (include/kq.h): one layer of kq_fit_layers."""
+    _fields_ = [("W", ctypes.c_void_p), ("n", ctypes.c_int64), ("K", ctypes.c_int32), ("sel", ctypes.c_void_p),
+                ("C", ctypes.c_void_p), ("idx", ctypes.c_void_p), ("counts", ctypes.c_void_p),
+                ("objective", ctypes.c_void_p), ("levels", ctypes.c_void_p), ("codes", ctypes.c_void_p),
+                ("W_out", ctypes.c_void_p), ("ws", ctypes.c_void_p), ("ws_bytes", ctypes.c_size_t)]
 
 
 class Report(ctypes.Structure):
@@ -80,6 +88,7 @@ def lib() -> ctypes.CDLL:
             "kq_quantize_reconstruct": ([P, i64, P, i32, P, P, P, P, sz, P], ctypes.c_int),
             "kq_search_codebook_size": ([P, i64, P, i32, ctypes.c_double, ctypes.c_double, i32, i32, P, P, P,
                                          P, P, P, P, P, P, sz, P], ctypes.c_int),
+            "kq_fit_layers": ([ctypes.POINTER(LayerJob), i32, i32, i32, i32, P], ctypes.c_int),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -237,6 +246,23 @@ def kq_fit_codebook(W, C_init, iters, C_out, idx, counts, objective, ws, stream=
         c.ptr(objective, "objective", torch.float64), ctypes.byref(run), c.ptr(ws, "ws", torch.uint8), ws.numel(),
         c.stream(stream))
     return run.value
+
+
+def kq_fit_layers(jobs, iters: int, level_iters: int = 100, flags: int = 0, stream=None) -> None:
+    """All layers of a network in one call (kq_layer_job per layer). Each job is a
+    dict with tensors W, C, idx, counts, ws and optionally sel, objective, levels,
+    codes, W_out (absent or None: not given); all on one device."""
+    c = _Call("kq_fit_layers")
+    arr = (LayerJob * len(jobs))()
+    for i, j in enumerate(jobs):
+        g = j.get
+        arr[i] = LayerJob(
+            c.ptr(j["W"], "W", torch.float32), _rows(j["W"]), _rows(j["C"]), c.ptr(g("sel"), "sel", torch.int64),
+            c.ptr(j["C"], "C", torch.float32), c.ptr(j["idx"], "idx", torch.int32),
+            c.ptr(j["counts"], "counts", torch.int32), c.ptr(g("objective"), "objective", torch.float64),
+            c.ptr(g("levels"), "levels", torch.float32), c.ptr(g("codes"), "codes", torch.uint8),
+            c.ptr(g("W_out"), "W_out", torch.float32), c.ptr(j["ws"], "ws", torch.uint8), j["ws"].numel())
+    c(arr, len(jobs), iters, level_iters, flags, c.stream(stream))
 
 
 def kq_quantize_codebook_6bit(C, counts, max_iters, levels, codes, iters_run, ws, stream=None) -> None:

@@ -37,7 +37,7 @@ def test_exports_every_declared_symbol(lib):
 
 
 def test_status_strings_and_version(lib):
-    assert kq.kq_abi_version() == 5
+    assert kq.kq_abi_version() == 6
     for code, name in kq.STATUS_NAMES.items():
         assert kq.kq_status_string(code) == name
     assert kq.kq_status_string(99) == "KQ_ERR_UNKNOWN"
@@ -168,6 +168,33 @@ def test_conventional_ratio_matches_oracle(lib):
         kq.kq_compression_report(0, 4)
 
 
+def _job(base, **kw):
+    g = lambda a: ctypes.c_void_p((1 << 20) + (base << 12) + a)  # distinct 256-byte aligned dummies
+    d = dict(W=g(0), n=1024, K=16, sel=None, C=g(256), idx=g(512), counts=g(768), objective=None, levels=None,
+             codes=None, W_out=None, ws=g(1024), ws_bytes=kq.kq_workspace_bytes(1024, 16))
+    d.update(kw)
+    return kq.LayerJob(**d)
+
+
+def test_fit_layers_arguments_checked_on_host(lib):
+    # every rejection happens before any CUDA call (the dummy pointers are never used)
+    assert ctypes.sizeof(kq.LayerJob) == 104  # the C struct: 12 pointer-sized fields and n, K (padded)
+    FL = lib.kq_fit_layers
+    one = (kq.LayerJob * 1)(_job(1))
+    assert FL(None, 1, 3, 10, 0, None) == 1
+    assert FL(one, 0, 3, 10, 0, None) == 1
+    assert FL(one, 1, -1, 10, 0, None) == 1
+    assert FL(one, 1, 3, 100001, 0, None) == 1
+    assert FL(one, 1, 3, 10, kq.STOP_ON_STABLE, None) == 1  # would synchronise per layer
+    bad = [_job(1, n=0), _job(1, K=2048), _job(1, W=None), _job(1, ws=None),
+           _job(1, levels=ctypes.c_void_p(1 << 24)),  # levels without codes
+           _job(1, W_out=ctypes.c_void_p(1 << 24))]  # recovery without codes
+    for j in bad:
+        assert FL((kq.LayerJob * 1)(j), 1, 3, 10, 0, None) == 1
+    two = (kq.LayerJob * 2)(_job(1), _job(2, ws=_job(1).ws))  # one workspace for two layers
+    assert FL(two, 2, 3, 10, 0, None) == 1
+
+
 def test_trace_arguments_checked_on_host(lib):
     assert lib.kq_trace_start(0) == 1
     assert lib.kq_trace_start((1 << 20) + 1) == 1
@@ -195,3 +222,5 @@ def test_cuda_failure_returns_status_without_device(lib):
     assert L.kq_quantize_reconstruct(good, 1024, good, 16, good, None, good, good, ws_bytes, None) == 4
     assert L.kq_device_status(good, ws_bytes, None, None) == 4
     assert L.kq_trace_start(4) == 4  # no device to make events on
+    jobs = (kq.LayerJob * 2)(_job(1), _job(2))
+    assert L.kq_fit_layers(jobs, 2, 3, 10, kq.FIT_PRUNE, None) == 4
