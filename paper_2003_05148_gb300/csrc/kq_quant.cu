@@ -328,6 +328,330 @@ cudaError_t launch_level_fit_t(const LevelArgs &args, int num_sms, cudaStream_t 
     return cudaGetLastError();
 }
 
+// ---- The same level fit on one thread-block cluster, for up to LFC_MAX_CL x
+// ~13K scalars (a codebook of up to ~23K codewords): every CTA of the cluster keeps
+// its slice of the scalars in shared memory for the whole fit (value, weight x
+// fixed-point value, code; the weights per codeword), the per-level integer sums
+// of the CTAs are exchanged through distributed shared memory, and the CTAs meet at
+// the cluster's hardware barrier instead of a grid barrier in global memory. Every
+// per-scalar decision and every sum is the grid kernel's (the same nearest-level
+// functions, the same fixed-point values, exact integer sums), so levels, codes
+// and iteration count are bit-identical to it. It occupies LFC_MAX_CL SMs or fewer,
+// so other work (another layer's fit) runs beside it.
+constexpr int LFC_THREADS = 1024;
+constexpr int LFC_WARPS = LFC_THREADS / 32;
+constexpr int LFC_MAX_CL = 16;
+constexpr int64_t LFC_MIN_PER_CTA = 4096;  // fewer CTAs while each would hold fewer scalars than this
+
+struct LfcPhase0 {
+    uint32_t lo_w, hi_w, lo_a, hi_a, maxv_w;  // ordered-int minima / maxima (maxv_w: fp32 bits)
+    uint32_t flags;
+    unsigned long long wt;
+};
+
+struct LfcShared {
+    uint32_t bins[LFC_WARPS][LEVELS][4];         // per warp: q lo, q hi, w lo, w hi (carry-propagated)
+    unsigned long long red[16][LEVELS][2];       // CTA reduction partials (w, q)
+    unsigned long long tot[2][LEVELS][2];        // CTA totals per level (w, q), by iteration parity
+    uint32_t chg[2];                             // "a code of this CTA changed", by parity
+    LfcPhase0 p0, all;                           // this CTA's phase-0 figures, and the cluster's
+    float L[LEVELS];
+    uint8_t Tb[Q_TABLE];
+    float tlo, tinv;
+    int sorted, any_changed;
+};
+
+// unsigned 64-bit add into a (lo, hi) pair of 32-bit shared words with two 32-bit
+// atomics: the carry out of the low word is the add's own (exact under any order)
+__device__ __forceinline__ void add64_carry(uint32_t *lohi, unsigned long long x) {
+    const uint32_t xl = (uint32_t)x;
+    const uint32_t old = atomicAdd(lohi, xl);
+    const uint32_t carry = (old + xl) < old ? 1u : 0u;
+    const uint32_t xh = (uint32_t)(x >> 32) + carry;
+    if (xh) atomicAdd(lohi + 1, xh);
+}
+
+__device__ __forceinline__ uint32_t cluster_map(const void *p, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"((uint32_t)__cvta_generic_to_shared(p)), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ unsigned long long dsmem_ld64(uint32_t a) {
+    unsigned long long v;
+    asm volatile("ld.shared::cluster.u64 %0, [%1];" : "=l"(v) : "r"(a) : "memory");
+    return v;
+}
+__device__ __forceinline__ uint32_t dsmem_ld32(uint32_t a) {
+    uint32_t v;
+    asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
+    return v;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+constexpr size_t LFC_HDR = (sizeof(LfcShared) + 15) / 16 * 16;
+
+// per: codewords (or, UNIT, scalars) per CTA; len_max = scalars per CTA at most.
+// Grid = one cluster. Shared memory: LfcShared, then the slice's weight x fixed-point
+// values (8 B), values (4 B), weights per codeword (4 B per 9) and codes (1 B).
+template <bool UNIT>
+__global__ void __launch_bounds__(LFC_THREADS, 1) level_fit_cluster_kernel(LevelArgs a, int64_t per, int64_t len_max) {
+    extern __shared__ __align__(16) unsigned char lfc_smem[];
+    LfcShared &S = *reinterpret_cast<LfcShared *>(lfc_smem);
+    unsigned long long *zq = reinterpret_cast<unsigned long long *>(lfc_smem + LFC_HDR);
+    float *vv = reinterpret_cast<float *>(zq + len_max);
+    int32_t *zz = reinterpret_cast<int32_t *>(vv + len_max);
+    uint8_t *cc = reinterpret_cast<uint8_t *>(zz + (UNIT ? 0 : len_max / D));
+    Header *h = a.hdr;
+    const int64_t N = a.N;
+    const uint32_t rank = blockIdx.x, cl = gridDim.x;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    int64_t e0, e1;  // this CTA's scalars
+    if (UNIT) {
+        e0 = min(N, (int64_t)rank * per);
+        e1 = min(N, e0 + per);
+    } else {
+        const int64_t K = N / D, k0 = min(K, (int64_t)rank * per), k1 = min(K, k0 + per);
+        e0 = k0 * D;
+        e1 = k1 * D;
+    }
+    const int len = (int)(e1 - e0);
+
+    // Phase 0 (as the grid kernel): value ranges, max |v|, total weight; the slice
+    // is loaded into shared memory on the way.
+    if (tid == 0) {
+        S.p0 = LfcPhase0{0xffffffffu, 0u, 0xffffffffu, 0u, 0u, 0u, 0ull};
+        S.all = S.p0;
+    }
+    __syncthreads();
+    {
+        float lo_w = __int_as_float(0x7f800000), hi_w = -lo_w, lo_a = lo_w, hi_a = -lo_w, mv = 0.f;
+        unsigned long long wt = 0;
+        bool ok = true, badc = false;
+        for (int i = tid; i < len; i += LFC_THREADS) {
+            const float v = a.C[e0 + i];
+            vv[i] = v;
+            int32_t z = UNIT ? 1 : a.counts[(e0 + i) / D];
+            if (z < 0) {
+                badc = true;
+                z = 0;
+            }
+            if (!UNIT && i % D == 0) zz[i / D] = z;
+            if (!isfinite(v)) {
+                ok = false;
+                continue;
+            }
+            lo_a = fminf(lo_a, v);
+            hi_a = fmaxf(hi_a, v);
+            if (z > 0) {
+                lo_w = fminf(lo_w, v);
+                hi_w = fmaxf(hi_w, v);
+                mv = fmaxf(mv, fabsf(v));
+                wt += (unsigned long long)z;
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            lo_w = fminf(lo_w, __shfl_xor_sync(0xffffffffu, lo_w, o));
+            hi_w = fmaxf(hi_w, __shfl_xor_sync(0xffffffffu, hi_w, o));
+            lo_a = fminf(lo_a, __shfl_xor_sync(0xffffffffu, lo_a, o));
+            hi_a = fmaxf(hi_a, __shfl_xor_sync(0xffffffffu, hi_a, o));
+            mv = fmaxf(mv, __shfl_xor_sync(0xffffffffu, mv, o));
+            wt += __shfl_xor_sync(0xffffffffu, wt, o);
+        }
+        const bool all_ok = __all_sync(0xffffffffu, ok), any_bad = __any_sync(0xffffffffu, badc);
+        if (lane == 0) {
+            atomicMin(&S.p0.lo_w, f2ord(lo_w));
+            atomicMax(&S.p0.hi_w, f2ord(hi_w));
+            atomicMin(&S.p0.lo_a, f2ord(lo_a));
+            atomicMax(&S.p0.hi_a, f2ord(hi_a));
+            atomicMax(&S.p0.maxv_w, __float_as_uint(mv));
+            if (wt) atomicAdd(&S.p0.wt, wt);
+            if (!all_ok) set_flag(&h->status, KQ_FLAG_NONFINITE);
+            if (any_bad) set_flag(&h->status, KQ_FLAG_INDEX_RANGE);
+        }
+    }
+    cluster_sync_all();
+    if (tid < (int)cl) {  // the cluster's figures from every CTA's
+        const uint32_t r = cluster_map(&S.p0, (uint32_t)tid);
+        const uint32_t lw = dsmem_ld32(r), hw = dsmem_ld32(r + 4), la = dsmem_ld32(r + 8), ha = dsmem_ld32(r + 12),
+                       mx = dsmem_ld32(r + 16);
+        const unsigned long long wt = dsmem_ld64(r + 24);
+        atomicMin(&S.all.lo_w, lw);
+        atomicMax(&S.all.hi_w, hw);
+        atomicMin(&S.all.lo_a, la);
+        atomicMax(&S.all.hi_a, ha);
+        atomicMax(&S.all.maxv_w, mx);
+        if (wt) atomicAdd(&S.all.wt, wt);
+    }
+    __syncthreads();
+
+    // Initial levels and the fixed-point scale (as the grid kernel)
+    const unsigned long long A = S.all.wt;
+    const bool any = A > 0;
+    const float lo = ord2f(any ? S.all.lo_w : S.all.lo_a);
+    const float hi = ord2f(any ? S.all.hi_w : S.all.hi_a);
+    const float M = __uint_as_float(S.all.maxv_w);
+    int Sx = 0;
+    if (any && M > 0.f) {
+        int e;
+        frexp(__dmul_rn(__ull2double_rn(A), (double)M), &e);
+        Sx = 62 - e;
+    }
+    const double down = ldexp(1.0, -Sx);
+    if (tid < LEVELS) {
+        const double t = __ddiv_rn(__dmul_rn(__dsub_rn((double)hi, (double)lo), (double)tid), 63.0);
+        S.L[tid] = __double2float_rn(__dadd_rn((double)lo, t));
+    }
+    for (int i = tid; i < len; i += LFC_THREADS) {
+        const int32_t z = UNIT ? 1 : zz[i / D];
+        zq[i] = z > 0 ? (unsigned long long)((long long)z * fixed_rn(vv[i], Sx)) : 0ull;
+    }
+    __syncthreads();
+    build_table(S.L, S.Tb, S.sorted, S.tlo, S.tinv, true);
+
+    int32_t updates = 0;
+    for (int32_t it = 0; it < a.max_iters; ++it) {
+        const int par = it & 1;
+        uint32_t *wb = &S.bins[warp][0][0];
+        for (int e = lane; e < LEVELS * 4; e += 32) wb[e] = 0u;
+        if (tid == 0) {
+            S.chg[par] = 0u;  // last read by the other CTAs before the previous cluster barrier
+            S.any_changed = 0;
+        }
+        __syncthreads();
+        bool changed = false;
+        const bool sorted = S.sorted;
+        const float tlo = S.tlo, tinv = S.tinv;
+        for (int i = tid; i < len; i += LFC_THREADS) {
+            const int code = sorted ? nearest_level_table(vv[i], S.L, S.Tb, tlo, tinv) : nearest_level(vv[i], S.L);
+            changed |= it > 0 && cc[i] != (uint8_t)code;
+            cc[i] = (uint8_t)code;
+            const int32_t z = UNIT ? 1 : zz[i / D];
+            if (z > 0) {
+                add64_carry(&S.bins[warp][code][0], zq[i]);
+                add64_carry(&S.bins[warp][code][2], (unsigned long long)z);
+            }
+        }
+        if (__any_sync(0xffffffffu, changed) && lane == 0) atomicOr(&S.chg[par], 1u);
+        __syncthreads();
+        {  // CTA totals per level: 16 partials of 2 warps each, then their sum
+            const int l = tid & (LEVELS - 1), part = tid >> 6;
+            unsigned long long sq = 0ull, sw = 0ull;
+#pragma unroll
+            for (int w = 2 * part; w < 2 * part + 2; ++w) {
+                const uint4 b = *reinterpret_cast<const uint4 *>(&S.bins[w][l][0]);
+                sq += ((unsigned long long)b.y << 32) | b.x;
+                sw += ((unsigned long long)b.w << 32) | b.z;
+            }
+            S.red[part][l][0] = sw;
+            S.red[part][l][1] = sq;
+        }
+        __syncthreads();
+        if (tid < LEVELS) {
+            unsigned long long sw = 0ull, sq = 0ull;
+#pragma unroll
+            for (int p = 0; p < 16; ++p) {
+                sw += S.red[p][tid][0];
+                sq += S.red[p][tid][1];
+            }
+            S.tot[par][tid][0] = sw;
+            S.tot[par][tid][1] = sq;
+        }
+        cluster_sync_all();
+        // the cluster's totals (each CTA sums every CTA's, in the same exact integers):
+        // thread (r, l) fetches CTA r's totals of level l (S.red is free again)
+        {
+            const int l = tid & (LEVELS - 1), r = tid >> 6;
+            if (r < (int)cl) {
+                const uint32_t ra = cluster_map(&S.tot[par][l][0], (uint32_t)r);
+                S.red[r][l][0] = dsmem_ld64(ra);
+                S.red[r][l][1] = dsmem_ld64(ra + 8);
+                if (l == 0 && dsmem_ld32(cluster_map(&S.chg[par], (uint32_t)r))) atomicOr(&S.any_changed, 1);
+            }
+        }
+        __syncthreads();
+        unsigned long long Wl = 0ull, Ql = 0ull;
+        if (tid < LEVELS)
+            for (int r = 0; r < (int)cl; ++r) {
+                Wl += S.red[r][tid][0];
+                Ql += S.red[r][tid][1];
+            }
+        if (it > 0 && S.any_changed == 0) break;  // the same decision in every CTA
+        if (tid < LEVELS && Wl > 0)
+            S.L[tid] = __double2float_rn(__ddiv_rn(__dmul_rn(__ll2double_rn((long long)Ql), down), __ull2double_rn(Wl)));
+        __syncthreads();
+        build_table(S.L, S.Tb, S.sorted, S.tlo, S.tinv, true);
+        ++updates;
+    }
+
+    // codes of the final levels
+    __syncthreads();
+    {
+        const bool sorted = S.sorted;
+        const float tlo = S.tlo, tinv = S.tinv;
+        for (int i = tid; i < len; i += LFC_THREADS)
+            a.codes[e0 + i] =
+                (uint8_t)(sorted ? nearest_level_table(vv[i], S.L, S.Tb, tlo, tinv) : nearest_level(vv[i], S.L));
+    }
+    if (rank == 0) {
+        if (tid < LEVELS) a.levels[tid] = S.L[tid];
+        if (tid == 0 && a.iters_run) *a.iters_run = updates;
+    }
+    cluster_sync_all();  // no CTA leaves while another may still read its shared memory
+}
+
+// Launches the cluster kernel when the fit fits one cluster; *launched = false
+// (and nothing enqueued) otherwise.
+template <bool UNIT>
+cudaError_t launch_level_fit_cluster_t(const LevelArgs &args, cudaStream_t s, bool *launched) {
+    *launched = false;
+    const int64_t units = UNIT ? args.N : args.N / D;  // scalars, or codewords of 9 scalars
+    const int64_t unit_len = UNIT ? 1 : D;
+    int dev = 0, optin = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    if (e != cudaSuccess) return e;
+    auto kern = level_fit_cluster_kernel<UNIT>;
+    for (int cap = LFC_MAX_CL; cap >= 8; cap /= 2) {
+        int cl = 1;
+        while (cl < cap && (units + cl - 1) / cl * unit_len > LFC_MIN_PER_CTA) cl *= 2;
+        const int64_t per = (units + cl - 1) / cl;
+        const int64_t len_max = per * unit_len;
+        const size_t smem = LFC_HDR + (size_t)len_max * (8 + 4 + 1) + (UNIT ? 0 : (size_t)per * 4);
+        if (smem > (size_t)optin) return cudaSuccess;  // too large for one cluster: the grid kernel
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e == cudaSuccess && cl > 8) e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (e != cudaSuccess) return e;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((unsigned)cl);
+        cfg.blockDim = dim3(LFC_THREADS);
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = s;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = (unsigned)cl;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int nclusters = 0;
+        if (cudaOccupancyMaxActiveClusters(&nclusters, kern, &cfg) != cudaSuccess || nclusters < 1) {
+            (void)cudaGetLastError();  // not schedulable at this size: try a smaller cluster
+            continue;
+        }
+        LevelArgs a = args;
+        launch_begin(s);
+        e = cudaLaunchKernelEx(&cfg, kern, a, per, len_max);
+        if (e != cudaSuccess) return e;
+        launch_end(s, "level_fit_cluster_kernel");
+        *launched = true;
+        return cudaGetLastError();
+    }
+    return cudaSuccess;
+}
+
 cudaError_t launch_level_fit(const float *C, int64_t N, const int32_t *counts, int32_t max_iters, float *levels,
                              uint8_t *codes, int32_t *iters_run, Header *hdr, int num_sms, cudaStream_t s) {
     // Clear everything but the sticky status word; minima start at the top of the order.
@@ -336,6 +660,12 @@ cudaError_t launch_level_fit(const float *C, int64_t N, const int32_t *counts, i
     e = cudaMemsetAsync(&hdr->lo_w, 0xff, 2 * sizeof(uint32_t), s);
     if (e != cudaSuccess) return e;
     const LevelArgs args{C, N, counts, max_iters, levels, codes, iters_run, hdr, 0};
+    if (!test_hooks(hdr)) {  // (the failure-detection tests exercise the grid kernel's bounded barrier)
+        bool launched = false;
+        e = counts ? launch_level_fit_cluster_t<false>(args, s, &launched)
+                   : launch_level_fit_cluster_t<true>(args, s, &launched);
+        if (e != cudaSuccess || launched) return e;
+    }
     return counts ? launch_level_fit_t<false>(args, num_sms, s) : launch_level_fit_t<true>(args, num_sms, s);
 }
 

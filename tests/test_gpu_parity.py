@@ -548,7 +548,8 @@ def test_fit_deterministic():
 
 # --------------------------------------------------------------------------- 6-bit quantisation
 
-@pytest.mark.parametrize("K,seed,high", [(1, 1, 5), (16, 2, 300), (256, 3, 600), (5000, 4, 100), (65536, 5, 128)])
+@pytest.mark.parametrize("K,seed,high", [(1, 1, 5), (16, 2, 300), (256, 3, 600), (5000, 4, 100), (16384, 6, 64),
+                                         (20000, 7, 40), (24000, 8, 40), (65536, 5, 128)])
 def test_quantize_random_codebooks(K, seed, high):
     C = synth.random_kernels(K, 9, seed, 0.02)
     counts = synth.random_counts(K, seed + 100, high)
