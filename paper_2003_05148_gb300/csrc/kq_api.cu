@@ -312,6 +312,24 @@ int ceil_log2_i64(int64_t k) {
 
 }  // namespace
 
+namespace kq {
+kq_status quantize_codebook(const float *C, int32_t K, const int32_t *counts, int32_t max_iters, float *levels,
+                            uint8_t *codes, int32_t *iters_run, void *ws, size_t ws_bytes, cudaStream_t s,
+                            bool shared_gpu) {
+    if (K < 1 || (int64_t)K * D >= (1LL << 31) || !C || !counts || !levels || !codes) return KQ_ERR_INVALID_ARG;
+    if (max_iters < 0 || max_iters > 100000) return KQ_ERR_INVALID_ARG;
+    if (!aligned(C, 4) || !aligned(counts, 4) || !aligned(levels, 4) || !aligned(iters_run, 4))
+        return KQ_ERR_ALIGNMENT;
+    kq_status st = check_ws_header(ws, ws_bytes);
+    if (st != KQ_OK) return st;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != KQ_OK) return st;
+    Header *h = static_cast<Header *>(ws);
+    return cuda_status(
+        launch_level_fit(C, (int64_t)K * D, counts, max_iters, levels, codes, iters_run, h, sms, s, shared_gpu));
+}
+}  // namespace kq
+
 extern "C" {
 
 const char *kq_status_string(kq_status s) {
@@ -573,17 +591,8 @@ kq_status kq_search_codebook_size(const float *W, int64_t n, const int64_t *sel,
 kq_status kq_quantize_codebook_6bit(const float *C, int32_t K, const int32_t *counts, int32_t max_iters,
                                     float *levels, uint8_t *codes, int32_t *iters_run, void *ws, size_t ws_bytes,
                                     kq_stream_t stream) {
-    if (K < 1 || (int64_t)K * D >= (1LL << 31) || !C || !counts || !levels || !codes) return KQ_ERR_INVALID_ARG;
-    if (max_iters < 0 || max_iters > 100000) return KQ_ERR_INVALID_ARG;
-    if (!aligned(C, 4) || !aligned(counts, 4) || !aligned(levels, 4) || !aligned(iters_run, 4))
-        return KQ_ERR_ALIGNMENT;
-    kq_status st = check_ws_header(ws, ws_bytes);
-    if (st != KQ_OK) return st;
-    int sms = 0;
-    if ((st = num_sms(&sms)) != KQ_OK) return st;
-    Header *h = static_cast<Header *>(ws);
-    return cuda_status(launch_level_fit(C, (int64_t)K * D, counts, max_iters, levels, codes, iters_run, h, sms,
-                                        reinterpret_cast<cudaStream_t>(stream)));
+    return quantize_codebook(C, K, counts, max_iters, levels, codes, iters_run, ws, ws_bytes,
+                             reinterpret_cast<cudaStream_t>(stream), false);
 }
 
 kq_status kq_quantize_scalars_6bit(const float *v, int64_t m, int32_t max_iters, float *levels, uint8_t *codes,

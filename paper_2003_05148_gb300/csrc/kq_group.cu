@@ -131,9 +131,9 @@ extern "C" kq_status kq_fit_layers(const kq_layer_job *jobs, int32_t count, int3
         if (st == KQ_OK)
             st = kq_fit_codebook(j.W, j.n, j.K, j.C, iters, flags, j.C, j.idx, j.counts, j.objective, nullptr, j.ws,
                                  j.ws_bytes, ls);
-        if (st == KQ_OK && j.codes)
-            st = kq_quantize_codebook_6bit(j.C, j.K, j.counts, level_iters, j.levels, j.codes, nullptr, j.ws,
-                                           j.ws_bytes, ls);
+        if (st == KQ_OK && j.codes)  // (the one-cluster level fit where it fits: other layers run beside it)
+            st = quantize_codebook(j.C, j.K, j.counts, level_iters, j.levels, j.codes, nullptr, j.ws, j.ws_bytes,
+                                   pool->s[li], true);
         if (st == KQ_OK && j.W_out)
             st = kq_reconstruct(j.idx, j.n, nullptr, j.K, j.codes, j.levels, j.W_out, j.ws, j.ws_bytes, ls);
     }

@@ -385,8 +385,15 @@ cudaError_t launch_small_fit(const float *W, int64_t n, const float *C0, int32_t
                              float *cbuf1, double *blocksum, int max_blocksum, Header *hdr, int num_sms,
                              cudaStream_t s, bool stop_on_stable = false);
 
+// shared_gpu: other work runs beside this fit (kq_fit_layers), so the one-cluster
+// kernel is taken wherever it fits; alone, only where it is also the faster one.
 cudaError_t launch_level_fit(const float *C, int64_t N, const int32_t *counts, int32_t max_iters, float *levels,
-                             uint8_t *codes, int32_t *iters_run, Header *hdr, int num_sms, cudaStream_t s);
+                             uint8_t *codes, int32_t *iters_run, Header *hdr, int num_sms, cudaStream_t s,
+                             bool shared_gpu = false);
+// kq_quantize_codebook_6bit with that choice (kq_api.cu)
+kq_status quantize_codebook(const float *C, int32_t K, const int32_t *counts, int32_t max_iters, float *levels,
+                            uint8_t *codes, int32_t *iters_run, void *ws, size_t ws_bytes, cudaStream_t s,
+                            bool shared_gpu);
 
 // Retraining with averaged gradients (Eq. 2): codebook finalise over the update's
 // accumulators, and the 64-level segment mean of the quantised codebook.

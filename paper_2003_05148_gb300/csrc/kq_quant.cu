@@ -342,6 +342,7 @@ constexpr int LFC_THREADS = 1024;
 constexpr int LFC_WARPS = LFC_THREADS / 32;
 constexpr int LFC_MAX_CL = 16;
 constexpr int64_t LFC_MIN_PER_CTA = 4096;  // fewer CTAs while each would hold fewer scalars than this
+constexpr int64_t LFC_ALONE_MAX_N = 9 * 8192;  // scalars up to which it also wins alone on the GPU
 
 struct LfcPhase0 {
     uint32_t lo_w, hi_w, lo_a, hi_a, maxv_w;  // ordered-int minima / maxima (maxv_w: fp32 bits)
@@ -653,14 +654,20 @@ cudaError_t launch_level_fit_cluster_t(const LevelArgs &args, cudaStream_t s, bo
 }
 
 cudaError_t launch_level_fit(const float *C, int64_t N, const int32_t *counts, int32_t max_iters, float *levels,
-                             uint8_t *codes, int32_t *iters_run, Header *hdr, int num_sms, cudaStream_t s) {
+                             uint8_t *codes, int32_t *iters_run, Header *hdr, int num_sms, cudaStream_t s,
+                             bool shared_gpu) {
     // Clear everything but the sticky status word; minima start at the top of the order.
     cudaError_t e = cudaMemsetAsync(&hdr->maxabs_bits, 0, sizeof(Header) - offsetof(Header, maxabs_bits), s);
     if (e != cudaSuccess) return e;
     e = cudaMemsetAsync(&hdr->lo_w, 0xff, 2 * sizeof(uint32_t), s);
     if (e != cudaSuccess) return e;
     const LevelArgs args{C, N, counts, max_iters, levels, codes, iters_run, hdr, 0};
-    if (!test_hooks(hdr)) {  // (the failure-detection tests exercise the grid kernel's bounded barrier)
+    // Alone on the GPU the cluster kernel is the faster one up to ~8K codewords (per
+    // iteration at K = 512 / 4096 / 16384: 5.1 / 6.3 / 11.1 us against the grid
+    // kernel's 6.2 / 6.9 / 9.4 us); beside other work it always is, as it leaves
+    // all but 16 SMs free. (The failure-detection tests exercise the grid kernel's
+    // bounded barrier.)
+    if ((shared_gpu || N <= LFC_ALONE_MAX_N) && !test_hooks(hdr)) {
         bool launched = false;
         e = counts ? launch_level_fit_cluster_t<false>(args, s, &launched)
                    : launch_level_fit_cluster_t<true>(args, s, &launched);
