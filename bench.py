@@ -475,7 +475,8 @@ def run_kq(args, rank, world, local_rank):
         a = bytes_per_launch / t / 1e9
         tc = statistics.mean(call_ms) / 1e3
         ac = call_bytes / tc / 1e9
-        return {"bound": "hbm", "achieved": a, "peak": hbm, "unit": "GB/s", "frac": a / hbm,
+        return {"bound": "hbm", "achieved": a, "peak": hbm, "unit": "GB/s", "frac": a / hbm, "target_frac": 0.6,
+                "target_met": a / hbm >= 0.6,
                 "traffic": traffic.get(kernel), "kernel": kernel, "launches": len(ms_list), "us_mean": 1e6 * t,
                 "algorithmic_bytes": int(bytes_per_launch), "note": note,
                 "whole_call": {"us_mean": 1e6 * tc, "calls": len(call_ms), "algorithmic_bytes": int(call_bytes),

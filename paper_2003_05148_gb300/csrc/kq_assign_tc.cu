@@ -95,11 +95,13 @@ namespace kq {
 constexpr int TC_M = 128;                  // rows per MMA (row tile)
 constexpr int TC_RT = 2;                   // row tiles per CTA
 constexpr int TC_ROWS = TC_M * TC_RT;      // kernels per CTA
-// Warm starts with 1024 to 4096 codewords (no global hint order) group a CTA's rows by
+// Warm starts with 256 to 4096 codewords (no global hint order) group a CTA's rows by
 // the 32-codeword chunk of their hint: at most 128 chunks, plus rows without a hint.
-// (With fewer codeword tiles the sort costs more than it saves: 86 vs 91 us at K = 512,
-// n = 262,144; 148 vs 142 us at K = 2048.)
-constexpr int32_t TC_LGROUP_MINK = 1024;
+// In a fit's later passes (few rows change codeword) this keeps a warp's exact-path
+// entries to its hints' few chunks: at n = 262,144, K = 512, 56 instead of 63 us per
+// pass (VGG-16's 13 layers 19.6 instead of 20.3 ms per fit); the first warm pass after
+// an update, where many rows move, gains nothing (85 us either way).
+constexpr int32_t TC_LGROUP_MINK = 256;
 constexpr int32_t TC_LGROUP_MAXK = 4096;
 constexpr int TC_LBINS = TC_LGROUP_MAXK / 32 + 1;
 // TC_N codewords per tile (N of every MMA), TC_KD = K of the GEMM in fp16 elements

@@ -184,6 +184,49 @@ def test_assign_paths_agree():
     assert np.array_equal(i_w, i_tc) and bits_equal(d_w, d_tc)
 
 
+@pytest.mark.parametrize("K", [1, 100, 256, 512, 1025, 1536])
+def test_assign_small_codebook_many_blocks(K):
+    # small codebooks (one to six codeword tiles) over several waves of row blocks
+    # and a ragged last block; cold and warm-started, the warm rows grouped by hinted
+    # chunk inside each CTA from 256 codewords on. Bit-identical to the CUDA-core
+    # kernel, and to the oracle on sampled rows.
+    n = 7 * TC_MIN_N + 77
+    W = synth.random_kernels(n, 9, 271 + K, 0.05)
+    C = W[synth.init_selection(n, K, 272 + K)]
+    i_tc, d_tc, st, _ = gpu_assign(W, C)
+    assert st == 0
+    i_cc, d_cc = gpu_assign_cuda_cores(W, C)
+    assert np.array_equal(i_tc, i_cc) and bits_equal(d_tc, d_cc)
+    hint = synth.below(synth.stream_key(273 + K, 9), n, K).astype(np.int32)
+    hint[::2] = i_tc[::2]
+    i_w, d_w, st, _ = gpu_assign(W, C, hint=hint)
+    assert st == 0 and np.array_equal(i_w, i_tc) and bits_equal(d_w, d_tc)
+    rows = np.sort(synth.below(synth.stream_key(274 + K, 9), 3000, n))
+    rows[-1] = n - 1
+    idx_ref, dist_ref = oracle.assign(W[rows], C, threads=THREADS)
+    assert check_indices(W, C, i_tc[rows], idx_ref, rows) == 0
+    assert bits_equal(d_tc[rows], dist_ref)
+
+
+def test_fit_small_codebook_objective():
+    # the fit's objective at a small codebook comes from the assign kernel's per-CTA
+    # partial sums (fixed order, rows grouped by hint inside each CTA): the oracle's
+    # objective of the same assignment; the final assignment and counts are those of
+    # the fit's own codebook
+    n, K = 3 * TC_MIN_N + 5, 700
+    W = synth.random_kernels(n, 9, 281, 0.05)
+    C0 = W[synth.init_selection(n, K, 282)]
+    C1, idx1, cnt1, obj = _gpu_fit(W, C0, 1)
+    idx_ref, dist_ref = oracle.assign(W, C0, threads=THREADS)
+    assert obj[0] == pytest.approx(oracle.objective(dist_ref), rel=1e-12)
+    C_ref, _ = oracle.update(W, idx_ref, C0)
+    check_centroids(C1, C_ref)
+    i2, d2 = oracle.assign(W, C1, threads=THREADS)
+    assert check_indices(W, C1, idx1, i2) == 0
+    assert np.array_equal(cnt1, np.bincount(idx1, minlength=K))
+    assert obj[1] == pytest.approx(oracle.objective(d2), rel=1e-12)
+
+
 @pytest.mark.parametrize("case", ["kd_leaf_hints", "pilot", "pilot_above_tree"])
 def test_assign_cold_start_paths(case):
     # Without a hint on the tensor-core path, the full pass is seeded with hints: on
