@@ -474,7 +474,7 @@ struct TcShared {
     int32_t lhint[TC_ROWS];  // CTA-local grouping: the hint of each CTA row
     uint32_t lcnt[TC_LBINS];
     float rowbest[TC_ROWS];  // each CTA row's distance, for the objective's partial sum in row order
-    double wsum[TC_EPI_WARPS / 2][TC_RT];
+    F2 wsum[TC_EPI_WARPS / 2][TC_RT];  // per-warp partial sums (double-float)
 };
 
 // Shared layout of the pruned kernel (assign_tc_pruned_kernel); the per-row bound
@@ -971,18 +971,16 @@ assign_tc_kernel(const float *__restrict__ W, int64_t n, const float *__restrict
         asm volatile("bar.sync 2, 128;" ::: "memory");  // the 128 threads of the first half
 #pragma unroll
         for (int t = 0; t < TC_RT; ++t) {
-            double sum = (double)S.rowbest[t * TC_M + r];
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+            const F2 sum = f2_warp_sum(S.rowbest[t * TC_M + r]);
             if (lane == 0) S.wsum[warp - TC_EPI_WARP0][t] = sum;
         }
     }
     __syncthreads();
-    if (tid == 0) {
-        double s = 0.0;
+    if (tid == 0) {  // rows 0-31, 32-63, ... of the CTA in turn, as dist_block_sums_kernel
+        F2 s{0.f, 0.f};
         for (int t = 0; t < TC_RT; ++t)
-            for (int w = 0; w < TC_EPI_WARPS / 2; ++w) s += S.wsum[w][t];
-        if (blocksum) blocksum[blockIdx.x] = s;
+            for (int w = 0; w < TC_EPI_WARPS / 2; ++w) s = f2_add(s, S.wsum[w][t]);
+        if (blocksum) blocksum[blockIdx.x] = f2_to_double(s);
     }
     if (warp == 1) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
@@ -1618,17 +1616,15 @@ __global__ void __launch_bounds__(256) hint_scatter_kernel(const int32_t *__rest
 // blocksum[b] = sum of dist over rows [256 b, 256 b + 256) in a fixed order (fp64).
 __global__ void __launch_bounds__(256) dist_block_sums_kernel(const float *__restrict__ dist, int64_t n,
                                                               double *__restrict__ blocksum) {
-    __shared__ double ws[8];
+    __shared__ F2 ws[8];
     const int64_t i = (int64_t)blockIdx.x * 256 + threadIdx.x;
-    double v = i < n ? (double)__ldcs(dist + i) : 0.0;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    const F2 v = f2_warp_sum(i < n ? __ldcs(dist + i) : 0.f);
     if ((threadIdx.x & 31) == 0) ws[threadIdx.x >> 5] = v;
     __syncthreads();
     if (threadIdx.x == 0) {
-        double t = 0.0;
-        for (int w = 0; w < 8; ++w) t += ws[w];
-        blocksum[blockIdx.x] = t;
+        F2 t{0.f, 0.f};
+        for (int w = 0; w < 8; ++w) t = f2_add(t, ws[w]);
+        blocksum[blockIdx.x] = f2_to_double(t);
     }
 }
 

@@ -256,6 +256,37 @@ __device__ __forceinline__ bool levels_sorted(const float *L) {
 }
 
 
+// Objective partial sums of a block of non-negative fp32 distances, in a fixed
+// order and in double-float: an fp32 pair (hi, lo) holds the running sum hi + lo.
+// One step: s = fl(a.hi + b.hi) with its exact rounding error (Knuth's TwoSum), the
+// low parts added to that error, renormalised (Dekker's FastTwoSum). With every term
+// non-negative each step is relatively accurate to ~2^-47, so a 256-term block sum is
+// within ~1e-13 of the exact sum; fp32 operations with explicit rounding (no FMA
+// contraction), far faster than GB300's fp64 pipe.
+struct F2 {
+    float hi, lo;
+};
+__device__ __forceinline__ F2 f2_add(F2 a, F2 b) {
+    const float s = __fadd_rn(a.hi, b.hi);
+    const float bb = __fsub_rn(s, a.hi);
+    float e = __fadd_rn(__fsub_rn(a.hi, __fsub_rn(s, bb)), __fsub_rn(b.hi, bb));
+    e = __fadd_rn(e, __fadd_rn(a.lo, b.lo));
+    const float hi = __fadd_rn(s, e);
+    return F2{hi, __fsub_rn(e, __fsub_rn(hi, s))};
+}
+// a warp's 32 values (lane i holds v), summed by an xor butterfly: every lane ends
+// with the same pair (each step is symmetric in its operands)
+__device__ __forceinline__ F2 f2_warp_sum(float v) {
+    F2 s{v, 0.f};
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const F2 t{__shfl_xor_sync(0xffffffffu, s.hi, o), __shfl_xor_sync(0xffffffffu, s.lo, o)};
+        s = f2_add(s, t);
+    }
+    return s;
+}
+__device__ __forceinline__ double f2_to_double(F2 s) { return (double)s.hi + (double)s.lo; }
+
 __device__ __forceinline__ bool finite9(const float *v) {
     bool ok = true;
 #pragma unroll
