@@ -50,13 +50,13 @@ struct SmallFitArgs {
 // p % SF_SPLIT == s (consecutive lanes read consecutive pairs: no bank conflicts), and
 // the lanes' (distance, index) minima merge lexicographically, so the lowest index
 // wins ties as in one sequential scan. Lane s < SF_ROWS then records kernel s.
-__device__ __forceinline__ double small_fit_assign(const SmallFitArgs &a, const unsigned long long (*cp)[SF_MAX_K / 2],
+__device__ __forceinline__ F2 small_fit_assign(const SmallFitArgs &a, const unsigned long long (*cp)[SF_MAX_K / 2],
                                                    int32_t npairs, int S, bool accumulate, bool &nonfinite,
                                                    bool compare, bool &moved) {
     const int lane = threadIdx.x & 31, slice = lane % SF_SPLIT;
     const unsigned gmask = 0xffu << (lane & ~(SF_SPLIT - 1));  // the group's lanes
     const int64_t gstride = (int64_t)gridDim.x * (SF_THREADS / SF_SPLIT);
-    double part = 0.0;
+    F2 part{0.f, 0.f};
     // groups of SF_ROWS kernels dealt round-robin over the CTAs, so every CTA has work
     for (int64_t g = (int64_t)(threadIdx.x / SF_SPLIT) * gridDim.x + blockIdx.x; g * SF_ROWS < a.n; g += gstride) {
         const int64_t r0 = g * SF_ROWS;
@@ -124,7 +124,7 @@ __device__ __forceinline__ double small_fit_assign(const SmallFitArgs &a, const 
         if (slice < SF_ROWS && row < a.n) {
             if (compare) moved |= a.idx[row] != mi;  // the previous assignment, written by this lane
             a.idx[row] = mi;
-            part += (double)mb;
+            part = f2_add(part, F2{mb, 0.f});
             unsigned long long *acc = a.acc + (int64_t)mi * ACC_WORDS;
             if (accumulate) {
 #pragma unroll
@@ -142,7 +142,7 @@ __device__ __forceinline__ double small_fit_assign(const SmallFitArgs &a, const 
 
 __global__ void __launch_bounds__(SF_THREADS) small_fit_kernel(SmallFitArgs a) {
     __shared__ unsigned long long cp[D][SF_MAX_K / 2];  // codewords 2p, 2p + 1 packed per coordinate
-    __shared__ double wsum[SF_THREADS / 32];
+    __shared__ F2 wsum[SF_THREADS / 32];
     Header *h = a.hdr;
     unsigned epoch = 0;
     const int64_t gtid = (int64_t)blockIdx.x * SF_THREADS + threadIdx.x;
@@ -178,18 +178,19 @@ __global__ void __launch_bounds__(SF_THREADS) small_fit_kernel(SmallFitArgs a) {
         }
         __syncthreads();
         bool moved = false;
-        double part = small_fit_assign(a, cp, npairs, S, !last, nonfinite, a.stop_on_stable && t > 0, moved);
+        F2 part = small_fit_assign(a, cp, npairs, S, !last, nonfinite, a.stop_on_stable && t > 0, moved);
         uint32_t *moved_word = (t & 1) ? &h->fit_moved1 : &h->fit_moved;
         if (__any_sync(0xffffffffu, moved) && (threadIdx.x & 31) == 0) atomicOr(moved_word, 1u);
         // per-CTA partial of the objective, fixed order
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+        for (int o = 16; o > 0; o >>= 1)
+            part = f2_add(part, F2{__shfl_xor_sync(0xffffffffu, part.hi, o), __shfl_xor_sync(0xffffffffu, part.lo, o)});
         if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = part;
         __syncthreads();
-        if (threadIdx.x == 0) {
-            double s = 0.0;
-            for (int w = 0; w < SF_THREADS / 32; ++w) s += wsum[w];
-            a.blocksum[blockIdx.x] = s;
+        if (threadIdx.x == 0) {  // the CTA's pair, in the 8 bytes of its block-sum slot
+            F2 s{0.f, 0.f};
+            for (int w = 0; w < SF_THREADS / 32; ++w) s = f2_add(s, wsum[w]);
+            reinterpret_cast<F2 *>(a.blocksum)[blockIdx.x] = s;
         }
         if (!grid_barrier(h, gridDim.x, epoch)) return;
         // a fixed point: this assignment is the final one (the same word in every CTA;
@@ -218,10 +219,18 @@ __global__ void __launch_bounds__(SF_THREADS) small_fit_kernel(SmallFitArgs a) {
 #pragma unroll
             for (int j = 0; j <= D; ++j) row[j] = 0ull;
         }
-        if (a.objective && gtid == 0) {
-            double s = 0.0;
-            for (unsigned b = 0; b < gridDim.x; ++b) s += __ldcg(a.blocksum + b);
-            for (int32_t u = t; u <= (stable ? a.iters : t); ++u) a.objective[u] = s;
+        if (a.objective && gtid < 32) {  // warp 0 of CTA 0: lane l takes CTAs l, l + 32, ..., then a butterfly
+            const F2 *bs = reinterpret_cast<const F2 *>(a.blocksum);
+            F2 s{0.f, 0.f};
+            for (unsigned b = (unsigned)gtid; b < gridDim.x; b += 32) {
+                const float2 v = __ldcg(reinterpret_cast<const float2 *>(bs + b));
+                s = f2_add(s, F2{v.x, v.y});
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1)
+                s = f2_add(s, F2{__shfl_xor_sync(0xffffffffu, s.hi, o), __shfl_xor_sync(0xffffffffu, s.lo, o)});
+            if (gtid == 0)
+                for (int32_t u = t; u <= (stable ? a.iters : t); ++u) a.objective[u] = f2_to_double(s);
         }
         if (gtid == 0 && fin) h->fit_iters = t;
         if (fin) break;
