@@ -100,3 +100,25 @@ def test_fit_layers_orders_against_the_callers_stream():
     for r, b, o in zip(ref, bufs, outs):
         assert np.array_equal(r["W_out"].view(np.uint8), o.cpu().numpy().view(np.uint8))
         assert np.array_equal(r["idx"], b["idx"].cpu().numpy())
+
+
+def test_fit_layers_reports_a_failing_layer():
+    # a layer whose workspace is too small fails with KQ_ERR_WORKSPACE; the call
+    # still joins the streams it forked, so the caller's stream stays usable and the
+    # layers enqueued before the failing one complete
+    lays = synth.workload(4).layers[:3]
+    T = 2
+    bufs = [_buffers(lay, T, with_sel=False) for lay in lays]
+    ref = []
+    for lay in lays:
+        b = _buffers(lay, T, with_sel=False)
+        _single(b, T, 30, 0)
+        ref.append(_outputs(b))
+    bufs[2]["ws"] = bufs[2]["ws"][:4096]  # the smallest layer is dealt last: its fit fails
+    with pytest.raises(kq.KQError) as err:
+        kq.kq_fit_layers(bufs, T, 30, 0)
+    assert err.value.status == 6  # KQ_ERR_WORKSPACE
+    torch.cuda.current_stream().synchronize()
+    for r, b in zip(ref[:2], bufs[:2]):
+        assert np.array_equal(r["idx"], b["idx"].cpu().numpy())
+        assert np.array_equal(r["W_out"].view(np.uint8), b["W_out"].cpu().numpy().view(np.uint8))
