@@ -288,10 +288,13 @@ kq_status kq_search_codebook_size(const float *W, int64_t n, const int64_t *sel,
  *   max_iters  0 .. 100000
  *   levels     64 fp32 output (device);  codes K x 9 uint8 output (device)
  *   iters_run  1 int32 output (device) or NULL: level updates performed
- * Uses only the first 4096 bytes of the workspace (ws_bytes >= 4096). The CTAs
- * of this call meet at grid barriers whose waits are bounded (~2 s): a wait that
- * runs out sets KQ_FLAG_TIMEOUT and the call ends without writing its outputs.
- * A negative count sets KQ_FLAG_INDEX_RANGE and is treated as 0. */
+ * Uses only the first 4096 bytes of the workspace (ws_bytes >= 4096). Up to 8192
+ * codewords the fit runs on one thread-block cluster of at most 16 CTAs (the
+ * cluster's hardware barrier, distributed shared memory; kq_fit_layers takes it
+ * up to ~23K codewords); otherwise the CTAs of the call meet at grid barriers
+ * whose waits are bounded (~2 s): a wait that runs out sets KQ_FLAG_TIMEOUT and
+ * the call ends without writing its outputs. Both give the same levels, codes
+ * and update count. A negative count sets KQ_FLAG_INDEX_RANGE and is treated as 0. */
 kq_status kq_quantize_codebook_6bit(const float *C, int32_t K, const int32_t *counts, int32_t max_iters,
                                     float *levels, uint8_t *codes, int32_t *iters_run, void *ws, size_t ws_bytes,
                                     kq_stream_t stream);
@@ -303,8 +306,9 @@ kq_status kq_quantize_codebook_6bit(const float *C, int32_t K, const int32_t *co
  *   max_iters  0 .. 100000
  *   levels     64 fp32 output (device);  codes m uint8 output (device)
  *   iters_run  1 int32 output (device) or NULL
- * Uses only the first 4096 bytes of the workspace (ws_bytes >= 4096). Bounded
- * grid barriers as in kq_quantize_codebook_6bit. */
+ * Uses only the first 4096 bytes of the workspace (ws_bytes >= 4096). Up to
+ * 73,728 scalars on one thread-block cluster, beyond that bounded grid barriers,
+ * as in kq_quantize_codebook_6bit. */
 kq_status kq_quantize_scalars_6bit(const float *v, int64_t m, int32_t max_iters, float *levels, uint8_t *codes,
                                    int32_t *iters_run, void *ws, size_t ws_bytes, kq_stream_t stream);
 
