@@ -32,7 +32,9 @@
  *   device can see (a non-finite input, an index or code out of range, a bounded
  *   device-side wait that gave up) set bits of a sticky status word in the
  *   workspace; kq_device_status() reads and clears it. Device code never traps
- *   and never waits without a bound. A CUDA launch error returns KQ_ERR_CUDA.
+ *   and never spins without a bound (the one-cluster level fit also uses the
+ *   cluster's hardware barrier, which every CTA of the cluster reaches by
+ *   construction). A CUDA launch error returns KQ_ERR_CUDA.
  * - Determinism. For identical inputs every output is bitwise identical from
  *   run to run (no floating-point atomics anywhere).
  * - Alignment. W and W_out must be 16-byte aligned; other float / int pointers
@@ -109,7 +111,8 @@ kq_status kq_trace_get(int32_t i, const char **name, float *ms);
  *   faults      KQ_TEST_SKIP_ARRIVAL: in the grid barriers of the cooperative
  *               kernels (6-bit quantisation, one-launch small fits, fused recovery,
  *               update fallback) CTA 0 never arrives, so the others wait until the
- *               limit; KQ_TEST_STOP_TILE_STREAM: the tensor-core assignment streams
+ *               limit (a workspace with a fault set always takes the grid-barrier
+ *               level fit, not the one-cluster one); KQ_TEST_STOP_TILE_STREAM: the tensor-core assignment streams
  *               no codeword tile beyond those it starts before its setup, so its
  *               MMA issuers wait until the limit. 0 clears both.
  *   wait_limit  polls before a bounded wait gives up (0: the normal limits, about
