@@ -1603,17 +1603,28 @@ __global__ void __launch_bounds__(SCAN_THREADS) scan_counts_kernel(const int32_t
 }
 
 // perm = the rows grouped by hint key (any order within a group).
+// Four rows per thread step, so that four returning atomics are in flight at once.
+constexpr int SCATTER_UNROLL = 4;
 __global__ void __launch_bounds__(256) hint_scatter_kernel(const int32_t *__restrict__ hint, int64_t n, int32_t K,
                                                            const int32_t *__restrict__ cpos, int32_t *cursor,
                                                            int32_t *__restrict__ perm) {
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
-        const int32_t pos = atomicAdd(cursor + hint_key(__ldcs(hint + i), K, cpos), 1);
-        if ((uint32_t)pos < (uint32_t)n) perm[pos] = (int32_t)i;  // counts that do not match the hints: no stray write
+    for (int64_t i0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i0 < n; i0 += SCATTER_UNROLL * stride) {
+        int32_t key[SCATTER_UNROLL], pos[SCATTER_UNROLL];
+#pragma unroll
+        for (int u = 0; u < SCATTER_UNROLL; ++u) {
+            const int64_t i = i0 + u * stride;
+            key[u] = i < n ? hint_key(__ldcs(hint + i), K, cpos) : -1;
+        }
+#pragma unroll
+        for (int u = 0; u < SCATTER_UNROLL; ++u) pos[u] = key[u] >= 0 ? atomicAdd(cursor + key[u], 1) : -1;
+#pragma unroll
+        for (int u = 0; u < SCATTER_UNROLL; ++u)  // counts that do not match the hints: no stray write
+            if ((uint32_t)pos[u] < (uint32_t)n) perm[pos[u]] = (int32_t)(i0 + u * stride);
     }
 }
 
-// blocksum[b] = sum of dist over rows [256 b, 256 b + 256) in a fixed order (fp64).
+// blocksum[b] = sum of dist over rows [256 b, 256 b + 256) in a fixed order (double-float).
 __global__ void __launch_bounds__(256) dist_block_sums_kernel(const float *__restrict__ dist, int64_t n,
                                                               double *__restrict__ blocksum) {
     __shared__ F2 ws[8];
@@ -1628,11 +1639,73 @@ __global__ void __launch_bounds__(256) dist_block_sums_kernel(const float *__res
     }
 }
 
+// The same histogram and scatter for at most HINT_SMEM_BINS keys (e.g. the k-d
+// leaves, 256 of them at 65,536 codewords, where millions of rows land on few keys
+// and one global atomic per row contends on a handful of addresses): each CTA takes
+// a contiguous run of rows, counts them per key in shared memory, and touches the
+// global array once per key it holds. The scatter counts its run first, reserves
+// one range per key with a single returning atomic, then places each row at that
+// range's base plus its rank among the run's rows of the key (the order within a
+// key is free).
+constexpr int HINT_SMEM_BINS = 4096;
+constexpr int HINT_SMEM_THREADS = 512;
+
+__device__ __forceinline__ void hint_run(int64_t n, int64_t &r0, int64_t &r1) {
+    const int64_t per = (n + gridDim.x - 1) / gridDim.x;
+    r0 = min(n, (int64_t)blockIdx.x * per);
+    r1 = min(n, r0 + per);
+}
+
+__global__ void __launch_bounds__(HINT_SMEM_THREADS) hint_histogram_smem_kernel(const int32_t *__restrict__ hint,
+                                                                                int64_t n, int32_t K,
+                                                                                const int32_t *__restrict__ cpos,
+                                                                                int32_t *cnt) {
+    __shared__ int32_t c[HINT_SMEM_BINS];
+    const int m = K + 1;
+    for (int b = threadIdx.x; b < m; b += HINT_SMEM_THREADS) c[b] = 0;
+    __syncthreads();
+    int64_t r0, r1;
+    hint_run(n, r0, r1);
+    for (int64_t i = r0 + threadIdx.x; i < r1; i += HINT_SMEM_THREADS) atomicAdd(&c[hint_key(__ldcs(hint + i), K, cpos)], 1);
+    __syncthreads();
+    for (int b = threadIdx.x; b < m; b += HINT_SMEM_THREADS)
+        if (c[b]) atomicAdd(cnt + b, c[b]);
+}
+
+__global__ void __launch_bounds__(HINT_SMEM_THREADS) hint_scatter_smem_kernel(const int32_t *__restrict__ hint,
+                                                                              int64_t n, int32_t K,
+                                                                              const int32_t *__restrict__ cpos,
+                                                                              int32_t *cursor, int32_t *__restrict__ perm) {
+    __shared__ int32_t c[HINT_SMEM_BINS];     // the run's rows per key, then the rank counters
+    __shared__ int32_t base[HINT_SMEM_BINS];  // the range reserved per key
+    const int m = K + 1;
+    for (int b = threadIdx.x; b < m; b += HINT_SMEM_THREADS) c[b] = 0;
+    __syncthreads();
+    int64_t r0, r1;
+    hint_run(n, r0, r1);
+    for (int64_t i = r0 + threadIdx.x; i < r1; i += HINT_SMEM_THREADS) atomicAdd(&c[hint_key(__ldcs(hint + i), K, cpos)], 1);
+    __syncthreads();
+    for (int b = threadIdx.x; b < m; b += HINT_SMEM_THREADS) {
+        base[b] = c[b] ? atomicAdd(cursor + b, c[b]) : 0;
+        c[b] = 0;
+    }
+    __syncthreads();
+    for (int64_t i = r0 + threadIdx.x; i < r1; i += HINT_SMEM_THREADS) {
+        const int32_t key = hint_key(__ldcs(hint + i), K, cpos);
+        const int32_t pos = base[key] + atomicAdd(&c[key], 1);
+        if ((uint32_t)pos < (uint32_t)n) perm[pos] = (int32_t)i;  // counts that do not match the hints: no stray write
+    }
+}
+
 cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, const int32_t *cpos,
                                     const int32_t *cperm, const int32_t *hint_counts, int32_t *cnt, int32_t *perm,
                                     int num_sms, cudaStream_t s) {
     int64_t blocks = (n + 255) / 256;
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
+    // few keys: runs of at least 4096 rows per CTA, up to two CTAs per SM
+    int64_t sblocks = (n + 4095) / 4096;
+    if (sblocks > 2LL * num_sms) sblocks = 2LL * num_sms;
+    if (sblocks < 1) sblocks = 1;
     if (hint_counts) {
         // the rows per hinted codeword are known (all hints valid): start offsets
         // straight from them, K + 1 entries with the last count 0
@@ -1643,16 +1716,26 @@ cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, c
         cudaError_t e = cudaMemsetAsync(cnt, 0, (size_t)(K + 1) * sizeof(int32_t), s);
         if (e != cudaSuccess) return e;
         launch_begin(s);
-        hint_histogram_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cpos, cnt);
-        launch_end(s, "hint_histogram_kernel");
+        if (K + 1 <= HINT_SMEM_BINS) {
+            hint_histogram_smem_kernel<<<(unsigned)sblocks, HINT_SMEM_THREADS, 0, s>>>(hint, n, K, cpos, cnt);
+            launch_end(s, "hint_histogram_smem_kernel");
+        } else {
+            hint_histogram_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cpos, cnt);
+            launch_end(s, "hint_histogram_kernel");
+        }
         // the scan turns cnt into start offsets in place
         launch_begin(s);
         scan_counts_kernel<<<1, SCAN_THREADS, 0, s>>>(cnt, K + 1, K + 1, cnt, nullptr);
         launch_end(s, "scan_counts_kernel");
     }
     launch_begin(s);
-    hint_scatter_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cpos, cnt, perm);
-    launch_end(s, "hint_scatter_kernel");
+    if (K + 1 <= HINT_SMEM_BINS) {
+        hint_scatter_smem_kernel<<<(unsigned)sblocks, HINT_SMEM_THREADS, 0, s>>>(hint, n, K, cpos, cnt, perm);
+        launch_end(s, "hint_scatter_smem_kernel");
+    } else {
+        hint_scatter_kernel<<<(unsigned)blocks, 256, 0, s>>>(hint, n, K, cpos, cnt, perm);
+        launch_end(s, "hint_scatter_kernel");
+    }
     return cudaGetLastError();
 }
 
