@@ -50,6 +50,7 @@ __global__ void __launch_bounds__(KD_THREADS) kd_split_kernel(const float *__res
     __shared__ unsigned long long s_prefix, s_mask;
     __shared__ long long s_rank;
     __shared__ unsigned int s_left, s_right;
+    __shared__ int s_unique;
 
     // mean (fixed summation order: per thread, then xor-shuffle tree, then warps in order)
     float acc[KD_COV];
@@ -144,10 +145,14 @@ __global__ void __launch_bounds__(KD_THREADS) kd_split_kernel(const float *__res
         s_prefix = 0ull;
         s_mask = 0ull;
         s_rank = r;
+        s_unique = 0;
     }
     __syncthreads();
-    // radix select of the key of rank r, 8 bits at a time from the top
-    for (int shift = 56; shift >= 0; shift -= 8) {
+    // radix select of the key of rank r, 8 bits at a time from the top; it stops as
+    // soon as one key alone carries the selected prefix: that key is the one of rank
+    // r, and comparing with the prefix (lower bits 0) puts exactly the r keys below
+    // it on the left
+    for (int shift = 56; shift >= 0 && !s_unique; shift -= 8) {
         for (int i = tid; i < 256; i += KD_THREADS) hist[i] = 0u;
         __syncthreads();
         const unsigned long long pre = s_prefix, msk = s_mask;
@@ -178,10 +183,11 @@ __global__ void __launch_bounds__(KD_THREADS) kd_split_kernel(const float *__res
             s_rank = rk - cum;
             s_left = 0u;
             s_right = 0u;
+            s_unique = hist[d] == 1u;
         }
         __syncthreads();
     }
-    const unsigned long long pivot = s_prefix;  // exactly r keys are below it
+    const unsigned long long pivot = s_prefix;  // exactly r keys are below it (lower bits 0 after an early stop)
     for (int64_t e0 = ea; e0 < eb; e0 += KD_THREADS) {  // warp-uniform trip count
         const int64_t e = e0 + tid;
         const bool in = e < eb;
@@ -273,38 +279,102 @@ __global__ void __launch_bounds__(256) kd_leaf_kernel(const float *__restrict__ 
 // hint[row] = the nearest codeword of row's leaf tile (fp32 direct form, first
 // position on ties), rows taken in the order of perm (grouped by leaf, so a CTA's
 // rows read the same few tiles). The tile's codewords are the fp32 part of the
-// packed tensor-core tile.
+// packed tensor-core tile. A thread takes LS_ROWS consecutive slots: when they
+// share a leaf (all but the slots at a leaf boundary) each codeword is loaded once
+// for all of them. (The hints only seed the tensor-core pass; any choice gives the
+// same assignment.)
+constexpr int LS_ROWS = 4;
 __global__ void __launch_bounds__(256) kd_leaf_search_kernel(const float *__restrict__ W, int64_t n,
                                                              const int32_t *__restrict__ perm,
                                                              const int32_t *__restrict__ leaf,
                                                              const unsigned char *__restrict__ Cpk,
                                                              const int32_t *__restrict__ cperm, int32_t K,
                                                              int32_t *__restrict__ hint) {
-    const int64_t s = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (s >= n) return;
-    const int64_t row = perm[s];
-    if ((uint64_t)row >= (uint64_t)n) return;
-    const int32_t g = leaf[row];
-    float x[D];
+    const int64_t s0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * LS_ROWS;
+    if (s0 >= n) return;
+    int64_t row[LS_ROWS];
+    int32_t g[LS_ROWS];
+    bool same = true;
 #pragma unroll
-    for (int u = 0; u < D; ++u) x[u] = W[row * D + u];
-    const float *cw = reinterpret_cast<const float *>(Cpk + (int64_t)g * TC_TILE_BYTES + TC_TILE_H);
-    const int cntw = min(256, K - g * 256);
-    float best = __int_as_float(0x7f800000);
-    int bk = 0;
-    for (int kl = 0; kl < cntw; ++kl) {
-        float acc = 0.f;
-#pragma unroll
-        for (int u = 0; u < D; ++u) {
-            const float t = x[u] - __ldg(cw + kl * D + u);
-            acc = fmaf(t, t, acc);
-        }
-        if (acc < best) {
-            best = acc;
-            bk = kl;
-        }
+    for (int r = 0; r < LS_ROWS; ++r) {
+        const int64_t s = s0 + r;
+        row[r] = s < n ? perm[s] : -1;
+        if ((uint64_t)row[r] >= (uint64_t)n) row[r] = -1;
+        g[r] = row[r] >= 0 ? leaf[row[r]] : -1;
+        same &= row[r] >= 0 && g[r] == g[0];
     }
-    hint[row] = cperm[g * 256 + bk];
+    if (same) {
+        // two codewords per packed fp32x2 operation (each half the scalar sequence)
+        unsigned long long x2[LS_ROWS][D];
+        float best[LS_ROWS];
+        int bk[LS_ROWS];
+#pragma unroll
+        for (int r = 0; r < LS_ROWS; ++r) {
+#pragma unroll
+            for (int u = 0; u < D; ++u) {
+                const float v = W[row[r] * D + u];
+                x2[r][u] = pack2(v, v);
+            }
+            best[r] = __int_as_float(0x7f800000);
+            bk[r] = 0;
+        }
+        const float *cw = reinterpret_cast<const float *>(Cpk + (int64_t)g[0] * TC_TILE_BYTES + TC_TILE_H);
+        const int cntw = min(256, K - g[0] * 256);
+        for (int kl = 0; kl < cntw; kl += 2) {
+            const bool two = kl + 1 < cntw;  // an odd last codeword pairs with +inf (never chosen)
+            unsigned long long c2[D];
+#pragma unroll
+            for (int u = 0; u < D; ++u)
+                c2[u] = pack2(__ldg(cw + kl * D + u), two ? __ldg(cw + (kl + 1) * D + u) : __int_as_float(0x7f800000));
+#pragma unroll
+            for (int r = 0; r < LS_ROWS; ++r) {
+                unsigned long long t = sub2(x2[r][0], c2[0]);
+                unsigned long long acc = mul2(t, t);
+#pragma unroll
+                for (int u = 1; u < D; ++u) {
+                    t = sub2(x2[r][u], c2[u]);
+                    acc = fma2(t, t, acc);
+                }
+                float d0, d1;
+                unpack2(acc, d0, d1);
+                if (d0 < best[r]) {
+                    best[r] = d0;
+                    bk[r] = kl;
+                }
+                if (d1 < best[r]) {
+                    best[r] = d1;
+                    bk[r] = kl + 1;
+                }
+            }
+        }
+#pragma unroll
+        for (int r = 0; r < LS_ROWS; ++r) hint[row[r]] = cperm[g[0] * 256 + bk[r]];
+        return;
+    }
+#pragma unroll
+    for (int r = 0; r < LS_ROWS; ++r) {  // a leaf boundary or the end: row by row
+        if (row[r] < 0) continue;
+        float x[D];
+#pragma unroll
+        for (int u = 0; u < D; ++u) x[u] = W[row[r] * D + u];
+        const float *cw = reinterpret_cast<const float *>(Cpk + (int64_t)g[r] * TC_TILE_BYTES + TC_TILE_H);
+        const int cntw = min(256, K - g[r] * 256);
+        float best = __int_as_float(0x7f800000);
+        int bk = 0;
+        for (int kl = 0; kl < cntw; ++kl) {
+            float acc = 0.f;
+#pragma unroll
+            for (int u = 0; u < D; ++u) {
+                const float t = x[u] - __ldg(cw + kl * D + u);
+                acc = fmaf(t, t, acc);
+            }
+            if (acc < best) {
+                best = acc;
+                bk = kl;
+            }
+        }
+        hint[row[r]] = cperm[g[r] * 256 + bk];
+    }
 }
 
 int kd_levels(int32_t T) {
@@ -348,8 +418,8 @@ cudaError_t launch_kd_hints(const float *W, int64_t n, const KdNode *nodes, int3
     if ((e = launch_hint_permutation(leaf, n, T, nullptr, nullptr, nullptr, cnt, perm, num_sms, s)) != cudaSuccess)
         return e;
     launch_begin(s);
-    kd_leaf_search_kernel<<<blocks, 256, 0, s>>>(W, n, perm, leaf, reinterpret_cast<const unsigned char *>(Cpk),
-                                                 cperm, K, hint);
+    kd_leaf_search_kernel<<<(unsigned)((n + 256 * LS_ROWS - 1) / (256 * LS_ROWS)), 256, 0, s>>>(
+        W, n, perm, leaf, reinterpret_cast<const unsigned char *>(Cpk), cperm, K, hint);
     launch_end(s, "kd_leaf_search_kernel");
     return cudaGetLastError();
 }
