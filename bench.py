@@ -445,7 +445,12 @@ def run_kq(args, rank, world, local_rank):
             "peak_basis": f"measured cuBLAS bf16 sustained {bf16:.1f} TFLOP/s (of measured; dense fp16 and bf16 "
                           f"share one rate); the kernel is timed inside the long step",
             "launches": len(tc_ms), "ms_mean": statistics.mean(tc_ms),
-            "ms_mean_full_pass": statistics.mean(full), "ms_mean_pilot": statistics.mean(
+            "ms_mean_full_pass": statistics.mean(full),
+            # the first full pass of a step starts from k-d leaf hints (cold), the later T from the
+            # previous assignment (warm)
+            "ms_first_pass": statistics.mean(full[0::T + 1]),
+            "ms_warm_pass": statistics.mean([ms for i, ms in enumerate(full) if i % (T + 1)]) if T else None,
+            "ms_mean_pilot": statistics.mean(
                 [ms for i, ms in enumerate(tc_ms) if i % per_step < pilots]) if pilots > 0 else None,
             "frac_of_burst": achieved / float(peaks.get("bf16_tflops", bf16)),
             "gemm": {"flops_per_pair": GEMM_FLOPS_PER_PAIR, "achieved": gemm, "frac_of_peak": gemm / bf16,

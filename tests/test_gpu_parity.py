@@ -227,17 +227,21 @@ def test_fit_small_codebook_objective():
     assert obj[1] == pytest.approx(oracle.objective(d2), rel=1e-12)
 
 
-@pytest.mark.parametrize("case", ["kd_leaf_hints", "pilot", "pilot_above_tree"])
+@pytest.mark.parametrize("case", ["kd_leaf_hints", "kd_leaf_hints_duplicates", "pilot", "pilot_above_tree"])
 def test_assign_cold_start_paths(case):
     # Without a hint on the tensor-core path, the full pass is seeded with hints: on
     # large problems (n K >= 1e10, up to 65536 codewords) each kernel's nearest codeword
     # in its k-d leaf tile, otherwise (from 16384 codewords) a pilot pass against the
-    # first K / 16 codewords. The answer is the plain argmin all the same (the CUDA-core
-    # kernel, the oracle on sampled rows, and a run warm-started from the answer).
-    n, K = {"kd_leaf_hints": (655360 + 123, 16384 + 77), "pilot": (2 * TC_MIN_N + 123, 16384 + 77),
-            "pilot_above_tree": (2 * TC_MIN_N + 123, 65536 + 1000)}[case]
+    # first K / 16 codewords.
+    # The answer is the plain argmin all the same (the CUDA-core kernel, the oracle on
+    # sampled rows, and a run warm-started from the answer); with every codeword
+    # present twice, the lower index of each tied pair.
+    n, K = {"kd_leaf_hints": (655360 + 123, 16384 + 77), "kd_leaf_hints_duplicates": (655360 + 45, 16384 + 77),
+            "pilot": (2 * TC_MIN_N + 123, 16384 + 77), "pilot_above_tree": (2 * TC_MIN_N + 123, 65536 + 1000)}[case]
     W = synth.random_kernels(n, 9, 261, 0.05)
     C = W[synth.init_selection(n, K, 262)]
+    if case == "kd_leaf_hints_duplicates":
+        C[K // 2:] = C[:K - K // 2]
     i0, d0, st, _ = gpu_assign(W, C)
     assert st == 0
     if K <= 65536:  # the allocation-free CUDA-core variant holds up to 65536 codewords
