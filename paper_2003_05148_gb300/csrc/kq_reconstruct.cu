@@ -128,30 +128,83 @@ __device__ __forceinline__ void gc_gather(const unsigned long long *__restrict__
     }
 }
 
+// A lane's float4 slots of a 32-kernel chunk (288 floats, 72 float4): float4 lane
+// and lane + 32 of every chunk (slots 0, 1), and float4 64 + (lane & 7) of the
+// first chunk of a pair (lanes 0-7) or of the second (lanes 8-15) (slot 2, both
+// chunks' last eight float4 in one pass). A slot's first element is code j0 of the
+// chunk's kernel ra; elements e < split belong to ra, the rest are codes 0-2 of
+// kernel ra + 1 (all in the low word of its code word).
+struct GcSlots {
+    int ra[3], j0[3], split[3];
+};
+__device__ __forceinline__ GcSlots gc_slots(int lane) {
+    GcSlots g;
+#pragma unroll
+    for (int s = 0; s < 3; ++s) {
+        const int v = s < 2 ? lane + 32 * s : 64 + (lane & 7);
+        g.ra[s] = (4 * v) / D;
+        g.j0[s] = 4 * v - D * g.ra[s];
+        g.split[s] = D - g.j0[s];
+    }
+    return g;
+}
+// The four weights of a slot: qa the code word of kernel ra, qb the low word of
+// kernel ra + 1's; lv the replicated level table.
+__device__ __forceinline__ float4 gc_decode(unsigned long long qa, uint32_t qb, int j0, int split,
+                                            const float (*lv)[32], int lane) {
+    float r[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const bool first = e < split;
+        const int j = first ? j0 + e : e - split;
+        r[e] = lv[((first ? qa : (unsigned long long)qb) >> (7 * j)) & 127u][lane];
+    }
+    return make_float4(r[0], r[1], r[2], r[3]);
+}
+
+// A warp's place in the loop of gather_codes_rows: its first chunk pair and the
+// indices of its first two pairs, loaded by gc_start (before the code words exist).
+struct GcPipe {
+    int64_t c2;
+    int32_t k[2], kn[2];
+};
+__device__ __forceinline__ void gc_start(const int32_t *__restrict__ idx, int64_t n, int64_t cta, int64_t ncta,
+                                         GcPipe &p) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t nch = n / 32;
+    const int64_t npairs = nch / 2 + (nch & 1);
+    const int64_t step = ncta * R_WARPS;
+    p.c2 = cta * R_WARPS + warp;
+    p.k[0] = p.k[1] = p.kn[0] = p.kn[1] = 0;
+    if (p.c2 < npairs) {
+        gc_load_idx(idx, nch, p.c2, lane, p.k);
+        if (p.c2 + step < npairs) gc_load_idx(idx, nch, p.c2 + step, lane, p.kn);
+    }
+}
+
 // The loop of gather_codes_kernel over the chunk pairs of CTA `cta` of `ncta` (and
-// the ragged end in CTA 0); lv is the replicated level table, ra/j0/split the lane's
-// float4 slots. Software-pipelined by one pair: while pair c2 is decoded and
-// stored, the code words of the warp's next pair and the indices of the one after
-// are already in flight, so a warp waits for neither the index read from DRAM nor
-// the gather from L2. Returns whether this thread saw an index outside [0, K).
+// the ragged end in CTA 0), from the state gc_start left; lv is the replicated level
+// table. Software-pipelined by one pair: while pair c2 is decoded and stored, the
+// code words of the warp's next pair and the indices of the one after are already in
+// flight, so a warp waits for neither the index read from DRAM nor the gather from
+// L2. Returns whether this thread saw an index outside [0, K).
 __device__ __forceinline__ bool gather_codes_rows(const int32_t *__restrict__ idx, int64_t n,
                                                   const unsigned long long *__restrict__ Cq, int32_t K,
-                                                  float *__restrict__ W_out, const float (*lv)[32], const int *ra,
-                                                  const int *j0, const int *split, int64_t cta, int64_t ncta) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+                                                  float *__restrict__ W_out, const float (*lv)[32], const GcSlots &sl,
+                                                  GcPipe p, int64_t cta, int64_t ncta) {
+    const int lane = threadIdx.x & 31;
     bool bad = false;
     const int64_t nch = n / 32;
     const int64_t npairs = nch / 2 + (nch & 1);
     const int64_t step = ncta * R_WARPS;
-    int64_t c2 = cta * R_WARPS + warp;
-    int32_t kn[2] = {0, 0};
+    int64_t c2 = p.c2;
+    int32_t kn[2] = {p.kn[0], p.kn[1]};
     unsigned long long q[2] = {0ull, 0ull};
-    if (c2 < npairs) {
-        int32_t k[2];
-        gc_load_idx(idx, nch, c2, lane, k);
-        if (c2 + step < npairs) gc_load_idx(idx, nch, c2 + step, lane, kn);
-        gc_gather(Cq, K, k, 2 * c2 + 1 < nch, q, bad);
-    }
+    if (c2 < npairs) gc_gather(Cq, K, p.k, 2 * c2 + 1 < nch, q, bad);
+    // slot 2 reads kernels 28-31 of both chunks from lanes 28-31 (first chunk) and
+    // 12-15 (second chunk, moved there by one shuffle pair)
+    const int off2 = lane < 8 ? 0 : 16;
+    const int sa2 = sl.ra[2] - off2, sb2 = min(sl.ra[2] + 1, 31) - off2;
     for (; c2 < npairs; c2 += step) {
         const int64_t c2n = c2 + step;
         unsigned long long qn[2] = {0ull, 0ull};
@@ -159,28 +212,34 @@ __device__ __forceinline__ bool gather_codes_rows(const int32_t *__restrict__ id
         if (c2n < npairs) gc_gather(Cq, K, kn, 2 * c2n + 1 < nch, qn, bad);
         if (c2n + step < npairs) gc_load_idx(idx, nch, c2n + step, lane, knn);
         const bool two = 2 * c2 + 1 < nch;
+        float4 *d4[2] = {reinterpret_cast<float4 *>(W_out + 2 * c2 * 32 * D),
+                         reinterpret_cast<float4 *>(W_out + (2 * c2 + 1) * 32 * D)};
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
             if (h == 1 && !two) break;
-            const int64_t r0 = (2 * c2 + h) * 32;
             const uint32_t qlo = (uint32_t)q[h], qhi = (uint32_t)(q[h] >> 32);
-            float4 *d4 = reinterpret_cast<float4 *>(W_out + r0 * D);
 #pragma unroll
-            for (int s = 0; s < 3; ++s) {
-                const int rb = min(ra[s] + 1, 31);
-                const unsigned long long qa = ((unsigned long long)__shfl_sync(0xffffffffu, qhi, ra[s]) << 32) |
-                                              __shfl_sync(0xffffffffu, qlo, ra[s]);
-                const unsigned long long qb = ((unsigned long long)__shfl_sync(0xffffffffu, qhi, rb) << 32) |
-                                              __shfl_sync(0xffffffffu, qlo, rb);
-                float r[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const bool first = e < split[s];
-                    const int j = first ? j0[s] + e : e - split[s];
-                    r[e] = lv[((first ? qa : qb) >> (7 * j)) & 127u][lane];
-                }
-                if (s < 2 || lane < 32 * D / 4 - 64) __stcs(d4 + lane + 32 * s, make_float4(r[0], r[1], r[2], r[3]));
+            for (int s = 0; s < 2; ++s) {
+                const int rb = min(sl.ra[s] + 1, 31);
+                const unsigned long long qa = ((unsigned long long)__shfl_sync(0xffffffffu, qhi, sl.ra[s]) << 32) |
+                                              __shfl_sync(0xffffffffu, qlo, sl.ra[s]);
+                const uint32_t qb = __shfl_sync(0xffffffffu, qlo, rb);
+                __stcs(d4[h] + lane + 32 * s, gc_decode(qa, qb, sl.j0[s], sl.split[s], lv, lane));
             }
+        }
+        {
+            const uint32_t t_lo = __shfl_sync(0xffffffffu, (uint32_t)q[1], (lane + 16) & 31);
+            const uint32_t t_hi = __shfl_sync(0xffffffffu, (uint32_t)(q[1] >> 32), (lane + 16) & 31);
+            const uint32_t wlo = lane >= 16 ? (uint32_t)q[0] : t_lo;
+            const uint32_t whi = lane >= 16 ? (uint32_t)(q[0] >> 32) : t_hi;
+            const unsigned long long qa = ((unsigned long long)__shfl_sync(0xffffffffu, whi, sa2) << 32) |
+                                          __shfl_sync(0xffffffffu, wlo, sa2);
+            const uint32_t qb = __shfl_sync(0xffffffffu, wlo, sb2);
+            const float4 v = gc_decode(qa, qb, sl.j0[2], sl.split[2], lv, lane);
+            if (lane < 8)
+                __stcs(d4[0] + 64 + lane, v);
+            else if (lane < 16 && two)
+                __stcs(d4[1] + 56 + lane, v);  // float4 64 + (lane - 8)
         }
         q[0] = qn[0];
         q[1] = qn[1];
@@ -218,22 +277,17 @@ __global__ void __launch_bounds__(R_THREADS, 4)
 gather_codes_kernel(const int32_t *__restrict__ idx, int64_t n, const unsigned long long *__restrict__ Cq,
                     const float *__restrict__ levels, int32_t K, float *__restrict__ W_out, uint32_t *status) {
     __shared__ float lv[LEVELS + 1][32];  // row LEVELS decodes out-of-range codes to 0
+    const int lane = threadIdx.x & 31;
+    // the first indices are in flight while the level table is built (the decode
+    // kernel does not write them; everything before it has completed)
+    GcPipe p;
+    gc_start(idx, n, blockIdx.x, gridDim.x, p);
     for (int e = threadIdx.x; e < (LEVELS + 1) * 32; e += R_THREADS)
         lv[e / 32][e % 32] = e / 32 < LEVELS ? levels[e / 32] : 0.f;
+    const GcSlots sl = gc_slots(lane);
     __syncthreads();
-    const int lane = threadIdx.x & 31;
-    // slot s: float4 v = lane + 32 s of the chunk; its first element is coordinate
-    // j0 of kernel ra, elements e < split belong to ra, the rest to ra + 1
-    int ra[3], j0[3], split[3];
-#pragma unroll
-    for (int s = 0; s < 3; ++s) {
-        const int v = min(lane + 32 * s, 32 * D / 4 - 1);
-        ra[s] = (4 * v) / D;
-        j0[s] = 4 * v - D * ra[s];
-        split[s] = D - j0[s];
-    }
     asm volatile("griddepcontrol.wait;" ::: "memory");  // Cq is written by the decode kernel
-    const bool bad = gather_codes_rows(idx, n, Cq, K, W_out, lv, ra, j0, split, blockIdx.x, gridDim.x);
+    const bool bad = gather_codes_rows(idx, n, Cq, K, W_out, lv, sl, p, blockIdx.x, gridDim.x);
     if (__any_sync(0xffffffffu, bad) && lane == 0) set_flag(status, KQ_FLAG_INDEX_RANGE);
 }
 
@@ -275,15 +329,9 @@ encode_gather_kernel(const float *__restrict__ C, int32_t K, const float *__rest
     unsigned epoch = 0;
     if (!grid_barrier(hdr, gridDim.x, epoch)) return;
     const int lane = threadIdx.x & 31;
-    int ra[3], j0[3], split[3];
-#pragma unroll
-    for (int s = 0; s < 3; ++s) {
-        const int v = min(lane + 32 * s, 32 * D / 4 - 1);
-        ra[s] = (4 * v) / D;
-        j0[s] = 4 * v - D * ra[s];
-        split[s] = D - j0[s];
-    }
-    const bool bad = gather_codes_rows(idx, n, Cq, K, W_out, lv, ra, j0, split, blockIdx.x, gridDim.x);
+    GcPipe p;
+    gc_start(idx, n, blockIdx.x, gridDim.x, p);
+    const bool bad = gather_codes_rows(idx, n, Cq, K, W_out, lv, gc_slots(lane), p, blockIdx.x, gridDim.x);
     if (__any_sync(0xffffffffu, bad) && lane == 0) set_flag(&hdr->status, KQ_FLAG_INDEX_RANGE);
 }
 
