@@ -647,8 +647,10 @@ def test_quantize_negative_count_flagged():
 
 # --------------------------------------------------------------------------- reconstruction
 
-@pytest.mark.parametrize("n,K", [(1, 1), (31, 5), (4096, 16), (100001, 256), (4194304, 65536)])
+@pytest.mark.parametrize("n,K", [(1, 1), (31, 5), (4096, 16), (100001, 256), (544775, 4096), (1000003, 65536),
+                                 (4194304, 65536)])
 def test_reconstruct(n, K):
+    # ragged ends, and sizes whose last round of chunk pairs leaves warps idle
     C = synth.random_kernels(K, 9, K, 0.05)
     idx = synth.below(synth.stream_key(n, 2), n, K).astype(np.int32)
     counts = np.bincount(idx, minlength=K).astype(np.int32)
