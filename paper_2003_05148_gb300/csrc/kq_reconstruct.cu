@@ -262,17 +262,18 @@ __device__ __forceinline__ bool gather_codes_rows(const int32_t *__restrict__ id
 
 // K+C recovery. A warp owns pairs of 32-kernel chunks (1152 output bytes = 72
 // float4 each). Each lane fetches the packed codes of its own kernel (one 8-byte
-// word, instead of a 36-byte row), then produces output float4 number lane,
-// lane + 32 and (lanes 0-7) lane + 64 of a chunk directly: the at most two
-// kernels a float4 spans send their code words by shuffle, and every code is
-// looked up in a level table replicated across the 32 shared-memory banks (level
-// l for lane L at [l][L]: no bank conflicts). The stores are coalesced streaming
-// float4 stores; one resident wave of CTAs, each warp's loop software-pipelined
-// (gather_codes_rows). Launched as a programmatic dependent of
-// decode_codebook_kernel (the launch and the level table overlap the decode; Cq is
-// read after griddepcontrol.wait). Stress layer (n = 4,194,304), minimum of 30
-// calls: 42.9 us with two waves and no pipelining, 41.5 us as here; decoding
-// each lane's own kernel into a staging tile instead of the shuffles: 42.8 us.
+// word, instead of a 36-byte row), then produces output float4 number lane and
+// lane + 32 of each chunk, and lanes 0-15 the last eight float4 of both chunks
+// (gc_slots), directly: the at most two kernels a float4 spans send their code
+// words by shuffle, and every code is looked up in a level table replicated across
+// the 32 shared-memory banks (level l for lane L at [l][L]: no bank conflicts). The
+// stores are coalesced streaming float4 stores; one resident wave of CTAs, each
+// warp's loop software-pipelined (gather_codes_rows). Launched as a programmatic
+// dependent of decode_codebook_kernel (the launch, the first index loads and the
+// level table overlap the decode; Cq is read after griddepcontrol.wait). Stress
+// layer (n = 4,194,304), whole kq_reconstruct call, minimum of 30 calls: 42.9 us with
+// two waves and no pipelining, 41.8 us pipelined, 40.3 us as here; decoding each
+// lane's own kernel into a staging tile instead of the shuffles was slower.
 __global__ void __launch_bounds__(R_THREADS, 4)
 gather_codes_kernel(const int32_t *__restrict__ idx, int64_t n, const unsigned long long *__restrict__ Cq,
                     const float *__restrict__ levels, int32_t K, float *__restrict__ W_out, uint32_t *status) {
