@@ -178,6 +178,13 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
             hint_counts = nullptr;
         }
         KQ_TRY(launch_pack_codebook_tc(C, K, w.cpk, w.hdr, s));
+        if (!hint && K < COLD_PILOT_MIN_K) {
+            // fewer codewords: each row seeded with the nearest of the first few (one
+            // CUDA-core pass), instead of testing its whole first tile exactly
+            KQ_TRY(launch_sample_hints(W, n, C, K < SAMPLE_HINT_MAX ? K : SAMPLE_HINT_MAX, idx, sms, s));
+            hint = idx;
+            hint_counts = nullptr;
+        }
         if (!hint && K >= COLD_PILOT_MIN_K) {
             int nbp = 0;
             KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K / COLD_PILOT_DIV, nullptr, nullptr, idx, nullptr, nullptr, &nbp,

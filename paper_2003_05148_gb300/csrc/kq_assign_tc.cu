@@ -1739,6 +1739,46 @@ cudaError_t launch_hint_permutation(const int32_t *hint, int64_t n, int32_t K, c
     return cudaGetLastError();
 }
 
+// Seeds for a cold assignment with few codeword tiles: hint[i] = the nearest of
+// codewords 0 .. S - 1 (fp32 direct form, first on ties; S <= SAMPLE_HINT_MAX), one
+// thread per kernel. Without a seed the tensor-core pass tests every row's first
+// tile exactly (no threshold yet); with it a row only meets the few codewords
+// nearer than its seed. (When the codebook was drawn from the kernels, the first S
+// codewords are a random sample of them.) The hints do not change the answer.
+__global__ void __launch_bounds__(256) sample_hint_kernel(const float *__restrict__ W, int64_t n,
+                                                          const float *__restrict__ C, int32_t S,
+                                                          int32_t *__restrict__ hint) {
+    __shared__ float cs[SAMPLE_HINT_MAX * D];
+    for (int e = threadIdx.x; e < S * D; e += blockDim.x) cs[e] = C[e];
+    __syncthreads();
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        float x[D];
+#pragma unroll
+        for (int j = 0; j < D; ++j) x[j] = W[i * D + j];
+        float best = __int_as_float(0x7f800000);
+        int32_t bk = 0;
+        for (int32_t k = 0; k < S; ++k) {
+            const float d = direct_distance(x, cs + k * D);
+            if (d < best) {
+                best = d;
+                bk = k;
+            }
+        }
+        hint[i] = bk;
+    }
+}
+
+cudaError_t launch_sample_hints(const float *W, int64_t n, const float *C, int32_t S, int32_t *hint, int num_sms,
+                                cudaStream_t s) {
+    if (S < 1 || S > SAMPLE_HINT_MAX) return cudaErrorInvalidValue;
+    const int64_t want = (n + 255) / 256;
+    const int64_t blocks = want < 8LL * num_sms ? want : 8LL * num_sms;
+    launch_begin(s);
+    sample_hint_kernel<<<(unsigned)blocks, 256, 0, s>>>(W, n, C, S, hint);
+    launch_end(s, "sample_hint_kernel");
+    return cudaGetLastError();
+}
+
 cudaError_t launch_dist_block_sums(const float *dist, int64_t n, double *blocksum, int *nblocksum, cudaStream_t s) {
     const int64_t blocks = (n + 255) / 256;
     launch_begin(s);

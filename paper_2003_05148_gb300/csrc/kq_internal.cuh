@@ -362,6 +362,10 @@ cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Heade
 cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const float *Cpk, int32_t K,
                              const int32_t *hint, const int32_t *perm, int32_t *idx, float *dist, double *blocksum,
                              int *nblocksum, Header *hdr, cudaStream_t s, const TcYy *yy = nullptr);
+// Cold-start seeds: hint[i] = the nearest of codewords 0 .. S - 1, S <= SAMPLE_HINT_MAX.
+constexpr int32_t SAMPLE_HINT_MAX = 64;
+cudaError_t launch_sample_hints(const float *W, int64_t n, const float *C, int32_t S, int32_t *hint, int num_sms,
+                                cudaStream_t s);
 // Rows grouped by their hinted codeword (cnt: K + 1 ints of scratch, perm: n ints).
 // cpos (nullable): groups ordered by cpos[hint] instead of the hint (the codebook's
 // tile order); cperm is its inverse (needed with hint_counts). hint_counts: the
