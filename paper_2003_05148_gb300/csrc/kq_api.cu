@@ -159,8 +159,11 @@ Ws carve(void *ws, int64_t n, int32_t K) {
 
 // One assignment, on the kernel tc_eligible picks. hint_counts: rows per hinted
 // codeword, when known (the fit's previous update counted them), or null.
+// packed: the workspace already holds C packed for the tensor cores (the fit's fused
+// step for small codebooks packs each new codebook).
 kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const int32_t *hint, int32_t *idx,
-                     float *dist, int *nb, const Ws &w, int sms, cudaStream_t s, const int32_t *hint_counts = nullptr) {
+                     float *dist, int *nb, const Ws &w, int sms, cudaStream_t s, const int32_t *hint_counts = nullptr,
+                     bool packed = false) {
     if (tc_eligible(n, K, sms)) {
         // A cold start with many tiles gets hints, written into idx (each row's hint is
         // read before its own answer is written, by the same CTA): on large problems
@@ -177,7 +180,7 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
             hint = idx;
             hint_counts = nullptr;
         }
-        KQ_TRY(launch_pack_codebook_tc(C, K, w.cpk, w.hdr, s));
+        if (!packed) KQ_TRY(launch_pack_codebook_tc(C, K, w.cpk, w.hdr, s));
         if (!hint && K < COLD_PILOT_MIN_K) {
             // fewer codewords: each row seeded with the nearest of the first few (one
             // CUDA-core pass), instead of testing its whole first tile exactly
@@ -255,9 +258,13 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
     // pruned assignments: the codebook's k-d order is taken once, from C_init
     const bool pruned = prune && K <= w.yy_cap && yy_sizes(K) && tc_eligible(n, K, sms);
     if (pruned) KQ_TRY(launch_codebook_order(cur, K, w.cperm, w.cpos, w.kdtmp, w.kdkey, w.nodes, w.hdr, s));
+    // small codebooks on the tensor-core path: the objective's sum, the finalise and the
+    // next codebook's packing in one launch per iteration
+    const bool fused = !pruned && !stop_on_stable && tc_eligible(n, K, sms) && tc_pack_small(K);
+    bool packed = false;  // cur is packed in the workspace
     auto assign = [&](int32_t t, const int32_t *hint, int32_t *out, const int32_t *hint_counts) -> kq_status {
         if (pruned) return run_assign_pruned(W, n, cur, K, hint, out, &nb, w, sms, s, hint_counts, nxt, t > 0);
-        return run_assign(W, n, cur, K, hint, out, nullptr, &nb, w, sms, s, hint_counts);
+        return run_assign(W, n, cur, K, hint, out, nullptr, &nb, w, sms, s, hint_counts, packed);
     };
     // Assignment t goes to idx when iters - t is even, else to the workspace's other
     // index buffer, so the final one lands in idx. Iteration t > 0 starts every row
@@ -268,7 +275,7 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
         int32_t *out = buf(t);
         const int32_t *hint = t > 0 ? buf(t - 1) : nullptr;
         if ((st = assign(t, hint, out, t > 0 ? counts : nullptr)) != KQ_OK) return st;
-        if (objective) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
+        if (objective && !fused) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
         if (t == 0) {
             KQ_TRY(launch_accumulate(W, n, out, K, w.hdr, w.acc, false, sms, s));
         } else if (!stop_on_stable) {
@@ -289,7 +296,13 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
                 return KQ_OK;
             }
         }
-        KQ_TRY(launch_finalize(w.acc, K, w.hdr, cur, nxt, counts, s, true));
+        if (fused) {
+            KQ_TRY(launch_finalize_pack_small(w.blocksum, nb, objective ? objective + t : nullptr, w.acc, K, w.hdr, cur,
+                                              nxt, counts, w.cpk, s));
+            packed = true;
+        } else {
+            KQ_TRY(launch_finalize(w.acc, K, w.hdr, cur, nxt, counts, s, true));
+        }
         float *tmp = cur;
         cur = nxt;
         nxt = tmp;

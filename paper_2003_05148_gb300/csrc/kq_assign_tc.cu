@@ -399,10 +399,10 @@ __global__ void __launch_bounds__(256) pack_codebook_tc_kernel(const float *__re
 // Both steps in one CTA, for small codebooks (one launch instead of two).
 constexpr int32_t TC_PACK_ONE_CTA = 2048;
 constexpr int TC_PACK_SMALL_THREADS = 1024;
-__global__ void __launch_bounds__(TC_PACK_SMALL_THREADS) pack_codebook_tc_small_kernel(const float *__restrict__ C,
-                                                                                       int32_t K, int32_t Kpad,
-                                                                                       float *__restrict__ Cpk,
-                                                                                       Header *hdr) {
+// The packing of a codebook of at most TC_PACK_ONE_CTA padded codewords by one CTA of
+// TC_PACK_SMALL_THREADS threads (the bounds in hdr start from 0).
+__device__ __forceinline__ void pack_small_body(const float *__restrict__ C, int32_t K, int32_t Kpad,
+                                                float *__restrict__ Cpk, Header *hdr) {
     constexpr int WARPS = TC_PACK_SMALL_THREADS / 32;
     __shared__ float s_m[WARPS];
     float m = 0.f;
@@ -424,6 +424,45 @@ __global__ void __launch_bounds__(TC_PACK_SMALL_THREADS) pack_codebook_tc_small_
         qmax = max_bits(qmax, c);
     }
     publish_bounds_tc(cmax, hmax, qmax, hdr);
+}
+
+__global__ void __launch_bounds__(TC_PACK_SMALL_THREADS) pack_codebook_tc_small_kernel(const float *__restrict__ C,
+                                                                                       int32_t K, int32_t Kpad,
+                                                                                       float *__restrict__ Cpk,
+                                                                                       Header *hdr) {
+    pack_small_body(C, K, Kpad, Cpk, hdr);
+}
+
+// One step of the fit for a small codebook (launch_finalize_pack_small): three
+// launches (the objective's sum, the finalise, the packing) in one CTA.
+__global__ void __launch_bounds__(TC_PACK_SMALL_THREADS)
+finalize_pack_small_kernel(const double *__restrict__ blocksum, int nblocks, double *obj,
+                           unsigned long long *__restrict__ acc, int32_t K, int32_t Kpad, Header *hdr,
+                           const float *C_prev, float *C_next, int32_t *__restrict__ counts, float *__restrict__ Cpk) {
+    // the objective in the order of sum_blocks_kernel: 256 strided partial sums, xor
+    // butterflies within the warps, the eight warp sums in order
+    __shared__ double wsum[8];
+    if (obj && threadIdx.x < 256) {
+        double v = 0.0;
+        for (int b = threadIdx.x; b < nblocks; b += 256) v += blocksum[b];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = v;
+    }
+    const int S = __ldcg(&hdr->upd_scale);
+    for (int k = threadIdx.x; k < K; k += TC_PACK_SMALL_THREADS) finalize_codeword(acc, k, S, C_prev, C_next, counts, true);
+    if (threadIdx.x == 0) {  // the packing's bounds start from 0
+        atomicExch(&hdr->cb_cmax, 0u);
+        atomicExch(&hdr->cb_hmax, 0u);
+        atomicExch(&hdr->cb_qmax, 0u);
+    }
+    __syncthreads();  // C_next, the warp sums and the cleared bounds, for the whole CTA
+    if (obj && threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < 8; ++w) t += wsum[w];
+        *obj = t;
+    }
+    pack_small_body(C_next, K, Kpad, Cpk, hdr);
 }
 
 // Per-row constants of the test: k0 = X2lo - Qmax (rounded down), k1 = |x| Cmax +
@@ -1482,6 +1521,21 @@ assign_tc_pruned_kernel(const float *__restrict__ W, int64_t n, const float *__r
 }
 
 int32_t tc_kpad(int32_t K) { return (K + TC_N - 1) / TC_N * TC_N; }
+
+bool tc_pack_small(int32_t K) { return tc_kpad(K) <= TC_PACK_ONE_CTA; }
+
+cudaError_t launch_finalize_pack_small(const double *blocksum, int nblocks, double *obj, unsigned long long *acc,
+                                       int32_t K, Header *hdr, const float *C_prev, float *C_next, int32_t *counts,
+                                       float *Cpk, cudaStream_t s) {
+    const int32_t Kpad = tc_kpad(K);
+    if (Kpad > TC_PACK_ONE_CTA) return cudaErrorInvalidValue;
+    launch_begin(s);
+    finalize_pack_small_kernel<<<1, TC_PACK_SMALL_THREADS, 0, s>>>(blocksum, nblocks, obj, acc, K, Kpad, hdr, C_prev,
+                                                                  C_next, counts, Cpk);
+    launch_end(s, "finalize_pack_small_kernel");
+    return cudaGetLastError();
+}
+
 
 // Which assignment kernel is faster, from measured costs on GB300: this kernel runs
 // ceil(n / 256) CTAs, one per SM at a time, each ~12K cycles of setup and teardown

@@ -362,6 +362,40 @@ cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Heade
 cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const float *Cpk, int32_t K,
                              const int32_t *hint, const int32_t *perm, int32_t *idx, float *dist, double *blocksum,
                              int *nblocksum, Header *hdr, cudaStream_t s, const TcYy *yy = nullptr);
+// The update's finalise of codeword k (sums at scale 2^S): c_k = (sum * 2^-S) / z_k
+// in fp32 (C_prev when z_k = 0), counts[k] = z_k; the accumulator row is cleared
+// unless keep. fp32 arithmetic (GB300's fp64 rate is low): sum -> fp32, exact
+// power-of-two scaling, one IEEE division; within ~1.5 ulp of the exact mean.
+__device__ __forceinline__ void finalize_codeword(unsigned long long *__restrict__ acc, int k, int S,
+                                                  const float *C_prev, float *C_next, int32_t *__restrict__ counts,
+                                                  bool keep) {
+    unsigned long long *a = acc + (int64_t)k * ACC_WORDS;
+    const long long z = (long long)a[D];
+    const float zf = (float)z;  // exact below 2^24, within half an ulp above
+    float c[D];
+#pragma unroll
+    for (int j = 0; j < D; ++j) {
+        const float sum = scalbnf(__ll2float_rn((long long)a[j]), -S);
+        c[j] = z > 0 ? __fdiv_rn(sum, zf) : C_prev[(int64_t)k * D + j];
+    }
+#pragma unroll
+    for (int j = 0; j < D; ++j) C_next[(int64_t)k * D + j] = c[j];
+    counts[k] = (int32_t)z;
+    if (keep) return;
+    ulonglong2 *a2 = reinterpret_cast<ulonglong2 *>(a);
+#pragma unroll
+    for (int w = 0; w < ACC_WORDS / 2; ++w) a2[w] = make_ulonglong2(0ull, 0ull);
+}
+
+// Codebooks the tensor-core path packs in one CTA (at most 2048 padded codewords).
+bool tc_pack_small(int32_t K);
+// One step of the fit for such codebooks, one CTA: the objective of the assignment
+// just made (obj nullable; the order of launch_sum_blocks), the update's finalise
+// with the sums kept (as launch_finalize), and C_next packed for the next assignment
+// (as launch_pack_codebook_tc).
+cudaError_t launch_finalize_pack_small(const double *blocksum, int nblocks, double *obj, unsigned long long *acc,
+                                       int32_t K, Header *hdr, const float *C_prev, float *C_next, int32_t *counts,
+                                       float *Cpk, cudaStream_t s);
 // Cold-start seeds: hint[i] = the nearest of codewords 0 .. S - 1, S <= SAMPLE_HINT_MAX.
 constexpr int32_t SAMPLE_HINT_MAX = 64;
 cudaError_t launch_sample_hints(const float *W, int64_t n, const float *C, int32_t S, int32_t *hint, int num_sms,

@@ -213,23 +213,7 @@ finalize_kernel(unsigned long long *__restrict__ acc, int32_t K, const Header *h
                 float *C_next, int32_t *__restrict__ counts, bool keep) {
     const int k = blockIdx.x * blockDim.x + threadIdx.x;
     if (k >= K) return;
-    const int S = __ldcg(&hdr->upd_scale);
-    unsigned long long *a = acc + (int64_t)k * ACC_WORDS;
-    const long long z = (long long)a[D];
-    const float zf = (float)z;  // exact below 2^24, within half an ulp above
-    float c[D];
-#pragma unroll
-    for (int j = 0; j < D; ++j) {
-        const float sum = scalbnf(__ll2float_rn((long long)a[j]), -S);
-        c[j] = z > 0 ? __fdiv_rn(sum, zf) : C_prev[(int64_t)k * D + j];
-    }
-#pragma unroll
-    for (int j = 0; j < D; ++j) C_next[(int64_t)k * D + j] = c[j];
-    counts[k] = (int32_t)z;
-    if (keep) return;
-    ulonglong2 *a2 = reinterpret_cast<ulonglong2 *>(a);
-#pragma unroll
-    for (int w = 0; w < ACC_WORDS / 2; ++w) a2[w] = make_ulonglong2(0ull, 0ull);
+    finalize_codeword(acc, k, __ldcg(&hdr->upd_scale), C_prev, C_next, counts, keep);
 }
 
 // The sums of idx_old (in acc, at the scale in hdr->upd_scale) become those of
