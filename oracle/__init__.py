@@ -228,9 +228,11 @@ def reconstruct(idx, C, codes=None, levels=None):
 
 
 def gather_rows(W, sel):
-    """Codeword initialisation: C_0[j] = W[sel[j]]."""
+    """Codeword initialisation: C_0[j] = W[sel[j]] (every sel[j] a row of W)."""
     W = _f32(W).reshape(-1, D)
     sel = np.ascontiguousarray(sel, dtype=np.int64)
+    if sel.size and (sel.min() < 0 or sel.max() >= W.shape[0]):
+        raise ValueError(f"row index outside [0, {W.shape[0]})")
     C0 = np.empty((sel.shape[0], D), np.float32)
     _load().kqo_gather_rows(_ptr(W), _ptr(sel), sel.shape[0], _ptr(C0))
     return C0

@@ -780,8 +780,8 @@ def test_fit_pruned_matches_plain(case):
              "iters0": 40000, "iters1": 40000}[case]
         K = {"k4097_ragged_tile": 4097, "k12345": 12345}.get(case, 4096)
         lay = synth.Layer("t", 64, n // 64, K, 4 * K, 70 + len(case))
-        W = synth.conv_weights(lay)[:n]
-        C0 = oracle.gather_rows(W, synth.init_selection(n, K, 71 + len(case)))
+        W = synth.conv_weights(lay)  # 64 (n // 64) kernels
+        C0 = oracle.gather_rows(W, synth.init_selection(W.shape[0], K, 71 + len(case)))
         if case == "dup_codewords":
             # exact ties between codewords far apart in the original numbering
             C0[[5, 700, 2900, 4000]] = C0[[3000, 4095, 12, 64]]

@@ -226,6 +226,15 @@ def test_k_equals_n_identity():
     assert np.array_equal(C.view(np.int32), W.view(np.int32))
 
 
+def test_gather_rows_rejects_rows_outside_w():
+    # an index past the last kernel would read past W
+    W = synth.random_kernels(100, 9, 5)
+    assert np.array_equal(oracle.gather_rows(W, [0, 99, 7]), W[[0, 99, 7]])
+    for bad in ([0, 100], [-1, 3]):
+        with pytest.raises(ValueError):
+            oracle.gather_rows(W, bad)
+
+
 def test_fit_objective_non_increasing_and_consistent():
     lay = synth.workload(1).layers[0]
     W, sel = synth.layer_inputs(lay)
