@@ -290,6 +290,25 @@ __global__ void __launch_bounds__(256) kd_leaf_search_kernel(const float *__rest
                                                              const unsigned char *__restrict__ Cpk,
                                                              const int32_t *__restrict__ cperm, int32_t K,
                                                              int32_t *__restrict__ hint) {
+    // The CTA's slots mostly share one leaf (rows are grouped by leaf): that of its first
+    // slot's row is staged in shared memory coordinate by coordinate (cs[u][kl], +inf
+    // past the tile's codewords), so a pair of codewords' coordinate u is one 8-byte load.
+    __shared__ __align__(16) float cs[D][256];
+    const int64_t cta0 = (int64_t)blockIdx.x * blockDim.x * LS_ROWS;
+    int gh = -1;
+    {
+        const int64_t r0 = perm[cta0];  // cta0 < n: the grid covers n slots
+        if ((uint64_t)r0 < (uint64_t)n) gh = leaf[r0];
+    }
+    if (gh >= 0) {
+        const float *cw = reinterpret_cast<const float *>(Cpk + (int64_t)gh * TC_TILE_BYTES + TC_TILE_H);
+        const int cntw = min(256, K - gh * 256);
+        for (int e = threadIdx.x; e < D * 256; e += blockDim.x) {
+            const int kl = e / D, u = e - kl * D;  // coalesced reads of the tile's rows
+            cs[u][kl] = kl < cntw ? __ldg(cw + e) : __int_as_float(0x7f800000);
+        }
+    }
+    __syncthreads();
     const int64_t s0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * LS_ROWS;
     if (s0 >= n) return;
     int64_t row[LS_ROWS];
@@ -320,12 +339,19 @@ __global__ void __launch_bounds__(256) kd_leaf_search_kernel(const float *__rest
         }
         const float *cw = reinterpret_cast<const float *>(Cpk + (int64_t)g[0] * TC_TILE_BYTES + TC_TILE_H);
         const int cntw = min(256, K - g[0] * 256);
+        const bool staged = g[0] == gh;
         for (int kl = 0; kl < cntw; kl += 2) {
             const bool two = kl + 1 < cntw;  // an odd last codeword pairs with +inf (never chosen)
             unsigned long long c2[D];
+            if (staged) {
 #pragma unroll
-            for (int u = 0; u < D; ++u)
-                c2[u] = pack2(__ldg(cw + kl * D + u), two ? __ldg(cw + (kl + 1) * D + u) : __int_as_float(0x7f800000));
+                for (int u = 0; u < D; ++u) c2[u] = *reinterpret_cast<const unsigned long long *>(&cs[u][kl]);
+            } else {
+#pragma unroll
+                for (int u = 0; u < D; ++u)
+                    c2[u] = pack2(__ldg(cw + kl * D + u),
+                                  two ? __ldg(cw + (kl + 1) * D + u) : __int_as_float(0x7f800000));
+            }
 #pragma unroll
             for (int r = 0; r < LS_ROWS; ++r) {
                 unsigned long long t = sub2(x2[r][0], c2[0]);
