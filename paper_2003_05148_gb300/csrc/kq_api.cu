@@ -275,7 +275,9 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
         int32_t *out = buf(t);
         const int32_t *hint = t > 0 ? buf(t - 1) : nullptr;
         if ((st = assign(t, hint, out, t > 0 ? counts : nullptr)) != KQ_OK) return st;
-        if (objective && !fused) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
+        // the objective of assignment t: with the finalise below (one launch fewer), or
+        // here when the fit may stop before it
+        if (objective && stop_on_stable) KQ_TRY(launch_sum_blocks(w.blocksum, nb, objective + t, s));
         if (t == 0) {
             KQ_TRY(launch_accumulate(W, n, out, K, w.hdr, w.acc, false, sms, s));
         } else if (!stop_on_stable) {
@@ -301,7 +303,8 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
                                               nxt, counts, w.cpk, s));
             packed = true;
         } else {
-            KQ_TRY(launch_finalize(w.acc, K, w.hdr, cur, nxt, counts, s, true));
+            KQ_TRY(launch_finalize(w.acc, K, w.hdr, cur, nxt, counts, s, true, w.blocksum, nb,
+                                   objective && !stop_on_stable ? objective + t : nullptr));
         }
         float *tmp = cur;
         cur = nxt;

@@ -434,8 +434,11 @@ cudaError_t launch_update_fallback(const float *W, int64_t n, const int32_t *idx
                                    unsigned long long *acc, int num_sms, cudaStream_t s);
 cudaError_t launch_histogram(const int32_t *idx, int64_t n, int32_t K, int32_t *counts, uint32_t *status,
                              int num_sms, cudaStream_t s);
+// obj (nullable): also the objective, the sum of the nblocks block sums (as
+// launch_sum_blocks, the same order).
 cudaError_t launch_finalize(unsigned long long *acc, int32_t K, const Header *hdr, const float *C_prev,
-                            float *C_next, int32_t *counts, cudaStream_t s, bool keep_sums = false);
+                            float *C_next, int32_t *counts, cudaStream_t s, bool keep_sums = false,
+                            const double *blocksum = nullptr, int nblocks = 0, double *obj = nullptr);
 // The fit's update after its first iteration: the exact fixed-point sums of idx_old
 // (held in acc) become those of idx_new by moving only the rows whose codeword changed.
 // moved (nullable): set to 1 when some row's codeword changed.

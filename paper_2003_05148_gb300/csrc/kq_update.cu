@@ -208,9 +208,27 @@ update_fallback_kernel(const float *__restrict__ W, int64_t n, const int32_t *__
 // only moves the rows whose codeword changed). fp32 arithmetic (GB300's fp64 rate is
 // low): sum -> fp32, exact power-of-two scaling, one IEEE division; within ~1.5 ulp
 // of the exact mean.
+// obj (nullable): CTA 0 also writes the objective of the assignment the update came
+// from, the sum of its nblocks block sums in the order of sum_blocks_kernel (256
+// strided partial sums, xor butterflies within the warps, the eight warp sums in order).
 __global__ void __launch_bounds__(256)
 finalize_kernel(unsigned long long *__restrict__ acc, int32_t K, const Header *hdr, const float *C_prev,
-                float *C_next, int32_t *__restrict__ counts, bool keep) {
+                float *C_next, int32_t *__restrict__ counts, bool keep, const double *__restrict__ blocksum,
+                int nblocks, double *obj) {
+    if (obj && blockIdx.x == 0) {
+        __shared__ double wsum[8];
+        double v = 0.0;
+        for (int b = threadIdx.x; b < nblocks; b += 256) v += blocksum[b];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = v;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            double t = 0.0;
+            for (int w = 0; w < 8; ++w) t += wsum[w];
+            *obj = t;
+        }
+    }
     const int k = blockIdx.x * blockDim.x + threadIdx.x;
     if (k >= K) return;
     finalize_codeword(acc, k, __ldcg(&hdr->upd_scale), C_prev, C_next, counts, keep);
@@ -366,9 +384,11 @@ cudaError_t launch_update_fallback(const float *W, int64_t n, const int32_t *idx
 }
 
 cudaError_t launch_finalize(unsigned long long *acc, int32_t K, const Header *hdr, const float *C_prev,
-                            float *C_next, int32_t *counts, cudaStream_t s, bool keep_sums) {
+                            float *C_next, int32_t *counts, cudaStream_t s, bool keep_sums, const double *blocksum,
+                            int nblocks, double *obj) {
     launch_begin(s);
-    finalize_kernel<<<(K + 255) / 256, 256, 0, s>>>(acc, K, hdr, C_prev, C_next, counts, keep_sums);
+    finalize_kernel<<<(K + 255) / 256, 256, 0, s>>>(acc, K, hdr, C_prev, C_next, counts, keep_sums, blocksum,
+                                                     nblocks, obj);
     launch_end(s, "finalize_kernel");
     return cudaGetLastError();
 }
