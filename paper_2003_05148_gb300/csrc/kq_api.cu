@@ -160,10 +160,15 @@ Ws carve(void *ws, int64_t n, int32_t K) {
 // One assignment, on the kernel tc_eligible picks. hint_counts: rows per hinted
 // codeword, when known (the fit's previous update counted them), or null.
 // packed: the workspace already holds C packed for the tensor cores (the fit's fused
-// step for small codebooks packs each new codebook).
+// step for small codebooks packs each new codebook). sums: where the objective's block
+// sums (w.blocksum) come from when the rows were processed in hint order: SUMS_NOW
+// (dist_block_sums_kernel), SUMS_NONE (nobody reads them), or SUMS_DEFER (the caller
+// sums *defer_dist itself; set to null when the block sums are already there).
+enum BlockSums { SUMS_NOW, SUMS_NONE, SUMS_DEFER };
 kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const int32_t *hint, int32_t *idx,
                      float *dist, int *nb, const Ws &w, int sms, cudaStream_t s, const int32_t *hint_counts = nullptr,
-                     bool packed = false) {
+                     bool packed = false, BlockSums sums = SUMS_NOW, const float **defer_dist = nullptr) {
+    if (defer_dist) *defer_dist = nullptr;
     if (tc_eligible(n, K, sms)) {
         // A cold start with many tiles gets hints, written into idx (each row's hint is
         // read before its own answer is written, by the same CTA): on large problems
@@ -203,7 +208,8 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
             KQ_TRY(launch_hint_permutation(hint, n, K, nullptr, nullptr, hint_counts, w.pcnt, w.perm, sms, s));
             float *d = dist ? dist : w.dist;
             KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K, hint, w.perm, idx, d, nullptr, nb, w.hdr, s));
-            KQ_TRY(launch_dist_block_sums(d, n, w.blocksum, nb, s));
+            if (sums == SUMS_NOW) KQ_TRY(launch_dist_block_sums(d, n, w.blocksum, nb, s));
+            if (sums == SUMS_DEFER) *defer_dist = d;
         } else {
             KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K, hint, nullptr, idx, dist, w.blocksum, nb, w.hdr, s));
         }
@@ -222,7 +228,9 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
 // first pass) the hints come from the k-d leaves, written into idx.
 kq_status run_assign_pruned(const float *W, int64_t n, const float *C, int32_t K, const int32_t *hint, int32_t *idx,
                             int *nb, const Ws &w, int sms, cudaStream_t s, const int32_t *hint_counts,
-                            const float *Cprev, bool read) {
+                            const float *Cprev, bool read, BlockSums sums = SUMS_NOW,
+                            const float **defer_dist = nullptr) {
+    if (defer_dist) *defer_dist = nullptr;
     const TcYy st{w.cperm, w.cpos, w.tdrift, w.yrec, w.ydist, yy_stride(w.yy_cap), read ? 1 : 0};
     KQ_TRY(launch_pack_codebook_tc(C, K, w.cpk, w.hdr, s, w.cperm, read ? Cprev : nullptr,
                                    read ? w.tdrift : nullptr));
@@ -233,7 +241,8 @@ kq_status run_assign_pruned(const float *W, int64_t n, const float *C, int32_t K
     }
     KQ_TRY(launch_hint_permutation(hint, n, K, w.cpos, w.cperm, hint_counts, w.pcnt, w.perm, sms, s));
     KQ_TRY(launch_assign_tc(W, n, C, w.cpk, K, hint, w.perm, idx, w.dist, nullptr, nb, w.hdr, s, &st));
-    KQ_TRY(launch_dist_block_sums(w.dist, n, w.blocksum, nb, s));
+    if (sums == SUMS_NOW) KQ_TRY(launch_dist_block_sums(w.dist, n, w.blocksum, nb, s));
+    if (sums == SUMS_DEFER) *defer_dist = w.dist;
     return KQ_OK;
 }
 
@@ -262,9 +271,15 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
     // next codebook's packing in one launch per iteration
     const bool fused = !pruned && !stop_on_stable && tc_eligible(n, K, sms) && tc_pack_small(K);
     bool packed = false;  // cur is packed in the workspace
+    // the block sums of an assignment made in hint order: summed by the delta update
+    // that follows it (one launch fewer), when the objective is wanted and that update runs
+    const bool want_sums = objective || final_obj;
+    const float *ddist = nullptr;  // the distances whose block sums the next delta update takes
     auto assign = [&](int32_t t, const int32_t *hint, int32_t *out, const int32_t *hint_counts) -> kq_status {
-        if (pruned) return run_assign_pruned(W, n, cur, K, hint, out, &nb, w, sms, s, hint_counts, nxt, t > 0);
-        return run_assign(W, n, cur, K, hint, out, nullptr, &nb, w, sms, s, hint_counts, packed);
+        const BlockSums bs = !want_sums ? SUMS_NONE : (t >= 1 && t < iters && !stop_on_stable) ? SUMS_DEFER : SUMS_NOW;
+        if (pruned)
+            return run_assign_pruned(W, n, cur, K, hint, out, &nb, w, sms, s, hint_counts, nxt, t > 0, bs, &ddist);
+        return run_assign(W, n, cur, K, hint, out, nullptr, &nb, w, sms, s, hint_counts, packed, bs, &ddist);
     };
     // Assignment t goes to idx when iters - t is even, else to the workspace's other
     // index buffer, so the final one lands in idx. Iteration t > 0 starts every row
@@ -281,7 +296,7 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
         if (t == 0) {
             KQ_TRY(launch_accumulate(W, n, out, K, w.hdr, w.acc, false, sms, s));
         } else if (!stop_on_stable) {
-            KQ_TRY(launch_accumulate_delta(W, n, hint, out, K, w.hdr, w.acc, sms, s));
+            KQ_TRY(launch_accumulate_delta(W, n, hint, out, K, w.hdr, w.acc, sms, s, nullptr, ddist, w.blocksum, &nb));
         } else {
             KQ_TRY(cudaMemsetAsync(&w.hdr->fit_moved, 0, sizeof(uint32_t), s));
             KQ_TRY(launch_accumulate_delta(W, n, hint, out, K, w.hdr, w.acc, sms, s, &w.hdr->fit_moved));
@@ -482,7 +497,7 @@ kq_status kq_assign(const float *W, int64_t n, const float *C, int32_t K, const 
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     Ws w = carve(ws, n, K);
     int nb = 0;
-    return run_assign(W, n, C, K, hint, idx, dist, &nb, w, sms, s);
+    return run_assign(W, n, C, K, hint, idx, dist, &nb, w, sms, s, nullptr, false, SUMS_NONE);  // no objective out
 }
 
 kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int32_t K, const float *C_prev,

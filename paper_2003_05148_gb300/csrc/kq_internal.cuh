@@ -441,10 +441,13 @@ cudaError_t launch_finalize(unsigned long long *acc, int32_t K, const Header *hd
                             const double *blocksum = nullptr, int nblocks = 0, double *obj = nullptr);
 // The fit's update after its first iteration: the exact fixed-point sums of idx_old
 // (held in acc) become those of idx_new by moving only the rows whose codeword changed.
-// moved (nullable): set to 1 when some row's codeword changed.
+// moved (nullable): set to 1 when some row's codeword changed. dist (nullable): also
+// the per-256-row sums of dist into blocksum (as launch_dist_block_sums), their count
+// into *nblocksum.
 cudaError_t launch_accumulate_delta(const float *W, int64_t n, const int32_t *idx_old, const int32_t *idx_new,
                                     int32_t K, Header *hdr, unsigned long long *acc, int num_sms, cudaStream_t s,
-                                    uint32_t *moved = nullptr);
+                                    uint32_t *moved = nullptr, const float *dist = nullptr,
+                                    double *blocksum = nullptr, int *nblocksum = nullptr);
 // obj[j] = obj[from] for from < j <= to (the objective of a fit stopped at a fixed point).
 cudaError_t launch_fill_objective(double *obj, int32_t from, int32_t to, cudaStream_t s);
 

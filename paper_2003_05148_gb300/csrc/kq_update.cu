@@ -239,14 +239,32 @@ finalize_kernel(unsigned long long *__restrict__ acc, int32_t K, const Header *h
 // and added to the new one's (the same fixed-point values the full accumulation
 // adds, so the result is the full accumulation's, bit for bit; integer arithmetic
 // is exact whatever the order). Rows that kept their codeword cost two index loads.
+// dist (nullable): the assignment's distances, whose per-256-row sums go to
+// blocksum[b] exactly as dist_block_sums_kernel computes them (the CTA works on whole
+// 256-row blocks, one thread per row).
 __global__ void __launch_bounds__(256)
 accumulate_delta_kernel(const float *__restrict__ W, int64_t n, const int32_t *__restrict__ idx_old,
                         const int32_t *__restrict__ idx_new, int32_t K, Header *hdr,
-                        unsigned long long *__restrict__ acc, uint32_t *moved) {
+                        unsigned long long *__restrict__ acc, uint32_t *moved, const float *__restrict__ dist,
+                        double *__restrict__ blocksum) {
+    __shared__ F2 ws[8];
     const int S = __ldcg(&hdr->upd_scale);
     bool bad = false, any = false;
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+    const int64_t nblk = (n + 255) / 256;
+    for (int64_t blk = blockIdx.x; blk < nblk; blk += gridDim.x) {  // block-uniform trip count
+        const int64_t i = blk * 256 + threadIdx.x;
+        if (dist) {
+            const F2 v = f2_warp_sum(i < n ? __ldcs(dist + i) : 0.f);
+            if ((threadIdx.x & 31) == 0) ws[threadIdx.x >> 5] = v;
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                F2 t{0.f, 0.f};
+                for (int w = 0; w < 8; ++w) t = f2_add(t, ws[w]);
+                blocksum[blk] = f2_to_double(t);
+            }
+            __syncthreads();  // ws is the next block's
+        }
+        if (i >= n) continue;
         const int32_t a = __ldcs(idx_old + i), b = __ldcs(idx_new + i);
         if (a == b) continue;
         any = true;
@@ -270,12 +288,14 @@ accumulate_delta_kernel(const float *__restrict__ W, int64_t n, const int32_t *_
 
 cudaError_t launch_accumulate_delta(const float *W, int64_t n, const int32_t *idx_old, const int32_t *idx_new,
                                     int32_t K, Header *hdr, unsigned long long *acc, int num_sms, cudaStream_t s,
-                                    uint32_t *moved) {
+                                    uint32_t *moved, const float *dist, double *blocksum, int *nblocksum) {
     int64_t blocks = (n + 255) / 256;
+    if (dist) *nblocksum = (int)blocks;
     if (blocks > 8LL * num_sms) blocks = 8LL * num_sms;
     if (blocks < 1) blocks = 1;
     launch_begin(s);
-    accumulate_delta_kernel<<<(unsigned)blocks, 256, 0, s>>>(W, n, idx_old, idx_new, K, hdr, acc, moved);
+    accumulate_delta_kernel<<<(unsigned)blocks, 256, 0, s>>>(W, n, idx_old, idx_new, K, hdr, acc, moved, dist,
+                                                             blocksum);
     launch_end(s, "accumulate_delta_kernel");
     return cudaGetLastError();
 }
