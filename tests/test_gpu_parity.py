@@ -585,6 +585,34 @@ def test_fit_zero_iterations_and_identity():
     assert bits_equal(C_g, W) and np.array_equal(idx_g, np.arange(500)) and np.all(obj_g == 0.0)
 
 
+@pytest.mark.parametrize("cfg,li,flags", [(2, 0, 0), (3, 8, 0), (4, 9, 0), (4, 9, kq.STOP_ON_STABLE),
+                                           (4, 9, kq.FIT_PRUNE)])
+def test_fit_objective_optional(cfg, li, flags):
+    # The objective's sums ride along with other kernels (the finalise, the delta update)
+    # or are skipped when no objective is asked for: codebook, indices and counts are
+    # the same either way, and the objective is that of a separate pass over the
+    # distances (dist_block_sums + sum_blocks order), i.e. the oracle's within 1e-12.
+    lay, W, C0 = _layer(cfg, li)
+    n, K, T = W.shape[0], C0.shape[0], 4
+    out = []
+    for with_obj in (True, False):
+        C = torch.empty(K, 9, dtype=torch.float32, device=dev())
+        idx = torch.empty(n, dtype=torch.int32, device=dev())
+        counts = torch.empty(K, dtype=torch.int32, device=dev())
+        obj = torch.full((T + 1,), float("nan"), dtype=torch.float64, device=dev()) if with_obj else None
+        ws = kq.workspace(n, K, dev())
+        kq.kq_fit_codebook(to_dev(W), to_dev(C0), T, C, idx, counts, obj, ws, flags=flags)
+        assert kq.kq_device_status(ws)[0] == 0
+        out.append((C.cpu().numpy(), idx.cpu().numpy(), counts.cpu().numpy(), None if obj is None else obj.cpu().numpy()))
+    (Ca, ia, ca, oa), (Cb, ib, cb, _) = out
+    assert bits_equal(Ca, Cb) and np.array_equal(ia, ib) and np.array_equal(ca, cb)
+    assert np.all(np.isfinite(oa))
+    # the last objective is the final assignment's: the oracle's distances to C, summed
+    idx_ref, dist_ref = oracle.assign(W, Ca, threads=THREADS)
+    assert check_indices(W, Ca, ia, idx_ref) == 0
+    assert oa[-1] == pytest.approx(oracle.objective(dist_ref), rel=1e-12)
+
+
 def test_fit_deterministic():
     lay, W, C0 = _layer(2)
     a = _gpu_fit(W, C0, 4)
