@@ -165,9 +165,12 @@ Ws carve(void *ws, int64_t n, int32_t K) {
 // (dist_block_sums_kernel), SUMS_NONE (nobody reads them), or SUMS_DEFER (the caller
 // sums *defer_dist itself; set to null when the block sums are already there).
 enum BlockSums { SUMS_NOW, SUMS_NONE, SUMS_DEFER };
+// normed: the packing bounds are cleared and C's largest norm is in place
+// (launch_finalize_norm_tc).
 kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const int32_t *hint, int32_t *idx,
                      float *dist, int *nb, const Ws &w, int sms, cudaStream_t s, const int32_t *hint_counts = nullptr,
-                     bool packed = false, BlockSums sums = SUMS_NOW, const float **defer_dist = nullptr) {
+                     bool packed = false, BlockSums sums = SUMS_NOW, const float **defer_dist = nullptr,
+                     bool normed = false) {
     if (defer_dist) *defer_dist = nullptr;
     if (tc_eligible(n, K, sms)) {
         // A cold start with many tiles gets hints, written into idx (each row's hint is
@@ -185,7 +188,7 @@ kq_status run_assign(const float *W, int64_t n, const float *C, int32_t K, const
             hint = idx;
             hint_counts = nullptr;
         }
-        if (!packed) KQ_TRY(launch_pack_codebook_tc(C, K, w.cpk, w.hdr, s));
+        if (!packed) KQ_TRY(launch_pack_codebook_tc(C, K, w.cpk, w.hdr, s, nullptr, nullptr, nullptr, normed));
         if (!hint && K < COLD_PILOT_MIN_K) {
             // fewer codewords: each row seeded with the nearest of the first few (one
             // CUDA-core pass), instead of testing its whole first tile exactly
@@ -271,6 +274,10 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
     // next codebook's packing in one launch per iteration
     const bool fused = !pruned && !stop_on_stable && tc_eligible(n, K, sms) && tc_pack_small(K);
     bool packed = false;  // cur is packed in the workspace
+    // larger codebooks on the tensor-core path: the finalise also takes the new
+    // codebook's largest norm (the packing's first step)
+    const bool fnorm = !pruned && !stop_on_stable && tc_eligible(n, K, sms) && !tc_pack_small(K);
+    bool normed = false;  // cur's largest norm is in place
     // the block sums of an assignment made in hint order: summed by the delta update
     // that follows it (one launch fewer), when the objective is wanted and that update runs
     const bool want_sums = objective || final_obj;
@@ -279,7 +286,7 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
         const BlockSums bs = !want_sums ? SUMS_NONE : (t >= 1 && t < iters && !stop_on_stable) ? SUMS_DEFER : SUMS_NOW;
         if (pruned)
             return run_assign_pruned(W, n, cur, K, hint, out, &nb, w, sms, s, hint_counts, nxt, t > 0, bs, &ddist);
-        return run_assign(W, n, cur, K, hint, out, nullptr, &nb, w, sms, s, hint_counts, packed, bs, &ddist);
+        return run_assign(W, n, cur, K, hint, out, nullptr, &nb, w, sms, s, hint_counts, packed, bs, &ddist, normed);
     };
     // Assignment t goes to idx when iters - t is even, else to the workspace's other
     // index buffer, so the final one lands in idx. Iteration t > 0 starts every row
@@ -317,6 +324,10 @@ kq_status run_fit(const float *W, int64_t n, int32_t K, const float *C_init, int
             KQ_TRY(launch_finalize_pack_small(w.blocksum, nb, objective ? objective + t : nullptr, w.acc, K, w.hdr, cur,
                                               nxt, counts, w.cpk, s));
             packed = true;
+        } else if (fnorm) {
+            KQ_TRY(launch_finalize_norm_tc(w.blocksum, nb, objective ? objective + t : nullptr, w.acc, K, w.hdr, cur,
+                                           nxt, counts, s));
+            normed = true;
         } else {
             KQ_TRY(launch_finalize(w.acc, K, w.hdr, cur, nxt, counts, s, true, w.blocksum, nb,
                                    objective && !stop_on_stable ? objective + t : nullptr));

@@ -439,16 +439,8 @@ __global__ void __launch_bounds__(TC_PACK_SMALL_THREADS)
 finalize_pack_small_kernel(const double *__restrict__ blocksum, int nblocks, double *obj,
                            unsigned long long *__restrict__ acc, int32_t K, int32_t Kpad, Header *hdr,
                            const float *C_prev, float *C_next, int32_t *__restrict__ counts, float *__restrict__ Cpk) {
-    // the objective in the order of sum_blocks_kernel: 256 strided partial sums, xor
-    // butterflies within the warps, the eight warp sums in order
     __shared__ double wsum[8];
-    if (obj && threadIdx.x < 256) {
-        double v = 0.0;
-        for (int b = threadIdx.x; b < nblocks; b += 256) v += blocksum[b];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-        if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = v;
-    }
+    if (obj) objective_sum_256(blocksum, nblocks, obj, wsum);  // block-uniform
     const int S = __ldcg(&hdr->upd_scale);
     for (int k = threadIdx.x; k < K; k += TC_PACK_SMALL_THREADS) finalize_codeword(acc, k, S, C_prev, C_next, counts, true);
     if (threadIdx.x == 0) {  // the packing's bounds start from 0
@@ -456,13 +448,26 @@ finalize_pack_small_kernel(const double *__restrict__ blocksum, int nblocks, dou
         atomicExch(&hdr->cb_hmax, 0u);
         atomicExch(&hdr->cb_qmax, 0u);
     }
-    __syncthreads();  // C_next, the warp sums and the cleared bounds, for the whole CTA
-    if (obj && threadIdx.x == 0) {
-        double t = 0.0;
-        for (int w = 0; w < 8; ++w) t += wsum[w];
-        *obj = t;
-    }
+    __syncthreads();  // C_next and the cleared bounds, for the whole CTA
     pack_small_body(C_next, K, Kpad, Cpk, hdr);
+}
+
+// The fit's finalise for larger codebooks (launch_finalize_norm_tc): finalize_kernel's
+// work (one codeword per thread, CTA 0 also the objective) and the new codewords'
+// largest norm into hdr->cb_craw (codebook_norm_tc_kernel's work), whose bounds the
+// launcher cleared.
+__global__ void __launch_bounds__(256)
+finalize_norm_tc_kernel(const double *__restrict__ blocksum, int nblocks, double *obj,
+                        unsigned long long *__restrict__ acc, int32_t K, Header *hdr, const float *C_prev,
+                        float *C_next, int32_t *__restrict__ counts) {
+    if (obj && blockIdx.x == 0) {
+        __shared__ double wsum[8];
+        objective_sum_256(blocksum, nblocks, obj, wsum);
+    }
+    const int k = blockIdx.x * blockDim.x + threadIdx.x;
+    if (k < K) finalize_codeword(acc, k, __ldcg(&hdr->upd_scale), C_prev, C_next, counts, true);
+    const float m = warp_max_bits(k < K ? codeword_norm_ru(C_next, k) : 0.f);  // this thread's own write
+    if ((threadIdx.x & 31) == 0) atomicMax(&hdr->cb_craw, __float_as_uint(m));
 }
 
 // Per-row constants of the test: k0 = X2lo - Qmax (rounded down), k1 = |x| Cmax +
@@ -1550,11 +1555,31 @@ bool tc_eligible(int64_t n, int32_t K, int num_sms) {
     return n >= (int64_t)TC_ROWS * num_sms || tc_us < cc_us;
 }
 
-cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Header *hdr, cudaStream_t s,
-                                    const int32_t *cperm, const float *Cprev, float *tdrift) {
+cudaError_t launch_finalize_norm_tc(const double *blocksum, int nblocks, double *obj, unsigned long long *acc,
+                                    int32_t K, Header *hdr, const float *C_prev, float *C_next, int32_t *counts,
+                                    cudaStream_t s) {
     cudaError_t e = cudaMemsetAsync(&hdr->cb_cmax, 0, 4 * sizeof(uint32_t), s);  // cb_cmax .. cb_craw
     if (e != cudaSuccess) return e;
+    launch_begin(s);
+    finalize_norm_tc_kernel<<<(K + 255) / 256, 256, 0, s>>>(blocksum, nblocks, obj, acc, K, hdr, C_prev, C_next,
+                                                            counts);
+    launch_end(s, "finalize_norm_tc_kernel");
+    return cudaGetLastError();
+}
+
+cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Header *hdr, cudaStream_t s,
+                                    const int32_t *cperm, const float *Cprev, float *tdrift, bool normed) {
+    cudaError_t e;
     const int32_t Kpad = tc_kpad(K);
+    if (normed && Kpad > TC_PACK_ONE_CTA) {  // bounds cleared, largest norm in place
+        launch_begin(s);
+        pack_codebook_tc_kernel<<<(Kpad + 255) / 256, 256, 0, s>>>(C, K, Kpad, Cpk, hdr, cperm,
+                                                                    tdrift ? Cprev : nullptr, Cprev ? tdrift : nullptr);
+        launch_end(s, "pack_codebook_tc_kernel");
+        return cudaGetLastError();
+    }
+    e = cudaMemsetAsync(&hdr->cb_cmax, 0, 4 * sizeof(uint32_t), s);  // cb_cmax .. cb_craw
+    if (e != cudaSuccess) return e;
     if (Kpad <= TC_PACK_ONE_CTA && !cperm && !tdrift) {
         launch_begin(s);
         pack_codebook_tc_small_kernel<<<1, TC_PACK_SMALL_THREADS, 0, s>>>(C, K, Kpad, Cpk, hdr);

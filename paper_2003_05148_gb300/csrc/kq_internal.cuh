@@ -355,9 +355,11 @@ cudaError_t launch_assign(const float *W, int64_t n, const float *Cd, const floa
 bool tc_eligible(int64_t n, int32_t K, int num_sms);
 // cperm (nullable): pack the codebook in that order; Cprev, tdrift (nullable): the
 // largest codeword move per tile since Cprev.
+// normed: the bounds are cleared and hdr->cb_craw holds C's largest norm already
+// (launch_finalize_norm_tc).
 cudaError_t launch_pack_codebook_tc(const float *C, int32_t K, float *Cpk, Header *hdr, cudaStream_t s,
                                     const int32_t *cperm = nullptr, const float *Cprev = nullptr,
-                                    float *tdrift = nullptr);
+                                    float *tdrift = nullptr, bool normed = false);
 // yy (nullable): the pruned assignment over a codebook packed in yy->cperm order.
 cudaError_t launch_assign_tc(const float *W, int64_t n, const float *C, const float *Cpk, int32_t K,
                              const int32_t *hint, const int32_t *perm, int32_t *idx, float *dist, double *blocksum,
@@ -387,6 +389,34 @@ __device__ __forceinline__ void finalize_codeword(unsigned long long *__restrict
     for (int w = 0; w < ACC_WORDS / 2; ++w) a2[w] = make_ulonglong2(0ull, 0ull);
 }
 
+// The objective of an assignment from its block sums, in the order of
+// sum_blocks_kernel: threads 0-255 take strided partial sums, xor butterflies within
+// their warps, then thread 0 adds the eight warp sums in order. Every thread of the
+// CTA calls it (a CTA barrier inside); wsum: 8 doubles of shared memory.
+__device__ __forceinline__ void objective_sum_256(const double *__restrict__ blocksum, int nblocks, double *obj,
+                                                  double *wsum) {
+    if (threadIdx.x < 256) {
+        double v = 0.0;
+        for (int b = threadIdx.x; b < nblocks; b += 256) v += blocksum[b];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = v;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < 8; ++w) t += wsum[w];
+        *obj = t;
+    }
+}
+
+// The fit's finalise for larger codebooks on the tensor-core path: launch_finalize
+// (sums kept; obj nullable as there) that also reduces the new codebook's largest norm
+// into hdr->cb_craw after clearing the packing bounds, so the next
+// launch_pack_codebook_tc can skip both (normed).
+cudaError_t launch_finalize_norm_tc(const double *blocksum, int nblocks, double *obj, unsigned long long *acc,
+                                    int32_t K, Header *hdr, const float *C_prev, float *C_next, int32_t *counts,
+                                    cudaStream_t s);
 // Codebooks the tensor-core path packs in one CTA (at most 2048 padded codewords).
 bool tc_pack_small(int32_t K);
 // One step of the fit for such codebooks, one CTA: the objective of the assignment

@@ -217,17 +217,7 @@ finalize_kernel(unsigned long long *__restrict__ acc, int32_t K, const Header *h
                 int nblocks, double *obj) {
     if (obj && blockIdx.x == 0) {
         __shared__ double wsum[8];
-        double v = 0.0;
-        for (int b = threadIdx.x; b < nblocks; b += 256) v += blocksum[b];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-        if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = v;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            double t = 0.0;
-            for (int w = 0; w < 8; ++w) t += wsum[w];
-            *obj = t;
-        }
+        objective_sum_256(blocksum, nblocks, obj, wsum);
     }
     const int k = blockIdx.x * blockDim.x + threadIdx.x;
     if (k >= K) return;
