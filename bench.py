@@ -614,6 +614,14 @@ def run_only(args):
         fc_it = torch.zeros(1, dtype=torch.int32, device=dev)
         calls["fcquant"] = lambda: kq.kq_quantize_scalars_6bit(v, 100, levels, fc_codes, fc_it, ws)
         n, K = args.m, 64
+    if args.only in ("fit", "prunefit"):
+        # the fit as a user calls it (the workload's iteration count, from the seeded
+        # initial codebook), without or with the tile pruning that stands for Yinyang
+        T_fit = synth.workload(WORKLOAD_CFG).iters
+        C_fit = torch.empty_like(C)
+        obj_fit = torch.empty(T_fit + 1, dtype=torch.float64, device=dev)
+        fit_flags = kq.FIT_PRUNE if args.only == "prunefit" else 0
+        calls[args.only] = lambda: kq.kq_fit_codebook(W, C, T_fit, C_fit, idx2, counts, obj_fit, ws, flags=fit_flags)
     f = calls[args.only]
     # --l2-drain: after every call, outside its events, read a 512 MB buffer (larger
     # than L2), so that the call's dirty L2 lines go to DRAM before the next call
@@ -633,6 +641,8 @@ def run_only(args):
         if drain is not None:
             drain.sum()
     torch.cuda.synchronize()
+    # the work of the last pruned fit (nothing else has run on ws since)
+    tiles = kq.kq_fit_prune_stats(ws) if args.only == "prunefit" else None
     st, flags = kq.kq_device_status(ws)
     ms = [a.elapsed_time(b) for a, b in evs]
     out = {"only": args.only, "n": n, "K": K, "reps": args.reps, "ms_mean": statistics.mean(ms),
@@ -644,6 +654,17 @@ def run_only(args):
         k_s, e_s, tr_s = search_out["r"]
         out["K_chosen"], out["error"], out["trials"] = k_s, e_s, len(tr_s)
         out["trace"] = [[a, round(b, 6)] for a, b in tr_s]
+    if args.only in ("fit", "prunefit"):
+        evals = (T_fit + 1) * n * K  # kernel x codeword distances the fit's assignments decide
+        out["iters"] = T_fit
+        out["effective_evals_per_s"] = evals / (statistics.mean(ms) * 1e-3)
+        if tiles is not None:
+            tiles_run, tiles_all = tiles
+            out["tiles_run"], out["tiles_all"] = tiles_run, tiles_all
+            frac = tiles_run / tiles_all if tiles_all else 1.0
+            out["executed_fraction"] = frac
+            # (256-kernel block, 256-codeword tile) pairs the tensor core processed
+            out["executed_evals_per_s"] = frac * out["effective_evals_per_s"]
     if args.only == "fcquant":
         it = int(fc_it.item())
         out["iters_run"] = it
@@ -756,7 +777,7 @@ def main():
     ap.add_argument("--ref-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--only", choices=["assign", "update", "quantize", "reconstruct", "gradstep", "levelgrad",
-                                       "fcquant", "search", "fusedrecon"],
+                                       "fcquant", "search", "fusedrecon", "fit", "prunefit"],
                     help="profiling aid: time one entry point on its own (no bench line)")
     ap.add_argument("--n", type=int, default=4194304)
     ap.add_argument("--K", type=int, default=65536)

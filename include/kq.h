@@ -229,9 +229,10 @@ kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int
  *              every update), and a tile that cannot hold a codeword as close as
  *              the kernel's previous one is skipped for a whole block of kernels.
  *              The outputs are identical either way; the workspace holds the
- *              bounds. (On the 2048 x 2048 stress layer it skips 16-46% of the
- *              tiles per update but each processed tile costs more, so it is not
- *              the default.)
+ *              bounds, and kq_fit_prune_stats reports the tiles processed. (On
+ *              the 2048 x 2048 stress layer it skips 16-46% of the tiles per
+ *              update, 29.5% of a 10-update fit's tile work, but each processed
+ *              tile costs more, so it is not the default.)
  *   idx        n int32 output: the final assignment (device)
  *   counts     K int32 output: cluster sizes of the final assignment (device)
  *   objective  iters + 1 fp64 outputs (device) or NULL: Eq. 1 objective per step,
@@ -244,6 +245,22 @@ kq_status kq_update_centroids(const float *W, int64_t n, const int32_t *idx, int
 kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_init, int32_t iters, int32_t flags,
                           float *C_out, int32_t *idx, int32_t *counts, double *objective, int32_t *iters_run,
                           void *ws, size_t ws_bytes, kq_stream_t stream);
+
+/* Work of a pruned fit (KQ_FIT_PRUNE; the tile skipping that stands for
+ * Yinyang k-means, Sec. 4.1), for reporting executed against effective
+ * distance evaluations. Call it after a kq_fit_codebook call with
+ * KQ_FIT_PRUNE and before any other call on the same workspace:
+ *   tiles_run  1 uint64 output (host): (256-kernel block, 256-codeword tile)
+ *              pairs the tensor core processed over all the fit's assignments
+ *   tiles_all  1 uint64 output (host): the pairs those assignments hold in
+ *              all, i.e. what the same fit processes without pruning
+ * Both are 0 when that fit did not take the pruned path (sizes outside
+ * 4096..65536 codewords or off the tensor-core path). Each pair stands for
+ * up to 65,536 kernel x codeword distances (fewer in a ragged last block or
+ * tile). Synchronises `stream`. Errors: KQ_ERR_INVALID_ARG for a NULL output;
+ * KQ_ERR_WORKSPACE / KQ_ERR_ALIGNMENT for a bad workspace. */
+kq_status kq_fit_prune_stats(void *ws, size_t ws_bytes, uint64_t *tiles_run, uint64_t *tiles_all,
+                             kq_stream_t stream);
 
 /* Adaptive codebook size, Algorithm 1 with Eq. 3 (Sec. 3.1): a binary search for
  * the smallest codebook that keeps a layer's quality above a target. The paper's

@@ -60,7 +60,7 @@ __global__ void test_inject_kernel(Header *h, uint32_t faults, uint32_t limit) {
 
 namespace {
 
-constexpr int32_t KQ_ABI_VERSION = 6;
+constexpr int32_t KQ_ABI_VERSION = 7;
 constexpr int32_t HINT_ORDER_MIN_K = 4096;  // warm starts in hint order from 16 codeword tiles on
 // Cold assignments with many codeword tiles start from a pilot pass: rows against the
 // first K / COLD_PILOT_DIV codewords (a random sample when the codebook was drawn from
@@ -467,6 +467,21 @@ kq_status kq_device_status(void *ws, size_t ws_bytes, kq_stream_t stream, uint32
     return KQ_OK;
 }
 
+kq_status kq_fit_prune_stats(void *ws, size_t ws_bytes, uint64_t *tiles_run, uint64_t *tiles_all,
+                             kq_stream_t stream) {
+    if (!tiles_run || !tiles_all) return KQ_ERR_INVALID_ARG;
+    kq_status st = check_ws_header(ws, ws_bytes);
+    if (st != KQ_OK) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    Header *h = static_cast<Header *>(ws);
+    unsigned long long v[2] = {0ull, 0ull};  // yy_tiles_run, yy_tiles_all (adjacent)
+    KQ_TRY(cudaMemcpyAsync(v, &h->yy_tiles_run, sizeof(v), cudaMemcpyDeviceToHost, s));
+    KQ_TRY(cudaStreamSynchronize(s));
+    *tiles_run = v[0];
+    *tiles_all = v[1];
+    return KQ_OK;
+}
+
 kq_status kq_test_inject_wait_fault(void *ws, size_t ws_bytes, uint32_t faults, uint32_t wait_limit,
                                     kq_stream_t stream) {
     if ((faults & ~(KQ_TEST_SKIP_ARRIVAL | KQ_TEST_STOP_TILE_STREAM)) != 0u) return KQ_ERR_INVALID_ARG;
@@ -545,6 +560,8 @@ kq_status kq_fit_codebook(const float *W, int64_t n, int32_t K, const float *C_i
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     const Ws w = carve(ws, n, K);
     const bool stop = (flags & KQ_STOP_ON_STABLE) != 0;
+    if (flags & KQ_FIT_PRUNE)  // the pruned passes' work counters (kq_fit_prune_stats)
+        KQ_TRY(cudaMemsetAsync(&w.hdr->yy_tiles_run, 0, 2 * sizeof(unsigned long long), s));
     if (small_fit_eligible(n, K)) {  // the whole fit in one cooperative launch
         const int nblk = (int)((n + 255) / 256) + MAX_PART_BLOCKS;
         KQ_TRY(launch_small_fit(W, n, C_init, K, iters, C_out, idx, counts, objective, w.acc, w.cbuf0, w.cbuf1,

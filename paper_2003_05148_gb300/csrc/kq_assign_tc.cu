@@ -1493,6 +1493,10 @@ assign_tc_pruned_kernel(const float *__restrict__ W, int64_t n, const float *__r
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TC_COLS) : "memory");
     }
+    if (tid == 0) {  // the work done against the work of an unpruned pass (kq_fit_prune_stats)
+        atomicAdd(&hdr->yy_tiles_run, (unsigned long long)nt);
+        atomicAdd(&hdr->yy_tiles_all, (unsigned long long)ntiles);
+    }
     if (epi && row < n) {
         idx[row] = bi;
         if (dist) dist[row] = best;

@@ -4,6 +4,7 @@
 
 #include <cuda_runtime.h>
 #include <stdint.h>
+#include <stddef.h>
 
 #include "kq.h"
 
@@ -74,8 +75,12 @@ struct Header {
     unsigned long long lacc[3][LEVELS][2];  // level fit: (weight sum, fixed-point sum) per level
     double obj;                         // codebook-size search: objective of the last fit
     uint32_t yy_cnorm;                  // pruned fit: largest norm of the initial codebook (fp32 bits)
+    unsigned long long yy_tiles_run;    // pruned fit: (row block, codeword tile) pairs processed, all passes
+    unsigned long long yy_tiles_all;    // pruned fit: the pairs the same passes hold in all
 };
 static_assert(sizeof(Header) <= 4096, "header too large");
+static_assert(offsetof(Header, yy_tiles_all) == offsetof(Header, yy_tiles_run) + 8,
+              "kq_fit_prune_stats reads both counters with one copy");
 
 struct WsLayout {
     size_t cd, acc, part, blocksum, cbuf0, cbuf1, cp, cq, cpk, dist, perm, pcnt, prev;

@@ -28,7 +28,7 @@ EXPORTS = ["kq_status_string", "kq_abi_version", "kq_kernel_launches", "kq_works
            "kq_compression_report", "kq_conventional_ratio", "kq_assign_noalloc", "kq_quantize_scalars_6bit",
            "kq_codebook_grad_step", "kq_levels_grad_step", "kq_search_codebook_size", "kq_quantize_reconstruct",
            "kq_seed_indices", "kq_trace_start", "kq_trace_stop", "kq_trace_count", "kq_trace_get",
-           "kq_test_inject_wait_fault", "kq_fit_layers"]
+           "kq_test_inject_wait_fault", "kq_fit_layers", "kq_fit_prune_stats"]
 
 
 class KQError(RuntimeError):
@@ -72,6 +72,7 @@ def lib() -> ctypes.CDLL:
             "kq_trace_get": ([i32, ctypes.POINTER(ctypes.c_char_p), ctypes.POINTER(ctypes.c_float)], ctypes.c_int),
             "kq_workspace_bytes": ([i64, i32], sz),
             "kq_device_status": ([P, sz, P, P], ctypes.c_int),
+            "kq_fit_prune_stats": ([P, sz, P, P, P], ctypes.c_int),
             "kq_init_codebook": ([P, i64, P, i32, P, P, sz, P], ctypes.c_int),
             "kq_assign": ([P, i64, P, i32, P, P, P, P, sz, P], ctypes.c_int),
             "kq_update_centroids": ([P, i64, P, i32, P, P, P, P, sz, P], ctypes.c_int),
@@ -205,6 +206,15 @@ def kq_device_status(ws: torch.Tensor, stream=None):
     with torch.cuda.device(c.device):
         st = lib().kq_device_status(ptr, ws.numel(), c.stream(stream), ctypes.byref(flags))
     return st, flags.value
+
+
+def kq_fit_prune_stats(ws, stream=None):
+    """(tiles_run, tiles_all): the (block, tile) pairs the last pruned fit on `ws` processed,
+    and those its assignments hold in all (synchronises the stream)."""
+    run, total = ctypes.c_uint64(0), ctypes.c_uint64(0)
+    c = _Call("kq_fit_prune_stats")
+    c(c.ptr(ws, "ws", torch.uint8), ws.numel(), ctypes.byref(run), ctypes.byref(total), c.stream(stream))
+    return run.value, total.value
 
 
 def kq_test_inject_wait_fault(ws, faults: int, wait_limit: int, stream=None) -> None:

@@ -37,7 +37,7 @@ def test_exports_every_declared_symbol(lib):
 
 
 def test_status_strings_and_version(lib):
-    assert kq.kq_abi_version() == 6
+    assert kq.kq_abi_version() == 7
     for code, name in kq.STATUS_NAMES.items():
         assert kq.kq_status_string(code) == name
     assert kq.kq_status_string(99) == "KQ_ERR_UNKNOWN"
@@ -96,6 +96,11 @@ def test_host_validation_before_any_device_work(lib):
     assert L.kq_reconstruct(good, 1024, good, 16, None, None, odd, good, ws_bytes, None) == 2  # W_out alignment
     assert L.kq_init_codebook(good, 1024, good, 2000, good, good, ws_bytes, None) == 1
     assert L.kq_device_status(None, 0, None, None) == 6
+    u64 = ctypes.c_uint64()
+    assert L.kq_fit_prune_stats(None, 0, ctypes.byref(u64), ctypes.byref(u64), None) == 6  # no workspace
+    assert L.kq_fit_prune_stats(good, 4096, None, ctypes.byref(u64), None) == 1  # no output
+    assert L.kq_fit_prune_stats(odd, 4096, ctypes.byref(u64), ctypes.byref(u64), None) == 2  # ws alignment
+    assert L.kq_fit_prune_stats(good, 4095, ctypes.byref(u64), ctypes.byref(u64), None) == 6  # too small
     nan = float("nan")
     assert L.kq_quantize_scalars_6bit(good, 0, 10, good, good, None, good, 4096, None) == 1  # m = 0
     assert L.kq_quantize_scalars_6bit(good, 100, 100001, good, good, None, good, 4096, None) == 1
@@ -221,6 +226,8 @@ def test_cuda_failure_returns_status_without_device(lib):
     assert L.kq_reconstruct(good, 1024, good, 16, None, None, good, good, ws_bytes, None) == 4
     assert L.kq_quantize_reconstruct(good, 1024, good, 16, good, None, good, good, ws_bytes, None) == 4
     assert L.kq_device_status(good, ws_bytes, None, None) == 4
+    u64 = ctypes.c_uint64()
+    assert L.kq_fit_prune_stats(good, ws_bytes, ctypes.byref(u64), ctypes.byref(u64), None) == 4
     assert L.kq_trace_start(4) == 4  # no device to make events on
     jobs = (kq.LayerJob * 2)(_job(1), _job(2))
     assert L.kq_fit_layers(jobs, 2, 3, 10, kq.FIT_PRUNE, None) == 4

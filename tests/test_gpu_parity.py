@@ -459,7 +459,7 @@ def test_fit_stepwise(cfg, li):
     assert np.all(obj_T[1:] <= obj_T[:-1] * (1 + 1e-6))
 
 
-def _gpu_fit_run(W, C0, iters, flags):
+def _gpu_fit_run(W, C0, iters, flags, stats=None):
     n, K = W.shape[0], C0.shape[0]
     C = torch.empty(K, 9, dtype=torch.float32, device=dev())
     idx = torch.empty(n, dtype=torch.int32, device=dev())
@@ -467,6 +467,8 @@ def _gpu_fit_run(W, C0, iters, flags):
     obj = torch.empty(iters + 1, dtype=torch.float64, device=dev())
     ws = kq.workspace(n, K, dev())
     run = kq.kq_fit_codebook(to_dev(W), to_dev(C0), iters, C, idx, counts, obj, ws, flags=flags)
+    if stats is not None:  # the pruned passes' work, read before any other call on ws
+        stats.extend(kq.kq_fit_prune_stats(ws))
     st, _ = kq.kq_device_status(ws)
     assert st == 0
     return (C.cpu().numpy(), idx.cpu().numpy(), counts.cpu().numpy(), obj.cpu().numpy()), run
@@ -790,9 +792,19 @@ def test_trace_times_every_launch_of_a_fit():
 # --------------------------------------------------------------------------- pruned fit
 
 def _fit_both(W, C0, iters):
-    pruned, run_p = _gpu_fit_run(W, C0, iters, kq.FIT_PRUNE)
-    plain, run_q = _gpu_fit_run(W, C0, iters, 0)
-    return pruned, plain
+    # both fits, and the pruned one's work: every assignment of the fit runs pruned, so
+    # its passes hold (iters + 1) x blocks x tiles (256-kernel block, 256-codeword tile)
+    # pairs, of which the first pass (no bounds yet) processes all
+    n, K = W.shape[0], C0.shape[0]
+    per_pass = -(-n // 256) * -(-K // 256)
+    work, none = [], []
+    pruned, run_p = _gpu_fit_run(W, C0, iters, kq.FIT_PRUNE, work)
+    plain, run_q = _gpu_fit_run(W, C0, iters, 0, none)
+    tiles_run, tiles_all = work
+    assert tiles_all == (iters + 1) * per_pass
+    assert per_pass <= tiles_run <= tiles_all
+    assert none == [0, 0]  # a fresh workspace, a fit without pruning
+    return pruned, plain, tiles_run / tiles_all
 
 
 @pytest.mark.parametrize("case", ["k4096", "k4097_ragged_tile", "k12345", "dup_codewords", "resnet_k16384",
@@ -814,7 +826,7 @@ def test_fit_pruned_matches_plain(case):
             # exact ties between codewords far apart in the original numbering
             C0[[5, 700, 2900, 4000]] = C0[[3000, 4095, 12, 64]]
         iters = {"iters0": 0, "iters1": 1}.get(case, iters)
-    pruned, plain = _fit_both(W, C0, iters)
+    pruned, plain, _ = _fit_both(W, C0, iters)
     for a, b in zip(pruned, plain):
         assert bits_equal(a, b)
 
@@ -847,9 +859,10 @@ def test_fit_pruned_full_size_stress():
     # codebook), 3 iterations, pruned and plain bit for bit; sampled rows of the
     # final assignment against the oracle
     lay, W, C0 = _layer(5)
-    pruned, plain = _fit_both(W, C0, 3)
+    pruned, plain, frac = _fit_both(W, C0, 3)
     for a, b in zip(pruned, plain):
         assert bits_equal(a, b)
+    assert frac < 1.0  # the later passes skip tiles
     C_T, idx_T = pruned[0], pruned[1]
     rows = np.sort(synth.below(synth.stream_key(lay.seed, 11), 2048, lay.n))
     idx_ref, _ = oracle.assign(W[rows], C_T, threads=THREADS)
